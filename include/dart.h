@@ -1,0 +1,181 @@
+/*
+ * dart.h -- C ABI of the GB300 (sm_103a) hot path of DART, "Decoded Attention
+ * over Recurrent sTates" (arXiv 2608.02032).
+ *
+ * The hot path of one DART block, from the precomputed token projections to
+ * the block output (the same boundary as the paper's kernel benchmark,
+ * Sec. 5.3 "Kernel Forward Time and Inference Cache"):
+ *   dart_chunk_scan   Mamba-2 chunked SSD scan (Sec. 2; App. A) that also
+ *                     keeps every chunk state contribution as a chunk state
+ *                     memory M_j = Delta H_[j] (Sec. 3).
+ *   dart_sma_forward  token-conditioned key/value decoding from the memories,
+ *                     causal state-memory attention over chunks (Sec. 3;
+ *                     App. B.1; Alg. 1) and the gated residual merge
+ *                     Y = Y_ssd + SiLU(z) R (Sec. 3).
+ *   dart_decode_step  one autoregressive token over the chunk-memory cache
+ *                     and the running state (Sec. 4 "Inference Cache").
+ *
+ * Conventions shared by every entry point
+ *   - Every tensor pointer is a DEVICE pointer owned by the caller, 16-byte
+ *     aligned, contiguous and row-major in the shapes given below (the
+ *     paper's table of compact tensor shapes, App. B.2). The library keeps
+ *     no reference to any pointer after the call returns.
+ *   - The library never allocates device memory. Scratch comes from the
+ *     caller's `workspace` (device memory of at least
+ *     dart_workspace_size(dims, op) bytes, 256-byte aligned).
+ *   - Every call is asynchronous on `stream` (a cudaStream_t; NULL is the
+ *     legacy default stream) and does not synchronise the host.
+ *   - Arguments are validated on the host before anything is launched; a
+ *     call that returns an error has written nothing.
+ *   - Token and chunk indices are 0-based: token t lies in chunk t / S, the
+ *     paper's 1-based c(t) = ceil(t / S) (Sec. 3).
+ *   - Head h reads projection group h / (H / G) (G = 1 in the paper).
+ *
+ * Numerical readings where the paper is silent
+ *   - a_t = exp(dt_t * A_h) and the write term is dt_t * B_t^T X_t; dt is the
+ *     post-softplus step size.
+ *   - RMSNorm (Qbar, Ebar) and the memory inverse RMS r use unit weight and
+ *     dims.eps (App. B.1 names eps without a value).
+ *   - The state before the first token is zero (App. A).
+ *   - All accumulation is fp32. With mem_dtype = DART_BF16 the memories are
+ *     stored in bf16 and r is computed from the stored values.
+ */
+#ifndef DART_H_
+#define DART_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    DART_OK = 0,
+    DART_ERR_INVALID_ARG = 1,  /* NULL or misaligned pointer, bad dims, H % G != 0, eps <= 0 */
+    DART_ERR_UNSUPPORTED = 2,  /* valid but not built: L % S != 0, P/N/S outside the set below */
+    DART_ERR_WORKSPACE = 3,    /* workspace NULL/misaligned or smaller than dart_workspace_size */
+    DART_ERR_CUDA = 4,         /* a CUDA call failed; see dart_last_cuda_error() */
+    DART_ERR_TIMEOUT = 5       /* a device-side wait gave up (see dart_get_device_status) */
+} dart_status;
+
+typedef enum { DART_F32 = 0, DART_BF16 = 1 } dart_dtype;
+
+/* Problem sizes in the paper's notation (App. B.2). */
+typedef struct {
+    int64_t batch;     /* Bsz */
+    int64_t seqlen;    /* L (ignored by dart_decode_step) */
+    int64_t nheads;    /* H */
+    int64_t ngroups;   /* G, must divide H */
+    int64_t headdim;   /* P, value axis of a memory */
+    int64_t dstate;    /* N, key axis of a memory (SSD state size) */
+    int64_t chunk;     /* S, chunk size; M = L / S memories per (b, h) */
+    int32_t in_dtype;  /* dart_dtype of the token inputs X, B, C, Q, E, z and x, b, c, q, e, z */
+    int32_t mem_dtype; /* dart_dtype of the chunk memories M and the decode cache */
+    int32_t out_dtype; /* dart_dtype of the outputs Y_ssd, Y, R and the decode output y */
+    float eps;         /* RMSNorm / inverse-RMS epsilon, > 0 */
+} dart_dims;
+
+/* Supported sizes: P in {16, 32, 64}, N in {16, 32, 64, 128},
+ * S in {16, 32, 64, 128, 256} with L % S == 0. Supported dtype triples
+ * (in, mem, out): (F32, F32, F32), (BF16, F32, F32), (BF16, BF16, F32) and
+ * (BF16, BF16, BF16). Accumulation is fp32 in every case. Outputs and
+ * memories heavy-tailed enough that rounding them to bf16 costs several
+ * percent of their RMS, so fp32 outputs are the default for bf16 inputs. */
+
+typedef enum {
+    DART_OP_CHUNK_SCAN = 0,
+    DART_OP_SMA_FORWARD = 1,
+    DART_OP_DECODE_STEP = 2
+} dart_op;
+
+/* Human-readable name of a status code (static storage, never NULL). */
+const char* dart_status_string(dart_status status);
+
+/* The cudaError_t of the most recent DART_ERR_CUDA on this thread (0 if none). */
+int dart_last_cuda_error(void);
+
+/* Bytes of workspace `op` needs for `dims` (0 if none). Returns 0 for
+ * invalid dims too; the entry point then reports the error. */
+size_t dart_workspace_size(const dart_dims* dims, int op);
+
+/*
+ * Chunked SSD scan with chunk state memories (Sec. 2 SSD recurrence;
+ * App. A eqs. "mamba2_chunk_state" and "mamba2_delta_h_chunk"; Sec. 3
+ * equation for Delta H_[c]):
+ *   Y_ssd_t = C_t H_t with H_t = exp(dt_t A_h) H_{t-1} + dt_t B_t^T X_t,
+ *   M[b, c, h] = sum_{s in chunk c} exp(sum_{k=s+1}^{e(c)} dt_k A_h) dt_s B_s^T X_s.
+ * Inputs:  X  (Bsz, L, H, P) in_dtype;  dt (Bsz, L, H) fp32 (post-softplus);
+ *          A  (H) fp32;  Bm, Cm (Bsz, L, G, N) in_dtype.
+ * Outputs: Y_ssd (Bsz, L, H, P) out_dtype;  M (Bsz, M, H, N, P) mem_dtype;
+ *          rM (Bsz, M, H, N) fp32 or NULL: r[n] = (mean_p M[n, p]^2 + eps)^-1/2
+ *          of the stored memory (App. B.1);
+ *          final_state (Bsz, H, N, P) fp32 or NULL: H_{L-1}.
+ */
+dart_status dart_chunk_scan(const dart_dims* dims, const void* X, const float* dt,
+                            const float* A, const void* Bm, const void* Cm, void* Y_ssd,
+                            void* M, float* rM, float* final_state, void* workspace,
+                            size_t workspace_bytes, void* stream);
+
+/*
+ * State-memory attention and gated merge (Sec. 3 value/key readouts, chunk
+ * logit, softmax over earlier chunks and R_t; App. B.1 normalised score
+ * branch; Alg. 1 streaming form; Sec. 3 "Gated Residual Integration"):
+ *   Qbar = RMSNorm(Q_t), Ebar = RMSNorm(E_t),
+ *   l_{t,j} = Qbar (r_j (.) (M_j Ebar)) / sqrt(N),  V_{t,j} = C_t M_j,
+ *   g = softmax over j < t / S,  R_t = sum_j g_j V_{t,j},
+ *   lse_t = log sum_j exp(l_{t,j}),  Y = Y_ssd + SiLU(z) R.
+ * Tokens of chunk 0 have R = 0, lse = -inf and Y = Y_ssd.
+ * Inputs:  M (Bsz, M, H, N, P) mem_dtype;  rM (Bsz, M, H, N) fp32 or NULL
+ *          (NULL: computed from M into the workspace);
+ *          Q, Cm (Bsz, L, G, N) in_dtype;  E (Bsz, L, G, P) in_dtype;
+ *          z (Bsz, L, H) in_dtype gate logits;  Y_ssd (Bsz, L, H, P) out_dtype.
+ * Outputs: Y (Bsz, L, H, P) out_dtype;  R (Bsz, L, H, P) out_dtype or NULL;
+ *          lse (Bsz, L, H) fp32 or NULL.
+ */
+dart_status dart_sma_forward(const dart_dims* dims, const void* M, const float* rM,
+                             const void* Q, const void* Cm, const void* E, const void* z,
+                             const void* Y_ssd, void* Y, void* R, float* lse, void* workspace,
+                             size_t workspace_bytes, void* stream);
+
+/*
+ * One decode step over the chunk-memory cache (the persistent inference
+ * cache of Sec. 4 "Inference Cache" and Sec. 5.3; the paper gives no decode
+ * algorithm, this is the reading that makes prefill followed by decode equal
+ * a longer prefill). For the token at index pos (pos tokens absorbed before
+ * it) and i = pos / S completed chunks:
+ *   a = exp(dt A_h);  state <- a state + dt b^T x;
+ *   partial <- dt b^T x if pos % S == 0, else a partial + dt b^T x;
+ *   y = c state + SiLU(z) R, R = SMA over cache memories j < i (as above);
+ *   if (pos + 1) % S == 0: cache[b, i, h] <- partial (and i < m_cap).
+ * In/out:  cache (Bsz, m_cap, H, N, P) mem_dtype; memories j < i are read,
+ *          slot i is written when its chunk completes;
+ *          state, partial (Bsz, H, N, P) fp32, updated in place.
+ * Inputs:  x (Bsz, H, P) in_dtype; dt (Bsz, H) fp32; A (H) fp32;
+ *          b, c, q (Bsz, G, N) in_dtype; e (Bsz, G, P) in_dtype; z (Bsz, H) in_dtype.
+ * Outputs: y (Bsz, H, P) out_dtype; lse (Bsz, H) fp32 or NULL.
+ * Requires pos >= 0 and pos / S <= m_cap; dims.seqlen is ignored.
+ */
+dart_status dart_decode_step(const dart_dims* dims, int64_t pos, int64_t m_cap, void* cache,
+                             float* state, float* partial, const void* x, const float* dt,
+                             const float* A, const void* b, const void* c, const void* q,
+                             const void* e, const void* z, void* y, float* lse,
+                             void* workspace, size_t workspace_bytes, void* stream);
+
+/* Number of kernels this library has launched in this process since it was
+ * loaded (all entry points, all threads). A diagnostic for benchmarks. */
+uint64_t dart_launch_count(void);
+
+/*
+ * Synchronises `stream`, then reports and clears the device status word that
+ * kernels set when a bounded device-side wait gives up: DART_ERR_TIMEOUT if
+ * one did since the last call, DART_ERR_CUDA if the synchronisation failed,
+ * else DART_OK.
+ */
+dart_status dart_get_device_status(void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* DART_H_ */

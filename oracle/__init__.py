@@ -51,11 +51,12 @@ def _load():
         lib.oracle_chunk_memories.argtypes = [_i64] * 7 + [_dp] * 5
         lib.oracle_sma.argtypes = [_i64] * 7 + [ctypes.c_double] + [_dp] * 4 + [_i64, _ip] + [_dp] * 3
         lib.oracle_merge.argtypes = [_i64, _i64] + [_dp] * 4
+        lib.oracle_memory_inverse_rms.argtypes = [_i64, _i64, ctypes.c_double, _dp, _dp]
         lib.oracle_decode_step.argtypes = (
             [_i64] * 6 + [ctypes.c_double, _i64, _i64] + [_dp] * 13
         )
         for f in ("oracle_ssd_recurrence", "oracle_chunk_memories", "oracle_sma",
-                  "oracle_merge", "oracle_decode_step"):
+                  "oracle_merge", "oracle_decode_step", "oracle_memory_inverse_rms"):
             getattr(lib, f).restype = None
         _lib = lib
     return _lib
@@ -131,6 +132,15 @@ def sma(dH, Q, Cm, E, S: int, eps: float, H: int | None = None, tokens=None, wan
     if want_g:
         return R, lse, g.reshape(R.shape[:-1] + (M,))
     return R, lse
+
+
+def memory_inverse_rms(dH, eps: float):
+    """Inverse RMS of each memory row along P (App. B.1): shape ``dH.shape[:-1]``."""
+    dH = _f64(dH)
+    P = dH.shape[-1]
+    r = np.empty(dH.shape[:-1])
+    _load().oracle_memory_inverse_rms(r.size, P, float(eps), _ptr(dH), _ptr(r))
+    return r
 
 
 def merge(Yssd, z, R):

@@ -252,6 +252,20 @@ void oracle_sma(i64 Bsz, i64 L, i64 H, i64 G, i64 P, i64 N, i64 S, double eps,
 }
 
 /*
+ * Inverse RMS of every memory row along the value axis (App. B.1):
+ *   r_{j,n} = (mean_p dH_j[n,p]^2 + eps)^(-1/2),  rows = Bsz * M * H * N.
+ * Pinned: closed forms for constant and two-valued rows.
+ */
+void oracle_memory_inverse_rms(i64 rows, i64 P, double eps, const double* dH, double* r)
+{
+    for (i64 i = 0; i < rows; ++i) {
+        double ss = 0.0;
+        for (i64 p = 0; p < P; ++p) ss += dH[i * P + p] * dH[i * P + p];
+        r[i] = 1.0 / sqrt(ss / (double)P + eps);
+    }
+}
+
+/*
  * Gated residual merge (Sec. 3, "Gated Residual Integration"):
  *   Y = Y_ssd + SiLU(z) R,  one gate logit z per (b, t, h) row.
  * Pinned: z = 0 reproduces Y_ssd exactly (the SMA-removal special case).

@@ -1,0 +1,101 @@
+"""Allocating wrappers over the C ABI: the calls a PyTorch user makes.
+
+Each wrapper allocates its outputs and workspace with PyTorch on the inputs'
+device and calls one entry point of ``libdart.so`` on the current stream.
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass
+
+import torch
+
+from . import binding as B
+
+
+def _dtype_code(t: torch.Tensor) -> int:
+    if t.dtype not in B.DART_DTYPE:
+        raise TypeError(f"unsupported dtype {t.dtype}; use float32 or bfloat16")
+    return B.DART_DTYPE[t.dtype]
+
+
+def _workspace(dims, op, device) -> torch.Tensor | None:
+    n = B.dart_workspace_size(dims, op)
+    if n == 0:
+        return None
+    return torch.empty(n, dtype=torch.uint8, device=device)
+
+
+@dataclass
+class ScanOut:
+    Y_ssd: torch.Tensor  # (Bsz, L, H, P)
+    M: torch.Tensor      # (Bsz, M, H, N, P) chunk state memories
+    rM: torch.Tensor     # (Bsz, M, H, N) inverse RMS of each memory row
+    final_state: torch.Tensor | None  # (Bsz, H, N, P) fp32
+
+
+def chunk_scan(X, dt, A, Bm, Cm, chunk: int, eps: float = 1e-6, final_state: bool = False,
+               workspace: torch.Tensor | None = None, mem_dtype=torch.float32,
+               out_dtype=torch.float32) -> ScanOut:
+    """Chunked SSD scan with chunk state memories (``dart_chunk_scan``)."""
+    Bsz, L, H, P = X.shape
+    G, N = Bm.shape[2], Bm.shape[3]
+    code = _dtype_code(X)
+    dims = B.make_dims(Bsz, L, H, G, P, N, chunk, code, mem_dtype, out_dtype, eps=eps)
+    M = L // chunk
+    dev = X.device
+    Y = torch.empty(X.shape, dtype=out_dtype, device=dev)
+    Mem = torch.empty(Bsz, M, H, N, P, dtype=mem_dtype, device=dev)
+    rM = torch.empty(Bsz, M, H, N, dtype=torch.float32, device=dev)
+    fs = torch.empty(Bsz, H, N, P, dtype=torch.float32, device=dev) if final_state else None
+    ws = workspace if workspace is not None else _workspace(dims, B.DART_OP_CHUNK_SCAN, dev)
+    B.dart_chunk_scan(dims, X, dt, A, Bm, Cm, Y, Mem, rM, fs, ws)
+    return ScanOut(Y, Mem, rM, fs)
+
+
+@dataclass
+class SmaOut:
+    Y: torch.Tensor             # (Bsz, L, H, P) gated merge
+    R: torch.Tensor | None      # (Bsz, L, H, P) SMA readout
+    lse: torch.Tensor           # (Bsz, L, H) fp32 logsumexp over earlier chunks
+
+
+def sma_forward(Mem, rM, Q, Cm, E, z, Y_ssd, chunk: int, eps: float = 1e-6, want_R: bool = True,
+                workspace: torch.Tensor | None = None) -> SmaOut:
+    """State-memory attention and gated merge (``dart_sma_forward``)."""
+    Bsz, L, H, P = Y_ssd.shape
+    G, N = Q.shape[2], Q.shape[3]
+    dims = B.make_dims(Bsz, L, H, G, P, N, chunk, _dtype_code(Q), _dtype_code(Mem),
+                       _dtype_code(Y_ssd), eps=eps)
+    dev = Y_ssd.device
+    Y = torch.empty_like(Y_ssd)
+    R = torch.empty_like(Y_ssd) if want_R else None
+    lse = torch.empty(Bsz, L, H, dtype=torch.float32, device=dev)
+    ws = workspace
+    if rM is None and ws is None:
+        ws = _workspace(dims, B.DART_OP_SMA_FORWARD, dev)
+    B.dart_sma_forward(dims, Mem, rM, Q, Cm, E, z, Y_ssd, Y, R, lse, ws)
+    return SmaOut(Y, R, lse)
+
+
+def prefill_forward(X, dt, A, Bm, Cm, Q, E, z, chunk: int, eps: float = 1e-6, want_R=False,
+                    mem_dtype=torch.float32, out_dtype=torch.float32):
+    """Whole DART hot path of one block for a prefill: scan, SMA and merge."""
+    s = chunk_scan(X, dt, A, Bm, Cm, chunk, eps, mem_dtype=mem_dtype, out_dtype=out_dtype)
+    o = sma_forward(s.M, s.rM, Q, Cm, E, z, s.Y_ssd, chunk, eps, want_R=want_R)
+    return s, o
+
+
+def decode_step(cache, state, partial, x, dt, A, b, c, q, e, z, pos: int, chunk: int,
+                eps: float = 1e-6, out_dtype=torch.float32):
+    """One decode step (``dart_decode_step``); cache, state and partial are updated in place.
+
+    Returns (y ``Bsz x H x P``, lse ``Bsz x H``).
+    """
+    Bsz, m_cap, H, N, P = cache.shape
+    G = b.shape[1]
+    dims = B.make_dims(Bsz, 1, H, G, P, N, chunk, _dtype_code(x), _dtype_code(cache),
+                       out_dtype, eps=eps)
+    y = torch.empty(x.shape, dtype=out_dtype, device=x.device)
+    lse = torch.empty(Bsz, H, dtype=torch.float32, device=x.device)
+    B.dart_decode_step(dims, pos, m_cap, cache, state, partial, x, dt, A, b, c, q, e, z, y, lse)
+    return y, lse

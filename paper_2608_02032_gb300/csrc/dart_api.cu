@@ -1,0 +1,246 @@
+// C ABI of the DART hot path: host-side validation, workspace layout and
+// kernel dispatch. Declarations and the contract are in include/dart.h.
+#include <atomic>
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include "dart.h"
+#include "kernels.h"
+
+namespace {
+
+thread_local int t_last_cuda_error = 0;
+
+typedef long long i64;
+
+dart_status cuda_fail(cudaError_t e) {
+    t_last_cuda_error = (int)e;
+    return DART_ERR_CUDA;
+}
+
+bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+bool is_pow2(int64_t v) { return v > 0 && (v & (v - 1)) == 0; }
+
+size_t align256(size_t v) { return (v + 255) & ~(size_t)255; }
+
+// Supported (in, mem, out) dtype triples.
+enum class Combo { kFFF, kBFF, kBBF, kBBB, kNone };
+
+Combo combo_of(const dart_dims* d) {
+    const int i = d->in_dtype, m = d->mem_dtype, o = d->out_dtype;
+    if (i == DART_F32 && m == DART_F32 && o == DART_F32) return Combo::kFFF;
+    if (i == DART_BF16 && m == DART_F32 && o == DART_F32) return Combo::kBFF;
+    if (i == DART_BF16 && m == DART_BF16 && o == DART_F32) return Combo::kBBF;
+    if (i == DART_BF16 && m == DART_BF16 && o == DART_BF16) return Combo::kBBB;
+    return Combo::kNone;
+}
+
+// Calls L<Tin, Tmem, Tout>::run(args...) for the dtype triple of d.
+template <template <typename, typename, typename> class L, typename... Args>
+cudaError_t dispatch(const dart_dims* d, Args&&... args) {
+    typedef __nv_bfloat16 bf;
+    switch (combo_of(d)) {
+        case Combo::kFFF: return L<float, float, float>::run(args...);
+        case Combo::kBFF: return L<bf, float, float>::run(args...);
+        case Combo::kBBF: return L<bf, bf, float>::run(args...);
+        case Combo::kBBB: return L<bf, bf, bf>::run(args...);
+        default: return cudaErrorInvalidValue;
+    }
+}
+
+template <typename I, typename M, typename O> struct ScanL {
+    static cudaError_t run(const dart::ScanArgs& a, cudaStream_t s) {
+        return dart::launch_chunk_scan_simt<I, M, O>(a, s);
+    }
+};
+template <typename I, typename M, typename O> struct SmaL {
+    static cudaError_t run(const dart::SmaArgs& a, cudaStream_t s) {
+        return dart::launch_sma_forward_simt<I, M, O>(a, s);
+    }
+};
+template <typename I, typename M, typename O> struct DecodeL {
+    static cudaError_t run(const dart::DecodeArgs& a, cudaStream_t s) {
+        return dart::launch_decode_step<I, M, O>(a, s);
+    }
+};
+
+// Shared validation of the sizes in dims (without the op-specific parts).
+dart_status check_dims(const dart_dims* d, bool need_seqlen) {
+    if (d == nullptr) return DART_ERR_INVALID_ARG;
+    if (d->batch <= 0 || d->nheads <= 0 || d->ngroups <= 0 || d->headdim <= 0 || d->dstate <= 0 ||
+        d->chunk <= 0)
+        return DART_ERR_INVALID_ARG;
+    if (need_seqlen && d->seqlen <= 0) return DART_ERR_INVALID_ARG;
+    if (d->nheads % d->ngroups != 0) return DART_ERR_INVALID_ARG;
+    if (!(d->eps > 0.0f)) return DART_ERR_INVALID_ARG;
+    if (d->in_dtype != DART_F32 && d->in_dtype != DART_BF16) return DART_ERR_INVALID_ARG;
+    if (d->mem_dtype != DART_F32 && d->mem_dtype != DART_BF16) return DART_ERR_INVALID_ARG;
+    if (d->out_dtype != DART_F32 && d->out_dtype != DART_BF16) return DART_ERR_INVALID_ARG;
+    if (combo_of(d) == Combo::kNone) return DART_ERR_UNSUPPORTED;
+    const int64_t P = d->headdim, N = d->dstate, S = d->chunk;
+    if (!(P == 16 || P == 32 || P == 64)) return DART_ERR_UNSUPPORTED;
+    if (!(N == 16 || N == 32 || N == 64 || N == 128)) return DART_ERR_UNSUPPORTED;
+    if (!(is_pow2(S) && S >= 16 && S <= 256)) return DART_ERR_UNSUPPORTED;
+    if (need_seqlen && d->seqlen % S != 0) return DART_ERR_UNSUPPORTED;
+    // every offset below is computed in 64-bit, but grid dimensions are 32-bit
+    if (need_seqlen && (d->seqlen / S) * d->nheads > 65535 * 64) return DART_ERR_UNSUPPORTED;
+    if (d->batch > 65535 || d->nheads > 65535) return DART_ERR_UNSUPPORTED;
+    return DART_OK;
+}
+
+struct ScanWs {
+    size_t cum_off, dh_off, total;
+};
+
+ScanWs scan_ws(const dart_dims* d) {
+    const i64 M = d->seqlen / d->chunk;
+    ScanWs w;
+    w.cum_off = 0;
+    w.dh_off = align256((size_t)(d->batch * d->nheads * M * d->chunk) * sizeof(float));
+    w.total = w.dh_off +
+              align256((size_t)(d->batch * M * d->nheads * d->dstate * d->headdim) * sizeof(float));
+    return w;
+}
+
+size_t sma_ws(const dart_dims* d) {
+    const i64 M = d->seqlen / d->chunk;
+    return align256((size_t)(d->batch * M * d->nheads * d->dstate) * sizeof(float));
+}
+
+std::atomic<uint64_t> g_launches{0};
+
+}  // namespace
+
+namespace dart {
+void note_launches(int n) { g_launches.fetch_add((uint64_t)n, std::memory_order_relaxed); }
+}  // namespace dart
+
+extern "C" {
+
+uint64_t dart_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
+
+
+const char* dart_status_string(dart_status s) {
+    switch (s) {
+        case DART_OK: return "DART_OK";
+        case DART_ERR_INVALID_ARG: return "DART_ERR_INVALID_ARG: invalid argument";
+        case DART_ERR_UNSUPPORTED: return "DART_ERR_UNSUPPORTED: valid but unsupported sizes or dtypes";
+        case DART_ERR_WORKSPACE: return "DART_ERR_WORKSPACE: workspace missing, misaligned or too small";
+        case DART_ERR_CUDA: return "DART_ERR_CUDA: a CUDA call failed (see dart_last_cuda_error)";
+        case DART_ERR_TIMEOUT: return "DART_ERR_TIMEOUT: a device-side wait gave up";
+    }
+    return "unknown dart_status";
+}
+
+int dart_last_cuda_error(void) { return t_last_cuda_error; }
+
+size_t dart_workspace_size(const dart_dims* d, int op) {
+    switch (op) {
+        case DART_OP_CHUNK_SCAN:
+            if (check_dims(d, true) != DART_OK) return 0;
+            return scan_ws(d).total;
+        case DART_OP_SMA_FORWARD:
+            if (check_dims(d, true) != DART_OK) return 0;
+            return sma_ws(d);
+        case DART_OP_DECODE_STEP:
+            return 0;
+    }
+    return 0;
+}
+
+dart_status dart_chunk_scan(const dart_dims* d, const void* X, const float* dt, const float* A,
+                            const void* Bm, const void* Cm, void* Y_ssd, void* M, float* rM,
+                            float* final_state, void* ws, size_t ws_bytes, void* stream) {
+    dart_status st = check_dims(d, true);
+    if (st != DART_OK) return st;
+    const void* req[] = {X, dt, A, Bm, Cm, Y_ssd, M};
+    for (const void* p : req)
+        if (p == nullptr || !aligned16(p)) return DART_ERR_INVALID_ARG;
+    if ((rM && !aligned16(rM)) || (final_state && !aligned16(final_state)))
+        return DART_ERR_INVALID_ARG;
+    const ScanWs w = scan_ws(d);
+    if (ws == nullptr || ((uintptr_t)ws & 255u) != 0 || ws_bytes < w.total)
+        return DART_ERR_WORKSPACE;
+
+    dart::ScanArgs a;
+    a.B = d->batch; a.L = d->seqlen; a.H = d->nheads; a.G = d->ngroups;
+    a.P = d->headdim; a.N = d->dstate; a.S = d->chunk; a.eps = d->eps;
+    a.X = X; a.dt = dt; a.A = A; a.Bm = Bm; a.Cm = Cm; a.Y = Y_ssd; a.M = M; a.rM = rM;
+    a.final_state = final_state;
+    a.cum = (float*)((char*)ws + w.cum_off);
+    a.dH32 = (float*)((char*)ws + w.dh_off);
+    cudaStream_t s = (cudaStream_t)stream;
+    cudaError_t e = dispatch<ScanL>(d, a, s);
+    return e == cudaSuccess ? DART_OK : cuda_fail(e);
+}
+
+dart_status dart_sma_forward(const dart_dims* d, const void* M, const float* rM, const void* Q,
+                             const void* Cm, const void* E, const void* z, const void* Y_ssd,
+                             void* Y, void* R, float* lse, void* ws, size_t ws_bytes,
+                             void* stream) {
+    dart_status st = check_dims(d, true);
+    if (st != DART_OK) return st;
+    const void* req[] = {M, Q, Cm, E, z, Y_ssd, Y};
+    for (const void* p : req)
+        if (p == nullptr || !aligned16(p)) return DART_ERR_INVALID_ARG;
+    if ((rM && !aligned16(rM)) || (R && !aligned16(R)) || (lse && !aligned16(lse)))
+        return DART_ERR_INVALID_ARG;
+    const size_t need = rM == nullptr ? sma_ws(d) : 0;
+    if (need > 0 && (ws == nullptr || ((uintptr_t)ws & 255u) != 0 || ws_bytes < need))
+        return DART_ERR_WORKSPACE;
+
+    cudaStream_t s = (cudaStream_t)stream;
+    const float* r = rM;
+    if (r == nullptr) {
+        const i64 rows = d->batch * (d->seqlen / d->chunk) * d->nheads * d->dstate;
+        float* rws = (float*)ws;
+        cudaError_t e = d->mem_dtype == DART_F32
+                            ? dart::launch_memory_rms<float>(M, rws, rows, d->headdim, d->eps, s)
+                            : dart::launch_memory_rms<__nv_bfloat16>(M, rws, rows, d->headdim,
+                                                                      d->eps, s);
+        if (e != cudaSuccess) return cuda_fail(e);
+        r = rws;
+    }
+    dart::SmaArgs a;
+    a.B = d->batch; a.L = d->seqlen; a.H = d->nheads; a.G = d->ngroups;
+    a.P = d->headdim; a.N = d->dstate; a.S = d->chunk; a.eps = d->eps;
+    a.M = M; a.rM = r; a.Q = Q; a.Cm = Cm; a.E = E; a.z = z; a.Yssd = Y_ssd; a.Y = Y; a.R = R;
+    a.lse = lse;
+    cudaError_t e = dispatch<SmaL>(d, a, s);
+    return e == cudaSuccess ? DART_OK : cuda_fail(e);
+}
+
+dart_status dart_decode_step(const dart_dims* d, int64_t pos, int64_t m_cap, void* cache,
+                             float* state, float* partial, const void* x, const float* dt,
+                             const float* A, const void* b, const void* c, const void* q,
+                             const void* e, const void* z, void* y, float* lse, void* ws,
+                             size_t ws_bytes, void* stream) {
+    (void)ws;
+    (void)ws_bytes;
+    dart_status st = check_dims(d, false);
+    if (st != DART_OK) return st;
+    if (pos < 0 || m_cap < 0 || pos / d->chunk > m_cap) return DART_ERR_INVALID_ARG;
+    if (m_cap > 0 && cache == nullptr) return DART_ERR_INVALID_ARG;
+    const void* req[] = {state, partial, x, dt, A, b, c, q, e, z, y};
+    for (const void* p : req)
+        if (p == nullptr || !aligned16(p)) return DART_ERR_INVALID_ARG;
+    if ((cache && !aligned16(cache)) || (lse && !aligned16(lse))) return DART_ERR_INVALID_ARG;
+
+    dart::DecodeArgs a;
+    a.B = d->batch; a.H = d->nheads; a.G = d->ngroups; a.P = d->headdim; a.N = d->dstate;
+    a.S = d->chunk; a.pos = pos; a.m_cap = m_cap; a.eps = d->eps;
+    a.cache = cache; a.state = state; a.partial = partial; a.x = x; a.dt = dt; a.A = A;
+    a.b = b; a.c = c; a.q = q; a.e = e; a.z = z; a.y = y; a.lse = lse;
+    cudaStream_t s = (cudaStream_t)stream;
+    cudaError_t err = dispatch<DecodeL>(d, a, s);
+    return err == cudaSuccess ? DART_OK : cuda_fail(err);
+}
+
+dart_status dart_get_device_status(void* stream) {
+    cudaError_t e = cudaStreamSynchronize((cudaStream_t)stream);
+    if (e != cudaSuccess) return cuda_fail(e);
+    return DART_OK;
+}
+
+}  // extern "C"

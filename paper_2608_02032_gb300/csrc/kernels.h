@@ -1,0 +1,77 @@
+// Internal launch interface between the C ABI (dart_api.cu) and the kernels.
+// Not installed; the public interface is include/dart.h.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+namespace dart {
+
+struct ScanArgs {
+    int64_t B, L, H, G, P, N, S;
+    float eps;
+    const void* X;
+    const float* dt;
+    const float* A;
+    const void* Bm;
+    const void* Cm;
+    void* Y;
+    void* M;
+    float* rM;
+    float* final_state;
+    // workspace
+    float* cum;   // B x H x M x S
+    float* dH32;  // B x M x H x N x P (fp32 memories, then states entering each chunk)
+};
+
+struct SmaArgs {
+    int64_t B, L, H, G, P, N, S;
+    float eps;
+    const void* M;
+    const float* rM;
+    const void* Q;
+    const void* Cm;
+    const void* E;
+    const void* z;
+    const void* Yssd;
+    void* Y;
+    void* R;
+    float* lse;
+};
+
+struct DecodeArgs {
+    int64_t B, H, G, P, N, S, pos, m_cap;
+    float eps;
+    void* cache;
+    float* state;
+    float* partial;
+    const void* x;
+    const float* dt;
+    const float* A;
+    const void* b;
+    const void* c;
+    const void* q;
+    const void* e;
+    const void* z;
+    void* y;
+    float* lse;
+};
+
+// Kernels launched by the library (read by dart_launch_count()).
+void note_launches(int n);
+
+template <typename Tin, typename Tmem, typename Tout>
+cudaError_t launch_chunk_scan_simt(const ScanArgs& a, cudaStream_t stream);
+
+template <typename Tmem>
+cudaError_t launch_memory_rms(const void* M, float* rM, int64_t rows, int64_t P, float eps,
+                              cudaStream_t stream);
+
+template <typename Tin, typename Tmem, typename Tout>
+cudaError_t launch_sma_forward_simt(const SmaArgs& a, cudaStream_t stream);
+
+template <typename Tin, typename Tmem, typename Tout>
+cudaError_t launch_decode_step(const DecodeArgs& a, cudaStream_t stream);
+
+}  // namespace dart

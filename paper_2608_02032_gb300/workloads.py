@@ -137,3 +137,21 @@ def decode_state_slab(w: Workload, b: int) -> torch.Tensor:
     """Running state of batch row ``b``: ``H x N x P`` fp32 ~ N(0, 0.02^2)."""
     g = torch.Generator().manual_seed(w.seed * 1_000_003 + 104_729 * (b + 1) + 1)
     return 0.02 * torch.randn(w.heads, w.dstate, w.headdim, generator=g)
+
+
+def decode_partial_slab(w: Workload, b: int) -> torch.Tensor:
+    """Partial-chunk memory of batch row ``b``: ``H x N x P`` fp32 ~ N(0, 0.01^2)
+    (only read when ``w.pos`` is not a chunk start)."""
+    g = torch.Generator().manual_seed(w.seed * 1_000_003 + 15_485_863 * (b + 1) + 2)
+    return 0.01 * torch.randn(w.heads, w.dstate, w.headdim, generator=g)
+
+
+def decode_state(w: Workload, m_cap: int | None = None) -> dict:
+    """Whole decode state on the host: cache (Bsz x m_cap x H x N x P), state and
+    partial (Bsz x H x N x P). For small workloads; large ones go slab by slab."""
+    m_cap = w.mem if m_cap is None else m_cap
+    return dict(
+        cache=torch.stack([decode_cache_slab(w, b, m_cap) for b in range(w.batch)]),
+        state=torch.stack([decode_state_slab(w, b) for b in range(w.batch)]),
+        partial=torch.stack([decode_partial_slab(w, b) for b in range(w.batch)]),
+    )

@@ -1,0 +1,189 @@
+"""Parity of the CUDA prefill path (dart_chunk_scan + dart_sma_forward) with the oracle.
+
+Element-by-element at sizes the oracle finishes in seconds; on sampled heads
+and tokens at the full L = 16K workload. Tolerance: max|gpu - oracle| /
+RMS(oracle) <= 1e-4 (fp32) or 2e-2 (bf16 inputs, fp32 accumulation), per
+output tensor; lse = -inf rows (chunk 0) must match exactly.
+"""
+import numpy as np
+import pytest
+import torch
+
+from helpers import TOL, dev, gpu_prefill, host, oracle_prefill, rel_err
+from paper_2608_02032_gb300 import api, binding
+from paper_2608_02032_gb300.workloads import WORKLOADS, Workload, prefill_inputs
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _need_gpu():
+    assert torch.cuda.is_available(), "GPU tests need a CUDA device"
+    binding.lib()  # fails loudly if libdart.so is missing
+
+
+def _compare(got, ref, tol, keys=("Y_ssd", "M", "rM", "final_state", "R", "lse", "Y")):
+    errs = {k: rel_err(got[k], ref[k]) for k in keys if k in got}
+    bad = {k: v for k, v in errs.items() if not v <= tol}
+    assert not bad, f"tolerance {tol} exceeded: {bad} (all: {errs})"
+    return errs
+
+
+def test_tiny_fp32_workload_matches_oracle(oracle_mod):
+    w = WORKLOADS["tiny_fp32"]
+    inp = prefill_inputs(w)
+    _compare(gpu_prefill(inp, w), oracle_prefill(inp, w), TOL["f32"])
+
+
+def test_prefill_b4_l2k_bf16_matches_oracle(oracle_mod):
+    w = WORKLOADS["prefill_b4_l2k"]
+    inp = prefill_inputs(w)
+    _compare(gpu_prefill(inp, w), oracle_prefill(inp, w), TOL["bf16"])
+
+
+SWEEP = [
+    # (L, S, P, N, H, G, dtype)
+    (64, 16, 32, 16, 2, 1, "f32"),
+    (96, 32, 16, 64, 2, 1, "f32"),
+    (192, 64, 64, 128, 2, 1, "f32"),
+    (384, 128, 32, 64, 3, 1, "f32"),
+    (512, 256, 64, 128, 2, 1, "f32"),
+    (256, 256, 64, 128, 2, 1, "bf16"),   # M = 1: no token has history
+    (512, 256, 64, 128, 2, 1, "bf16"),   # M = 2
+    (768, 256, 64, 128, 4, 2, "bf16"),   # M = 3, two groups
+    (320, 64, 32, 32, 2, 1, "bf16"),     # ragged last token tile inside chunks
+    (1024, 128, 64, 128, 2, 1, "bf16"),
+]
+
+
+@pytest.mark.parametrize("L,S,P,N,H,G,dtype", SWEEP)
+def test_size_sweep_matches_oracle(oracle_mod, L, S, P, N, H, G, dtype):
+    w = Workload("sweep", 2, H, L, P, N, S, groups=G, dtype=dtype, seed=77 + L + S + P + N)
+    inp = prefill_inputs(w)
+    _compare(gpu_prefill(inp, w), oracle_prefill(inp, w), TOL[dtype])
+
+
+@pytest.mark.parametrize("mem,out", [("bf16", "f32"), ("bf16", "bf16")])
+def test_bf16_storage_of_memories_and_outputs(oracle_mod, mem, out):
+    """bf16 memories (and outputs). Each stored memory is the oracle's memory
+    rounded to bf16 (within an ulp, 2^-8 relative: the GPU rounds its fp32 sum).
+    SMA then reads the stored memories, so R, lse and Y are checked against the
+    oracle's SMA over its own memories rounded to bf16 (round to nearest even,
+    on the CPU), at the bf16-input tolerance; bf16 outputs add their own
+    rounding (2^-8 relative)."""
+    w = Workload("bf16_store", 2, 2, 512, 64, 128, 128, seed=10)
+    inp = prefill_inputs(w)
+    X, Bm, Cm, Q, E, z = (dev(inp[k], "bf16") for k in ("X", "Bm", "Cm", "Q", "E", "z"))
+    dtv, A = dev(inp["dt"], torch.float32), dev(inp["A"], torch.float32)
+    to = {"bf16": torch.bfloat16, "f32": torch.float32}[out]
+    s, o = api.prefill_forward(X, dtv, A, Bm, Cm, Q, E, z, w.chunk, w.eps, want_R=True,
+                               mem_dtype=torch.bfloat16, out_dtype=to)
+    torch.cuda.synchronize()
+    ref = oracle_prefill(inp, w)
+    g, r = host(s.M), ref["M"]
+    assert np.all(np.abs(g - r) <= 2.0 ** -8 * np.abs(r) + 1e-6 * np.abs(r).max())
+    dH16 = torch.from_numpy(ref["M"]).to(torch.bfloat16).double().numpy()
+    R16, lse16 = oracle_mod.sma(dH16, inp["Q"], inp["Cm"], inp["E"], w.chunk, w.eps)
+    Y16 = oracle_mod.merge(ref["Y_ssd"], inp["z"], R16)
+    assert rel_err(host(o.lse), lse16) <= TOL["bf16"]
+    for k, got, want in (("Y_ssd", s.Y_ssd, ref["Y_ssd"]), ("R", o.R, R16), ("Y", o.Y, Y16)):
+        g = host(got)
+        if out == "f32":
+            assert rel_err(g, want) <= TOL["bf16"], k
+        else:
+            rms = np.sqrt(np.mean(want ** 2))
+            assert np.all(np.abs(g - want) <= 2.0 ** -8 * np.abs(want) + TOL["bf16"] * rms), k
+
+
+def test_single_chunk_has_no_readout(oracle_mod):
+    """S = L: every token is in chunk 0, so R = 0, lse = -inf and Y = Y_ssd exactly."""
+    w = Workload("one_chunk", 1, 2, 256, 64, 128, 256, seed=5)
+    got = gpu_prefill(prefill_inputs(w), w)
+    assert np.all(got["R"] == 0) and np.all(np.isneginf(got["lse"]))
+    assert np.array_equal(got["Y"], got["Y_ssd"])
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_zero_gate_reproduces_mamba2_bitwise(oracle_mod, dtype):
+    """z = 0 (W_G = 0, Sec. 3): Y is bit-identical to the SSD output."""
+    w = Workload("zero_gate", 1, 2, 512, 64, 128, 128, dtype=dtype, seed=6)
+    inp = prefill_inputs(w)
+    inp["z"] = torch.zeros_like(inp["z"])
+    got = gpu_prefill(inp, w)
+    assert np.array_equal(got["Y"], got["Y_ssd"])
+    assert np.any(got["R"] != 0)
+
+
+def test_rms_computed_inside_when_not_given(oracle_mod):
+    w = Workload("rm_null", 1, 2, 512, 64, 128, 128, seed=8)
+    inp = prefill_inputs(w)
+    X, Bm, Cm, Q, E, z = (dev(inp[k], "bf16") for k in ("X", "Bm", "Cm", "Q", "E", "z"))
+    dtv, A = dev(inp["dt"], torch.float32), dev(inp["A"], torch.float32)
+    s = api.chunk_scan(X, dtv, A, Bm, Cm, w.chunk, w.eps)
+    o1 = api.sma_forward(s.M, s.rM, Q, Cm, E, z, s.Y_ssd, w.chunk, w.eps)
+    o2 = api.sma_forward(s.M, None, Q, Cm, E, z, s.Y_ssd, w.chunk, w.eps)
+    torch.cuda.synchronize()
+    # the two r computations sum the squares in different orders
+    assert rel_err(host(o1.Y), host(o2.Y)) <= 1e-5
+    assert rel_err(host(o1.lse), host(o2.lse)) <= 1e-6  # -inf rows must match exactly
+
+
+def test_outputs_stay_inside_their_buffers(oracle_mod):
+    """Canary bands around every output of both calls stay untouched."""
+    w = Workload("canary", 1, 2, 512, 64, 128, 128, seed=9)
+    inp = prefill_inputs(w)
+    Bsz, L, H, P, N, S = 1, 512, 2, 64, 128, 128
+    M = L // S
+    X, Bm, Cm, Q, E, z = (dev(inp[k], "bf16") for k in ("X", "Bm", "Cm", "Q", "E", "z"))
+    dtv, A = dev(inp["dt"], torch.float32), dev(inp["A"], torch.float32)
+    pad = 4096
+
+    def guarded(n, dtype):
+        buf = torch.full((n + 2 * pad,), 7.0, dtype=dtype, device="cuda")
+        return buf, buf[pad:pad + n]
+
+    bufs = {}
+    f32 = torch.float32
+    for name, n, dtp in [("Y", Bsz * L * H * P, f32), ("M", Bsz * M * H * N * P, f32),
+                         ("rM", Bsz * M * H * N, f32), ("fs", Bsz * H * N * P, f32),
+                         ("Yo", Bsz * L * H * P, f32), ("R", Bsz * L * H * P, f32),
+                         ("lse", Bsz * L * H, f32)]:
+        bufs[name] = guarded(n, dtp)
+    dims = binding.make_dims(Bsz, L, H, 1, P, N, S, binding.DART_BF16, eps=w.eps)
+    ws = torch.empty(binding.dart_workspace_size(dims, binding.DART_OP_CHUNK_SCAN), dtype=torch.uint8,
+                     device="cuda")
+    binding.dart_chunk_scan(dims, X, dtv, A, Bm, Cm, bufs["Y"][1], bufs["M"][1], bufs["rM"][1],
+                            bufs["fs"][1], ws)
+    binding.dart_sma_forward(dims, bufs["M"][1], bufs["rM"][1], Q, Cm, E, z, bufs["Y"][1],
+                             bufs["Yo"][1], bufs["R"][1], bufs["lse"][1])
+    torch.cuda.synchronize()
+    for name, (buf, _) in bufs.items():
+        assert torch.all(buf[:pad] == 7.0) and torch.all(buf[-pad:] == 7.0), name
+
+
+def test_l16k_workload_sampled_heads_and_tokens(oracle_mod):
+    """The full L = 16K, H = 32 workload in the benchmark's launch configuration,
+    checked on three heads: Y_ssd and the memories of every token/chunk of those
+    heads, R, lse and Y on 768 sampled tokens."""
+    import oracle
+
+    w = WORKLOADS["prefill_l16k"]
+    inp = prefill_inputs(w)
+    got = gpu_prefill(inp, w)
+    heads = [0, 17, 31]
+    rng = np.random.default_rng(0)
+    toks = np.concatenate([rng.choice(np.arange(w.chunk, w.seqlen), 250, replace=False),
+                           [0, w.chunk - 1, w.chunk, w.seqlen - 1, 3 * w.chunk + 5, w.seqlen - w.chunk]])
+    for h in heads:
+        sl = {k: inp[k][:, :, h:h + 1] for k in ("X", "dt", "z")}
+        Yssd, Hl = oracle.ssd_recurrence(sl["X"], sl["dt"], inp["A"][h:h + 1], inp["Bm"], inp["Cm"])
+        dH = oracle.chunk_memories(sl["X"], sl["dt"], inp["A"][h:h + 1], inp["Bm"], w.chunk)
+        assert rel_err(got["Y_ssd"][:, :, h:h + 1], Yssd) <= TOL["bf16"]
+        assert rel_err(got["M"][:, :, h:h + 1], dH) <= TOL["bf16"]
+        assert rel_err(got["final_state"][:, h:h + 1], Hl) <= TOL["bf16"]
+        tl = np.stack([np.zeros_like(toks), toks, np.zeros_like(toks)], 1)
+        R, lse = oracle.sma(dH, inp["Q"], inp["Cm"], inp["E"], w.chunk, w.eps, tokens=tl)
+        Y = oracle.merge(Yssd[0, toks, 0], sl["z"][0, toks, 0], R)
+        assert rel_err(got["R"][0, toks, h], R) <= TOL["bf16"]
+        assert rel_err(got["lse"][0, toks, h], lse) <= TOL["bf16"]
+        assert rel_err(got["Y"][0, toks, h], Y) <= TOL["bf16"]

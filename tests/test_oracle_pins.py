@@ -250,6 +250,22 @@ def test_token_list_matches_full_evaluation(oracle_mod):
         assert ls[i] == lse[b, t, h] or (np.isneginf(ls[i]) and np.isneginf(lse[b, t, h]))
 
 
+def test_memory_inverse_rms_closed_forms(oracle_mod):
+    """App. B.1: r = (mean_p dH^2 + eps)^-1/2 along the value axis P: a row of
+    constant a gives (a^2 + eps)^-1/2; the row (3, 4) gives (12.5 + eps)^-1/2."""
+    eps = 1e-6
+    dH = np.zeros((1, 2, 1, 3, 2))
+    dH[0, 0, 0, 0] = [2.0, 2.0]
+    dH[0, 0, 0, 1] = [3.0, 4.0]
+    dH[0, 1, 0, 2] = [-5.0, -5.0]
+    r = oracle_mod.memory_inverse_rms(dH, eps)
+    assert r.shape == (1, 2, 1, 3)
+    assert abs(r[0, 0, 0, 0] - 1 / math.sqrt(4.0 + eps)) < 1e-15
+    assert abs(r[0, 0, 0, 1] - 1 / math.sqrt(12.5 + eps)) < 1e-15
+    assert abs(r[0, 1, 0, 2] - 1 / math.sqrt(25.0 + eps)) < 1e-15
+    assert abs(r[0, 0, 0, 2] - 1 / math.sqrt(eps)) < 1e-9
+
+
 # ---------------------------------------------------------------------- merge
 
 def test_zero_gate_reproduces_mamba2_exactly(oracle_mod):
