@@ -56,7 +56,8 @@ typedef enum {
     DART_ERR_UNSUPPORTED = 2,  /* valid but not built: L % S != 0, P/N/S outside the set below */
     DART_ERR_WORKSPACE = 3,    /* workspace NULL/misaligned or smaller than dart_workspace_size */
     DART_ERR_CUDA = 4,         /* a CUDA call failed; see dart_last_cuda_error() */
-    DART_ERR_TIMEOUT = 5       /* a device-side wait gave up (see dart_get_device_status) */
+    DART_ERR_TIMEOUT = 5,      /* a device-side wait gave up (see dart_get_device_status) */
+    DART_ERR_TOO_LARGE = 6     /* beyond the fixed scratch of dart_sma_forward_noalloc */
 } dart_status;
 
 typedef enum { DART_F32 = 0, DART_BF16 = 1 } dart_dtype;
@@ -161,6 +162,36 @@ dart_status dart_decode_step(const dart_dims* dims, int64_t pos, int64_t m_cap, 
                              const float* A, const void* b, const void* c, const void* q,
                              const void* e, const void* z, void* y, float* lse,
                              void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * dart_sma_forward_noalloc: dart_sma_forward with rM = NULL, for callers that
+ * cannot allocate device memory and cannot pass a workspace. The paper has no
+ * counterpart; this entry point exists for integration. Typical callers: a
+ * host framework that hands a plugin only its input and output buffers and
+ * owns all other device memory; a latency-critical service that forbids
+ * allocation after start-up (cudaMalloc and cudaFree can synchronise the
+ * device); a process under a fixed device-memory budget.
+ * It computes exactly what dart_sma_forward computes when rM is NULL. Its only
+ * scratch, the inverse RMS of every memory row, lives in a fixed device array
+ * of 2^20 fp32 values (4 MiB) inside the library, which every GPU that loads
+ * the library holds until the process exits. It calls no cudaMalloc, no
+ * cudaFree and no allocating library routine.
+ * Arguments: as dart_sma_forward, without rM and the workspace. The caller
+ * still passes (and owns) every input and output.
+ * Limit: Bsz * (L / S) * H * N <= 2^20 memory rows (e.g. B1 H32 L16384 N128
+ * S256 uses 2^18); larger problems return DART_ERR_TOO_LARGE before anything
+ * is launched.
+ * Set-up: the first call on a device looks up the array's device address on
+ * that device (with that device current) and caches it; make that first call
+ * before any stream capture. All calls share the array and it keeps the last
+ * call's contents (every entry read is first written by the same call, so
+ * nothing needs clearing). Calls that overlap on the GPU, on any streams,
+ * race on the array: serialise them.
+ */
+dart_status dart_sma_forward_noalloc(const dart_dims* dims, const void* M, const void* Q,
+                                     const void* Cm, const void* E, const void* z,
+                                     const void* Y_ssd, void* Y, void* R, float* lse,
+                                     void* stream);
 
 /* Number of kernels this library has launched in this process since it was
  * loaded (all entry points, all threads). A diagnostic for benchmarks. */

@@ -21,14 +21,15 @@ DART_OK = 0
 DART_F32, DART_BF16 = 0, 1
 DART_OP_CHUNK_SCAN, DART_OP_SMA_FORWARD, DART_OP_DECODE_STEP = 0, 1, 2
 STATUS_NAMES = {0: "DART_OK", 1: "DART_ERR_INVALID_ARG", 2: "DART_ERR_UNSUPPORTED",
-                3: "DART_ERR_WORKSPACE", 4: "DART_ERR_CUDA", 5: "DART_ERR_TIMEOUT"}
+                3: "DART_ERR_WORKSPACE", 4: "DART_ERR_CUDA", 5: "DART_ERR_TIMEOUT",
+                6: "DART_ERR_TOO_LARGE"}
 
 TORCH_DTYPE = {DART_F32: torch.float32, DART_BF16: torch.bfloat16}
 DART_DTYPE = {torch.float32: DART_F32, torch.bfloat16: DART_BF16}
 
 EXPORTED = ("dart_status_string", "dart_last_cuda_error", "dart_workspace_size",
-            "dart_chunk_scan", "dart_sma_forward", "dart_decode_step", "dart_launch_count",
-            "dart_get_device_status")
+            "dart_chunk_scan", "dart_sma_forward", "dart_decode_step", "dart_sma_forward_noalloc",
+            "dart_launch_count", "dart_get_device_status")
 
 
 class DartError(RuntimeError):
@@ -84,6 +85,8 @@ def lib() -> ctypes.CDLL:
         L.dart_decode_step.restype = ctypes.c_int
         L.dart_decode_step.argtypes = ([dp, ctypes.c_int64, ctypes.c_int64] + [_vp] * 14
                                        + [ctypes.c_size_t, _vp])
+        L.dart_sma_forward_noalloc.restype = ctypes.c_int
+        L.dart_sma_forward_noalloc.argtypes = [dp] + [_vp] * 10
         L.dart_launch_count.restype = ctypes.c_uint64
         L.dart_launch_count.argtypes = []
         L.dart_get_device_status.restype = ctypes.c_int
@@ -146,6 +149,15 @@ def dart_sma_forward(dims, M, rM, Q, Cm, E, z, Y_ssd, Y, R=None, lse=None, works
         ctypes.byref(dims), _ptr(M, "M"), _ptr(rM, "rM"), _ptr(Q, "Q"), _ptr(Cm, "Cm"),
         _ptr(E, "E"), _ptr(z, "z"), _ptr(Y_ssd, "Y_ssd"), _ptr(Y, "Y"), _ptr(R, "R"),
         _ptr(lse, "lse"), w, nb, _stream(stream)))
+
+
+def dart_sma_forward_noalloc(dims, M, Q, Cm, E, z, Y_ssd, Y, R=None, lse=None, stream=None) -> None:
+    """dart_sma_forward with rM = NULL for callers that cannot allocate: its
+    scratch is a fixed 4 MiB array inside the library (see include/dart.h)."""
+    _check("dart_sma_forward_noalloc", lib().dart_sma_forward_noalloc(
+        ctypes.byref(dims), _ptr(M, "M"), _ptr(Q, "Q"), _ptr(Cm, "Cm"), _ptr(E, "E"),
+        _ptr(z, "z"), _ptr(Y_ssd, "Y_ssd"), _ptr(Y, "Y"), _ptr(R, "R"), _ptr(lse, "lse"),
+        _stream(stream)))
 
 
 def dart_decode_step(dims, pos, m_cap, cache, state, partial, x, dt, A, b, c, q, e, z, y,

@@ -114,6 +114,8 @@ std::atomic<uint64_t> g_launches{0};
 
 namespace dart {
 void note_launches(int n) { g_launches.fetch_add((uint64_t)n, std::memory_order_relaxed); }
+dart_status validate_dims(const dart_dims* d, bool need_seqlen) { return check_dims(d, need_seqlen); }
+dart_status record_cuda_error(cudaError_t e) { return cuda_fail(e); }
 }  // namespace dart
 
 extern "C" {
@@ -129,6 +131,8 @@ const char* dart_status_string(dart_status s) {
         case DART_ERR_WORKSPACE: return "DART_ERR_WORKSPACE: workspace missing, misaligned or too small";
         case DART_ERR_CUDA: return "DART_ERR_CUDA: a CUDA call failed (see dart_last_cuda_error)";
         case DART_ERR_TIMEOUT: return "DART_ERR_TIMEOUT: a device-side wait gave up";
+        case DART_ERR_TOO_LARGE:
+            return "DART_ERR_TOO_LARGE: problem exceeds the fixed scratch of dart_sma_forward_noalloc";
     }
     return "unknown dart_status";
 }

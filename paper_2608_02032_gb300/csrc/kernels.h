@@ -6,7 +6,14 @@
 #include <stddef.h>
 #include <stdint.h>
 
+#include "dart.h"
+
 namespace dart {
+
+// Validation of dims shared by the entry points (dart_api.cu).
+dart_status validate_dims(const dart_dims* d, bool need_seqlen);
+// Records e for dart_last_cuda_error() and returns DART_ERR_CUDA.
+dart_status record_cuda_error(cudaError_t e);
 
 struct ScanArgs {
     int64_t B, L, H, G, P, N, S;

@@ -40,7 +40,7 @@ def test_binding_covers_the_header():
 
 
 def test_status_strings(L):
-    for s in range(6):
+    for s in range(7):
         assert L.dart_status_string(s)
     assert b"unknown" in L.dart_status_string(99)
 
@@ -108,3 +108,14 @@ def test_decode_validation(L):
     bad[3] = v(FAKE + 4)
     assert L.dart_decode_step(ctypes.byref(d), 5, 3, v(FAKE), *bad, None, 0, None) == 1
     assert B.STATUS_NAMES[1] == "DART_ERR_INVALID_ARG"
+
+
+def test_noalloc_rejects_problems_beyond_its_scratch(L):
+    """2^20 memory rows is the fixed limit; one more row is refused before any launch."""
+    v = ctypes.c_void_p
+    ok = _dims(batch=1, seqlen=2 ** 20 // (2 * 128) * 128, nheads=2, chunk=128)  # exactly 2^20 rows
+    big = _dims(batch=2, seqlen=2 ** 20 // (2 * 128) * 128, nheads=2, chunk=128)
+    assert L.dart_sma_forward_noalloc(ctypes.byref(big), *[v(FAKE)] * 9, None) == 6
+    assert L.dart_sma_forward_noalloc(ctypes.byref(ok), *[v(FAKE)] * 6, v(0), v(FAKE), v(FAKE),
+                                      None) == 1  # a NULL output is still caught first
+    assert L.dart_sma_forward_noalloc(ctypes.byref(_dims(headdim=48)), *[v(FAKE)] * 9, None) == 2
