@@ -266,6 +266,8 @@ def run_dart(args) -> None:
     Y = torch.empty_like(Yssd)
     lse = torch.empty(Bsz, L, H, dtype=torch.float32, device=dev)
     ws = torch.empty(Bd.dart_workspace_size(dims, Bd.DART_OP_CHUNK_SCAN), dtype=torch.uint8, device=dev)
+    ws_sma = torch.empty(max(Bd.dart_workspace_size(dims, Bd.DART_OP_SMA_FORWARD), 256),
+                         dtype=torch.uint8, device=dev)
     flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream(dev)
 
@@ -275,7 +277,7 @@ def run_dart(args) -> None:
         ev_mid = torch.cuda.Event(enable_timing=True)
         ev_mid.record(stream)
         Bd.dart_sma_forward(dims, Mem, rM, d_in["Q"], d_in["Cm"], d_in["E"], d_in["z"], Yssd, Y, None,
-                            lse, None, stream)
+                            lse, ws_sma, stream)
         return ev_mid
 
     for _ in range(args.warmup):

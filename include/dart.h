@@ -133,6 +133,11 @@ dart_status dart_chunk_scan(const dart_dims* dims, const void* X, const float* d
  *          z (Bsz, L, H) in_dtype gate logits;  Y_ssd (Bsz, L, H, P) out_dtype.
  * Outputs: Y (Bsz, L, H, P) out_dtype;  R (Bsz, L, H, P) out_dtype or NULL;
  *          lse (Bsz, L, H) fp32 or NULL.
+ * Workspace: dart_workspace_size(dims, DART_OP_SMA_FORWARD) bytes. Always
+ *          needed on the tensor-core path (bf16 inputs, P = 64, N = 128,
+ *          S % 128 == 0, H / G a multiple of 4), where it holds each memory's
+ *          MMA operands (48 KiB per memory and head); elsewhere only when rM is
+ *          NULL (for r).
  */
 dart_status dart_sma_forward(const dart_dims* dims, const void* M, const float* rM,
                              const void* Q, const void* Cm, const void* E, const void* z,
@@ -196,6 +201,17 @@ dart_status dart_sma_forward_noalloc(const dart_dims* dims, const void* M, const
 /* Number of kernels this library has launched in this process since it was
  * loaded (all entry points, all threads). A diagnostic for benchmarks. */
 uint64_t dart_launch_count(void);
+
+/*
+ * Bound on every device-side wait of the tensor-core kernels, in nanoseconds
+ * of wall-clock time per wait (default 2 s; 0 restores the default). A wait
+ * that runs out makes the kernel stop its pipeline, finish its own copies and
+ * MMAs in flight, free its tensor memory and record DART_ERR_TIMEOUT for
+ * dart_get_device_status(); the outputs of that call are then undefined.
+ * Tests set a tiny bound to exercise that path without faulting the GPU.
+ * Process-wide; takes effect for launches after the call.
+ */
+void dart_set_wait_limit_ns(uint64_t limit_ns);
 
 /*
  * Synchronises `stream`, then reports and clears the device status word that

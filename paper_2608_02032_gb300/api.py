@@ -70,9 +70,7 @@ def sma_forward(Mem, rM, Q, Cm, E, z, Y_ssd, chunk: int, eps: float = 1e-6, want
     Y = torch.empty_like(Y_ssd)
     R = torch.empty_like(Y_ssd) if want_R else None
     lse = torch.empty(Bsz, L, H, dtype=torch.float32, device=dev)
-    ws = workspace
-    if rM is None and ws is None:
-        ws = _workspace(dims, B.DART_OP_SMA_FORWARD, dev)
+    ws = workspace if workspace is not None else _workspace(dims, B.DART_OP_SMA_FORWARD, dev)
     B.dart_sma_forward(dims, Mem, rM, Q, Cm, E, z, Y_ssd, Y, R, lse, ws)
     return SmaOut(Y, R, lse)
 

@@ -29,7 +29,7 @@ DART_DTYPE = {torch.float32: DART_F32, torch.bfloat16: DART_BF16}
 
 EXPORTED = ("dart_status_string", "dart_last_cuda_error", "dart_workspace_size",
             "dart_chunk_scan", "dart_sma_forward", "dart_decode_step", "dart_sma_forward_noalloc",
-            "dart_launch_count", "dart_get_device_status")
+            "dart_launch_count", "dart_set_wait_limit_ns", "dart_get_device_status")
 
 
 class DartError(RuntimeError):
@@ -89,6 +89,8 @@ def lib() -> ctypes.CDLL:
         L.dart_sma_forward_noalloc.argtypes = [dp] + [_vp] * 10
         L.dart_launch_count.restype = ctypes.c_uint64
         L.dart_launch_count.argtypes = []
+        L.dart_set_wait_limit_ns.restype = None
+        L.dart_set_wait_limit_ns.argtypes = [ctypes.c_uint64]
         L.dart_get_device_status.restype = ctypes.c_int
         L.dart_get_device_status.argtypes = [_vp]
         _lib = L
@@ -177,3 +179,8 @@ def dart_get_device_status(stream=None) -> None:
 def dart_launch_count() -> int:
     """Kernels the library has launched in this process."""
     return int(lib().dart_launch_count())
+
+
+def dart_set_wait_limit_ns(limit_ns: int) -> None:
+    """Bound on each device-side wait of the tensor-core kernels (0 = default 2 s)."""
+    lib().dart_set_wait_limit_ns(int(limit_ns))

@@ -103,10 +103,26 @@ ScanWs scan_ws(const dart_dims* d) {
     return w;
 }
 
+dart::SmaArgs sma_args(const dart_dims* d) {
+    dart::SmaArgs a{};
+    a.B = d->batch; a.L = d->seqlen; a.H = d->nheads; a.G = d->ngroups;
+    a.P = d->headdim; a.N = d->dstate; a.S = d->chunk; a.eps = d->eps;
+    return a;
+}
+
+// The tensor-core SMA serves bf16 token inputs at its tile shape; everything
+// else runs on the FFMA kernel.
+bool sma_uses_tc(const dart_dims* d) {
+    return d->in_dtype == DART_BF16 && dart::sma_tc_supported(sma_args(d));
+}
+
 size_t sma_ws(const dart_dims* d) {
     const i64 M = d->seqlen / d->chunk;
+    if (sma_uses_tc(d)) return align256(dart::sma_tc_workspace(d->batch, M, d->nheads));
     return align256((size_t)(d->batch * M * d->nheads * d->dstate) * sizeof(float));
 }
+
+std::atomic<unsigned long long> g_wait_limit_ns{2000000000ull};
 
 std::atomic<uint64_t> g_launches{0};
 
@@ -190,11 +206,27 @@ dart_status dart_sma_forward(const dart_dims* d, const void* M, const float* rM,
         if (p == nullptr || !aligned16(p)) return DART_ERR_INVALID_ARG;
     if ((rM && !aligned16(rM)) || (R && !aligned16(R)) || (lse && !aligned16(lse)))
         return DART_ERR_INVALID_ARG;
-    const size_t need = rM == nullptr ? sma_ws(d) : 0;
+    const bool tc = sma_uses_tc(d);
+    const size_t need = (tc || rM == nullptr) ? sma_ws(d) : 0;
     if (need > 0 && (ws == nullptr || ((uintptr_t)ws & 255u) != 0 || ws_bytes < need))
         return DART_ERR_WORKSPACE;
 
     cudaStream_t s = (cudaStream_t)stream;
+    if (tc) {
+        dart::SmaArgs a = sma_args(d);
+        a.M = M; a.rM = rM; a.Q = Q; a.Cm = Cm; a.E = E; a.z = z; a.Yssd = Y_ssd; a.Y = Y;
+        a.R = R; a.lse = lse;
+        const unsigned long long lim = g_wait_limit_ns.load();
+        typedef __nv_bfloat16 bf;
+        cudaError_t e;
+        if (d->mem_dtype == DART_F32)
+            e = dart::launch_sma_forward_tc<float, float>(a, ws, lim, s);
+        else if (d->out_dtype == DART_F32)
+            e = dart::launch_sma_forward_tc<bf, float>(a, ws, lim, s);
+        else
+            e = dart::launch_sma_forward_tc<bf, bf>(a, ws, lim, s);
+        return e == cudaSuccess ? DART_OK : cuda_fail(e);
+    }
     const float* r = rM;
     if (r == nullptr) {
         const i64 rows = d->batch * (d->seqlen / d->chunk) * d->nheads * d->dstate;
@@ -244,7 +276,13 @@ dart_status dart_decode_step(const dart_dims* d, int64_t pos, int64_t m_cap, voi
 dart_status dart_get_device_status(void* stream) {
     cudaError_t e = cudaStreamSynchronize((cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(e);
-    return DART_OK;
+    const int code = dart::take_tc_status();
+    if (code < 0) return cuda_fail(cudaGetLastError());
+    return code != 0 ? DART_ERR_TIMEOUT : DART_OK;
+}
+
+void dart_set_wait_limit_ns(uint64_t limit_ns) {
+    g_wait_limit_ns.store(limit_ns == 0 ? 2000000000ull : (unsigned long long)limit_ns);
 }
 
 }  // extern "C"

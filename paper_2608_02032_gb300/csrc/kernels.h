@@ -81,4 +81,13 @@ cudaError_t launch_sma_forward_simt(const SmaArgs& a, cudaStream_t stream);
 template <typename Tin, typename Tmem, typename Tout>
 cudaError_t launch_decode_step(const DecodeArgs& a, cudaStream_t stream);
 
+// Tensor-core SMA (sma_tc.cu): bf16 token inputs, P = 64, N = 128, S % 128 == 0.
+bool sma_tc_supported(const SmaArgs& a);
+size_t sma_tc_workspace(int64_t B, int64_t Mc, int64_t H);
+template <typename Tmem, typename Tout>
+cudaError_t launch_sma_forward_tc(const SmaArgs& a, void* ws, unsigned long long wait_limit_ns,
+                                  cudaStream_t stream);
+// Reads and clears the tensor-core kernels' timeout code (0 = none, -1 = read failed).
+int take_tc_status();
+
 }  // namespace dart

@@ -76,6 +76,21 @@ extern "C" dart_status dart_sma_forward_noalloc(const dart_dims* d, const void* 
             ? dart::launch_memory_rms<float>(M, r, rows, d->headdim, d->eps, s)
             : dart::launch_memory_rms<__nv_bfloat16>(M, r, rows, d->headdim, d->eps, s);
     if (e != cudaSuccess) return dart::record_cuda_error(e);
-    // The rest is dart_sma_forward with the r computed above.
-    return dart_sma_forward(d, M, r, Q, Cm, E, z, Y_ssd, Y, R, lse, nullptr, 0, stream);
+    // The rest is the FFMA SMA kernel of dart_sma_forward with the r computed
+    // above (it needs no scratch beyond r).
+    dart::SmaArgs a{};
+    a.B = d->batch; a.L = d->seqlen; a.H = d->nheads; a.G = d->ngroups;
+    a.P = d->headdim; a.N = d->dstate; a.S = d->chunk; a.eps = d->eps;
+    a.M = M; a.rM = r; a.Q = Q; a.Cm = Cm; a.E = E; a.z = z; a.Yssd = Y_ssd; a.Y = Y; a.R = R;
+    a.lse = lse;
+    typedef __nv_bfloat16 bf;
+    if (d->in_dtype == DART_F32)
+        e = dart::launch_sma_forward_simt<float, float, float>(a, s);
+    else if (d->mem_dtype == DART_F32)
+        e = dart::launch_sma_forward_simt<bf, float, float>(a, s);
+    else if (d->out_dtype == DART_F32)
+        e = dart::launch_sma_forward_simt<bf, bf, float>(a, s);
+    else
+        e = dart::launch_sma_forward_simt<bf, bf, bf>(a, s);
+    return e == cudaSuccess ? DART_OK : dart::record_cuda_error(e);
 }

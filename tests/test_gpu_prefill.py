@@ -53,6 +53,12 @@ SWEEP = [
     (768, 256, 64, 128, 4, 2, "bf16"),   # M = 3, two groups
     (320, 64, 32, 32, 2, 1, "bf16"),     # ragged last token tile inside chunks
     (1024, 128, 64, 128, 2, 1, "bf16"),
+    # tensor-core SMA shapes (bf16, P 64, N 128, S % 128 == 0, 4 heads per CTA)
+    (512, 128, 64, 128, 4, 1, "bf16"),     # first tile of each chunk ... M = 4
+    (256, 128, 64, 128, 4, 1, "bf16"),     # M = 2
+    (128, 128, 64, 128, 4, 1, "bf16"),     # M = 1: only chunk-0 tiles
+    (1024, 256, 64, 128, 8, 1, "bf16"),    # two head groups
+    (768, 256, 64, 128, 8, 2, "bf16"),     # G = 2, four heads per group
 ]
 
 
