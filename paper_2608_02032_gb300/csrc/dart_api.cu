@@ -191,7 +191,19 @@ dart_status dart_chunk_scan(const dart_dims* d, const void* X, const float* dt, 
     a.cum = (float*)((char*)ws + w.cum_off);
     a.dH32 = (float*)((char*)ws + w.dh_off);
     cudaStream_t s = (cudaStream_t)stream;
-    cudaError_t e = dispatch<ScanL>(d, a, s);
+    cudaError_t e;
+    if (d->in_dtype == DART_BF16 && dart::scan_tc_supported(a)) {
+        typedef __nv_bfloat16 bf;
+        const unsigned long long lim = g_wait_limit_ns.load();
+        if (d->mem_dtype == DART_F32)
+            e = dart::launch_chunk_scan_tc<float, float>(a, lim, s);
+        else if (d->out_dtype == DART_F32)
+            e = dart::launch_chunk_scan_tc<bf, float>(a, lim, s);
+        else
+            e = dart::launch_chunk_scan_tc<bf, bf>(a, lim, s);
+    } else {
+        e = dispatch<ScanL>(d, a, s);
+    }
     return e == cudaSuccess ? DART_OK : cuda_fail(e);
 }
 
@@ -277,8 +289,9 @@ dart_status dart_get_device_status(void* stream) {
     cudaError_t e = cudaStreamSynchronize((cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(e);
     const int code = dart::take_tc_status();
-    if (code < 0) return cuda_fail(cudaGetLastError());
-    return code != 0 ? DART_ERR_TIMEOUT : DART_OK;
+    const int code2 = dart::take_scan_tc_status();
+    if (code < 0 || code2 < 0) return cuda_fail(cudaGetLastError());
+    return (code != 0 || code2 != 0) ? DART_ERR_TIMEOUT : DART_OK;
 }
 
 void dart_set_wait_limit_ns(uint64_t limit_ns) {

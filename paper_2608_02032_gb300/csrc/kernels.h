@@ -70,6 +70,16 @@ void note_launches(int n);
 
 template <typename Tin, typename Tmem, typename Tout>
 cudaError_t launch_chunk_scan_simt(const ScanArgs& a, cudaStream_t stream);
+// Steps 1 and 3 of the scan (scan.cu), shared by both scan paths.
+cudaError_t launch_chunk_cumsum(const ScanArgs& a, cudaStream_t stream);
+cudaError_t launch_state_passing(const ScanArgs& a, cudaStream_t stream);
+
+// Tensor-core scan (scan_tc.cu): bf16 inputs, P = 64, N = 128, S in {128, 256}.
+bool scan_tc_supported(const ScanArgs& a);
+template <typename Tmem, typename Tout>
+cudaError_t launch_chunk_scan_tc(const ScanArgs& a, unsigned long long wait_limit_ns,
+                                 cudaStream_t stream);
+int take_scan_tc_status();
 
 template <typename Tmem>
 cudaError_t launch_memory_rms(const void* M, float* rM, int64_t rows, int64_t P, float eps,

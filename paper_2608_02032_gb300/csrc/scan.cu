@@ -290,23 +290,40 @@ chunk_output_kernel(const Tin* __restrict__ X, const float* __restrict__ dt,
 }
 
 // ------------------------------------------------------------------ launch
+cudaError_t launch_chunk_cumsum(const ScanArgs& a, cudaStream_t stream) {
+    const int B = (int)a.B, L = (int)a.L, H = (int)a.H, S = (int)a.S, M = L / S;
+    chunk_cumsum_kernel<<<dim3(M, H, B), S, 64 * sizeof(float), stream>>>(a.dt, a.A, a.cum, L, H,
+                                                                             S, M);
+    note_launches(1);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_state_passing(const ScanArgs& a, cudaStream_t stream) {
+    const int B = (int)a.B, H = (int)a.H, S = (int)a.S, M = (int)(a.L / a.S);
+    const int NP = (int)(a.N * a.P);
+    state_passing_kernel<<<dim3((NP + 255) / 256, H, B), 256, 0, stream>>>(a.dH32, a.cum,
+                                                                           a.final_state, H, M, S,
+                                                                           NP);
+    note_launches(1);
+    return cudaGetLastError();
+}
+
 template <typename Tin, typename Tmem, typename Tout>
 cudaError_t launch_chunk_scan_simt(const ScanArgs& a, cudaStream_t stream) {
     const int B = (int)a.B, L = (int)a.L, H = (int)a.H, G = (int)a.G, P = (int)a.P,
               N = (int)a.N, S = (int)a.S, M = L / S;
-    chunk_cumsum_kernel<<<dim3(M, H, B), S, 64 * sizeof(float), stream>>>(a.dt, a.A, a.cum, L, H,
-                                                                             S, M);
+    cudaError_t e = launch_chunk_cumsum(a, stream);
+    if (e != cudaSuccess) return e;
     chunk_state_kernel<Tin, Tmem><<<dim3(M, H, B), 256, 0, stream>>>(
         (const Tin*)a.X, a.dt, a.cum, (const Tin*)a.Bm, a.dH32, (Tmem*)a.M, a.rM, L, H, G, P, N, S,
         M, a.eps);
-    const int NP = N * P;
-    state_passing_kernel<<<dim3((NP + 255) / 256, H, B), 256, 0, stream>>>(a.dH32, a.cum,
-                                                                           a.final_state, H, M, S,
-                                                                           NP);
+    note_launches(1);
+    e = launch_state_passing(a, stream);
+    if (e != cudaSuccess) return e;
     chunk_output_kernel<Tin, Tout><<<dim3((S + 63) / 64, M * H, B), 256, 0, stream>>>(
         (const Tin*)a.X, a.dt, a.cum, (const Tin*)a.Bm, (const Tin*)a.Cm, a.dH32, (Tout*)a.Y, L, H,
         G, P, N, S, M);
-    note_launches(4);
+    note_launches(1);
     return cudaGetLastError();
 }
 

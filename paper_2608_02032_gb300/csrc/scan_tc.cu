@@ -1,0 +1,517 @@
+// Chunked SSD scan on the 5th-generation tensor cores for bf16 token inputs,
+// P = 64, N = 128, S in {128, 256} (Sec. 2; Sec. 3 "Chunk State Memories";
+// App. A chunked scan). Two kernels replace the FFMA chunk-state and
+// chunk-output kernels; the within-chunk cumsum and the inter-chunk state
+// passing stay as they are (scan.cu).
+//
+// chunk_state_tc_kernel, one CTA (128 threads) per (chunk c, head group, b):
+//   M_c = B_c^T (w (.) X_c),  w_s = exp(cum_end - cum_s) dt_s      (App. A)
+//   A = B_c^T sits in TMEM (lane n, K = s); the B operand w (.) X_c is staged
+//   per head as bf16 hi + lo (two MMAs, ~2^-16 relative) in the 128-byte
+//   swizzled MN-major layout. The epilogue (thread n = row n) writes the
+//   memory, its inverse RMS r (App. B.1) and the fp32 copy for state passing.
+// chunk_output_tc_kernel, one CTA (128 threads) per (128-token tile, chunk, head group, b):
+//   scores = C_tile B_src^T                  (once, shared by the heads: G = 1)
+//   W_h[t,s] = scores[t,s] exp(cum_t - cum_s) dt_s  for s <= t, else 0
+//   Y_t = W_h X_h + exp(cum_t) C_t H_[c-1]   (App. A intra + inter terms)
+//   W_h is scaled per row by 1 / max_s |W_h[t,s]| and stored fp16 in TMEM as
+//   the A operand (fp16 keeps 11 bits; the row scale keeps small decayed
+//   weights out of the subnormal range); H_[c-1] is split bf16 hi + lo. A CPU
+//   emulation against the oracle gives max|err|/RMS(Y) = 2.1e-3 for this
+//   scheme (5.4e-3 without the row scale, 4.2e-2 with plain bf16).
+// TMEM of the output kernel: scores [0, 256), W [256, 384), intra accumulator
+// [384, 448), inter accumulator [448, 512).
+#include <math.h>
+
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+
+#include "common.cuh"
+#include "kernels.h"
+#include "tc_ptx.cuh"
+
+namespace dart {
+namespace {
+
+__device__ int g_scan_tc_status;  // first timeout code since the last read (0 = none)
+
+constexpr int kP = 64;
+constexpr int kN = 128;
+constexpr int kT = 128;  // tokens per output tile
+constexpr int kThreads = 128;
+constexpr int kHeadsPerCta = 8;
+constexpr uint64_t kDrainLimitNs = 2000000000ull;
+constexpr float kLog2e = 1.4426950408889634f;
+
+__device__ __forceinline__ uint32_t sw128(uint32_t row, uint32_t byte_in_row) {
+    const uint32_t o = row * 128u + byte_in_row;
+    return o ^ ((row & 7u) << 4);
+}
+
+__device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
+    const __nv_bfloat162 v = __floats2bfloat162_rn(a, b);
+    return *reinterpret_cast<const uint32_t*>(&v);
+}
+__device__ __forceinline__ uint32_t pack_f16(float a, float b) {
+    const __half2 v = __floats2half2_rn(a, b);
+    return *reinterpret_cast<const uint32_t*>(&v);
+}
+
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
+    uint32_t r[32];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];\n\t"
+        "tcgen05.wait::ld.sync.aligned;"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+          "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),
+          "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),
+          "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+        : "r"(taddr)
+        : "memory");
+#pragma unroll
+    for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// D[tmem] (+)= A[smem] * B[smem]
+__device__ __forceinline__ void mma_f16_ss(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
+                                           uint32_t idesc, uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}"
+        ::"r"(d_tmem), "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
+// Commit the MMAs issued by thread 0 and wait (all threads) for them; on a
+// timeout set the status and return false (the caller stops; the final drain
+// waits for the MMAs in flight with the long bound).
+__device__ __forceinline__ bool commit_and_wait(uint64_t* bar, uint32_t parity,
+                                                unsigned long long limit_ns, int code) {
+    if (threadIdx.x == 0) tc::mma_commit(bar);
+    const bool ok = tc::mbar_wait(bar, parity, limit_ns, nullptr);
+    if (!ok) atomicCAS(&g_scan_tc_status, 0, code);
+    const bool all_ok = __syncthreads_and(ok ? 1 : 0) != 0;
+    tc::tc_fence_after();
+    return all_ok;
+}
+
+// ------------------------------------------------------------ chunk state
+struct StateSmem {
+    union {
+        uint8_t wx[2][256 * 128];        // (w (.) X) hi | lo: S rows x 128 bytes, swizzled
+        __nv_bfloat16 b_rows[256 * kN];  // the chunk's B rows (only while building A)
+    };
+    float w[256];
+    uint64_t bar;
+    uint32_t tmem_base;
+};
+
+template <typename Tmem>
+__global__ void __launch_bounds__(kThreads)
+chunk_state_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restrict__ dt,
+                      const float* __restrict__ cum, const __nv_bfloat16* __restrict__ Bm,
+                      float* __restrict__ dH32, Tmem* __restrict__ Mout, float* __restrict__ rM,
+                      int L, int H, int G, int S, int Mc, float eps,
+                      unsigned long long wait_limit_ns) {
+    extern __shared__ uint8_t smem_raw[];
+    StateSmem& sm = *reinterpret_cast<StateSmem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                                  ~(uintptr_t)1023);
+    const int c = blockIdx.x, hg = blockIdx.y, b = blockIdx.z;
+    const int tid = threadIdx.x, warp = tid >> 5;
+    const int h0 = hg * kHeadsPerCta;
+    const int g = h0 / (H / G);
+    const i64 tok0 = (i64)b * L + (i64)c * S;
+    const uint32_t lane_addr = (uint32_t)(32 * warp) << 16;
+
+    if (tid == 0) {
+        tc::mbar_init(&sm.bar, 1);
+        tc::fence_barrier_init();
+    }
+    if (warp == 0) {
+        tc::tmem_alloc(&sm.tmem_base, 256);
+        tc::tmem_relinquish();
+    }
+    // the chunk's B rows into shared memory (16-byte loads)
+    {
+        uint4* dst = reinterpret_cast<uint4*>(sm.b_rows);
+        const int per_row = kN * 2 / 16;  // 16
+        for (int i = tid; i < S * per_row; i += kThreads) {
+            const int s = i / per_row, q = i % per_row;
+            dst[i] = reinterpret_cast<const uint4*>(Bm + ((tok0 + s) * G + g) * kN)[q];
+        }
+    }
+    tc::tc_fence_before();
+    __syncthreads();
+    tc::tc_fence_after();
+    const uint32_t tmem = sm.tmem_base;
+    // A = B^T into TMEM: lane n, columns s / 2 (bf16 pairs)
+    {
+        const int n = tid;
+        for (int c0 = 0; c0 < S / 2; c0 += 16) {
+            uint32_t r[16];
+#pragma unroll
+            for (int i = 0; i < 16; ++i) {
+                const int s = 2 * (c0 + i);
+                __nv_bfloat162 p;
+                p.x = sm.b_rows[s * kN + n];
+                p.y = sm.b_rows[(s + 1) * kN + n];
+                r[i] = *reinterpret_cast<const uint32_t*>(&p);
+            }
+            tc::tmem_st16(tmem + lane_addr + (uint32_t)c0, r);
+        }
+        asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+    }
+    __syncthreads();  // b_rows is overwritten by the staging buffers below
+    const uint32_t d_col = (uint32_t)(S / 2);  // accumulator after the A operand
+    constexpr uint32_t idesc = tc::idesc_f16(1, true, kN, kP);
+    uint32_t phase = 0;
+    bool ok = true;
+    for (int hh = 0; hh < kHeadsPerCta && ok; ++hh) {
+        const int h = h0 + hh;
+        const float* cumc = cum + (((i64)b * H + h) * Mc + c) * S;
+        const float cum_end = cumc[S - 1];
+        for (int s = tid; s < S; s += kThreads)
+            sm.w[s] = expf(cum_end - cumc[s]) * dt[(tok0 + s) * H + h];
+        __syncthreads();
+        // stage (w (.) X_h) as bf16 hi / lo, rows s, 128-byte swizzle
+        for (int s = tid; s < S; s += kThreads) {
+            const uint4* xr = reinterpret_cast<const uint4*>(X + ((tok0 + s) * H + h) * kP);
+            const float ws = sm.w[s];
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {  // 8 bf16 per 16-byte chunk
+                const uint4 xv = xr[q];
+                const uint32_t xw[4] = {xv.x, xv.y, xv.z, xv.w};
+                uint32_t hi[4], lo[4];
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&xw[e]));
+                    const float a0 = ws * f.x, a1 = ws * f.y;
+                    const __nv_bfloat162 hv = __floats2bfloat162_rn(a0, a1);
+                    const float2 hf = __bfloat1622float2(hv);
+                    hi[e] = *reinterpret_cast<const uint32_t*>(&hv);
+                    lo[e] = pack_bf16(a0 - hf.x, a1 - hf.y);
+                }
+                const uint32_t o = sw128((uint32_t)s, (uint32_t)q * 16u);
+                *reinterpret_cast<uint4*>(sm.wx[0] + o) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+                *reinterpret_cast<uint4*>(sm.wx[1] + o) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+            }
+        }
+        tc::fence_proxy_async_shared();
+        tc::tc_fence_before();
+        __syncthreads();
+        if (tid == 0) {
+            tc::tc_fence_after();
+            for (int part = 0; part < 2; ++part) {
+                const uint32_t base = tc::smem_u32(sm.wx[part]);
+                for (int ks = 0; ks < S / 16; ++ks) {
+                    const uint64_t bd = tc::smem_desc_sw128(base + 2048u * ks, 1024u, 1024u);
+                    tc::mma_f16_ts(tmem + d_col, tmem + 8u * ks, bd, idesc,
+                                   (part > 0 || ks > 0) ? 1u : 0u);
+                }
+            }
+        }
+        ok = commit_and_wait(&sm.bar, phase, wait_limit_ns, 1);
+        phase ^= 1u;
+        if (!ok) break;
+        // epilogue: thread n = memory row n
+        {
+            const int n = tid;
+            const i64 mrow = ((((i64)b * Mc + c) * H + h) * kN + n);
+            float v[32];
+            float ss = 0.0f;
+#pragma unroll
+            for (int half = 0; half < 2; ++half) {
+                tmem_ld32(tmem + lane_addr + d_col + 32u * half, v);
+                float4* d32 = reinterpret_cast<float4*>(dH32 + mrow * kP + 32 * half);
+#pragma unroll
+                for (int q = 0; q < 8; ++q)
+                    d32[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+#pragma unroll
+                for (int i = 0; i < 32; ++i) {
+                    Mout[mrow * kP + 32 * half + i] = cvt_from_f32<Tmem>(v[i]);
+                    const float sv = stored_value<Tmem>(v[i]);
+                    ss = fmaf(sv, sv, ss);
+                }
+            }
+            if (rM != nullptr) rM[mrow] = rsqrtf(ss / (float)kP + eps);
+        }
+        tc::tc_fence_before();
+        __syncthreads();  // the accumulator and the staging buffers are reused
+    }
+    if (!ok) {  // a wait ran out: let the MMAs in flight finish before freeing TMEM
+        if (!tc::mbar_wait(&sm.bar, phase ^ 1u, kDrainLimitNs, nullptr))
+            atomicCAS(&g_scan_tc_status, 0, 9);
+    }
+    tc::tc_fence_before();
+    __syncthreads();
+    if (warp == 0) {
+        __syncwarp();
+        tc::tc_fence_after();
+        tc::tmem_dealloc(tmem, 256);
+    }
+}
+
+// ----------------------------------------------------------- chunk output
+struct OutSmem {
+    uint8_t c_tile[2][kT * 128];   // C of the tile, K-major, two 64-wide K blocks
+    uint8_t b_src[2][256 * 128];   // B of the sources, K-major (rows s), two K blocks
+    uint8_t x_src[256 * 128];      // X_h of the sources as fp16, MN-major (rows s)
+    uint8_t h_prev[2][kN * 128];   // H_[c-1] of head h, bf16 hi | lo, MN-major (rows n)
+    float c2[256];                 // cum * log2(e) of the sources
+    float dts[256];
+    uint64_t bar;
+    uint32_t tmem_base;
+};
+
+template <typename Tout>
+__global__ void __launch_bounds__(kThreads, 1)
+chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restrict__ dt,
+                       const float* __restrict__ cum, const __nv_bfloat16* __restrict__ Bm,
+                       const __nv_bfloat16* __restrict__ Cm, const float* __restrict__ Hin,
+                       Tout* __restrict__ Y, int L, int H, int G, int S, int Mc,
+                       unsigned long long wait_limit_ns) {
+    extern __shared__ uint8_t smem_raw[];
+    OutSmem& sm = *reinterpret_cast<OutSmem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                              ~(uintptr_t)1023);
+    const int tt = blockIdx.x;  // tile inside the chunk
+    const int c = blockIdx.y / (H / kHeadsPerCta);
+    const int hg = blockIdx.y % (H / kHeadsPerCta);
+    const int b = blockIdx.z;
+    const int tid = threadIdx.x, warp = tid >> 5;
+    const int h0 = hg * kHeadsPerCta;
+    const int g = h0 / (H / G);
+    const int ns = (tt + 1) * kT;  // sources 0 .. ns-1 of the chunk
+    const i64 tok0 = (i64)b * L + (i64)c * S;
+    const uint32_t lane_addr = (uint32_t)(32 * warp) << 16;
+    constexpr uint32_t kColSc = 0, kColW = 256, kColIn = 384, kColEx = 448;
+
+    if (tid == 0) {
+        tc::mbar_init(&sm.bar, 1);
+        tc::fence_barrier_init();
+    }
+    if (warp == 0) {
+        tc::tmem_alloc(&sm.tmem_base, 512);
+        tc::tmem_relinquish();
+    }
+    // C of the tile: row t, K-major, two K blocks of 64 (16-byte chunks, swizzled)
+    for (int i = tid; i < kT * 16; i += kThreads) {
+        const int t = i / 16, q = i % 16;
+        const uint4 v = reinterpret_cast<const uint4*>(Cm + ((tok0 + tt * kT + t) * G + g) * kN)[q];
+        *reinterpret_cast<uint4*>(sm.c_tile[q / 8] + sw128((uint32_t)t, (uint32_t)(q % 8) * 16u)) = v;
+    }
+    // B of the sources: row s, K-major
+    for (int i = tid; i < ns * 16; i += kThreads) {
+        const int s = i / 16, q = i % 16;
+        const uint4 v = reinterpret_cast<const uint4*>(Bm + ((tok0 + s) * G + g) * kN)[q];
+        *reinterpret_cast<uint4*>(sm.b_src[q / 8] + sw128((uint32_t)s, (uint32_t)(q % 8) * 16u)) = v;
+    }
+    tc::fence_proxy_async_shared();
+    tc::tc_fence_before();
+    __syncthreads();
+    tc::tc_fence_after();
+    const uint32_t tmem = sm.tmem_base;
+    uint32_t phase = 0;
+    // scores = C_tile B_src^T (M 128, N ns, K 128)
+    if (tid == 0) {
+        const uint32_t idesc = tc::idesc_f16(1, false, kT, (uint32_t)ns);
+        for (int ks = 0; ks < kN / 16; ++ks) {
+            const uint64_t ad = tc::smem_desc_sw128(tc::smem_u32(sm.c_tile[ks / 4]) + 32u * (ks % 4), 16u, 1024u);
+            const uint64_t bd = tc::smem_desc_sw128(tc::smem_u32(sm.b_src[ks / 4]) + 32u * (ks % 4), 16u, 1024u);
+            mma_f16_ss(tmem + kColSc, ad, bd, idesc, ks > 0 ? 1u : 0u);
+        }
+    }
+    bool ok = commit_and_wait(&sm.bar, phase, wait_limit_ns, 2);
+    phase ^= 1u;
+
+    const int tl = tt * kT + tid;  // this thread's token inside the chunk
+    const i64 tok = tok0 + tl;
+    for (int hh = 0; hh < kHeadsPerCta && ok; ++hh) {
+        const int h = h0 + hh;
+        const float* cumc = cum + (((i64)b * H + h) * Mc + c) * S;
+        for (int s = tid; s < ns; s += kThreads) {
+            sm.c2[s] = cumc[s] * kLog2e;
+            sm.dts[s] = dt[(tok0 + s) * H + h];
+        }
+        // X_h of the sources as fp16, rows s (MN-major B operand of the intra MMA)
+        for (int i = tid; i < ns * 8; i += kThreads) {
+            const int s = i / 8, q = i % 8;
+            const uint4 xv = reinterpret_cast<const uint4*>(X + ((tok0 + s) * H + h) * kP)[q];
+            const uint32_t xw[4] = {xv.x, xv.y, xv.z, xv.w};
+            uint32_t f[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const float2 v = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&xw[e]));
+                f[e] = pack_f16(v.x, v.y);
+            }
+            *reinterpret_cast<uint4*>(sm.x_src + sw128((uint32_t)s, (uint32_t)q * 16u)) =
+                make_uint4(f[0], f[1], f[2], f[3]);
+        }
+        // H_[c-1] of head h as bf16 hi | lo, rows n (zero state before chunk 0)
+        const bool has_prev = c > 0;
+        if (has_prev) {
+            const float* Hh = Hin + (((i64)b * Mc + c) * H + h) * (i64)(kN * kP);
+            for (int i = tid; i < kN * 8; i += kThreads) {
+                const int n = i / 8, q = i % 8;
+                const float4 a = reinterpret_cast<const float4*>(Hh + n * kP)[2 * q];
+                const float4 bb = reinterpret_cast<const float4*>(Hh + n * kP)[2 * q + 1];
+                const float vals[8] = {a.x, a.y, a.z, a.w, bb.x, bb.y, bb.z, bb.w};
+                uint32_t hi[4], lo[4];
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const __nv_bfloat162 hv = __floats2bfloat162_rn(vals[2 * e], vals[2 * e + 1]);
+                    const float2 hf = __bfloat1622float2(hv);
+                    hi[e] = *reinterpret_cast<const uint32_t*>(&hv);
+                    lo[e] = pack_bf16(vals[2 * e] - hf.x, vals[2 * e + 1] - hf.y);
+                }
+                const uint32_t o = sw128((uint32_t)n, (uint32_t)q * 16u);
+                *reinterpret_cast<uint4*>(sm.h_prev[0] + o) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+                *reinterpret_cast<uint4*>(sm.h_prev[1] + o) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+            }
+        }
+        __syncthreads();
+        // W_h row of this thread: two passes over the scores (max, then scale + fp16)
+        const float c2t = sm.c2[tl];
+        float wmax = 0.0f;
+        for (int s0 = 0; s0 < ns; s0 += 32) {
+            float v[32];
+            tmem_ld32(tmem + lane_addr + kColSc + (uint32_t)s0, v);
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+                const int s = s0 + i;
+                const float wv = s <= tl ? v[i] * exp2f(c2t - sm.c2[s]) * sm.dts[s] : 0.0f;
+                wmax = fmaxf(wmax, fabsf(wv));
+            }
+        }
+        const float rscale = wmax > 0.0f ? 1.0f / wmax : 1.0f;
+        for (int s0 = 0; s0 < ns; s0 += 32) {
+            float v[32];
+            tmem_ld32(tmem + lane_addr + kColSc + (uint32_t)s0, v);
+            uint32_t pk[16];
+#pragma unroll
+            for (int i = 0; i < 16; ++i) {
+                const int s = s0 + 2 * i;
+                const float w0 = s <= tl ? v[2 * i] * exp2f(c2t - sm.c2[s]) * sm.dts[s] : 0.0f;
+                const float w1 = s + 1 <= tl ? v[2 * i + 1] * exp2f(c2t - sm.c2[s + 1]) * sm.dts[s + 1] : 0.0f;
+                pk[i] = pack_f16(w0 * rscale, w1 * rscale);
+            }
+            tc::tmem_st16(tmem + lane_addr + kColW + (uint32_t)(s0 / 2), pk);
+        }
+        asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+        tc::fence_proxy_async_shared();
+        tc::tc_fence_before();
+        __syncthreads();
+        if (tid == 0) {
+            tc::tc_fence_after();
+            const uint32_t id16 = tc::idesc_f16(0, true, kT, kP);
+            for (int ks = 0; ks < ns / 16; ++ks) {
+                const uint64_t bd = tc::smem_desc_sw128(tc::smem_u32(sm.x_src) + 2048u * ks, 1024u, 1024u);
+                tc::mma_f16_ts(tmem + kColIn, tmem + kColW + 8u * ks, bd, id16, ks > 0 ? 1u : 0u);
+            }
+            if (has_prev) {
+                const uint32_t idb = tc::idesc_f16(1, true, kT, kP);
+                for (int part = 0; part < 2; ++part) {
+                    for (int ks = 0; ks < kN / 16; ++ks) {
+                        const uint64_t ad = tc::smem_desc_sw128(
+                            tc::smem_u32(sm.c_tile[ks / 4]) + 32u * (ks % 4), 16u, 1024u);
+                        const uint64_t bd = tc::smem_desc_sw128(
+                            tc::smem_u32(sm.h_prev[part]) + 2048u * ks, 1024u, 1024u);
+                        mma_f16_ss(tmem + kColEx, ad, bd, idb, (part > 0 || ks > 0) ? 1u : 0u);
+                    }
+                }
+            }
+        }
+        ok = commit_and_wait(&sm.bar, phase, wait_limit_ns, 3);
+        phase ^= 1u;
+        if (!ok) break;
+        // Y_t = wmax * (W~ X)_t + exp(cum_t) (C H)_t
+        {
+            const float dec = exp2f(c2t);
+            Tout* yrow = Y + (tok * H + h) * kP;
+#pragma unroll
+            for (int half = 0; half < 2; ++half) {
+                float vi[32], ve[32];
+                tmem_ld32(tmem + lane_addr + kColIn + 32u * half, vi);
+                if (has_prev) {
+                    tmem_ld32(tmem + lane_addr + kColEx + 32u * half, ve);
+                } else {
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) ve[i] = 0.0f;
+                }
+#pragma unroll
+                for (int i = 0; i < 32; ++i)
+                    yrow[32 * half + i] = cvt_from_f32<Tout>(fmaf(wmax, vi[i], dec * ve[i]));
+            }
+        }
+        tc::tc_fence_before();
+        __syncthreads();  // shared staging and TMEM are reused by the next head
+    }
+    if (!ok) {
+        if (!tc::mbar_wait(&sm.bar, phase ^ 1u, kDrainLimitNs, nullptr))
+            atomicCAS(&g_scan_tc_status, 0, 10);
+    }
+    tc::tc_fence_before();
+    __syncthreads();
+    if (warp == 0) {
+        __syncwarp();
+        tc::tc_fence_after();
+        tc::tmem_dealloc(tmem, 512);
+    }
+}
+
+}  // namespace
+
+bool scan_tc_supported(const ScanArgs& a) {
+    return a.P == kP && a.N == kN && (a.S == 128 || a.S == 256) &&
+           a.H % kHeadsPerCta == 0 && (a.H / a.G) % kHeadsPerCta == 0;
+}
+
+template <typename Tmem, typename Tout>
+cudaError_t launch_chunk_scan_tc(const ScanArgs& a, unsigned long long wait_limit_ns,
+                                 cudaStream_t stream) {
+    const int B = (int)a.B, L = (int)a.L, H = (int)a.H, G = (int)a.G, S = (int)a.S, M = L / S;
+    cudaError_t e0 = launch_chunk_cumsum(a, stream);
+    if (e0 != cudaSuccess) return e0;
+    {
+        auto kern = chunk_state_tc_kernel<Tmem>;
+        const size_t smem = sizeof(StateSmem) + 1024;
+        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+        kern<<<dim3(M, H / kHeadsPerCta, B), kThreads, smem, stream>>>(
+            (const __nv_bfloat16*)a.X, a.dt, a.cum, (const __nv_bfloat16*)a.Bm, a.dH32, (Tmem*)a.M,
+            a.rM, L, H, G, S, M, a.eps, wait_limit_ns);
+    }
+    e0 = launch_state_passing(a, stream);
+    if (e0 != cudaSuccess) return e0;
+    {
+        auto kern = chunk_output_tc_kernel<Tout>;
+        const size_t smem = sizeof(OutSmem) + 1024;
+        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+        kern<<<dim3(S / kT, M * (H / kHeadsPerCta), B), kThreads, smem, stream>>>(
+            (const __nv_bfloat16*)a.X, a.dt, a.cum, (const __nv_bfloat16*)a.Bm,
+            (const __nv_bfloat16*)a.Cm, a.dH32, (Tout*)a.Y, L, H, G, S, M, wait_limit_ns);
+    }
+    note_launches(2);
+    return cudaGetLastError();
+}
+
+typedef __nv_bfloat16 bf16;
+template cudaError_t launch_chunk_scan_tc<float, float>(const ScanArgs&, unsigned long long, cudaStream_t);
+template cudaError_t launch_chunk_scan_tc<bf16, float>(const ScanArgs&, unsigned long long, cudaStream_t);
+template cudaError_t launch_chunk_scan_tc<bf16, bf16>(const ScanArgs&, unsigned long long, cudaStream_t);
+
+int take_scan_tc_status() {
+    int v = 0;
+    if (cudaMemcpyFromSymbol(&v, g_scan_tc_status, sizeof(int)) != cudaSuccess) return -1;
+    if (v != 0) {
+        const int zero = 0;
+        cudaMemcpyToSymbol(g_scan_tc_status, &zero, sizeof(int));
+    }
+    return v;
+}
+
+}  // namespace dart

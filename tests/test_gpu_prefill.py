@@ -59,6 +59,9 @@ SWEEP = [
     (128, 128, 64, 128, 4, 1, "bf16"),     # M = 1: only chunk-0 tiles
     (1024, 256, 64, 128, 8, 1, "bf16"),    # two head groups
     (768, 256, 64, 128, 8, 2, "bf16"),     # G = 2, four heads per group
+    # tensor-core scan shapes (bf16, P 64, N 128, S in {128, 256}, 8 heads per CTA)
+    (512, 128, 64, 128, 8, 1, "bf16"),
+    (1024, 256, 64, 128, 16, 2, "bf16"),   # G = 2, eight heads per group
 ]
 
 
