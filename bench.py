@@ -249,7 +249,7 @@ def run_dart(args) -> None:
         dist.init_process_group("nccl", device_id=dev)
     Bd.lib()
     peaks = _peaks()
-    w = WORKLOADS[PREFILL]
+    w = WORKLOADS[args.workload]
     inp = prefill_inputs(w)
     tdt = torch.bfloat16
     Bsz, L, H, G, P, N, S = w.batch, w.seqlen, w.heads, w.groups, w.headdim, w.dstate, w.chunk
@@ -454,6 +454,7 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-heads", type=int, default=4, help="heads in the oracle CPU sample")
     ap.add_argument("--ref-heads", type=int, default=1, help="heads per reference-arm step")
+    ap.add_argument("--workload", default=PREFILL, help="prefill workload (smaller ones for profiling)")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "dart":
         print("note: at least 3 warm-up steps are required; using 3", file=sys.stderr)

@@ -29,6 +29,82 @@ template <> __device__ __forceinline__ float stored_value<__nv_bfloat16>(float v
     return __bfloat162float(__float2bfloat16_rn(v));
 }
 
+// 32 consecutive values of a row (16-byte aligned) as vector loads / stores.
+__device__ __forceinline__ void load_row32(const float* src, float* v) {
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+        const float4 f = reinterpret_cast<const float4*>(src)[q];
+        v[4 * q] = f.x; v[4 * q + 1] = f.y; v[4 * q + 2] = f.z; v[4 * q + 3] = f.w;
+    }
+}
+__device__ __forceinline__ void load_row32(const __nv_bfloat16* src, float* v) {
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        const uint4 u = reinterpret_cast<const uint4*>(src)[q];
+        const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w[e]));
+            v[8 * q + 2 * e] = f.x; v[8 * q + 2 * e + 1] = f.y;
+        }
+    }
+}
+__device__ __forceinline__ void store_row32(float* dst, const float* v) {
+#pragma unroll
+    for (int q = 0; q < 8; ++q)
+        reinterpret_cast<float4*>(dst)[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+}
+__device__ __forceinline__ void store_row32(__nv_bfloat16* dst, const float* v) {
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        uint32_t w[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const __nv_bfloat162 p = __floats2bfloat162_rn(v[8 * q + 2 * e], v[8 * q + 2 * e + 1]);
+            w[e] = *reinterpret_cast<const uint32_t*>(&p);
+        }
+        reinterpret_cast<uint4*>(dst)[q] = make_uint4(w[0], w[1], w[2], w[3]);
+    }
+}
+
+// 16-value variants (half the registers).
+__device__ __forceinline__ void load_row16(const float* src, float* v) {
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        const float4 f = reinterpret_cast<const float4*>(src)[q];
+        v[4 * q] = f.x; v[4 * q + 1] = f.y; v[4 * q + 2] = f.z; v[4 * q + 3] = f.w;
+    }
+}
+__device__ __forceinline__ void load_row16(const __nv_bfloat16* src, float* v) {
+#pragma unroll
+    for (int q = 0; q < 2; ++q) {
+        const uint4 u = reinterpret_cast<const uint4*>(src)[q];
+        const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w[e]));
+            v[8 * q + 2 * e] = f.x; v[8 * q + 2 * e + 1] = f.y;
+        }
+    }
+}
+__device__ __forceinline__ void store_row16(float* dst, const float* v) {
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+        reinterpret_cast<float4*>(dst)[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+}
+__device__ __forceinline__ void store_row16(__nv_bfloat16* dst, const float* v) {
+#pragma unroll
+    for (int q = 0; q < 2; ++q) {
+        uint32_t w[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const __nv_bfloat162 p = __floats2bfloat162_rn(v[8 * q + 2 * e], v[8 * q + 2 * e + 1]);
+            w[e] = *reinterpret_cast<const uint32_t*>(&p);
+        }
+        reinterpret_cast<uint4*>(dst)[q] = make_uint4(w[0], w[1], w[2], w[3]);
+    }
+}
+
 // SiLU(z) = z * sigmoid(z), the SMA residual gate (Sec. 3).
 __device__ __forceinline__ float silu_f32(float z) { return z / (1.0f + expf(-z)); }
 

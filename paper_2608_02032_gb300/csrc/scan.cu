@@ -145,12 +145,27 @@ __global__ void state_passing_kernel(float* __restrict__ dH32, const float* __re
     const int h = blockIdx.y, b = blockIdx.z;
     if (e >= NP) return;
     const float* cumh = cum + ((i64)b * H + h) * M * S;
+    const i64 stride = (i64)H * NP;  // between chunk slots of the same element
+    float* base = dH32 + ((i64)b * M * H + h) * NP + e;
     float st = 0.0f;
-    for (int c = 0; c < M; ++c) {
-        const i64 o = (((i64)b * M + c) * H + h) * NP + e;
-        const float d = dH32[o];
-        dH32[o] = st;  // state entering chunk c
-        st = fmaf(expf(cumh[(i64)c * S + S - 1]), st, d);
+    // groups of 16 chunks: issue the independent loads first, then the chain
+    for (int c0 = 0; c0 < M; c0 += 16) {
+        const int n = min(16, M - c0);
+        float d[16], dec[16];
+#pragma unroll
+        for (int k = 0; k < 16; ++k) {
+            if (k < n) {
+                d[k] = base[(i64)(c0 + k) * stride];
+                dec[k] = expf(cumh[(i64)(c0 + k) * S + S - 1]);
+            }
+        }
+#pragma unroll
+        for (int k = 0; k < 16; ++k) {
+            if (k < n) {
+                base[(i64)(c0 + k) * stride] = st;  // state entering chunk c0 + k
+                st = fmaf(dec[k], st, d[k]);
+            }
+        }
     }
     if (final_state != nullptr) final_state[((i64)b * H + h) * NP + e] = st;
 }

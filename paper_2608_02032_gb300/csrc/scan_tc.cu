@@ -181,9 +181,12 @@ chunk_state_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restri
         for (int s = tid; s < S; s += kThreads) {
             const uint4* xr = reinterpret_cast<const uint4*>(X + ((tok0 + s) * H + h) * kP);
             const float ws = sm.w[s];
+            uint4 xrow[8];
+#pragma unroll
+            for (int q = 0; q < 8; ++q) xrow[q] = xr[q];
 #pragma unroll
             for (int q = 0; q < 8; ++q) {  // 8 bf16 per 16-byte chunk
-                const uint4 xv = xr[q];
+                const uint4 xv = xrow[q];
                 const uint32_t xw[4] = {xv.x, xv.y, xv.z, xv.w};
                 uint32_t hi[4], lo[4];
 #pragma unroll
@@ -230,9 +233,9 @@ chunk_state_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restri
 #pragma unroll
                 for (int q = 0; q < 8; ++q)
                     d32[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+                store_row32(Mout + mrow * kP + 32 * half, v);
 #pragma unroll
                 for (int i = 0; i < 32; ++i) {
-                    Mout[mrow * kP + 32 * half + i] = cvt_from_f32<Tmem>(v[i]);
                     const float sv = stored_value<Tmem>(v[i]);
                     ss = fmaf(sv, sv, ss);
                 }
@@ -336,28 +339,49 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
             sm.c2[s] = cumc[s] * kLog2e;
             sm.dts[s] = dt[(tok0 + s) * H + h];
         }
-        // X_h of the sources as fp16, rows s (MN-major B operand of the intra MMA)
-        for (int i = tid; i < ns * 8; i += kThreads) {
-            const int s = i / 8, q = i % 8;
-            const uint4 xv = reinterpret_cast<const uint4*>(X + ((tok0 + s) * H + h) * kP)[q];
-            const uint32_t xw[4] = {xv.x, xv.y, xv.z, xv.w};
-            uint32_t f[4];
+        // X_h of the sources as fp16, rows s (MN-major B operand of the intra MMA);
+        // all of a thread's 16-byte loads are issued before any is used
+        {
+            const int iters = ns * 8 / kThreads;  // 8 or 16
+            uint4 xv[16];
 #pragma unroll
-            for (int e = 0; e < 4; ++e) {
-                const float2 v = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&xw[e]));
-                f[e] = pack_f16(v.x, v.y);
+            for (int k = 0; k < 16; ++k) {
+                if (k < iters) {
+                    const int i = tid + k * kThreads, s = i / 8, q = i % 8;
+                    xv[k] = reinterpret_cast<const uint4*>(X + ((tok0 + s) * H + h) * kP)[q];
+                }
             }
-            *reinterpret_cast<uint4*>(sm.x_src + sw128((uint32_t)s, (uint32_t)q * 16u)) =
-                make_uint4(f[0], f[1], f[2], f[3]);
+#pragma unroll
+            for (int k = 0; k < 16; ++k) {
+                if (k < iters) {
+                    const int i = tid + k * kThreads, s = i / 8, q = i % 8;
+                    const uint32_t xw[4] = {xv[k].x, xv[k].y, xv[k].z, xv[k].w};
+                    uint32_t f[4];
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        const float2 v = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&xw[e]));
+                        f[e] = pack_f16(v.x, v.y);
+                    }
+                    *reinterpret_cast<uint4*>(sm.x_src + sw128((uint32_t)s, (uint32_t)q * 16u)) =
+                        make_uint4(f[0], f[1], f[2], f[3]);
+                }
+            }
         }
         // H_[c-1] of head h as bf16 hi | lo, rows n (zero state before chunk 0)
         const bool has_prev = c > 0;
         if (has_prev) {
             const float* Hh = Hin + (((i64)b * Mc + c) * H + h) * (i64)(kN * kP);
-            for (int i = tid; i < kN * 8; i += kThreads) {
-                const int n = i / 8, q = i % 8;
-                const float4 a = reinterpret_cast<const float4*>(Hh + n * kP)[2 * q];
-                const float4 bb = reinterpret_cast<const float4*>(Hh + n * kP)[2 * q + 1];
+            float4 hv4[16];
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+                const int i = tid + k * kThreads, n = i / 8, q = i % 8;
+                hv4[2 * k] = reinterpret_cast<const float4*>(Hh + n * kP)[2 * q];
+                hv4[2 * k + 1] = reinterpret_cast<const float4*>(Hh + n * kP)[2 * q + 1];
+            }
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+                const int i = tid + k * kThreads, n = i / 8, q = i % 8;
+                const float4 a = hv4[2 * k], bb = hv4[2 * k + 1];
                 const float vals[8] = {a.x, a.y, a.z, a.w, bb.x, bb.y, bb.z, bb.w};
                 uint32_t hi[4], lo[4];
 #pragma unroll
@@ -442,8 +466,8 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
                     for (int i = 0; i < 32; ++i) ve[i] = 0.0f;
                 }
 #pragma unroll
-                for (int i = 0; i < 32; ++i)
-                    yrow[32 * half + i] = cvt_from_f32<Tout>(fmaf(wmax, vi[i], dec * ve[i]));
+                for (int i = 0; i < 32; ++i) vi[i] = fmaf(wmax, vi[i], dec * ve[i]);
+                store_row32(yrow + 32 * half, vi);
             }
         }
         tc::tc_fence_before();

@@ -4,33 +4,46 @@
 // logit, softmax over earlier chunks and R_t; App. B.1 normalised score
 // branch; Alg. 1 streaming order; Sec. 3 gated merge).
 //
-// For a tile of 128 tokens (one TMEM lane each) and a memory M_j of head h
-// the kernel needs, per token t,
-//   U_t = Q_t (r_j (.) M_j)          (N = 128 -> P = 64)
-//   V_t = C_t M_j                    (N = 128 -> P = 64)
+// For a tile of 128 tokens (one TMEM lane each) and memory M_j of head h the
+// kernel needs, per token t,
+//   U_t = Q_t (r_j (.) M_j),   V_t = C_t M_j     (N = 128 -> P = 64 each)
 //   l_{t,j} = (U_t . Ebar_t) / (rms(Q_t) sqrt(N))
-// U and V are GEMMs with the token operands Q, C fixed for the whole tile
-// (they sit in TMEM as the A operand) and the memory as the B operand.
-// Precision: rounding the memory operand to bf16 moves the logits enough to
+// U and V are GEMMs whose token operands Q, C stay fixed for the whole tile
+// (they sit in TMEM as the A operand) while the memories stream through as
+// the B operand.
+//
+// Precision. Rounding the memory operand to bf16 moves the logits enough to
 // break the 2e-2 parity bar, so W = r (.) M is split into bf16 hi + lo parts
-// (two MMAs into one accumulator, ~2^-16 relative) and the value path runs
-// in fp16 on M / max|M_j| (scale re-applied in the epilogue). Q and C are
+// (two MMA chains into one accumulator, ~2^-16 relative) and the value path
+// runs in fp16 on M / max|M_j| (scale re-applied in the epilogue). Q and C are
 // exact (bf16 inputs; C widened to fp16 exactly); Qbar's RMS scale and Ebar
 // stay fp32 in the epilogue.
 //
-// Kernel 1 (sma_operands_kernel) writes, per memory, the three 16 KiB
-// operand tiles already in the 128-byte-swizzled shared-memory layout, so the
-// main kernel fetches one contiguous 48 KiB block per (memory, head) with a
-// single bulk copy.
-// Kernel 2 (sma_tc_kernel), one CTA per (batch, 128-token tile, 4 heads),
-// heaviest tiles first. Warp roles:
-//   warp 0      producer: bulk copies of operand blocks into a 4-stage ring
+// Shape. A tcgen05.mma with M = 128, K = 16 costs about the same for any
+// N <= 128 and only reaches the tensor peak at N >= 192 (measured on GB300:
+// ~90-99 cycles at N <= 128, ~137 at N = 256 with A in TMEM). So one job is
+// one memory j for the CTA's two heads: U is one N = 256 chain over the tiles
+// [W_hi h0 | W_lo h0 | W_hi h1 | W_lo h1] (the epilogue adds hi + lo), V is
+// one N = 128 chain over [M16 h0 | M16 h1]. U and V have one TMEM buffer each
+// and alternate, so each buffer is read by the epilogue while the other one
+// is being computed.
+//
+// Kernel 1 (sma_operands_kernel) writes per (memory, pair of heads) a 64 KiB
+// U part and a 32 KiB V part, already in the 128-byte-swizzled shared-memory
+// layout, so each part is one bulk copy.
+// Kernel 2 (sma_tc_kernel), one CTA per (batch, 128-token tile, 2 heads),
+// heaviest tiles first:
+//   warp 0      producer: bulk copies of the parts into a 3-stage ring
 //   warp 1      TMEM allocation; one thread issues the MMAs
-//   warps 2..5  epilogue (one thread per token row): stage Q and C into TMEM,
-//               then per job read U, V from TMEM, online softmax, and per
-//               head R = O / d, lse, Y = Y_ssd + SiLU(z) R.
-// TMEM: columns [0,64) Q (bf16 pairs), [64,128) C (fp16 pairs), then three
-// accumulator stages of 128 columns (U | V).
+//   warps 2, 3  idle (they complete warpgroup 0 for the register split)
+//   warps 4..7  epilogue warpgroup 0: head 0 of the pair
+//   warps 8..11 epilogue warpgroup 1: head 1 of the pair
+// An epilogue thread owns one token row of its head: it reads U and V from
+// TMEM with wide loads (three waits per job), runs the online softmax, and
+// finally writes R = O / d, lse and Y = Y_ssd + SiLU(z) R. Warpgroup 0 also
+// stages Q and C into TMEM, warpgroup 1 writes Ebar to shared memory.
+// TMEM: [0,64) Q (bf16 pairs), [64,128) C (fp16 pairs), [128,384) U,
+// [384,512) V.
 #include <math.h>
 
 #include <cuda_bf16.h>
@@ -48,19 +61,25 @@ __device__ int g_tc_status;  // first timeout code since the last read (0 = none
 constexpr int kRows = 128;   // tokens per tile (TMEM lanes)
 constexpr int kP = 64;
 constexpr int kN = 128;
-constexpr int kTile = kN * kP * 2;     // bytes of one 16-bit N x P operand tile
-constexpr int kJob = 3 * kTile;        // W_hi | W_lo | M16
-constexpr int kStages = 4;
-constexpr int kAcc = 3;
-constexpr int kHeadsPerCta = 4;
-constexpr int kThreads = 192;
+constexpr int kHeadsPerCta = 2;
+constexpr int kTile = kN * kP * 2;            // bytes of one 16-bit N x P operand tile
+constexpr int kPartU = 4 * kTile;             // W_hi h0 | W_lo h0 | W_hi h1 | W_lo h1
+constexpr int kPartV = 2 * kTile;             // M16 h0 | M16 h1
+constexpr int kPair = kPartU + kPartV;        // operand bytes per (memory, head pair)
+constexpr int kStages = 3;                    // ring of kPartU-sized stages
+constexpr int kThreads = 384;
+// Register split: launched at 168 per thread (384 x 168 = 64512 of the 65536
+// of an SM); warpgroup 0 (producer, MMA, two idle warps) drops to 56 and the
+// epilogue warpgroups rise to 224: 128 x 56 + 256 x 224 = 64512, within the
+// launch pool, and per sub-partition (56 + 2 x 224) x 32 = 16128 <= 16384.
+constexpr int kRegsLow = 56, kRegsHigh = 224;
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kColQ = 0, kColC = 64, kColAcc = 128;
+constexpr uint32_t kColQ = 0, kColC = 64, kColU = 128, kColV = 384;
 // Bound on the final waits for this CTA's own copies and MMAs (never cut short).
 constexpr uint64_t kDrainLimitNs = 2000000000ull;
 
-constexpr uint32_t kIdescBf16 = tc::idesc_f16(1, true, kRows, kP);
-constexpr uint32_t kIdescF16 = tc::idesc_f16(0, true, kRows, kP);
+constexpr uint32_t kIdescU = tc::idesc_f16(1, true, kRows, 4 * kP);  // bf16, N = 256
+constexpr uint32_t kIdescV = tc::idesc_f16(0, true, kRows, 2 * kP);  // fp16, N = 128
 
 // Byte offset of element (n, p) of a 128-row x 128-byte tile in the
 // 128-byte-swizzled layout: the 16-byte chunk index is XORed with n mod 8.
@@ -71,7 +90,9 @@ __device__ __forceinline__ uint32_t sw128(int n, int p) {
 
 // ------------------------------------------------------------ kernel 1
 // One block of 256 threads per (j, h, b) memory. Warp w owns rows n = w + 8k;
-// lane owns columns p = lane, lane + 32.
+// lane owns columns p = lane, lane + 32. Head h = 2 hp + x writes
+//   W_hi to  ops + ((b Mc + j) (H/2) + hp) kPair + 2x kTile,
+//   W_lo one tile further, M16 to  ... + kPartU + x kTile.
 template <typename Tmem>
 __global__ void __launch_bounds__(256)
 sma_operands_kernel(const Tmem* __restrict__ M, const float* __restrict__ rM,
@@ -81,7 +102,10 @@ sma_operands_kernel(const Tmem* __restrict__ M, const float* __restrict__ rM,
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const i64 mem = ((i64)b * Mc + j) * H + h;
     const Tmem* src = M + mem * (kN * kP);
-    uint8_t* dst = ops + mem * kJob;
+    const i64 pair = ((i64)b * Mc + j) * (H / kHeadsPerCta) + h / kHeadsPerCta;
+    const int x = h % kHeadsPerCta;
+    uint8_t* dst_u = ops + pair * kPair + 2 * x * kTile;
+    uint8_t* dst_v = ops + pair * kPair + kPartU + x * kTile;
     __shared__ float s_max[8];
 
     float v0[16], v1[16], rr[16];
@@ -118,21 +142,21 @@ sma_operands_kernel(const Tmem* __restrict__ M, const float* __restrict__ rM,
             const __nv_bfloat16 lo = __float2bfloat16_rn(wv - __bfloat162float(hi));
             const __half m16 = __float2half_rn(v * inv_s);
             const uint32_t o = sw128(n, p);
-            *reinterpret_cast<__nv_bfloat16*>(dst + o) = hi;
-            *reinterpret_cast<__nv_bfloat16*>(dst + kTile + o) = lo;
-            *reinterpret_cast<__half*>(dst + 2 * kTile + o) = m16;
+            *reinterpret_cast<__nv_bfloat16*>(dst_u + o) = hi;
+            *reinterpret_cast<__nv_bfloat16*>(dst_u + kTile + o) = lo;
+            *reinterpret_cast<__half*>(dst_v + o) = m16;
         }
     }
 }
 
 // ------------------------------------------------------------ kernel 2
 struct TcSmem {
-    uint8_t stage[kStages][kJob];  // 1024-aligned by placement
+    uint8_t stage[kStages][kPartU];  // 1024-aligned by placement
+    float4 ebar[kRows][kP / 4];      // Ebar rows, 16-byte chunks swizzled by row
     uint64_t full[kStages];
     uint64_t empty[kStages];
-    uint64_t acc_full[kAcc];
-    uint64_t acc_empty[kAcc];
-    uint64_t a_ready;
+    uint64_t u_full, u_free, v_full, v_free;
+    uint64_t a_ready, drain;
     uint32_t tmem_base;
     int abort;
 };
@@ -142,23 +166,70 @@ __device__ __forceinline__ void fail(volatile int* abort, int code) {
     atomicCAS(&g_tc_status, 0, code);
 }
 
-// tcgen05.ld of 32 consecutive fp32 columns of this thread's lane, waited.
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
-    uint32_t r[32];
+// tcgen05.ld of 16 consecutive fp32 columns of this thread's lane, waited.
+__device__ __forceinline__ void tmem_ld16w(uint32_t taddr, float (&v)[16]) {
+    uint32_t r[16];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];\n\t"
+        "tcgen05.wait::ld.sync.aligned;"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+          "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr)
+        : "memory");
+#pragma unroll
+    for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// Warp-uniform bounded wait (every lane waits; all lanes see the same outcome).
+__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, uint64_t limit_ns,
+                                          volatile int* abort) {
+    const bool got = tc::mbar_wait(bar, parity, limit_ns, abort);
+    return __all_sync(0xffffffffu, got);
+}
+
+// tcgen05.ld of 32 + 32 fp32 columns (two addresses) of this thread's lane, one wait.
+__device__ __forceinline__ void tmem_ld32x2(uint32_t ta, uint32_t tb, float (&v)[64]) {
+    uint32_t r[64];
     asm volatile(
         "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
         "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
-        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];\n\t"
+        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%64];\n\t"
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+        "{%32,%33,%34,%35,%36,%37,%38,%39,%40,%41,%42,%43,%44,%45,%46,%47,"
+        "%48,%49,%50,%51,%52,%53,%54,%55,%56,%57,%58,%59,%60,%61,%62,%63}, [%65];\n\t"
         "tcgen05.wait::ld.sync.aligned;"
         : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
           "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
           "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),
           "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),
-          "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
-        : "r"(taddr)
+          "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31]),
+          "=r"(r[32]), "=r"(r[33]), "=r"(r[34]), "=r"(r[35]), "=r"(r[36]), "=r"(r[37]),
+          "=r"(r[38]), "=r"(r[39]), "=r"(r[40]), "=r"(r[41]), "=r"(r[42]), "=r"(r[43]),
+          "=r"(r[44]), "=r"(r[45]), "=r"(r[46]), "=r"(r[47]), "=r"(r[48]), "=r"(r[49]),
+          "=r"(r[50]), "=r"(r[51]), "=r"(r[52]), "=r"(r[53]), "=r"(r[54]), "=r"(r[55]),
+          "=r"(r[56]), "=r"(r[57]), "=r"(r[58]), "=r"(r[59]), "=r"(r[60]), "=r"(r[61]),
+          "=r"(r[62]), "=r"(r[63])
+        : "r"(ta), "r"(tb)
         : "memory");
 #pragma unroll
-    for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+    for (int i = 0; i < 64; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// Dot product of 16 columns of U with Ebar[p0 .. p0+15] of row `row`.
+__device__ __forceinline__ float dot16(const float (&u)[16], const TcSmem& sm, int row, int p0) {
+    float acc = 0.0f;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        const int chunk = (p0 / 4 + q) ^ (row & 15);
+        const float4 e = sm.ebar[row][chunk];
+        acc = fmaf(u[4 * q], e.x, acc);
+        acc = fmaf(u[4 * q + 1], e.y, acc);
+        acc = fmaf(u[4 * q + 2], e.z, acc);
+        acc = fmaf(u[4 * q + 3], e.w, acc);
+    }
+    return acc;
 }
 
 template <typename Tout>
@@ -176,15 +247,15 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
 
     // work item: heaviest token tiles first
     const int tiles = L / kRows;
-    const int hgroups = H / kHeadsPerCta;
+    const int hpairs = H / kHeadsPerCta;
     const int item = blockIdx.x;
-    const int tt = tiles - 1 - item / (Bsz * hgroups);
-    const int rem = item % (Bsz * hgroups);
-    const int b = rem / hgroups;
-    const int h0 = (rem % hgroups) * kHeadsPerCta;
+    const int tt = tiles - 1 - item / (Bsz * hpairs);
+    const int rem = item % (Bsz * hpairs);
+    const int b = rem / hpairs;
+    const int hp = rem % hpairs;
+    const int h0 = hp * kHeadsPerCta;
     const int t0 = tt * kRows;
-    const int njobs_per_head = (t0 + kRows - 1) / S;  // memories the last token sees
-    const int njobs = njobs_per_head * kHeadsPerCta;
+    const int nj = (t0 + kRows - 1) / S;  // memories the last token of the tile sees
     volatile int* abort = &sm.abort;
 
     if (threadIdx.x == 0) {
@@ -192,11 +263,12 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
             tc::mbar_init(&sm.full[s], 1);
             tc::mbar_init(&sm.empty[s], 1);
         }
-        for (int a = 0; a < kAcc; ++a) {
-            tc::mbar_init(&sm.acc_full[a], 1);
-            tc::mbar_init(&sm.acc_empty[a], 128);
-        }
-        tc::mbar_init(&sm.a_ready, 128);
+        tc::mbar_init(&sm.u_full, 1);
+        tc::mbar_init(&sm.u_free, 256);
+        tc::mbar_init(&sm.v_full, 1);
+        tc::mbar_init(&sm.v_free, 256);
+        tc::mbar_init(&sm.a_ready, 256);  // Q from warpgroup 0, C from warpgroup 1
+        tc::mbar_init(&sm.drain, 1);
         sm.abort = 0;
         tc::fence_barrier_init();
     }
@@ -209,33 +281,34 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
     tc::tc_fence_after();
     const uint32_t tmem = sm.tmem_base;
 
-    if (warp == 0) {
+    if (warp < 4) {
+      asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegsLow));
+      if (warp == 0) {
         // ------------------------------------------------------- producer
+        // parts in order U(0), V(0), U(1), V(1), ...; part k uses stage k % 3
         if (lane == 0) {
-            int issued_phase[kStages];
-            bool issued[kStages];
-            for (int s = 0; s < kStages; ++s) issued[s] = false;
-            for (int k = 0; k < njobs; ++k) {
+            const int nparts = 2 * nj;
+            int k = 0;
+            for (; k < nparts; ++k) {
                 const int st = k % kStages;
                 const uint32_t round = (uint32_t)(k / kStages);
                 if (!tc::mbar_wait(&sm.empty[st], (round & 1u) ^ 1u, wait_limit_ns, abort)) {
                     fail(abort, 1);
                     break;
                 }
-                const int h = h0 + k / njobs_per_head;
-                const int j = k % njobs_per_head;
-                const uint8_t* src = ops + (((i64)b * Mc + j) * H + h) * kJob;
-                tc::mbar_arrive_expect_tx(&sm.full[st], kJob);
-                tc::bulk_g2s(sm.stage[st], src, kJob, &sm.full[st]);
-                issued[st] = true;
-                issued_phase[st] = (int)(round & 1u);
+                const int j = k >> 1;
+                const bool is_v = (k & 1) != 0;
+                const uint8_t* src = ops + (((i64)b * Mc + j) * hpairs + hp) * (i64)kPair +
+                                     (is_v ? kPartU : 0);
+                const uint32_t bytes = is_v ? (uint32_t)kPartV : (uint32_t)kPartU;
+                tc::mbar_arrive_expect_tx(&sm.full[st], bytes);
+                tc::bulk_g2s(sm.stage[st], src, bytes, &sm.full[st]);
             }
             // never leave a copy in flight behind: wait for the last one of each stage
-            for (int s = 0; s < kStages; ++s) {
-                if (issued[s] && !tc::mbar_wait(&sm.full[s], (uint32_t)issued_phase[s],
-                                                kDrainLimitNs, nullptr)) {
+            for (int kk = k - 1; kk >= 0 && kk >= k - kStages; --kk) {
+                if (!tc::mbar_wait(&sm.full[kk % kStages], (uint32_t)((kk / kStages) & 1),
+                                   kDrainLimitNs, nullptr))
                     atomicCAS(&g_tc_status, 0, 5);
-                }
             }
         }
     } else if (warp == 1) {
@@ -244,168 +317,209 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
             bool ok = tc::mbar_wait(&sm.a_ready, 0, wait_limit_ns, abort);
             if (!ok) fail(abort, 2);
             tc::tc_fence_after();
-            int k = 0;
-            for (; ok && k < njobs; ++k) {
+            bool issued = false;
+            for (int k = 0; ok && k < 2 * nj; ++k) {
+                const int j = k >> 1;
+                const bool is_v = (k & 1) != 0;
                 const int st = k % kStages;
-                const uint32_t round = (uint32_t)(k / kStages);
-                const int as = k % kAcc;
-                const uint32_t around = (uint32_t)(k / kAcc);
-                if (!tc::mbar_wait(&sm.acc_empty[as], (around & 1u) ^ 1u, wait_limit_ns, abort) ||
-                    !tc::mbar_wait(&sm.full[st], round & 1u, wait_limit_ns, abort)) {
+                const uint32_t ph = (uint32_t)(j & 1);
+                // the buffer is free once the epilogue has read the previous job's contents
+                if (!tc::mbar_wait(is_v ? &sm.v_free : &sm.u_free, ph ^ 1u, wait_limit_ns, abort) ||
+                    !tc::mbar_wait(&sm.full[st], (uint32_t)((k / kStages) & 1), wait_limit_ns, abort)) {
                     fail(abort, 3);
+                    ok = false;
                     break;
                 }
                 tc::tc_fence_after();
-                const uint32_t sbase = tc::smem_u32(sm.stage[st]);
-                const uint32_t d_u = tmem + kColAcc + 128u * (uint32_t)as;
-                const uint32_t d_v = d_u + 64u;
+                const uint32_t sb = tc::smem_u32(sm.stage[st]);
 #pragma unroll
-                for (int s = 0; s < kN / 16; ++s) {
-                    const uint64_t bd = tc::smem_desc_sw128(sbase + 2048u * s, 1024u, 1024u);
-                    tc::mma_f16_ts(d_u, tmem + kColQ + 8u * s, bd, kIdescBf16, s > 0 ? 1u : 0u);
+                for (int ks = 0; ks < kN / 16; ++ks) {
+                    const uint64_t bd = tc::smem_desc_sw128(sb + 2048u * ks, (uint32_t)kTile, 1024u);
+                    if (is_v)
+                        tc::mma_f16_ts(tmem + kColV, tmem + kColC + 8u * ks, bd, kIdescV, ks > 0 ? 1u : 0u);
+                    else
+                        tc::mma_f16_ts(tmem + kColU, tmem + kColQ + 8u * ks, bd, kIdescU, ks > 0 ? 1u : 0u);
                 }
-#pragma unroll
-                for (int s = 0; s < kN / 16; ++s) {
-                    const uint64_t bd = tc::smem_desc_sw128(sbase + kTile + 2048u * s, 1024u, 1024u);
-                    tc::mma_f16_ts(d_u, tmem + kColQ + 8u * s, bd, kIdescBf16, 1u);
-                }
-#pragma unroll
-                for (int s = 0; s < kN / 16; ++s) {
-                    const uint64_t bd =
-                        tc::smem_desc_sw128(sbase + 2 * kTile + 2048u * s, 1024u, 1024u);
-                    tc::mma_f16_ts(d_v, tmem + kColC + 8u * s, bd, kIdescF16, s > 0 ? 1u : 0u);
-                }
+                issued = true;
                 tc::mma_commit(&sm.empty[st]);
-                tc::mma_commit(&sm.acc_full[as]);
+                tc::mma_commit(is_v ? &sm.v_full : &sm.u_full);
             }
-            if (k > 0) {
-                // drain: the last commit arrives once every issued MMA is done
-                const int last = k - 1;
-                if (!tc::mbar_wait(&sm.acc_full[last % kAcc], (uint32_t)((last / kAcc) & 1),
-                                   kDrainLimitNs, nullptr))
+            if (!ok && issued) {
+                // drain: this commit arrives once every MMA issued so far is done
+                tc::mma_commit(&sm.drain);
+                if (!tc::mbar_wait(&sm.drain, 0, kDrainLimitNs, nullptr))
                     atomicCAS(&g_tc_status, 0, 6);
             }
         }
+      }
     } else {
+        asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(kRegsHigh));
         // ------------------------------------------------------- epilogue
+        const int wg = (warp - 4) >> 2;  // head h0 + wg
+        const int h = h0 + wg;
         const int row = 32 * (warp & 3) + lane;
         const uint32_t lane_addr = (uint32_t)(32 * (warp & 3)) << 16;
         const int t = t0 + row;
         const i64 tok = (i64)b * L + t;
         const int g = h0 / (H / G);
         const int nh = t / S;
-        // stage A operands: Q (bf16 pairs) and C (fp16 pairs); rms of Q
         float ssq = 0.0f;
-        {
+        if (wg == 0) {
+            // A operand Q (bf16 pairs) into TMEM
             const uint4* qrow = reinterpret_cast<const uint4*>(Q + (tok * G + g) * kN);
-            const uint4* crow = reinterpret_cast<const uint4*>(Cm + (tok * G + g) * kN);
+            uint4 qv[16];
+#pragma unroll
+            for (int u = 0; u < 16; ++u) qv[u] = qrow[u];
 #pragma unroll
             for (int c = 0; c < 4; ++c) {
-                uint32_t qa[16], ca[16];
+                uint32_t qa[16];
 #pragma unroll
                 for (int u = 0; u < 4; ++u) {
-                    const uint4 qv = qrow[c * 4 + u];
-                    const uint4 cv = crow[c * 4 + u];
-                    const uint32_t qw[4] = {qv.x, qv.y, qv.z, qv.w};
-                    const uint32_t cw[4] = {cv.x, cv.y, cv.z, cv.w};
+                    const uint32_t qw[4] = {qv[c * 4 + u].x, qv[c * 4 + u].y, qv[c * 4 + u].z, qv[c * 4 + u].w};
 #pragma unroll
                     for (int e = 0; e < 4; ++e) {
                         qa[u * 4 + e] = qw[e];
                         const float2 qf = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&qw[e]));
                         ssq = fmaf(qf.x, qf.x, fmaf(qf.y, qf.y, ssq));
+                    }
+                }
+                tc::tmem_st16(tmem + lane_addr + kColQ + 16u * c, qa);
+            }
+        } else {
+            // A operand C (fp16 pairs) into TMEM, and the Q row's sum of squares
+            const uint4* crow = reinterpret_cast<const uint4*>(Cm + (tok * G + g) * kN);
+            const uint4* qrow = reinterpret_cast<const uint4*>(Q + (tok * G + g) * kN);
+            uint4 cv[16];
+#pragma unroll
+            for (int u = 0; u < 16; ++u) cv[u] = crow[u];
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                uint32_t ca[16];
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    const uint32_t cw[4] = {cv[c * 4 + u].x, cv[c * 4 + u].y, cv[c * 4 + u].z, cv[c * 4 + u].w};
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
                         const float2 cf = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&cw[e]));
                         const __half2 ch = __floats2half2_rn(cf.x, cf.y);
                         ca[u * 4 + e] = *reinterpret_cast<const uint32_t*>(&ch);
                     }
                 }
-                tc::tmem_st16(tmem + lane_addr + kColQ + 16u * c, qa);
                 tc::tmem_st16(tmem + lane_addr + kColC + 16u * c, ca);
             }
-            tc::tmem_wait_st();
-        }
-        tc::tc_fence_before();
-        tc::mbar_arrive(&sm.a_ready);
-        // Ebar (fp32, registers) and the logit scale 1 / (rms(Q) sqrt(N))
-        float ebar[kP];
-        {
+#pragma unroll
+            for (int u = 0; u < 16; ++u) cv[u] = qrow[u];
+#pragma unroll
+            for (int u = 0; u < 16; ++u) {
+                const uint32_t qw[4] = {cv[u].x, cv[u].y, cv[u].z, cv[u].w};
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const float2 qf = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&qw[e]));
+                    ssq = fmaf(qf.x, qf.x, fmaf(qf.y, qf.y, ssq));
+                }
+            }
+            // Ebar row (fp32) into shared memory, 16-byte chunks swizzled by row
             const uint4* erow = reinterpret_cast<const uint4*>(E + (tok * G + g) * kP);
+            uint4 ev[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) ev[u] = erow[u];
+            float e[kP];
             float sse = 0.0f;
 #pragma unroll
             for (int u = 0; u < 8; ++u) {
-                const uint4 ev = erow[u];
-                const uint32_t ew[4] = {ev.x, ev.y, ev.z, ev.w};
+                const uint32_t ew[4] = {ev[u].x, ev[u].y, ev[u].z, ev[u].w};
 #pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&ew[e]));
-                    ebar[u * 8 + 2 * e] = f.x;
-                    ebar[u * 8 + 2 * e + 1] = f.y;
+                for (int q = 0; q < 4; ++q) {
+                    const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&ew[q]));
+                    e[u * 8 + 2 * q] = f.x;
+                    e[u * 8 + 2 * q + 1] = f.y;
                     sse = fmaf(f.x, f.x, fmaf(f.y, f.y, sse));
                 }
             }
             const float ie = rsqrtf(sse / (float)kP + eps);
 #pragma unroll
-            for (int p = 0; p < kP; ++p) ebar[p] *= ie;
+            for (int c = 0; c < kP / 4; ++c)
+                sm.ebar[row][c ^ (row & 15)] =
+                    make_float4(e[4 * c] * ie, e[4 * c + 1] * ie, e[4 * c + 2] * ie, e[4 * c + 3] * ie);
         }
+        asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+        tc::tc_fence_before();
+        tc::mbar_arrive(&sm.a_ready);
+        asm volatile("bar.sync 1, 256;" ::: "memory");  // Ebar rows visible to both warpgroups
         const float lscale = rsqrtf(ssq / (float)kN + eps) * rsqrtf((float)kN);
 
-        int k = 0;
+        float O[kP];
+#pragma unroll
+        for (int p = 0; p < kP; ++p) O[p] = 0.0f;
+        float m = -INFINITY, dsum = 0.0f;
         bool ok = true;
-        for (int hh = 0; hh < kHeadsPerCta; ++hh) {
-            const int h = h0 + hh;
-            float O[kP];
-#pragma unroll
-            for (int p = 0; p < kP; ++p) O[p] = 0.0f;
-            float m = -INFINITY, dsum = 0.0f;
-            for (int j = 0; j < njobs_per_head && ok; ++j, ++k) {
-                const int as = k % kAcc;
-                // warp-uniform outcome: tcgen05.ld below must be executed by every lane
-                const bool got = tc::mbar_wait(&sm.acc_full[as], (uint32_t)((k / kAcc) & 1),
-                                               wait_limit_ns, abort);
-                if (!__all_sync(0xffffffffu, got)) {
-                    fail(abort, 4);
-                    ok = false;
-                    break;
-                }
-                tc::tc_fence_after();
-                const uint32_t ua = tmem + lane_addr + kColAcc + 128u * (uint32_t)as;
-                float v[32];
-                float l = 0.0f;
-                tmem_ld32(ua, v);
-#pragma unroll
-                for (int i = 0; i < 32; ++i) l = fmaf(v[i], ebar[i], l);
-                tmem_ld32(ua + 32u, v);
-#pragma unroll
-                for (int i = 0; i < 32; ++i) l = fmaf(v[i], ebar[32 + i], l);
-                l *= lscale;
-                const bool use = j < nh;
-                const float mn = use ? fmaxf(m, l) : m;
-                const float sc = use ? expf(m - mn) : 1.0f;
-                const float pe = use ? expf(l - mn) : 0.0f;
-                const float w = pe * __ldg(scale + ((i64)b * Mc + j) * H + h);
-                dsum = fmaf(dsum, sc, pe);
-                m = mn;
-                tmem_ld32(ua + 64u, v);
-#pragma unroll
-                for (int i = 0; i < 32; ++i) O[i] = fmaf(O[i], sc, w * v[i]);
-                tmem_ld32(ua + 96u, v);
-#pragma unroll
-                for (int i = 0; i < 32; ++i) O[32 + i] = fmaf(O[32 + i], sc, w * v[i]);
-                tc::tc_fence_before();
-                tc::mbar_arrive(&sm.acc_empty[as]);
+        const uint32_t ua = tmem + lane_addr + kColU + (uint32_t)(128 * wg);  // hi | lo of head h
+        const uint32_t va = tmem + lane_addr + kColV + (uint32_t)(64 * wg);
+        for (int j = 0; j < nj; ++j) {
+            const uint32_t ph = (uint32_t)(j & 1);
+            if (!warp_wait(&sm.u_full, ph, wait_limit_ns, abort)) {
+                fail(abort, 4);
+                ok = false;
+                break;
             }
-            if (!ok) break;
-            // per-head epilogue: R = O / d, lse, gated merge
+            tc::tc_fence_after();
+            float l = 0.0f;
+#pragma unroll
+            for (int half = 0; half < 2; ++half) {  // columns 0..31 then 32..63, hi and lo
+                float v[64];
+                tmem_ld32x2(ua + 32u * half, ua + 64u + 32u * half, v);
+#pragma unroll
+                for (int q = 0; q < 8; ++q) {
+                    const float4 e = sm.ebar[row][(8 * half + q) ^ (row & 15)];
+                    l = fmaf(v[4 * q] + v[32 + 4 * q], e.x, l);
+                    l = fmaf(v[4 * q + 1] + v[33 + 4 * q], e.y, l);
+                    l = fmaf(v[4 * q + 2] + v[34 + 4 * q], e.z, l);
+                    l = fmaf(v[4 * q + 3] + v[35 + 4 * q], e.w, l);
+                }
+            }
+            tc::tc_fence_before();
+            tc::mbar_arrive(&sm.u_free);
+            l *= lscale;
+            const bool use = j < nh;
+            const float mn = use ? fmaxf(m, l) : m;
+            const float sc = use ? expf(m - mn) : 1.0f;
+            const float pe = use ? expf(l - mn) : 0.0f;
+            const float w = pe * __ldg(scale + ((i64)b * Mc + j) * H + h);
+            dsum = fmaf(dsum, sc, pe);
+            m = mn;
+            if (!warp_wait(&sm.v_full, ph, wait_limit_ns, abort)) {
+                fail(abort, 4);
+                ok = false;
+                break;
+            }
+            tc::tc_fence_after();
+            {
+                float v[64];
+                tmem_ld32x2(va, va + 32u, v);
+                tc::tc_fence_before();
+                tc::mbar_arrive(&sm.v_free);
+#pragma unroll
+                for (int p = 0; p < kP; ++p) O[p] = fmaf(O[p], sc, w * v[p]);
+            }
+        }
+        if (ok) {
+            // R = O / d, lse, gated merge (the row's loads issued first)
             const i64 rowo = tok * H + h;
             const bool has = nh > 0;
             const float inv_d = has ? 1.0f / dsum : 0.0f;
             const float gate = silu_f32(__bfloat162float(z[rowo]));
-            const Tout* ys = Yssd + rowo * kP;
-            Tout* yo = Y + rowo * kP;
+            float ys[kP];
+#pragma unroll
+            for (int c = 0; c < 4; ++c) load_row16(Yssd + rowo * kP + 16 * c, ys + 16 * c);
 #pragma unroll
             for (int p = 0; p < kP; ++p) {
-                const float r = has ? O[p] * inv_d : 0.0f;
-                yo[p] = cvt_from_f32<Tout>(ld_f32(ys + p) + gate * r);
-                if (R != nullptr) R[rowo * kP + p] = cvt_from_f32<Tout>(r);
+                O[p] = has ? O[p] * inv_d : 0.0f;
+                ys[p] = fmaf(gate, O[p], ys[p]);
+            }
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                store_row16(Y + rowo * kP + 16 * c, ys + 16 * c);
+                if (R != nullptr) store_row16(R + rowo * kP + 16 * c, O + 16 * c);
             }
             if (lse != nullptr) lse[rowo] = has ? m + logf(dsum) : -INFINITY;
         }
@@ -423,7 +537,7 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
 }  // namespace
 
 size_t sma_tc_workspace(int64_t B, int64_t Mc, int64_t H) {
-    const size_t ops = (size_t)(B * Mc * H) * kJob;
+    const size_t ops = (size_t)(B * Mc * (H / kHeadsPerCta)) * kPair;
     const size_t sc = (size_t)(B * Mc * H) * sizeof(float);
     return ops + ((sc + 255) & ~(size_t)255);
 }
@@ -438,7 +552,7 @@ cudaError_t launch_sma_forward_tc(const SmaArgs& a, void* ws, unsigned long long
                                   cudaStream_t stream) {
     const int Bsz = (int)a.B, L = (int)a.L, H = (int)a.H, Mc = (int)(a.L / a.S);
     uint8_t* ops = (uint8_t*)ws;
-    float* scale = (float*)(ops + (size_t)(a.B * Mc * H) * kJob);
+    float* scale = (float*)(ops + (size_t)(a.B * Mc * (H / kHeadsPerCta)) * kPair);
     if (Mc > 1) {
         sma_operands_kernel<Tmem><<<dim3(Mc - 1, H, Bsz), 256, 0, stream>>>(
             (const Tmem*)a.M, a.rM, ops, scale, Mc, H, a.eps);

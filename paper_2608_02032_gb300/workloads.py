@@ -67,6 +67,8 @@ WORKLOADS = {
                                notes="B4 H16 L2048 P64 N128 S256, bf16"),
     "prefill_l16k": Workload("prefill_l16k", 1, 32, 16384, 64, 128, 256, seed=1002,
                              notes="B1 H32 L16384 P64 N128 S256, bf16, 64 chunk memories"),
+    "prefill_l8k": Workload("prefill_l8k", 1, 32, 8192, 64, 128, 256, seed=1006,
+                            notes="B1 H32 L8192 P64 N128 S256, bf16 (profiling size)"),
     "decode_b64": Workload("decode_b64", 64, 32, 1, 64, 128, 256, seed=1003, mem=64, pos=16384,
                            notes="B64 H32 P64 N128 S256, 64 cached memories, pos 16384"),
     "train_b8_l4k_s128": Workload("train_b8_l4k_s128", 8, 24, 4096, 64, 128, 128, seed=1004,

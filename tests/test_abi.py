@@ -62,7 +62,12 @@ def test_workspace_sizes(L):
     cum = 1 * 2 * M * 128 * 4
     dh = 1 * M * 2 * 128 * 64 * 4
     assert B.dart_workspace_size(d, B.DART_OP_CHUNK_SCAN) == cum + dh
-    assert B.dart_workspace_size(d, B.DART_OP_SMA_FORWARD) == (1 * M * 2 * 128 * 4 + 255) // 256 * 256
+    # bf16 tensor-core path: 96 KiB of pre-swizzled operands per (memory, head pair) + per-memory scales
+    ops = 1 * M * 1 * 96 * 1024
+    assert B.dart_workspace_size(d, B.DART_OP_SMA_FORWARD) == ops + (1 * M * 2 * 4 + 255) // 256 * 256
+    # fp32 inputs take the CUDA-core path: one inverse RMS per memory row
+    d32 = _dims(dtype=B.DART_F32)
+    assert B.dart_workspace_size(d32, B.DART_OP_SMA_FORWARD) == (1 * M * 2 * 128 * 4 + 255) // 256 * 256
     assert B.dart_workspace_size(d, B.DART_OP_DECODE_STEP) == 0
     assert B.dart_workspace_size(_dims(headdim=48), B.DART_OP_CHUNK_SCAN) == 0
 
