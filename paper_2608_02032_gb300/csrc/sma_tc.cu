@@ -10,40 +10,42 @@
 //   l_{t,j} = (U_t . Ebar_t) / (rms(Q_t) sqrt(N))
 // U and V are GEMMs whose token operands Q, C stay fixed for the whole tile
 // (they sit in TMEM as the A operand) while the memories stream through as
-// the B operand.
+// the B operand. Heads of one group share Q, C and E, so one job is one
+// memory j for two heads of the same group: both heads' tiles side by side
+// make an N = 128 B operand.
 //
 // Precision. Rounding the memory operand to bf16 moves the logits enough to
 // break the 2e-2 parity bar, so W = r (.) M is split into bf16 hi + lo parts
 // (two MMA chains into one accumulator, ~2^-16 relative) and the value path
-// runs in fp16 on M / max|M_j| (scale re-applied in the epilogue). Q and C are
-// exact (bf16 inputs; C widened to fp16 exactly); Qbar's RMS scale and Ebar
-// stay fp32 in the epilogue.
+// runs in fp16 on M / max|M_j| (scale re-applied in the epilogue). Q is exact
+// (bf16); C is widened to fp16 after a per-row power-of-two scale that puts
+// its largest entry in [2^14, 2^15), which is exact and keeps any bf16 row
+// inside the fp16 range (the scale is undone on R). Qbar's RMS scale and
+// Ebar stay fp32 in the epilogue.
 //
-// Shape. A tcgen05.mma with M = 128, K = 16 costs about the same for any
-// N <= 128 and only reaches the tensor peak at N >= 192 (measured on GB300:
-// ~90-99 cycles at N <= 128, ~137 at N = 256 with A in TMEM). So one job is
-// one memory j for the CTA's two heads: U is one N = 256 chain over the tiles
-// [W_hi h0 | W_lo h0 | W_hi h1 | W_lo h1] (the epilogue adds hi + lo), V is
-// one N = 128 chain over [M16 h0 | M16 h1]. U and V have one TMEM buffer each
-// and alternate, so each buffer is read by the epilogue while the other one
-// is being computed.
+// Cost model (measured on GB300, A in TMEM): a tcgen05.mma with M = 128,
+// K = 16 takes ~64 cycles at N = 128 and ~128 at N = 256, i.e. the full
+// 8192 flop/cycle/SM from N = 128 up. One job is three N = 128 chains of
+// eight MMAs (hi, lo into U; value into V): ~1536 cycles, fed by three
+// 32 KiB operand parts.
 //
-// Kernel 1 (sma_operands_kernel) writes per (memory, pair of heads) a 64 KiB
-// U part and a 32 KiB V part, already in the 128-byte-swizzled shared-memory
-// layout, so each part is one bulk copy.
+// Kernel 1 (sma_operands_kernel) writes per (memory, pair of heads) the three
+// 32 KiB parts [W_hi h0 | W_hi h1], [W_lo h0 | W_lo h1], [M16 h0 | M16 h1],
+// already in the 128-byte-swizzled shared-memory layout, so each part is one
+// bulk copy.
 // Kernel 2 (sma_tc_kernel), one CTA per (batch, 128-token tile, 2 heads),
 // heaviest tiles first:
-//   warp 0      producer: bulk copies of the parts into a 3-stage ring
+//   warp 0      producer: bulk copies of the parts into a 6-stage ring
 //   warp 1      TMEM allocation; one thread issues the MMAs
 //   warps 2, 3  idle (they complete warpgroup 0 for the register split)
-//   warps 4..7  epilogue warpgroup 0: head 0 of the pair
-//   warps 8..11 epilogue warpgroup 1: head 1 of the pair
-// An epilogue thread owns one token row of its head: it reads U and V from
-// TMEM with wide loads (three waits per job), runs the online softmax, and
-// finally writes R = O / d, lse and Y = Y_ssd + SiLU(z) R. Warpgroup 0 also
-// stages Q and C into TMEM, warpgroup 1 writes Ebar to shared memory.
-// TMEM: [0,64) Q (bf16 pairs), [64,128) C (fp16 pairs), [128,384) U,
-// [384,512) V.
+//   warps 4..7  epilogue warpgroup 0: head 0 of the pair (stages Q)
+//   warps 8..11 epilogue warpgroup 1: head 1 of the pair (stages C)
+// An epilogue thread owns one token row of its head: it reads its 64 columns
+// of U and of V from TMEM, runs the online softmax (the running sum is only
+// rescaled when the maximum moves), and finally writes R = O / d, lse and
+// Y = Y_ssd + SiLU(z) R.
+// TMEM: [0,64) Q (bf16 pairs), [64,128) C (fp16 pairs), [128,256) and
+// [256,384) U (two buffers, jobs alternate), [384,512) V.
 #include <math.h>
 
 #include <cuda_bf16.h>
@@ -63,23 +65,23 @@ constexpr int kP = 64;
 constexpr int kN = 128;
 constexpr int kHeadsPerCta = 2;
 constexpr int kTile = kN * kP * 2;            // bytes of one 16-bit N x P operand tile
-constexpr int kPartU = 4 * kTile;             // W_hi h0 | W_lo h0 | W_hi h1 | W_lo h1
-constexpr int kPartV = 2 * kTile;             // M16 h0 | M16 h1
-constexpr int kPair = kPartU + kPartV;        // operand bytes per (memory, head pair)
-constexpr int kStages = 3;                    // ring of kPartU-sized stages
+constexpr int kPart = kHeadsPerCta * kTile;   // one N = 128 B operand: both heads' tiles
+constexpr int kPartsPerJob = 3;               // W_hi, W_lo, M16
+constexpr int kPair = kPartsPerJob * kPart;   // operand bytes per (memory, head pair)
+constexpr int kStages = 6;                    // ring of kPart-sized stages
 constexpr int kThreads = 384;
 // Register split: launched at 168 per thread (384 x 168 = 64512 of the 65536
-// of an SM); warpgroup 0 (producer, MMA, two idle warps) drops to 56 and the
-// epilogue warpgroups rise to 224: 128 x 56 + 256 x 224 = 64512, within the
-// launch pool, and per sub-partition (56 + 2 x 224) x 32 = 16128 <= 16384.
-constexpr int kRegsLow = 56, kRegsHigh = 224;
+// of an SM); warpgroup 0 (producer, MMA, two idle warps) drops to 80 and the
+// epilogue warpgroups rise to 208: 128 x 80 + 256 x 208 = 63488, within the
+// launch pool, and per sub-partition (80 + 2 x 208) x 32 = 15872 <= 16384.
+constexpr int kRegsLow = 80, kRegsHigh = 208;
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kColQ = 0, kColC = 64, kColU = 128, kColV = 384;
 // Bound on the final waits for this CTA's own copies and MMAs (never cut short).
 constexpr uint64_t kDrainLimitNs = 2000000000ull;
 
-constexpr uint32_t kIdescU = tc::idesc_f16(1, true, kRows, 4 * kP);  // bf16, N = 256
-constexpr uint32_t kIdescV = tc::idesc_f16(0, true, kRows, 2 * kP);  // fp16, N = 128
+constexpr uint32_t kIdescU = tc::idesc_f16(1, true, kRows, kHeadsPerCta * kP);  // bf16, N = 128
+constexpr uint32_t kIdescV = tc::idesc_f16(0, true, kRows, kHeadsPerCta * kP);  // fp16, N = 128
 
 // Byte offset of element (n, p) of a 128-row x 128-byte tile in the
 // 128-byte-swizzled layout: the 16-byte chunk index is XORed with n mod 8.
@@ -90,9 +92,8 @@ __device__ __forceinline__ uint32_t sw128(int n, int p) {
 
 // ------------------------------------------------------------ kernel 1
 // One block of 256 threads per (j, h, b) memory. Warp w owns rows n = w + 8k;
-// lane owns columns p = lane, lane + 32. Head h = 2 hp + x writes
-//   W_hi to  ops + ((b Mc + j) (H/2) + hp) kPair + 2x kTile,
-//   W_lo one tile further, M16 to  ... + kPartU + x kTile.
+// lane owns columns p = lane, lane + 32. Head h = 2 hp + x writes its tile x
+// of each of the three parts of ops + ((b Mc + j) (H/2) + hp) kPair.
 template <typename Tmem>
 __global__ void __launch_bounds__(256)
 sma_operands_kernel(const Tmem* __restrict__ M, const float* __restrict__ rM,
@@ -104,8 +105,9 @@ sma_operands_kernel(const Tmem* __restrict__ M, const float* __restrict__ rM,
     const Tmem* src = M + mem * (kN * kP);
     const i64 pair = ((i64)b * Mc + j) * (H / kHeadsPerCta) + h / kHeadsPerCta;
     const int x = h % kHeadsPerCta;
-    uint8_t* dst_u = ops + pair * kPair + 2 * x * kTile;
-    uint8_t* dst_v = ops + pair * kPair + kPartU + x * kTile;
+    uint8_t* dst_hi = ops + pair * kPair + x * kTile;
+    uint8_t* dst_lo = dst_hi + kPart;
+    uint8_t* dst_v = dst_hi + 2 * kPart;
     __shared__ float s_max[8];
 
     float v0[16], v1[16], rr[16];
@@ -142,8 +144,8 @@ sma_operands_kernel(const Tmem* __restrict__ M, const float* __restrict__ rM,
             const __nv_bfloat16 lo = __float2bfloat16_rn(wv - __bfloat162float(hi));
             const __half m16 = __float2half_rn(v * inv_s);
             const uint32_t o = sw128(n, p);
-            *reinterpret_cast<__nv_bfloat16*>(dst_u + o) = hi;
-            *reinterpret_cast<__nv_bfloat16*>(dst_u + kTile + o) = lo;
+            *reinterpret_cast<__nv_bfloat16*>(dst_hi + o) = hi;
+            *reinterpret_cast<__nv_bfloat16*>(dst_lo + o) = lo;
             *reinterpret_cast<__half*>(dst_v + o) = m16;
         }
     }
@@ -151,11 +153,12 @@ sma_operands_kernel(const Tmem* __restrict__ M, const float* __restrict__ rM,
 
 // ------------------------------------------------------------ kernel 2
 struct TcSmem {
-    uint8_t stage[kStages][kPartU];  // 1024-aligned by placement
-    float4 ebar[kRows][kP / 4];      // Ebar rows, 16-byte chunks swizzled by row
+    uint8_t stage[kStages][kPart];  // 1024-aligned by placement
+    float lq[kRows];                // per-row logit factor 1 / (rms(Q_t) sqrt(N))
+    float cdown[kRows];             // per-row power of two undoing C's scale
     uint64_t full[kStages];
     uint64_t empty[kStages];
-    uint64_t u_full, u_free, v_full, v_free;
+    uint64_t u_full[2], u_free[2], v_full, v_free;
     uint64_t a_ready, drain;
     uint32_t tmem_base;
     int abort;
@@ -166,22 +169,6 @@ __device__ __forceinline__ void fail(volatile int* abort, int code) {
     atomicCAS(&g_tc_status, 0, code);
 }
 
-// tcgen05.ld of 16 consecutive fp32 columns of this thread's lane, waited.
-__device__ __forceinline__ void tmem_ld16w(uint32_t taddr, float (&v)[16]) {
-    uint32_t r[16];
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
-        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];\n\t"
-        "tcgen05.wait::ld.sync.aligned;"
-        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
-          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
-          "=r"(r[14]), "=r"(r[15])
-        : "r"(taddr)
-        : "memory");
-#pragma unroll
-    for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
-}
-
 // Warp-uniform bounded wait (every lane waits; all lanes see the same outcome).
 __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, uint64_t limit_ns,
                                           volatile int* abort) {
@@ -189,47 +176,61 @@ __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, uint64
     return __all_sync(0xffffffffu, got);
 }
 
-// tcgen05.ld of 32 + 32 fp32 columns (two addresses) of this thread's lane, one wait.
-__device__ __forceinline__ void tmem_ld32x2(uint32_t ta, uint32_t tb, float (&v)[64]) {
-    uint32_t r[64];
+// tcgen05.ld of 32 consecutive fp32 columns of this thread's lane, waited; the
+// values come back as 16 packed pairs (column 2i in the low half).
+__device__ __forceinline__ void tmem_ld32p(uint32_t taddr, uint64_t (&v)[16]) {
+    uint32_t r[32];
     asm volatile(
         "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
         "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
-        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%64];\n\t"
-        "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
-        "{%32,%33,%34,%35,%36,%37,%38,%39,%40,%41,%42,%43,%44,%45,%46,%47,"
-        "%48,%49,%50,%51,%52,%53,%54,%55,%56,%57,%58,%59,%60,%61,%62,%63}, [%65];\n\t"
+        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];\n\t"
         "tcgen05.wait::ld.sync.aligned;"
         : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
           "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
           "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),
           "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),
-          "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31]),
-          "=r"(r[32]), "=r"(r[33]), "=r"(r[34]), "=r"(r[35]), "=r"(r[36]), "=r"(r[37]),
-          "=r"(r[38]), "=r"(r[39]), "=r"(r[40]), "=r"(r[41]), "=r"(r[42]), "=r"(r[43]),
-          "=r"(r[44]), "=r"(r[45]), "=r"(r[46]), "=r"(r[47]), "=r"(r[48]), "=r"(r[49]),
-          "=r"(r[50]), "=r"(r[51]), "=r"(r[52]), "=r"(r[53]), "=r"(r[54]), "=r"(r[55]),
-          "=r"(r[56]), "=r"(r[57]), "=r"(r[58]), "=r"(r[59]), "=r"(r[60]), "=r"(r[61]),
-          "=r"(r[62]), "=r"(r[63])
-        : "r"(ta), "r"(tb)
+          "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+        : "r"(taddr)
         : "memory");
 #pragma unroll
-    for (int i = 0; i < 64; ++i) v[i] = __uint_as_float(r[i]);
+    for (int i = 0; i < 16; ++i)
+        asm("mov.b64 %0, {%1, %2};" : "=l"(v[i]) : "r"(r[2 * i]), "r"(r[2 * i + 1]));
 }
 
-// Dot product of 16 columns of U with Ebar[p0 .. p0+15] of row `row`.
-__device__ __forceinline__ float dot16(const float (&u)[16], const TcSmem& sm, int row, int p0) {
-    float acc = 0.0f;
+// Packed fp32 pairs (x in the low half). The epilogue's multiply-adds run as
+// fma.rn.f32x2, two lanes of fp32 per instruction: same rounding as two
+// scalar fmaf, half the issue slots, which matters here because the MMA warp
+// shares each sub-partition's issue slots with two epilogue warps.
+__device__ __forceinline__ uint64_t f2_pack(float x, float y) {
+    uint64_t r;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(x), "f"(y));
+    return r;
+}
+__device__ __forceinline__ void f2_unpack(uint64_t v, float& x, float& y) {
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(x), "=f"(y) : "l"(v));
+}
+__device__ __forceinline__ uint64_t f2_fma(uint64_t a, uint64_t b, uint64_t c) {
+    uint64_t d;
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+    return d;
+}
+__device__ __forceinline__ uint64_t f2_mul(uint64_t a, uint64_t b) {
+    uint64_t d;
+    asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+    return d;
+}
+
+// The two bf16 values packed in a 32-bit word, as floats (low half first).
+__device__ __forceinline__ float bf_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf_hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
+
+// Issues the eight K = 16 MMAs of one N = 128 part: D (+)= A[tmem] * B[stage].
+// `first_acc` is 0 when the first MMA starts a fresh accumulator.
+template <uint32_t kIdesc, uint32_t first_acc>
+__device__ __forceinline__ void issue_part(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc) {
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
-        const int chunk = (p0 / 4 + q) ^ (row & 15);
-        const float4 e = sm.ebar[row][chunk];
-        acc = fmaf(u[4 * q], e.x, acc);
-        acc = fmaf(u[4 * q + 1], e.y, acc);
-        acc = fmaf(u[4 * q + 2], e.z, acc);
-        acc = fmaf(u[4 * q + 3], e.w, acc);
-    }
-    return acc;
+    for (uint32_t ks = 0; ks < kN / 16; ++ks)  // +2048 bytes (+128 in the address field) per K step
+        tc::mma_f16_ts(d_tmem, a_tmem + 8u * ks, b_desc + 128u * ks, kIdesc, ks > 0 ? 1u : first_acc);
 }
 
 template <typename Tout>
@@ -255,7 +256,9 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
     const int hp = rem % hpairs;
     const int h0 = hp * kHeadsPerCta;
     const int t0 = tt * kRows;
-    const int nj = (t0 + kRows - 1) / S;  // memories the last token of the tile sees
+    // S is a multiple of the tile height, so every token of the tile lies in
+    // chunk t0 / S and sees exactly the memories j < t0 / S.
+    const int nj = t0 / S;
     volatile int* abort = &sm.abort;
 
     if (threadIdx.x == 0) {
@@ -263,8 +266,10 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
             tc::mbar_init(&sm.full[s], 1);
             tc::mbar_init(&sm.empty[s], 1);
         }
-        tc::mbar_init(&sm.u_full, 1);
-        tc::mbar_init(&sm.u_free, 256);
+        for (int u = 0; u < 2; ++u) {
+            tc::mbar_init(&sm.u_full[u], 1);
+            tc::mbar_init(&sm.u_free[u], 256);
+        }
         tc::mbar_init(&sm.v_full, 1);
         tc::mbar_init(&sm.v_free, 256);
         tc::mbar_init(&sm.a_ready, 256);  // Q from warpgroup 0, C from warpgroup 1
@@ -285,9 +290,11 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
       asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegsLow));
       if (warp == 0) {
         // ------------------------------------------------------- producer
-        // parts in order U(0), V(0), U(1), V(1), ...; part k uses stage k % 3
+        // parts in order hi(0), lo(0), v(0), hi(1), ...; part k uses stage k % kStages
         if (lane == 0) {
-            const int nparts = 2 * nj;
+            const int nparts = kPartsPerJob * nj;
+            const uint8_t* src = ops + ((i64)b * Mc * hpairs + hp) * (i64)kPair;
+            const i64 job_stride = (i64)hpairs * kPair;
             int k = 0;
             for (; k < nparts; ++k) {
                 const int st = k % kStages;
@@ -296,13 +303,10 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
                     fail(abort, 1);
                     break;
                 }
-                const int j = k >> 1;
-                const bool is_v = (k & 1) != 0;
-                const uint8_t* src = ops + (((i64)b * Mc + j) * hpairs + hp) * (i64)kPair +
-                                     (is_v ? kPartU : 0);
-                const uint32_t bytes = is_v ? (uint32_t)kPartV : (uint32_t)kPartU;
-                tc::mbar_arrive_expect_tx(&sm.full[st], bytes);
-                tc::bulk_g2s(sm.stage[st], src, bytes, &sm.full[st]);
+                const int j = k / kPartsPerJob, part = k - j * kPartsPerJob;
+                tc::mbar_arrive_expect_tx(&sm.full[st], (uint32_t)kPart);
+                tc::bulk_g2s(sm.stage[st], src + j * job_stride + part * kPart, (uint32_t)kPart,
+                             &sm.full[st]);
             }
             // never leave a copy in flight behind: wait for the last one of each stage
             for (int kk = k - 1; kk >= 0 && kk >= k - kStages; --kk) {
@@ -318,31 +322,39 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
             if (!ok) fail(abort, 2);
             tc::tc_fence_after();
             bool issued = false;
-            for (int k = 0; ok && k < 2 * nj; ++k) {
-                const int j = k >> 1;
-                const bool is_v = (k & 1) != 0;
-                const int st = k % kStages;
-                const uint32_t ph = (uint32_t)(j & 1);
-                // the buffer is free once the epilogue has read the previous job's contents
-                if (!tc::mbar_wait(is_v ? &sm.v_free : &sm.u_free, ph ^ 1u, wait_limit_ns, abort) ||
-                    !tc::mbar_wait(&sm.full[st], (uint32_t)((k / kStages) & 1), wait_limit_ns, abort)) {
+            // descriptor of stage 0; stage st is kPart * st bytes further (>> 4 in the address field)
+            const uint64_t desc0 = tc::smem_desc_sw128(tc::smem_u32(sm.stage[0]), (uint32_t)kTile, 1024u);
+            int st = 0;
+            uint32_t round = 0;
+            for (int j = 0; ok && j < nj; ++j) {
+                const int ub = j & 1;
+                const uint32_t dU = tmem + kColU + 128u * (uint32_t)ub;
+                // U buffer ub is free once the epilogue has read job j - 2's contents
+                ok = tc::mbar_wait(&sm.u_free[ub], (uint32_t)((j >> 1) & 1) ^ 1u, wait_limit_ns, abort);
+#pragma unroll
+                for (int part = 0; part < kPartsPerJob && ok; ++part) {
+                    if (part == 2)
+                        ok = tc::mbar_wait(&sm.v_free, (uint32_t)(j & 1) ^ 1u, wait_limit_ns, abort);
+                    ok = ok && tc::mbar_wait(&sm.full[st], round & 1u, wait_limit_ns, abort);
+                    if (!ok) break;
+                    tc::tc_fence_after();
+                    const uint64_t bd = desc0 + (uint64_t)((st * kPart) >> 4);
+                    if (part == 0) issue_part<kIdescU, 0u>(dU, tmem + kColQ, bd);
+                    if (part == 1) issue_part<kIdescU, 1u>(dU, tmem + kColQ, bd);
+                    if (part == 2) issue_part<kIdescV, 0u>(tmem + kColV, tmem + kColC, bd);
+                    issued = true;
+                    tc::mma_commit(&sm.empty[st]);
+                    if (part == 1) tc::mma_commit(&sm.u_full[ub]);
+                    if (part == 2) tc::mma_commit(&sm.v_full);
+                    if (++st == kStages) {
+                        st = 0;
+                        ++round;
+                    }
+                }
+                if (!ok) {
                     fail(abort, 3);
-                    ok = false;
                     break;
                 }
-                tc::tc_fence_after();
-                const uint32_t sb = tc::smem_u32(sm.stage[st]);
-#pragma unroll
-                for (int ks = 0; ks < kN / 16; ++ks) {
-                    const uint64_t bd = tc::smem_desc_sw128(sb + 2048u * ks, (uint32_t)kTile, 1024u);
-                    if (is_v)
-                        tc::mma_f16_ts(tmem + kColV, tmem + kColC + 8u * ks, bd, kIdescV, ks > 0 ? 1u : 0u);
-                    else
-                        tc::mma_f16_ts(tmem + kColU, tmem + kColQ + 8u * ks, bd, kIdescU, ks > 0 ? 1u : 0u);
-                }
-                issued = true;
-                tc::mma_commit(&sm.empty[st]);
-                tc::mma_commit(is_v ? &sm.v_full : &sm.u_full);
             }
             if (!ok && issued) {
                 // drain: this commit arrives once every MMA issued so far is done
@@ -362,164 +374,170 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
         const int t = t0 + row;
         const i64 tok = (i64)b * L + t;
         const int g = h0 / (H / G);
-        const int nh = t / S;
-        float ssq = 0.0f;
-        if (wg == 0) {
-            // A operand Q (bf16 pairs) into TMEM
-            const uint4* qrow = reinterpret_cast<const uint4*>(Q + (tok * G + g) * kN);
-            uint4 qv[16];
+
+        // One round of loads per warpgroup: the E row (both) and Q (wg 0) or C (wg 1).
+        const uint4* erow = reinterpret_cast<const uint4*>(E + (tok * G + g) * kP);
+        const uint4* arow = reinterpret_cast<const uint4*>((wg == 0 ? Q : Cm) + (tok * G + g) * kN);
+        uint4 av[16];
+        uint32_t e2[kP / 2];  // the E row as bf16 pairs; Ebar = E * ie
 #pragma unroll
-            for (int u = 0; u < 16; ++u) qv[u] = qrow[u];
+        for (int u = 0; u < 16; ++u) av[u] = arow[u];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+            const uint4 w = erow[u];
+            e2[4 * u] = w.x; e2[4 * u + 1] = w.y; e2[4 * u + 2] = w.z; e2[4 * u + 3] = w.w;
+        }
+        float sse = 0.0f;
+#pragma unroll
+        for (int i = 0; i < kP / 2; ++i) {
+            const float a = bf_lo(e2[i]), c = bf_hi(e2[i]);
+            sse = fmaf(a, a, fmaf(c, c, sse));
+        }
+        const float ie = rsqrtf(sse / (float)kP + eps);
+        uint64_t eb[kP / 2];  // Ebar row as fp32 pairs
+#pragma unroll
+        for (int i = 0; i < kP / 2; ++i) eb[i] = f2_pack(bf_lo(e2[i]) * ie, bf_hi(e2[i]) * ie);
+        if (wg == 0) {
+            // A operand Q (bf16 pairs, exact) into TMEM; 1 / (rms(Q_t) sqrt(N)) to shared memory
+            float ssq = 0.0f;
 #pragma unroll
             for (int c = 0; c < 4; ++c) {
                 uint32_t qa[16];
 #pragma unroll
                 for (int u = 0; u < 4; ++u) {
-                    const uint32_t qw[4] = {qv[c * 4 + u].x, qv[c * 4 + u].y, qv[c * 4 + u].z, qv[c * 4 + u].w};
+                    const uint32_t qw[4] = {av[c * 4 + u].x, av[c * 4 + u].y, av[c * 4 + u].z, av[c * 4 + u].w};
 #pragma unroll
                     for (int e = 0; e < 4; ++e) {
                         qa[u * 4 + e] = qw[e];
-                        const float2 qf = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&qw[e]));
-                        ssq = fmaf(qf.x, qf.x, fmaf(qf.y, qf.y, ssq));
+                        const float a = bf_lo(qw[e]), d = bf_hi(qw[e]);
+                        ssq = fmaf(a, a, fmaf(d, d, ssq));
                     }
                 }
                 tc::tmem_st16(tmem + lane_addr + kColQ + 16u * c, qa);
             }
+            sm.lq[row] = rsqrtf(ssq / (float)kN + eps) * rsqrtf((float)kN);
         } else {
-            // A operand C (fp16 pairs) into TMEM, and the Q row's sum of squares
-            const uint4* crow = reinterpret_cast<const uint4*>(Cm + (tok * G + g) * kN);
-            const uint4* qrow = reinterpret_cast<const uint4*>(Q + (tok * G + g) * kN);
-            uint4 cv[16];
+            // A operand C into TMEM as fp16 after an exact power-of-two row scale
+            float cmax = 0.0f;
 #pragma unroll
-            for (int u = 0; u < 16; ++u) cv[u] = crow[u];
+            for (int u = 0; u < 16; ++u) {
+                const uint32_t cw[4] = {av[u].x, av[u].y, av[u].z, av[u].w};
+#pragma unroll
+                for (int e = 0; e < 4; ++e) cmax = fmaxf(cmax, fmaxf(fabsf(bf_lo(cw[e])), fabsf(bf_hi(cw[e]))));
+            }
+            // cmax = 1.f * 2^(ebits - 127): scale by 2^k with k = 141 - ebits puts it in [2^14, 2^15)
+            const int ebits = (__float_as_int(cmax) >> 23) & 0xff;
+            const int k = cmax > 0.0f ? min(max(141 - ebits, -60), 60) : 0;
+            const float up = __int_as_float((127 + k) << 23);
+            sm.cdown[row] = __int_as_float((127 - k) << 23);
 #pragma unroll
             for (int c = 0; c < 4; ++c) {
                 uint32_t ca[16];
 #pragma unroll
                 for (int u = 0; u < 4; ++u) {
-                    const uint32_t cw[4] = {cv[c * 4 + u].x, cv[c * 4 + u].y, cv[c * 4 + u].z, cv[c * 4 + u].w};
+                    const uint32_t cw[4] = {av[c * 4 + u].x, av[c * 4 + u].y, av[c * 4 + u].z, av[c * 4 + u].w};
 #pragma unroll
                     for (int e = 0; e < 4; ++e) {
-                        const float2 cf = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&cw[e]));
-                        const __half2 ch = __floats2half2_rn(cf.x, cf.y);
+                        const __half2 ch = __floats2half2_rn(bf_lo(cw[e]) * up, bf_hi(cw[e]) * up);
                         ca[u * 4 + e] = *reinterpret_cast<const uint32_t*>(&ch);
                     }
                 }
                 tc::tmem_st16(tmem + lane_addr + kColC + 16u * c, ca);
             }
-#pragma unroll
-            for (int u = 0; u < 16; ++u) cv[u] = qrow[u];
-#pragma unroll
-            for (int u = 0; u < 16; ++u) {
-                const uint32_t qw[4] = {cv[u].x, cv[u].y, cv[u].z, cv[u].w};
-#pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    const float2 qf = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&qw[e]));
-                    ssq = fmaf(qf.x, qf.x, fmaf(qf.y, qf.y, ssq));
-                }
-            }
-            // Ebar row (fp32) into shared memory, 16-byte chunks swizzled by row
-            const uint4* erow = reinterpret_cast<const uint4*>(E + (tok * G + g) * kP);
-            uint4 ev[8];
-#pragma unroll
-            for (int u = 0; u < 8; ++u) ev[u] = erow[u];
-            float e[kP];
-            float sse = 0.0f;
-#pragma unroll
-            for (int u = 0; u < 8; ++u) {
-                const uint32_t ew[4] = {ev[u].x, ev[u].y, ev[u].z, ev[u].w};
-#pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&ew[q]));
-                    e[u * 8 + 2 * q] = f.x;
-                    e[u * 8 + 2 * q + 1] = f.y;
-                    sse = fmaf(f.x, f.x, fmaf(f.y, f.y, sse));
-                }
-            }
-            const float ie = rsqrtf(sse / (float)kP + eps);
-#pragma unroll
-            for (int c = 0; c < kP / 4; ++c)
-                sm.ebar[row][c ^ (row & 15)] =
-                    make_float4(e[4 * c] * ie, e[4 * c + 1] * ie, e[4 * c + 2] * ie, e[4 * c + 3] * ie);
         }
         asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
         tc::tc_fence_before();
         tc::mbar_arrive(&sm.a_ready);
-        asm volatile("bar.sync 1, 256;" ::: "memory");  // Ebar rows visible to both warpgroups
-        const float lscale = rsqrtf(ssq / (float)kN + eps) * rsqrtf((float)kN);
+        asm volatile("bar.sync 1, 256;" ::: "memory");  // lq and cdown visible to both warpgroups
+        const float lfac = sm.lq[row];
+        const float cdown = sm.cdown[row];
 
-        float O[kP];
+        uint64_t O[kP / 2];  // running sum of w_j V_j as fp32 pairs
 #pragma unroll
-        for (int p = 0; p < kP; ++p) O[p] = 0.0f;
+        for (int i = 0; i < kP / 2; ++i) O[i] = 0ull;
         float m = -INFINITY, dsum = 0.0f;
         bool ok = true;
-        const uint32_t ua = tmem + lane_addr + kColU + (uint32_t)(128 * wg);  // hi | lo of head h
-        const uint32_t va = tmem + lane_addr + kColV + (uint32_t)(64 * wg);
+        const float* scl = scale + (i64)b * Mc * H + h;  // scale of memory j at scl[j H]
+        float s_next = nj > 0 ? __ldg(scl) : 0.0f;
+        const uint32_t ua = tmem + lane_addr + kColU + (uint32_t)(kP * wg);
+        const uint32_t va = tmem + lane_addr + kColV + (uint32_t)(kP * wg);
         for (int j = 0; j < nj; ++j) {
-            const uint32_t ph = (uint32_t)(j & 1);
-            if (!warp_wait(&sm.u_full, ph, wait_limit_ns, abort)) {
+            const int ub = j & 1;
+            const float s_j = s_next;
+            if (j + 1 < nj) s_next = __ldg(scl + (i64)(j + 1) * H);  // one job ahead
+            if (!warp_wait(&sm.u_full[ub], (uint32_t)((j >> 1) & 1), wait_limit_ns, abort)) {
                 fail(abort, 4);
                 ok = false;
                 break;
             }
             tc::tc_fence_after();
-            float l = 0.0f;
+            float l;
+            {
+                uint64_t acc = 0ull, v[16];
+                tmem_ld32p(ua + 128u * ub, v);
 #pragma unroll
-            for (int half = 0; half < 2; ++half) {  // columns 0..31 then 32..63, hi and lo
-                float v[64];
-                tmem_ld32x2(ua + 32u * half, ua + 64u + 32u * half, v);
+                for (int i = 0; i < 16; ++i) acc = f2_fma(v[i], eb[i], acc);
+                tmem_ld32p(ua + 128u * ub + 32u, v);
+                tc::tc_fence_before();
+                tc::mbar_arrive(&sm.u_free[ub]);
 #pragma unroll
-                for (int q = 0; q < 8; ++q) {
-                    const float4 e = sm.ebar[row][(8 * half + q) ^ (row & 15)];
-                    l = fmaf(v[4 * q] + v[32 + 4 * q], e.x, l);
-                    l = fmaf(v[4 * q + 1] + v[33 + 4 * q], e.y, l);
-                    l = fmaf(v[4 * q + 2] + v[34 + 4 * q], e.z, l);
-                    l = fmaf(v[4 * q + 3] + v[35 + 4 * q], e.w, l);
-                }
+                for (int i = 0; i < 16; ++i) acc = f2_fma(v[i], eb[16 + i], acc);
+                float lx, ly;
+                f2_unpack(acc, lx, ly);
+                l = (lx + ly) * lfac;
             }
-            tc::tc_fence_before();
-            tc::mbar_arrive(&sm.u_free);
-            l *= lscale;
-            const bool use = j < nh;
-            const float mn = use ? fmaxf(m, l) : m;
-            const float sc = use ? expf(m - mn) : 1.0f;
-            const float pe = use ? expf(l - mn) : 0.0f;
-            const float w = pe * __ldg(scale + ((i64)b * Mc + j) * H + h);
-            dsum = fmaf(dsum, sc, pe);
-            m = mn;
-            if (!warp_wait(&sm.v_full, ph, wait_limit_ns, abort)) {
+            // online softmax; the running sums are rescaled only when the maximum moves
+            if (l > m) {
+                const float sc = expf(m - l);
+                const uint64_t sc2 = f2_pack(sc, sc);
+#pragma unroll
+                for (int i = 0; i < kP / 2; ++i) O[i] = f2_mul(O[i], sc2);
+                dsum *= sc;
+                m = l;
+            }
+            const float pe = expf(l - m);
+            dsum += pe;
+            const float w = pe * s_j;
+            const uint64_t w2 = f2_pack(w, w);
+            if (!warp_wait(&sm.v_full, (uint32_t)(j & 1), wait_limit_ns, abort)) {
                 fail(abort, 4);
                 ok = false;
                 break;
             }
             tc::tc_fence_after();
             {
-                float v[64];
-                tmem_ld32x2(va, va + 32u, v);
+                uint64_t v[16];
+                tmem_ld32p(va, v);
+#pragma unroll
+                for (int i = 0; i < 16; ++i) O[i] = f2_fma(w2, v[i], O[i]);
+                tmem_ld32p(va + 32u, v);
                 tc::tc_fence_before();
                 tc::mbar_arrive(&sm.v_free);
 #pragma unroll
-                for (int p = 0; p < kP; ++p) O[p] = fmaf(O[p], sc, w * v[p]);
+                for (int i = 0; i < 16; ++i) O[16 + i] = f2_fma(w2, v[i], O[16 + i]);
             }
         }
         if (ok) {
-            // R = O / d, lse, gated merge (the row's loads issued first)
+            // R = O / d (C's row scale undone), lse, gated merge
             const i64 rowo = tok * H + h;
-            const bool has = nh > 0;
-            const float inv_d = has ? 1.0f / dsum : 0.0f;
+            const bool has = nj > 0;
+            const float inv_d = has ? cdown / dsum : 0.0f;
             const float gate = silu_f32(__bfloat162float(z[rowo]));
-            float ys[kP];
+            float ys[kP], r[kP];
 #pragma unroll
             for (int c = 0; c < 4; ++c) load_row16(Yssd + rowo * kP + 16 * c, ys + 16 * c);
 #pragma unroll
-            for (int p = 0; p < kP; ++p) {
-                O[p] = has ? O[p] * inv_d : 0.0f;
-                ys[p] = fmaf(gate, O[p], ys[p]);
+            for (int i = 0; i < kP / 2; ++i) {
+                f2_unpack(O[i], r[2 * i], r[2 * i + 1]);
+                r[2 * i] *= inv_d;
+                r[2 * i + 1] *= inv_d;
+                ys[2 * i] = fmaf(gate, r[2 * i], ys[2 * i]);
+                ys[2 * i + 1] = fmaf(gate, r[2 * i + 1], ys[2 * i + 1]);
             }
 #pragma unroll
             for (int c = 0; c < 4; ++c) {
                 store_row16(Y + rowo * kP + 16 * c, ys + 16 * c);
-                if (R != nullptr) store_row16(R + rowo * kP + 16 * c, O + 16 * c);
+                if (R != nullptr) store_row16(R + rowo * kP + 16 * c, r + 16 * c);
             }
             if (lse != nullptr) lse[rowo] = has ? m + logf(dsum) : -INFINITY;
         }
