@@ -46,6 +46,15 @@
 // Y = Y_ssd + SiLU(z) R.
 // TMEM: [0,64) Q (bf16 pairs), [64,128) C (fp16 pairs), [128,256) and
 // [256,384) U (two buffers, jobs alternate), [384,512) V.
+//
+// Synchronisation, job j, b = j & 1 (the MMA thread pays for every barrier
+// operation with idle tensor cycles, so it does four waits and two commits
+// per job): the producer refills stages 3b .. 3b+2 once job j - 2 is done
+// with them (uready[b], vready[b]); the MMA thread waits for each part
+// (full), commits uready[b] after the two U chains and vready[b] after the V
+// chain; the epilogue reads U on uready[b] and V on vready[b], then arrives on
+// v_free, which the MMA thread waits for before the next V chain. That one
+// arrival also frees job j's U buffer for job j + 2.
 #include <math.h>
 
 #include <cuda_bf16.h>
@@ -68,14 +77,24 @@ constexpr int kTile = kN * kP * 2;            // bytes of one 16-bit N x P opera
 constexpr int kPart = kHeadsPerCta * kTile;   // one N = 128 B operand: both heads' tiles
 constexpr int kPartsPerJob = 3;               // W_hi, W_lo, M16
 constexpr int kPair = kPartsPerJob * kPart;   // operand bytes per (memory, head pair)
-constexpr int kStages = 6;                    // ring of kPart-sized stages
+constexpr int kStages = 6;                    // ring of kPart-sized stages: two jobs
+static_assert(kStages == 2 * kPartsPerJob, "stage of part p of job j is 3 (j & 1) + p");
 constexpr int kThreads = 384;
 // Register split: launched at 168 per thread (384 x 168 = 64512 of the 65536
-// of an SM); warpgroup 0 (producer, MMA, two idle warps) drops to 80 and the
-// epilogue warpgroups rise to 208: 128 x 80 + 256 x 208 = 63488, within the
-// launch pool, and per sub-partition (80 + 2 x 208) x 32 = 15872 <= 16384.
-constexpr int kRegsLow = 80, kRegsHigh = 208;
+// of an SM); warpgroup 0 (producer, MMA, two idle warps) drops to 64 and the
+// epilogue warpgroups rise to 216: 128 x 64 + 256 x 216 = 63488, within the
+// launch pool, and per sub-partition (64 + 2 x 216) x 32 = 15872 <= 16384.
+constexpr int kRegsLow = 64, kRegsHigh = 216;
 constexpr uint32_t kTmemCols = 512;
+// Row staging in shared memory: every epilogue lane bulk-copies its own rows
+// into slots padded to 272 (144) bytes, so a warp's 16-byte shared accesses
+// hit all 32 banks and the global side moves whole rows.
+constexpr int kRowPad = 272;                          // slot of a 256-byte row
+constexpr int kERowPad = 144;                         // slot of a 128-byte E row
+constexpr int kStgQE = 32 * kRowPad + 32 * kERowPad;  // warp of warpgroup 0: Q rows, E rows
+constexpr int kStgC = 32 * kRowPad;                   // warp of warpgroup 1: C rows
+static_assert(4 * kStgQE + 4 * kStgC <= kPartsPerJob * kPart, "prologue staging fits stages 3..5");
+static_assert(4 * kRows * kRowPad <= kStages * kPart, "merge staging fits the ring");
 constexpr uint32_t kColQ = 0, kColC = 64, kColU = 128, kColV = 384;
 // Bound on the final waits for this CTA's own copies and MMAs (never cut short).
 constexpr uint64_t kDrainLimitNs = 2000000000ull;
@@ -156,10 +175,13 @@ struct TcSmem {
     uint8_t stage[kStages][kPart];  // 1024-aligned by placement
     float lq[kRows];                // per-row logit factor 1 / (rms(Q_t) sqrt(N))
     float cdown[kRows];             // per-row power of two undoing C's scale
-    uint64_t full[kStages];
-    uint64_t empty[kStages];
-    uint64_t u_full[2], u_free[2], v_full, v_free;
+    uint64_t full[kStages];  // part landed (producer -> MMA)
+    uint64_t uready[2];      // U of job j done, i.e. its hi and lo stages consumed (MMA -> epilogue, producer)
+    uint64_t vready[2];      // V of job j done, its value stage consumed (MMA -> epilogue, producer)
+    uint64_t v_free;         // epilogue finished reading job j (MMA waits before the next V)
     uint64_t a_ready, drain;
+    uint64_t stg[8];         // prologue row copies of epilogue warp w
+    uint64_t ybar[8];        // Y_ssd row copies of epilogue warp w
     uint32_t tmem_base;
     int abort;
 };
@@ -262,18 +284,18 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
     volatile int* abort = &sm.abort;
 
     if (threadIdx.x == 0) {
-        for (int s = 0; s < kStages; ++s) {
-            tc::mbar_init(&sm.full[s], 1);
-            tc::mbar_init(&sm.empty[s], 1);
-        }
+        for (int s = 0; s < kStages; ++s) tc::mbar_init(&sm.full[s], 1);
         for (int u = 0; u < 2; ++u) {
-            tc::mbar_init(&sm.u_full[u], 1);
-            tc::mbar_init(&sm.u_free[u], 256);
+            tc::mbar_init(&sm.uready[u], 1);
+            tc::mbar_init(&sm.vready[u], 1);
         }
-        tc::mbar_init(&sm.v_full, 1);
         tc::mbar_init(&sm.v_free, 256);
         tc::mbar_init(&sm.a_ready, 256);  // Q from warpgroup 0, C from warpgroup 1
         tc::mbar_init(&sm.drain, 1);
+        for (int w = 0; w < 8; ++w) {
+            tc::mbar_init(&sm.stg[w], 1);
+            tc::mbar_init(&sm.ybar[w], 1);
+        }
         sm.abort = 0;
         tc::fence_barrier_init();
     }
@@ -290,28 +312,41 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
       asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegsLow));
       if (warp == 0) {
         // ------------------------------------------------------- producer
-        // parts in order hi(0), lo(0), v(0), hi(1), ...; part k uses stage k % kStages
+        // parts in order hi(0), lo(0), v(0), hi(1), ...: with 6 stages and 3 parts a
+        // job, part p of job j sits in stage 3 (j & 1) + p, in its (j >> 1)-th use
         if (lane == 0) {
-            const int nparts = kPartsPerJob * nj;
             const uint8_t* src = ops + ((i64)b * Mc * hpairs + hp) * (i64)kPair;
             const i64 job_stride = (i64)hpairs * kPair;
-            int k = 0;
-            for (; k < nparts; ++k) {
-                const int st = k % kStages;
-                const uint32_t round = (uint32_t)(k / kStages);
-                if (!tc::mbar_wait(&sm.empty[st], (round & 1u) ^ 1u, wait_limit_ns, abort)) {
+            bool ok = true;
+            int nparts = 0;  // copies issued
+            for (int j = 0; ok && j < nj; ++j) {
+                const int s0 = kPartsPerJob * (j & 1);
+                // stages 3..5 hold the epilogue's row staging until the operands are in TMEM
+                if (j == 1 && !tc::mbar_wait(&sm.a_ready, 0, wait_limit_ns, abort)) {
                     fail(abort, 1);
                     break;
                 }
-                const int j = k / kPartsPerJob, part = k - j * kPartsPerJob;
-                tc::mbar_arrive_expect_tx(&sm.full[st], (uint32_t)kPart);
-                tc::bulk_g2s(sm.stage[st], src + j * job_stride + part * kPart, (uint32_t)kPart,
-                             &sm.full[st]);
+                // the stages were last used by job j - 2: wait for its U (hi, lo) and V
+                const uint32_t par = (uint32_t)((j >> 1) & 1) ^ 1u;
+#pragma unroll
+                for (int part = 0; part < kPartsPerJob; ++part) {
+                    if ((part == 0 && !tc::mbar_wait(&sm.uready[j & 1], par, wait_limit_ns, abort)) ||
+                        (part == 2 && !tc::mbar_wait(&sm.vready[j & 1], par, wait_limit_ns, abort))) {
+                        fail(abort, 1);
+                        ok = false;
+                        break;
+                    }
+                    tc::mbar_arrive_expect_tx(&sm.full[s0 + part], (uint32_t)kPart);
+                    tc::bulk_g2s(sm.stage[s0 + part], src + j * job_stride + part * kPart,
+                                 (uint32_t)kPart, &sm.full[s0 + part]);
+                    ++nparts;
+                }
             }
-            // never leave a copy in flight behind: wait for the last one of each stage
-            for (int kk = k - 1; kk >= 0 && kk >= k - kStages; --kk) {
-                if (!tc::mbar_wait(&sm.full[kk % kStages], (uint32_t)((kk / kStages) & 1),
-                                   kDrainLimitNs, nullptr))
+            // never leave a copy in flight behind: wait for the last copy into every stage
+            for (int k = nparts - 1; k >= 0 && k >= nparts - kStages; --k) {
+                const int jj = k / kPartsPerJob;
+                const int st = kPartsPerJob * (jj & 1) + (k - jj * kPartsPerJob);
+                if (!tc::mbar_wait(&sm.full[st], (uint32_t)((jj >> 1) & 1), kDrainLimitNs, nullptr))
                     atomicCAS(&g_tc_status, 0, 5);
             }
         }
@@ -324,38 +359,35 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
             bool issued = false;
             // descriptor of stage 0; stage st is kPart * st bytes further (>> 4 in the address field)
             const uint64_t desc0 = tc::smem_desc_sw128(tc::smem_u32(sm.stage[0]), (uint32_t)kTile, 1024u);
-            int st = 0;
-            uint32_t round = 0;
+            // U buffer j & 1 was last read by the epilogue in job j - 2, which it finished
+            // before arriving on v_free for job j - 2; this thread waited for that before V(j - 1).
             for (int j = 0; ok && j < nj; ++j) {
                 const int ub = j & 1;
                 const uint32_t dU = tmem + kColU + 128u * (uint32_t)ub;
-                // U buffer ub is free once the epilogue has read job j - 2's contents
-                ok = tc::mbar_wait(&sm.u_free[ub], (uint32_t)((j >> 1) & 1) ^ 1u, wait_limit_ns, abort);
-#pragma unroll
-                for (int part = 0; part < kPartsPerJob && ok; ++part) {
-                    if (part == 2)
-                        ok = tc::mbar_wait(&sm.v_free, (uint32_t)(j & 1) ^ 1u, wait_limit_ns, abort);
-                    ok = ok && tc::mbar_wait(&sm.full[st], round & 1u, wait_limit_ns, abort);
-                    if (!ok) break;
-                    tc::tc_fence_after();
-                    const uint64_t bd = desc0 + (uint64_t)((st * kPart) >> 4);
-                    if (part == 0) issue_part<kIdescU, 0u>(dU, tmem + kColQ, bd);
-                    if (part == 1) issue_part<kIdescU, 1u>(dU, tmem + kColQ, bd);
-                    if (part == 2) issue_part<kIdescV, 0u>(tmem + kColV, tmem + kColC, bd);
-                    issued = true;
-                    tc::mma_commit(&sm.empty[st]);
-                    if (part == 1) tc::mma_commit(&sm.u_full[ub]);
-                    if (part == 2) tc::mma_commit(&sm.v_full);
-                    if (++st == kStages) {
-                        st = 0;
-                        ++round;
-                    }
-                }
-                if (!ok) {
-                    fail(abort, 3);
+                const int s0 = kPartsPerJob * ub;  // stages of this job's parts: s0, s0 + 1, s0 + 2
+                const uint32_t par = (uint32_t)((j >> 1) & 1);
+                const uint64_t bd = desc0 + (uint64_t)((s0 * kPart) >> 4);
+                if (!tc::mbar_wait(&sm.full[s0], par, wait_limit_ns, abort)) {
+                    ok = false;
                     break;
                 }
+                issue_part<kIdescU, 0u>(dU, tmem + kColQ, bd);
+                issued = true;
+                if (!tc::mbar_wait(&sm.full[s0 + 1], par, wait_limit_ns, abort)) {
+                    ok = false;
+                    break;
+                }
+                issue_part<kIdescU, 1u>(dU, tmem + kColQ, bd + (uint64_t)(kPart >> 4));
+                tc::mma_commit(&sm.uready[ub]);
+                // V is free once the epilogue has finished job j - 1
+                ok = tc::mbar_wait(&sm.v_free, (uint32_t)(j & 1) ^ 1u, wait_limit_ns, abort);
+                tc::tc_fence_after();
+                ok = ok && tc::mbar_wait(&sm.full[s0 + 2], par, wait_limit_ns, abort);
+                if (!ok) break;
+                issue_part<kIdescV, 0u>(tmem + kColV, tmem + kColC, bd + (uint64_t)((2 * kPart) >> 4));
+                tc::mma_commit(&sm.vready[ub]);
             }
+            if (!ok) fail(abort, 3);
             if (!ok && issued) {
                 // drain: this commit arrives once every MMA issued so far is done
                 tc::mma_commit(&sm.drain);
@@ -375,16 +407,32 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
         const i64 tok = (i64)b * L + t;
         const int g = h0 / (H / G);
 
-        // One round of loads per warpgroup: the E row (both) and Q (wg 0) or C (wg 1).
-        const uint4* erow = reinterpret_cast<const uint4*>(E + (tok * G + g) * kP);
-        const uint4* arow = reinterpret_cast<const uint4*>((wg == 0 ? Q : Cm) + (tok * G + g) * kN);
+        // Rows in through shared memory: Q and E (warpgroup 0) or C (warpgroup 1).
+        // Warpgroup 1 reads the E rows that warpgroup 0's warp of its quadrant staged.
+        const int q4 = warp & 3;
+        uint8_t* qe_warp = sm.stage[kPartsPerJob] + q4 * kStgQE;
+        uint8_t* a_slot = (wg == 0 ? qe_warp : sm.stage[kPartsPerJob] + 4 * kStgQE + q4 * kStgC) +
+                          lane * kRowPad;
+        const uint8_t* e_slot = qe_warp + 32 * kRowPad + lane * kERowPad;
+        if (lane == 0)
+            tc::mbar_arrive_expect_tx(&sm.stg[warp - 4], (uint32_t)(32 * (wg == 0 ? 2 * (kN + kP) : 2 * kN)));
+        __syncwarp();
+        tc::bulk_g2s(a_slot, (wg == 0 ? Q : Cm) + (tok * G + g) * kN, 2 * kN, &sm.stg[warp - 4]);
+        if (wg == 0) tc::bulk_g2s((void*)e_slot, E + (tok * G + g) * kP, 2 * kP, &sm.stg[warp - 4]);
+        bool staged = warp_wait(&sm.stg[warp - 4], 0, wait_limit_ns, abort);
+        if (wg == 1) staged = staged && warp_wait(&sm.stg[q4], 0, wait_limit_ns, abort);
+        if (!staged) {
+            fail(abort, 7);
+            // never leave a copy in flight behind
+            if (!tc::mbar_wait(&sm.stg[warp - 4], 0, kDrainLimitNs, nullptr)) atomicCAS(&g_tc_status, 0, 5);
+        }
         uint4 av[16];
         uint32_t e2[kP / 2];  // the E row as bf16 pairs; Ebar = E * ie
 #pragma unroll
-        for (int u = 0; u < 16; ++u) av[u] = arow[u];
+        for (int u = 0; u < 16; ++u) av[u] = reinterpret_cast<const uint4*>(a_slot)[u];
 #pragma unroll
         for (int u = 0; u < 8; ++u) {
-            const uint4 w = erow[u];
+            const uint4 w = reinterpret_cast<const uint4*>(e_slot)[u];
             e2[4 * u] = w.x; e2[4 * u + 1] = w.y; e2[4 * u + 2] = w.z; e2[4 * u + 3] = w.w;
         }
         float sse = 0.0f;
@@ -448,7 +496,9 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
         asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
         tc::tc_fence_before();
         tc::mbar_arrive(&sm.a_ready);
-        asm volatile("bar.sync 1, 256;" ::: "memory");  // lq and cdown visible to both warpgroups
+        // lq and cdown visible to both warpgroups; all staging reads done before
+        // the merge reuses the ring
+        asm volatile("bar.sync 1, 256;" ::: "memory");
         const float lfac = sm.lq[row];
         const float cdown = sm.cdown[row];
 
@@ -456,7 +506,7 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
 #pragma unroll
         for (int i = 0; i < kP / 2; ++i) O[i] = 0ull;
         float m = -INFINITY, dsum = 0.0f;
-        bool ok = true;
+        bool ok = staged;
         const float* scl = scale + (i64)b * Mc * H + h;  // scale of memory j at scl[j H]
         float s_next = nj > 0 ? __ldg(scl) : 0.0f;
         const uint32_t ua = tmem + lane_addr + kColU + (uint32_t)(kP * wg);
@@ -465,7 +515,7 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
             const int ub = j & 1;
             const float s_j = s_next;
             if (j + 1 < nj) s_next = __ldg(scl + (i64)(j + 1) * H);  // one job ahead
-            if (!warp_wait(&sm.u_full[ub], (uint32_t)((j >> 1) & 1), wait_limit_ns, abort)) {
+            if (!warp_wait(&sm.uready[ub], (uint32_t)((j >> 1) & 1), wait_limit_ns, abort)) {
                 fail(abort, 4);
                 ok = false;
                 break;
@@ -478,8 +528,6 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
 #pragma unroll
                 for (int i = 0; i < 16; ++i) acc = f2_fma(v[i], eb[i], acc);
                 tmem_ld32p(ua + 128u * ub + 32u, v);
-                tc::tc_fence_before();
-                tc::mbar_arrive(&sm.u_free[ub]);
 #pragma unroll
                 for (int i = 0; i < 16; ++i) acc = f2_fma(v[i], eb[16 + i], acc);
                 float lx, ly;
@@ -499,7 +547,7 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
             dsum += pe;
             const float w = pe * s_j;
             const uint64_t w2 = f2_pack(w, w);
-            if (!warp_wait(&sm.v_full, (uint32_t)(j & 1), wait_limit_ns, abort)) {
+            if (!warp_wait(&sm.vready[ub], (uint32_t)((j >> 1) & 1), wait_limit_ns, abort)) {
                 fail(abort, 4);
                 ok = false;
                 break;
@@ -518,28 +566,49 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
             }
         }
         if (ok) {
-            // R = O / d (C's row scale undone), lse, gated merge
+            // R = O / d (C's row scale undone), lse, gated merge. Every MMA is done
+            // (the last job's V was read, or there were no jobs), so the ring is free:
+            // Y_ssd comes in and Y, R go out through per-lane row slots.
+            constexpr uint32_t kRowB = (uint32_t)(kP * sizeof(Tout));
             const i64 rowo = tok * H + h;
+            uint8_t* y_slot = sm.stage[0] + (wg * kRows + row) * kRowPad;
+            uint8_t* r_slot = sm.stage[0] + ((2 + wg) * kRows + row) * kRowPad;
+            if (lane == 0) tc::mbar_arrive_expect_tx(&sm.ybar[warp - 4], 32 * kRowB);
+            __syncwarp();
+            tc::bulk_g2s(y_slot, Yssd + rowo * kP, kRowB, &sm.ybar[warp - 4]);
             const bool has = nj > 0;
             const float inv_d = has ? cdown / dsum : 0.0f;
             const float gate = silu_f32(__bfloat162float(z[rowo]));
-            float ys[kP], r[kP];
-#pragma unroll
-            for (int c = 0; c < 4; ++c) load_row16(Yssd + rowo * kP + 16 * c, ys + 16 * c);
+            float r[kP];
 #pragma unroll
             for (int i = 0; i < kP / 2; ++i) {
                 f2_unpack(O[i], r[2 * i], r[2 * i + 1]);
                 r[2 * i] *= inv_d;
                 r[2 * i + 1] *= inv_d;
-                ys[2 * i] = fmaf(gate, r[2 * i], ys[2 * i]);
-                ys[2 * i + 1] = fmaf(gate, r[2 * i + 1], ys[2 * i + 1]);
             }
+            Tout* rs = reinterpret_cast<Tout*>(r_slot);
 #pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                store_row16(Y + rowo * kP + 16 * c, ys + 16 * c);
-                if (R != nullptr) store_row16(R + rowo * kP + 16 * c, r + 16 * c);
-            }
+            for (int c = 0; c < 4; ++c) store_row16(rs + 16 * c, r + 16 * c);
             if (lse != nullptr) lse[rowo] = has ? m + logf(dsum) : -INFINITY;
+            if (warp_wait(&sm.ybar[warp - 4], 0, wait_limit_ns, abort)) {
+                Tout* ys = reinterpret_cast<Tout*>(y_slot);
+#pragma unroll
+                for (int c = 0; c < 4; ++c) {
+                    float y[16];
+                    load_row16(ys + 16 * c, y);
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) y[i] = fmaf(gate, r[16 * c + i], y[i]);
+                    store_row16(ys + 16 * c, y);
+                }
+                tc::fence_proxy_async_shared();
+                tc::bulk_s2g(Y + rowo * kP, y_slot, kRowB);
+                if (R != nullptr) tc::bulk_s2g(R + rowo * kP, r_slot, kRowB);
+                tc::bulk_commit_group();
+                tc::bulk_wait_read_all();
+            } else {
+                fail(abort, 8);
+                if (!tc::mbar_wait(&sm.ybar[warp - 4], 0, kDrainLimitNs, nullptr)) atomicCAS(&g_tc_status, 0, 5);
+            }
         }
     }
 

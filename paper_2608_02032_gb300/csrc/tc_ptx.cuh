@@ -57,11 +57,10 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
     return ok != 0;
 }
 
-// Waits for the phase with the given parity to complete. Returns false once
-// limit_ns of wall-clock time have passed without completion, or as soon as
-// *abort (when given) becomes non-zero.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint64_t limit_ns,
-                                          volatile int* abort) {
+// Slow path of mbar_wait: keeps trying, returns false once limit_ns of
+// wall-clock time have passed or *abort (when given) becomes non-zero.
+__device__ __forceinline__ bool mbar_wait_slow(uint64_t* bar, uint32_t parity, uint64_t limit_ns,
+                                            volatile int* abort) {
     uint32_t spins = 0;
     uint64_t t0 = 0;
     while (!mbar_try_wait(bar, parity)) {
@@ -78,6 +77,16 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint64
     return true;
 }
 
+// Waits for the phase with the given parity to complete. Returns false once
+// limit_ns of wall-clock time have passed without completion, or as soon as
+// *abort (when given) becomes non-zero. A phase that has already completed
+// costs one try_wait (the MMA-issuing thread depends on this being short).
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint64_t limit_ns,
+                                          volatile int* abort) {
+    if (mbar_try_wait(bar, parity)) return true;
+    return mbar_wait_slow(bar, parity, limit_ns, abort);
+}
+
 // ------------------------------------------------------------- bulk copies
 // 1D bulk copy global -> shared, completion counted on bar (bytes: multiple of
 // 16, both addresses 16-byte aligned).
@@ -87,6 +96,23 @@ __device__ __forceinline__ void bulk_g2s(void* smem_dst, const void* gmem_src, u
         "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
         ::"r"(smem_u32(smem_dst)), "l"(gmem_src), "r"(bytes), "r"(smem_u32(bar))
         : "memory");
+}
+
+// 1D bulk copy shared -> global in this thread's bulk group (same size and
+// alignment rules). Shared-memory writes made by ordinary stores must be
+// made visible to the async proxy first (fence_proxy_async_shared).
+__device__ __forceinline__ void bulk_s2g(void* gmem_dst, const void* smem_src, uint32_t bytes) {
+    asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;"
+                 ::"l"(gmem_dst), "r"(smem_u32(smem_src)), "r"(bytes)
+                 : "memory");
+}
+__device__ __forceinline__ void bulk_commit_group() {
+    asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+}
+// Waits until every committed bulk group of this thread has finished reading
+// its shared-memory source.
+__device__ __forceinline__ void bulk_wait_read_all() {
+    asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
 }
 
 // ---------------------------------------------------------------- tcgen05
