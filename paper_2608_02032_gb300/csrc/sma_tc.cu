@@ -44,17 +44,19 @@
 // of U and of V from TMEM, runs the online softmax (the running sum is only
 // rescaled when the maximum moves), and finally writes R = O / d, lse and
 // Y = Y_ssd + SiLU(z) R.
-// TMEM: [0,64) Q (bf16 pairs), [64,128) C (fp16 pairs), [128,256) and
-// [256,384) U (two buffers, jobs alternate), [384,512) V.
+// TMEM: [0,64) Q (bf16 pairs), [64,128) C (fp16 pairs), [128,256) U,
+// [256,384) and [384,512) V (two buffers, jobs alternate).
 //
-// Synchronisation, job j, b = j & 1 (the MMA thread pays for every barrier
-// operation with idle tensor cycles, so it does four waits and two commits
-// per job): the producer refills stages 3b .. 3b+2 once job j - 2 is done
-// with them (uready[b], vready[b]); the MMA thread waits for each part
-// (full), commits uready[b] after the two U chains and vready[b] after the V
-// chain; the epilogue reads U on uready[b] and V on vready[b], then arrives on
-// v_free, which the MMA thread waits for before the next V chain. That one
-// arrival also frees job j's U buffer for job j + 2.
+// Synchronisation, job j, b = j & 1. The MMA thread pays for barrier
+// operations with idle tensor cycles, and most for a wait right after a
+// commit (measured: ~100 cycles each time), so it does all of a job's waits
+// first and commits only between MMA chains: wait u_free (the epilogue has
+// read U of job j - 1), v_free[b] (it has read V of job j - 2) and the
+// job's parts (full[b], one copy), then hi, lo, commit uready[b], V into buffer b, commit
+// vready[b]. The producer refills stages 3b .. 3b+2 once job j - 2 is done
+// with them (uready[b], vready[b]); the epilogue reads U on uready[b] and V on
+// vready[b]. Every barrier's waiter is at most one phase behind it, which the
+// parity waits need.
 #include <math.h>
 
 #include <cuda_bf16.h>
@@ -86,16 +88,14 @@ constexpr int kThreads = 384;
 // launch pool, and per sub-partition (64 + 2 x 216) x 32 = 15872 <= 16384.
 constexpr int kRegsLow = 64, kRegsHigh = 216;
 constexpr uint32_t kTmemCols = 512;
-// Row staging in shared memory: every epilogue lane bulk-copies its own rows
-// into slots padded to 272 (144) bytes, so a warp's 16-byte shared accesses
-// hit all 32 banks and the global side moves whole rows.
-constexpr int kRowPad = 272;                          // slot of a 256-byte row
-constexpr int kERowPad = 144;                         // slot of a 128-byte E row
-constexpr int kStgQE = 32 * kRowPad + 32 * kERowPad;  // warp of warpgroup 0: Q rows, E rows
-constexpr int kStgC = 32 * kRowPad;                   // warp of warpgroup 1: C rows
-static_assert(4 * kStgQE + 4 * kStgC <= kPartsPerJob * kPart, "prologue staging fits stages 3..5");
-static_assert(4 * kRows * kRowPad <= kStages * kPart, "merge staging fits the ring");
-constexpr uint32_t kColQ = 0, kColC = 64, kColU = 128, kColV = 384;
+// Row transposes in shared memory: an epilogue warp moves the 32 rows of its
+// quadrant between global memory (whole rows per vector load or store,
+// coalesced) and row slots padded by 16 bytes (a lane's 16-byte accesses to
+// its own row then hit all 32 banks across the warp).
+constexpr int kSlots = 32 * (256 + 16);  // one warp's slots for rows of up to 256 bytes
+static_assert(8 * kSlots <= kPartsPerJob * kPart, "prologue slots fit stages 3..5");
+static_assert(16 * kSlots <= kStages * kPart, "merge slots fit the ring");
+constexpr uint32_t kColQ = 0, kColC = 64, kColU = 128, kColV = 256;  // V buffer b at kColV + 128 b
 // Bound on the final waits for this CTA's own copies and MMAs (never cut short).
 constexpr uint64_t kDrainLimitNs = 2000000000ull;
 
@@ -175,13 +175,12 @@ struct TcSmem {
     uint8_t stage[kStages][kPart];  // 1024-aligned by placement
     float lq[kRows];                // per-row logit factor 1 / (rms(Q_t) sqrt(N))
     float cdown[kRows];             // per-row power of two undoing C's scale
-    uint64_t full[kStages];  // part landed (producer -> MMA)
+    uint64_t full[2];        // job j's three parts landed in stages 3b .. 3b+2 (producer -> MMA)
     uint64_t uready[2];      // U of job j done, i.e. its hi and lo stages consumed (MMA -> epilogue, producer)
     uint64_t vready[2];      // V of job j done, its value stage consumed (MMA -> epilogue, producer)
-    uint64_t v_free;         // epilogue finished reading job j (MMA waits before the next V)
+    uint64_t u_free;         // epilogue read U of job j (MMA waits before job j + 1); 8 warps
+    uint64_t v_free[2];      // epilogue read V of job j from buffer j & 1 (MMA waits before job j + 2)
     uint64_t a_ready, drain;
-    uint64_t stg[8];         // prologue row copies of epilogue warp w
-    uint64_t ybar[8];        // Y_ssd row copies of epilogue warp w
     uint32_t tmem_base;
     int abort;
 };
@@ -196,6 +195,14 @@ __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, uint64
                                           volatile int* abort) {
     const bool got = tc::mbar_wait(bar, parity, limit_ns, abort);
     return __all_sync(0xffffffffu, got);
+}
+
+// The warp's TMEM loads are complete (each lane waited on them): one arrival
+// for the whole warp (the barrier counts warps, keeping its traffic low).
+__device__ __forceinline__ void warp_release(uint64_t* bar) {
+    tc::tc_fence_before();
+    __syncwarp();
+    if ((threadIdx.x & 31) == 0) tc::mbar_arrive(bar);
 }
 
 // tcgen05.ld of 32 consecutive fp32 columns of this thread's lane, waited; the
@@ -246,6 +253,30 @@ __device__ __forceinline__ uint64_t f2_mul(uint64_t a, uint64_t b) {
 __device__ __forceinline__ float bf_lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float bf_hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
 
+// Warp-cooperative row transposes. Rows r = 0..31 of a warp start at
+// base + r * stride (16-byte aligned) and hold RB bytes; slot r is at
+// slots + r * (RB + 16). Each vector access of the warp covers 512 bytes of
+// whole rows on the global side.
+template <int RB>
+__device__ __forceinline__ void rows_to_slots(uint8_t* slots, const uint8_t* base, i64 stride, int lane) {
+    constexpr int kCpr = RB / 16, kRpi = 32 / kCpr;  // 16-byte chunks per row, rows per access
+    uint4 v[kCpr];
+#pragma unroll
+    for (int i = 0; i < kCpr; ++i)
+        v[i] = *reinterpret_cast<const uint4*>(base + (i64)(i * kRpi + lane / kCpr) * stride + (lane % kCpr) * 16);
+#pragma unroll
+    for (int i = 0; i < kCpr; ++i)
+        *reinterpret_cast<uint4*>(slots + (i * kRpi + lane / kCpr) * (RB + 16) + (lane % kCpr) * 16) = v[i];
+}
+template <int RB>
+__device__ __forceinline__ void slots_to_rows(uint8_t* base, i64 stride, const uint8_t* slots, int lane) {
+    constexpr int kCpr = RB / 16, kRpi = 32 / kCpr;
+#pragma unroll
+    for (int i = 0; i < kCpr; ++i)
+        *reinterpret_cast<uint4*>(base + (i64)(i * kRpi + lane / kCpr) * stride + (lane % kCpr) * 16) =
+            *reinterpret_cast<const uint4*>(slots + (i * kRpi + lane / kCpr) * (RB + 16) + (lane % kCpr) * 16);
+}
+
 // Issues the eight K = 16 MMAs of one N = 128 part: D (+)= A[tmem] * B[stage].
 // `first_acc` is 0 when the first MMA starts a fresh accumulator.
 template <uint32_t kIdesc, uint32_t first_acc>
@@ -284,18 +315,18 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
     volatile int* abort = &sm.abort;
 
     if (threadIdx.x == 0) {
-        for (int s = 0; s < kStages; ++s) tc::mbar_init(&sm.full[s], 1);
+        tc::mbar_init(&sm.full[0], 1);
+        tc::mbar_init(&sm.full[1], 1);
         for (int u = 0; u < 2; ++u) {
             tc::mbar_init(&sm.uready[u], 1);
             tc::mbar_init(&sm.vready[u], 1);
         }
-        tc::mbar_init(&sm.v_free, 256);
+        tc::mbar_init(&sm.u_free, 8);  // one arrival per epilogue warp
+        tc::mbar_init(&sm.v_free[0], 8);
+        tc::mbar_init(&sm.v_free[1], 8);
         tc::mbar_init(&sm.a_ready, 256);  // Q from warpgroup 0, C from warpgroup 1
         tc::mbar_init(&sm.drain, 1);
-        for (int w = 0; w < 8; ++w) {
-            tc::mbar_init(&sm.stg[w], 1);
-            tc::mbar_init(&sm.ybar[w], 1);
-        }
+
         sm.abort = 0;
         tc::fence_barrier_init();
     }
@@ -312,43 +343,33 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
       asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegsLow));
       if (warp == 0) {
         // ------------------------------------------------------- producer
-        // parts in order hi(0), lo(0), v(0), hi(1), ...: with 6 stages and 3 parts a
-        // job, part p of job j sits in stage 3 (j & 1) + p, in its (j >> 1)-th use
+        // one 96 KiB copy per job: part p of job j lands in stage 3 (j & 1) + p
         if (lane == 0) {
             const uint8_t* src = ops + ((i64)b * Mc * hpairs + hp) * (i64)kPair;
             const i64 job_stride = (i64)hpairs * kPair;
             bool ok = true;
-            int nparts = 0;  // copies issued
-            for (int j = 0; ok && j < nj; ++j) {
-                const int s0 = kPartsPerJob * (j & 1);
-                // stages 3..5 hold the epilogue's row staging until the operands are in TMEM
-                if (j == 1 && !tc::mbar_wait(&sm.a_ready, 0, wait_limit_ns, abort)) {
+            int njobs = 0;  // jobs whose copy was issued
+            for (int j = 0; j < nj; ++j) {
+                const int ub = j & 1;
+                // stages 3..5 hold the epilogue's row staging until the operands are in TMEM;
+                // stages 3b .. 3b+2 were last used by job j - 2: wait for its U and V
+                const uint32_t par = (uint32_t)((j >> 1) & 1) ^ 1u;
+                ok = (j != 1 || tc::mbar_wait(&sm.a_ready, 0, wait_limit_ns, abort)) &&
+                     tc::mbar_wait(&sm.uready[ub], par, wait_limit_ns, abort) &&
+                     tc::mbar_wait(&sm.vready[ub], par, wait_limit_ns, abort);
+                if (!ok) {
                     fail(abort, 1);
                     break;
                 }
-                // the stages were last used by job j - 2: wait for its U (hi, lo) and V
-                const uint32_t par = (uint32_t)((j >> 1) & 1) ^ 1u;
-#pragma unroll
-                for (int part = 0; part < kPartsPerJob; ++part) {
-                    if ((part == 0 && !tc::mbar_wait(&sm.uready[j & 1], par, wait_limit_ns, abort)) ||
-                        (part == 2 && !tc::mbar_wait(&sm.vready[j & 1], par, wait_limit_ns, abort))) {
-                        fail(abort, 1);
-                        ok = false;
-                        break;
-                    }
-                    tc::mbar_arrive_expect_tx(&sm.full[s0 + part], (uint32_t)kPart);
-                    tc::bulk_g2s(sm.stage[s0 + part], src + j * job_stride + part * kPart,
-                                 (uint32_t)kPart, &sm.full[s0 + part]);
-                    ++nparts;
-                }
+                // the job's hi, lo and value parts are contiguous in global and in the ring
+                tc::mbar_arrive_expect_tx(&sm.full[ub], (uint32_t)kPair);
+                tc::bulk_g2s(sm.stage[kPartsPerJob * ub], src + j * job_stride, (uint32_t)kPair, &sm.full[ub]);
+                ++njobs;
             }
-            // never leave a copy in flight behind: wait for the last copy into every stage
-            for (int k = nparts - 1; k >= 0 && k >= nparts - kStages; --k) {
-                const int jj = k / kPartsPerJob;
-                const int st = kPartsPerJob * (jj & 1) + (k - jj * kPartsPerJob);
-                if (!tc::mbar_wait(&sm.full[st], (uint32_t)((jj >> 1) & 1), kDrainLimitNs, nullptr))
+            // never leave a copy in flight behind: wait for the last copy into each half
+            for (int j = njobs - 1; j >= 0 && j >= njobs - 2; --j)
+                if (!tc::mbar_wait(&sm.full[j & 1], (uint32_t)((j >> 1) & 1), kDrainLimitNs, nullptr))
                     atomicCAS(&g_tc_status, 0, 5);
-            }
         }
     } else if (warp == 1) {
         // ------------------------------------------------------- MMA issuer
@@ -359,33 +380,23 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
             bool issued = false;
             // descriptor of stage 0; stage st is kPart * st bytes further (>> 4 in the address field)
             const uint64_t desc0 = tc::smem_desc_sw128(tc::smem_u32(sm.stage[0]), (uint32_t)kTile, 1024u);
-            // U buffer j & 1 was last read by the epilogue in job j - 2, which it finished
-            // before arriving on v_free for job j - 2; this thread waited for that before V(j - 1).
             for (int j = 0; ok && j < nj; ++j) {
                 const int ub = j & 1;
-                const uint32_t dU = tmem + kColU + 128u * (uint32_t)ub;
                 const int s0 = kPartsPerJob * ub;  // stages of this job's parts: s0, s0 + 1, s0 + 2
                 const uint32_t par = (uint32_t)((j >> 1) & 1);
                 const uint64_t bd = desc0 + (uint64_t)((s0 * kPart) >> 4);
-                if (!tc::mbar_wait(&sm.full[s0], par, wait_limit_ns, abort)) {
-                    ok = false;
-                    break;
-                }
-                issue_part<kIdescU, 0u>(dU, tmem + kColQ, bd);
-                issued = true;
-                if (!tc::mbar_wait(&sm.full[s0 + 1], par, wait_limit_ns, abort)) {
-                    ok = false;
-                    break;
-                }
-                issue_part<kIdescU, 1u>(dU, tmem + kColQ, bd + (uint64_t)(kPart >> 4));
-                tc::mma_commit(&sm.uready[ub]);
-                // V is free once the epilogue has finished job j - 1
-                ok = tc::mbar_wait(&sm.v_free, (uint32_t)(j & 1) ^ 1u, wait_limit_ns, abort);
+                ok = tc::mbar_wait(&sm.u_free, (uint32_t)ub ^ 1u, wait_limit_ns, abort) &&
+                     tc::mbar_wait(&sm.v_free[ub], par ^ 1u, wait_limit_ns, abort);
                 tc::tc_fence_after();
-                ok = ok && tc::mbar_wait(&sm.full[s0 + 2], par, wait_limit_ns, abort);
+                ok = ok && tc::mbar_wait(&sm.full[ub], par, wait_limit_ns, abort);
                 if (!ok) break;
-                issue_part<kIdescV, 0u>(tmem + kColV, tmem + kColC, bd + (uint64_t)((2 * kPart) >> 4));
+                issue_part<kIdescU, 0u>(tmem + kColU, tmem + kColQ, bd);
+                issue_part<kIdescU, 1u>(tmem + kColU, tmem + kColQ, bd + (uint64_t)(kPart >> 4));
+                tc::mma_commit(&sm.uready[ub]);
+                issue_part<kIdescV, 0u>(tmem + kColV + 128u * (uint32_t)ub, tmem + kColC,
+                                        bd + (uint64_t)((2 * kPart) >> 4));
                 tc::mma_commit(&sm.vready[ub]);
+                issued = true;
             }
             if (!ok) fail(abort, 3);
             if (!ok && issued) {
@@ -407,32 +418,23 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
         const i64 tok = (i64)b * L + t;
         const int g = h0 / (H / G);
 
-        // Rows in through shared memory: Q and E (warpgroup 0) or C (warpgroup 1).
-        // Warpgroup 1 reads the E rows that warpgroup 0's warp of its quadrant staged.
-        const int q4 = warp & 3;
-        uint8_t* qe_warp = sm.stage[kPartsPerJob] + q4 * kStgQE;
-        uint8_t* a_slot = (wg == 0 ? qe_warp : sm.stage[kPartsPerJob] + 4 * kStgQE + q4 * kStgC) +
-                          lane * kRowPad;
-        const uint8_t* e_slot = qe_warp + 32 * kRowPad + lane * kERowPad;
-        if (lane == 0)
-            tc::mbar_arrive_expect_tx(&sm.stg[warp - 4], (uint32_t)(32 * (wg == 0 ? 2 * (kN + kP) : 2 * kN)));
-        __syncwarp();
-        tc::bulk_g2s(a_slot, (wg == 0 ? Q : Cm) + (tok * G + g) * kN, 2 * kN, &sm.stg[warp - 4]);
-        if (wg == 0) tc::bulk_g2s((void*)e_slot, E + (tok * G + g) * kP, 2 * kP, &sm.stg[warp - 4]);
-        bool staged = warp_wait(&sm.stg[warp - 4], 0, wait_limit_ns, abort);
-        if (wg == 1) staged = staged && warp_wait(&sm.stg[q4], 0, wait_limit_ns, abort);
-        if (!staged) {
-            fail(abort, 7);
-            // never leave a copy in flight behind
-            if (!tc::mbar_wait(&sm.stg[warp - 4], 0, kDrainLimitNs, nullptr)) atomicCAS(&g_tc_status, 0, 5);
-        }
+        // Rows in through shared memory (stages 3..5 are not needed before job 1):
+        // Q (warpgroup 0) or C (warpgroup 1), then E, 32 rows per warp.
+        uint8_t* slots = sm.stage[kPartsPerJob] + (warp - 4) * kSlots;
+        const i64 tok0 = tok - lane;  // first token of this warp's rows
         uint4 av[16];
         uint32_t e2[kP / 2];  // the E row as bf16 pairs; Ebar = E * ie
+        rows_to_slots<2 * kN>(slots, reinterpret_cast<const uint8_t*>((wg == 0 ? Q : Cm) + (tok0 * G + g) * kN),
+                              (i64)G * kN * 2, lane);
+        __syncwarp();
 #pragma unroll
-        for (int u = 0; u < 16; ++u) av[u] = reinterpret_cast<const uint4*>(a_slot)[u];
+        for (int u = 0; u < 16; ++u) av[u] = reinterpret_cast<const uint4*>(slots + lane * (2 * kN + 16))[u];
+        __syncwarp();
+        rows_to_slots<2 * kP>(slots, reinterpret_cast<const uint8_t*>(E + (tok0 * G + g) * kP), (i64)G * kP * 2, lane);
+        __syncwarp();
 #pragma unroll
         for (int u = 0; u < 8; ++u) {
-            const uint4 w = reinterpret_cast<const uint4*>(e_slot)[u];
+            const uint4 w = reinterpret_cast<const uint4*>(slots + lane * (2 * kP + 16))[u];
             e2[4 * u] = w.x; e2[4 * u + 1] = w.y; e2[4 * u + 2] = w.z; e2[4 * u + 3] = w.w;
         }
         float sse = 0.0f;
@@ -506,11 +508,11 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
 #pragma unroll
         for (int i = 0; i < kP / 2; ++i) O[i] = 0ull;
         float m = -INFINITY, dsum = 0.0f;
-        bool ok = staged;
+        bool ok = true;
         const float* scl = scale + (i64)b * Mc * H + h;  // scale of memory j at scl[j H]
         float s_next = nj > 0 ? __ldg(scl) : 0.0f;
         const uint32_t ua = tmem + lane_addr + kColU + (uint32_t)(kP * wg);
-        const uint32_t va = tmem + lane_addr + kColV + (uint32_t)(kP * wg);
+        const uint32_t va = tmem + lane_addr + kColV + (uint32_t)(kP * wg);  // + 128 per V buffer
         for (int j = 0; j < nj; ++j) {
             const int ub = j & 1;
             const float s_j = s_next;
@@ -524,10 +526,11 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
             float l;
             {
                 uint64_t acc = 0ull, v[16];
-                tmem_ld32p(ua + 128u * ub, v);
+                tmem_ld32p(ua, v);
 #pragma unroll
                 for (int i = 0; i < 16; ++i) acc = f2_fma(v[i], eb[i], acc);
-                tmem_ld32p(ua + 128u * ub + 32u, v);
+                tmem_ld32p(ua + 32u, v);
+                warp_release(&sm.u_free);
 #pragma unroll
                 for (int i = 0; i < 16; ++i) acc = f2_fma(v[i], eb[16 + i], acc);
                 float lx, ly;
@@ -555,30 +558,29 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
             tc::tc_fence_after();
             {
                 uint64_t v[16];
-                tmem_ld32p(va, v);
+                tmem_ld32p(va + 128u * ub, v);
 #pragma unroll
                 for (int i = 0; i < 16; ++i) O[i] = f2_fma(w2, v[i], O[i]);
-                tmem_ld32p(va + 32u, v);
-                tc::tc_fence_before();
-                tc::mbar_arrive(&sm.v_free);
+                tmem_ld32p(va + 128u * ub + 32u, v);
+                warp_release(&sm.v_free[ub]);
 #pragma unroll
                 for (int i = 0; i < 16; ++i) O[16 + i] = f2_fma(w2, v[i], O[16 + i]);
             }
         }
         if (ok) {
             // R = O / d (C's row scale undone), lse, gated merge. Every MMA is done
-            // (the last job's V was read, or there were no jobs), so the ring is free:
-            // Y_ssd comes in and Y, R go out through per-lane row slots.
-            constexpr uint32_t kRowB = (uint32_t)(kP * sizeof(Tout));
+            // (the last job's V was read, or there were no jobs), so the ring is free
+            // for the row transposes: Y_ssd in, Y and R out.
+            constexpr int kRowB = kP * (int)sizeof(Tout);
             const i64 rowo = tok * H + h;
-            uint8_t* y_slot = sm.stage[0] + (wg * kRows + row) * kRowPad;
-            uint8_t* r_slot = sm.stage[0] + ((2 + wg) * kRows + row) * kRowPad;
-            if (lane == 0) tc::mbar_arrive_expect_tx(&sm.ybar[warp - 4], 32 * kRowB);
-            __syncwarp();
-            tc::bulk_g2s(y_slot, Yssd + rowo * kP, kRowB, &sm.ybar[warp - 4]);
+            const i64 row0 = tok0 * H + h;  // this warp's first output row
+            uint8_t* yslots = sm.stage[0] + (warp - 4) * 2 * kSlots;
+            uint8_t* rslots = yslots + kSlots;
+            const i64 rstride = (i64)H * kRowB;
             const bool has = nj > 0;
             const float inv_d = has ? cdown / dsum : 0.0f;
             const float gate = silu_f32(__bfloat162float(z[rowo]));
+            rows_to_slots<kRowB>(yslots, reinterpret_cast<const uint8_t*>(Yssd + row0 * kP), rstride, lane);
             float r[kP];
 #pragma unroll
             for (int i = 0; i < kP / 2; ++i) {
@@ -586,29 +588,23 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
                 r[2 * i] *= inv_d;
                 r[2 * i + 1] *= inv_d;
             }
-            Tout* rs = reinterpret_cast<Tout*>(r_slot);
+            Tout* rs = reinterpret_cast<Tout*>(rslots + lane * (kRowB + 16));
+            Tout* ys = reinterpret_cast<Tout*>(yslots + lane * (kRowB + 16));
 #pragma unroll
             for (int c = 0; c < 4; ++c) store_row16(rs + 16 * c, r + 16 * c);
             if (lse != nullptr) lse[rowo] = has ? m + logf(dsum) : -INFINITY;
-            if (warp_wait(&sm.ybar[warp - 4], 0, wait_limit_ns, abort)) {
-                Tout* ys = reinterpret_cast<Tout*>(y_slot);
+            __syncwarp();
 #pragma unroll
-                for (int c = 0; c < 4; ++c) {
-                    float y[16];
-                    load_row16(ys + 16 * c, y);
+            for (int c = 0; c < 4; ++c) {
+                float y[16];
+                load_row16(ys + 16 * c, y);
 #pragma unroll
-                    for (int i = 0; i < 16; ++i) y[i] = fmaf(gate, r[16 * c + i], y[i]);
-                    store_row16(ys + 16 * c, y);
-                }
-                tc::fence_proxy_async_shared();
-                tc::bulk_s2g(Y + rowo * kP, y_slot, kRowB);
-                if (R != nullptr) tc::bulk_s2g(R + rowo * kP, r_slot, kRowB);
-                tc::bulk_commit_group();
-                tc::bulk_wait_read_all();
-            } else {
-                fail(abort, 8);
-                if (!tc::mbar_wait(&sm.ybar[warp - 4], 0, kDrainLimitNs, nullptr)) atomicCAS(&g_tc_status, 0, 5);
+                for (int i = 0; i < 16; ++i) y[i] = fmaf(gate, r[16 * c + i], y[i]);
+                store_row16(ys + 16 * c, y);
             }
+            __syncwarp();
+            slots_to_rows<kRowB>(reinterpret_cast<uint8_t*>(Y + row0 * kP), rstride, yslots, lane);
+            if (R != nullptr) slots_to_rows<kRowB>(reinterpret_cast<uint8_t*>(R + row0 * kP), rstride, rslots, lane);
         }
     }
 
