@@ -277,6 +277,15 @@ __device__ __forceinline__ void slots_to_rows(uint8_t* base, i64 stride, const u
             *reinterpret_cast<const uint4*>(slots + (i * kRpi + lane / kCpr) * (RB + 16) + (lane % kCpr) * 16);
 }
 
+// Prefetches an RB-byte row and one gate value into L2.
+template <int RB, typename T>
+__device__ __forceinline__ void prefetch_row(const T* row, const __nv_bfloat16* zv) {
+#pragma unroll
+    for (int o = 0; o < RB; o += 128)
+        asm volatile("prefetch.global.L2 [%0];" ::"l"(reinterpret_cast<const uint8_t*>(row) + o));
+    asm volatile("prefetch.global.L2 [%0];" ::"l"(zv));
+}
+
 // Issues the eight K = 16 MMAs of one N = 128 part: D (+)= A[tmem] * B[stage].
 // `first_acc` is 0 when the first MMA starts a fresh accumulator.
 template <uint32_t kIdesc, uint32_t first_acc>
@@ -513,9 +522,14 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
         float s_next = nj > 0 ? __ldg(scl) : 0.0f;
         const uint32_t ua = tmem + lane_addr + kColU + (uint32_t)(kP * wg);
         const uint32_t va = tmem + lane_addr + kColV + (uint32_t)(kP * wg);  // + 128 per V buffer
+        // the merge's Y_ssd row and gate come from L2 if fetched a few jobs ahead
+        const i64 rowo_pf = tok * H + h;
+        const int pf_job = nj > 4 ? nj - 4 : 0;
+        if (nj == 0) prefetch_row<kP * (int)sizeof(Tout)>(Yssd + rowo_pf * kP, z + rowo_pf);
         for (int j = 0; j < nj; ++j) {
             const int ub = j & 1;
             const float s_j = s_next;
+            if (j == pf_job) prefetch_row<kP * (int)sizeof(Tout)>(Yssd + rowo_pf * kP, z + rowo_pf);
             if (j + 1 < nj) s_next = __ldg(scl + (i64)(j + 1) * H);  // one job ahead
             if (!warp_wait(&sm.uready[ub], (uint32_t)((j >> 1) & 1), wait_limit_ns, abort)) {
                 fail(abort, 4);
