@@ -55,8 +55,11 @@ def _load():
         lib.oracle_decode_step.argtypes = (
             [_i64] * 6 + [ctypes.c_double, _i64, _i64] + [_dp] * 13
         )
+        lib.oracle_ssd_backward.argtypes = [_i64] * 7 + [_dp] * 12
+        lib.oracle_sma_backward.argtypes = [_i64] * 7 + [ctypes.c_double] + [_dp] * 11
         for f in ("oracle_ssd_recurrence", "oracle_chunk_memories", "oracle_sma",
-                  "oracle_merge", "oracle_decode_step", "oracle_memory_inverse_rms"):
+                  "oracle_merge", "oracle_decode_step", "oracle_memory_inverse_rms",
+                  "oracle_ssd_backward", "oracle_sma_backward"):
             getattr(lib, f).restype = None
         _lib = lib
     return _lib
@@ -179,3 +182,51 @@ def forward(X, dt, A, Bm, Cm, Q, E, z, S: int, eps: float):
     R, lse = sma(dH, Q, Cm, E, S, eps)
     Y = merge(Yssd, z, R)
     return Yssd, dH, R, lse, Y
+
+
+def ssd_backward(X, dt, A, Bm, Cm, dY, dMem, S: int):
+    """Gradients of the SSD scan (chain rule on the token recurrence of Sec. 2 / App. A).
+
+    dY: gradient w.r.t. Y_ssd (``Bsz x L x H x P``); dMem: gradient w.r.t. the
+    chunk memories (``Bsz x M x H x N x P``) or None. Returns (dX, d_dt, dA, dB,
+    dC); dB and dC are summed over the heads of a group.
+    """
+    X, dt, A, Bm, Cm, dY = map(_f64, (X, dt, A, Bm, Cm, dY))
+    dMem = None if dMem is None else _f64(dMem)
+    Bsz, L, H, P = X.shape
+    G, N = Bm.shape[2], Bm.shape[3]
+    dX, ddt, dA = np.empty_like(X), np.empty_like(dt), np.empty_like(A)
+    dB, dC = np.empty_like(Bm), np.empty_like(Cm)
+    _load().oracle_ssd_backward(Bsz, L, H, G, P, N, S, _ptr(X), _ptr(dt), _ptr(A), _ptr(Bm),
+                                _ptr(Cm), _ptr(dY), _ptr(dMem), _ptr(dX), _ptr(ddt), _ptr(dA),
+                                _ptr(dB), _ptr(dC))
+    return dX, ddt, dA, dB, dC
+
+
+def sma_backward(dH, Q, Cm, E, z, dY, S: int, eps: float):
+    """Gradients of state-memory attention + gated merge (Sec. 3 / App. B.1) w.r.t.
+    the memories, Q, C, E and the gate logit z, for a loss gradient dY on
+    Y = Y_ssd + SiLU(z) R. Returns (dMem, dQ, dC, dE, dz); the gradient w.r.t.
+    Y_ssd is dY itself.
+    """
+    dH, Q, Cm, E, z, dY = map(_f64, (dH, Q, Cm, E, z, dY))
+    Bsz, M, H, N, P = dH.shape
+    L, G = Q.shape[1], Q.shape[2]
+    dMem, dQ, dC, dE = np.empty_like(dH), np.empty_like(Q), np.empty_like(Cm), np.empty_like(E)
+    dz = np.empty((Bsz, L, H))
+    _load().oracle_sma_backward(Bsz, L, H, G, P, N, S, float(eps), _ptr(dH), _ptr(Q), _ptr(Cm),
+                                _ptr(E), _ptr(z), _ptr(dY), _ptr(dMem), _ptr(dQ), _ptr(dC),
+                                _ptr(dE), _ptr(dz))
+    return dMem, dQ, dC, dE, dz
+
+
+def backward(X, dt, A, Bm, Cm, Q, E, z, dY, S: int, eps: float):
+    """Whole-layer backward for a loss gradient dY on Y: (dX, d_dt, dA, dB, dC, dQ, dE, dz).
+
+    The SMA backward's memory gradient feeds the scan backward, and dC sums
+    the SSD and SMA contributions.
+    """
+    dH = chunk_memories(X, dt, A, Bm, S)
+    dMem, dQ, dC_sma, dE, dz = sma_backward(dH, Q, Cm, E, z, dY, S, eps)
+    dX, ddt, dA, dB, dC_ssd = ssd_backward(X, dt, A, Bm, Cm, dY, dMem, S)
+    return dX, ddt, dA, dB, dC_ssd + dC_sma, dQ, dE, dz

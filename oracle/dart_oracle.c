@@ -341,3 +341,272 @@ void oracle_decode_step(i64 Bsz, i64 H, i64 G, i64 P, i64 N, i64 S, double eps,
         }
     }
 }
+
+/*
+ * Backward of the SSD scan (gradients of the paper's selective-SSM forms,
+ * Sec. 2 and App. A; the paper prints no backward, so this is the chain rule
+ * on the token recurrence, written out by hand).
+ * Outputs of the forward that a loss can depend on: Y_ssd (through dY, the
+ * same layout as Y) and the chunk memories dH_[c] (through dMem, the layout of
+ * oracle_chunk_memories; NULL means zero).
+ * Forward, per (b, h):  H_t = a_t H_{t-1} + u_t,  u_t = dt_t B_t^T X_t,
+ * a_t = exp(dt_t A_h), Y_t = C_t H_t; the memory of chunk c is the state of
+ * the same recurrence restarted from zero at the chunk's first token and
+ * read at its last token.
+ * Adjoints (reverse order over t): dH_t = C_t^T dY_t + a_{t+1} dH_{t+1};
+ * the chunk-local adjoint starts from dMem_[c] at the chunk's last token and
+ * dies at its first; du_t = dH_t + dHloc_t gives dX_t = dt_t B_t du_t,
+ * dB_t = dt_t du_t X_t, d(dt_t) = B_t du_t X_t; dC_t = H_t dY_t; the decay
+ * gives da_t = <dH_t, H_{t-1}> + <dHloc_t, Hloc_{t-1}>, d(dt_t) += A_h a_t
+ * da_t and dA_h += dt_t a_t da_t.
+ * dX (Bsz x L x H x P), ddt (Bsz x L x H), dA (H), dB, dC (Bsz x L x G x N,
+ * summed over the heads of a group). All outputs are overwritten.
+ * Pinned: central finite differences of a weighted sum of Y_ssd and the
+ * memories (tests/test_oracle_backward.py).
+ */
+void oracle_ssd_backward(i64 Bsz, i64 L, i64 H, i64 G, i64 P, i64 N, i64 S,
+                         const double* X, const double* dt, const double* A,
+                         const double* Bm, const double* Cm, const double* dY,
+                         const double* dMem, double* dX, double* ddt, double* dA,
+                         double* dB, double* dC)
+{
+    i64 M = (L + S - 1) / S;
+    i64 NP = N * P;
+    memset(dX, 0, (size_t)(Bsz * L * H * P) * sizeof(double));
+    memset(ddt, 0, (size_t)(Bsz * L * H) * sizeof(double));
+    memset(dA, 0, (size_t)H * sizeof(double));
+    memset(dB, 0, (size_t)(Bsz * L * G * N) * sizeof(double));
+    memset(dC, 0, (size_t)(Bsz * L * G * N) * sizeof(double));
+    /* heads of one group write the same dB, dC rows: parallel over b only */
+#pragma omp parallel for schedule(static)
+    for (i64 b = 0; b < Bsz; ++b) {
+        double* ckpt = (double*)calloc((size_t)(M * NP), sizeof(double));
+        double* Hg = (double*)malloc((size_t)(S * NP) * sizeof(double));
+        double* Hl = (double*)malloc((size_t)(S * NP) * sizeof(double));
+        double* dHg = (double*)malloc((size_t)NP * sizeof(double));
+        double* dHl = (double*)malloc((size_t)NP * sizeof(double));
+        for (i64 h = 0; h < H; ++h) {
+            i64 g = group_of(h, H, G);
+            /* forward once: the global state entering every chunk */
+            double* St = (double*)calloc((size_t)NP, sizeof(double));
+            for (i64 t = 0; t < L; ++t) {
+                if (t % S == 0) memcpy(ckpt + (t / S) * NP, St, (size_t)NP * sizeof(double));
+                double d = dt[(b * L + t) * H + h], a = exp(d * A[h]);
+                const double* Bt = Bm + ((b * L + t) * G + g) * N;
+                const double* Xt = X + ((b * L + t) * H + h) * P;
+                for (i64 n = 0; n < N; ++n)
+                    for (i64 p = 0; p < P; ++p)
+                        St[n * P + p] = a * St[n * P + p] + d * Bt[n] * Xt[p];
+            }
+            free(St);
+            double dAh = 0.0;
+            for (i64 i = 0; i < NP; ++i) dHg[i] = 0.0;
+            for (i64 c = M - 1; c >= 0; --c) {
+                i64 first = c * S, last = (c + 1) * S < L ? (c + 1) * S - 1 : L - 1;
+                /* recompute the chunk's global and local states */
+                for (i64 t = first; t <= last; ++t) {
+                    i64 k = t - first;
+                    double d = dt[(b * L + t) * H + h], a = exp(d * A[h]);
+                    const double* Bt = Bm + ((b * L + t) * G + g) * N;
+                    const double* Xt = X + ((b * L + t) * H + h) * P;
+                    const double* gprev = k > 0 ? Hg + (k - 1) * NP : ckpt + c * NP;
+                    for (i64 n = 0; n < N; ++n) {
+                        for (i64 p = 0; p < P; ++p) {
+                            double u = d * Bt[n] * Xt[p];
+                            Hg[k * NP + n * P + p] = a * gprev[n * P + p] + u;
+                            Hl[k * NP + n * P + p] = (k > 0 ? a * Hl[(k - 1) * NP + n * P + p] : 0.0) + u;
+                        }
+                    }
+                }
+                const double* dm = dMem ? dMem + ((b * M + c) * H + h) * NP : NULL;
+                for (i64 i = 0; i < NP; ++i) dHl[i] = dm ? dm[i] : 0.0;
+                for (i64 t = last; t >= first; --t) {
+                    i64 k = t - first;
+                    double d = dt[(b * L + t) * H + h], a = exp(d * A[h]);
+                    const double* Bt = Bm + ((b * L + t) * G + g) * N;
+                    const double* Ct = Cm + ((b * L + t) * G + g) * N;
+                    const double* Xt = X + ((b * L + t) * H + h) * P;
+                    const double* dYt = dY + ((b * L + t) * H + h) * P;
+                    double* dXt = dX + ((b * L + t) * H + h) * P;
+                    double* dBt = dB + ((b * L + t) * G + g) * N;
+                    double* dCt = dC + ((b * L + t) * G + g) * N;
+                    /* Y_t = C_t H_t */
+                    for (i64 n = 0; n < N; ++n) {
+                        double acc = 0.0;
+                        for (i64 p = 0; p < P; ++p) {
+                            dHg[n * P + p] += Ct[n] * dYt[p];
+                            acc += Hg[k * NP + n * P + p] * dYt[p];
+                        }
+                        dCt[n] += acc;
+                    }
+                    /* u_t = dt_t B_t^T X_t */
+                    double dd = 0.0;
+                    for (i64 n = 0; n < N; ++n) {
+                        double acc = 0.0;
+                        for (i64 p = 0; p < P; ++p) {
+                            double du = dHg[n * P + p] + dHl[n * P + p];
+                            acc += du * Xt[p];
+                            dXt[p] += d * Bt[n] * du;
+                        }
+                        dBt[n] += d * acc;
+                        dd += Bt[n] * acc;
+                    }
+                    /* a_t = exp(dt_t A_h) */
+                    const double* gprev = k > 0 ? Hg + (k - 1) * NP : ckpt + c * NP;
+                    double da = 0.0;
+                    for (i64 i = 0; i < NP; ++i) {
+                        da += dHg[i] * gprev[i];
+                        if (k > 0) da += dHl[i] * Hl[(k - 1) * NP + i];
+                    }
+                    ddt[(b * L + t) * H + h] = dd + A[h] * a * da;
+                    dAh += d * a * da;
+                    for (i64 i = 0; i < NP; ++i) {
+                        dHg[i] *= a;
+                        dHl[i] *= a;
+                    }
+                }
+            }
+#pragma omp atomic
+            dA[h] += dAh;
+        }
+        free(ckpt); free(Hg); free(Hl); free(dHg); free(dHl);
+    }
+}
+
+/*
+ * Backward of state-memory attention and the gated merge (Sec. 3 readouts,
+ * logit, softmax over earlier chunks, R_t and Y = Y_ssd + SiLU(z) R; App. B.1
+ * normalisations). The paper prints no backward; this is the chain rule on
+ * the plain per-token forms of oracle_sma, with the exact softmax Jacobian.
+ * For each (b, t, h) with history: dR = SiLU(z) dY, dz = (dY . R) SiLU'(z),
+ * dV_j = g_j dR, dl_j = g_j (dR . V_j - dR . R); through V_j = c dH_j and
+ * l_j = Qbar (r_j (.) dH_j Ebar) / sqrt(N) into dMem, dQbar, dEbar, dc, and
+ * through r_{j,n} = (mean_p dH_j[n,p]^2 + eps)^(-1/2) into dMem; the unit-
+ * weight RMSNorms take dQbar, dEbar back to dQ, dE. dY_ssd = dY and is not
+ * written here.
+ * dMem: Bsz x M x H x N x P; dQ, dC: Bsz x L x G x N; dE: Bsz x L x G x P
+ * (summed over the heads of a group); dz: Bsz x L x H. All overwritten.
+ * Pinned: central finite differences of a weighted sum of Y
+ * (tests/test_oracle_backward.py), and the closed form dz = dY . R / 2 at z = 0.
+ */
+void oracle_sma_backward(i64 Bsz, i64 L, i64 H, i64 G, i64 P, i64 N, i64 S, double eps,
+                         const double* dHm, const double* Q, const double* Cm, const double* E,
+                         const double* z, const double* dY, double* dMem, double* dQ,
+                         double* dC, double* dE, double* dz)
+{
+    i64 M = (L + S - 1) / S;
+    i64 NP = N * P;
+    memset(dMem, 0, (size_t)(Bsz * M * H * NP) * sizeof(double));
+    memset(dQ, 0, (size_t)(Bsz * L * G * N) * sizeof(double));
+    memset(dC, 0, (size_t)(Bsz * L * G * N) * sizeof(double));
+    memset(dE, 0, (size_t)(Bsz * L * G * P) * sizeof(double));
+    memset(dz, 0, (size_t)(Bsz * L * H) * sizeof(double));
+    double rsn = 1.0 / sqrt((double)N);
+#pragma omp parallel for schedule(static)
+    for (i64 b = 0; b < Bsz; ++b) {
+        double* qbar = (double*)malloc((size_t)N * sizeof(double));
+        double* ebar = (double*)malloc((size_t)P * sizeof(double));
+        double* r = (double*)malloc((size_t)(M * N) * sizeof(double));
+        double* Kraw = (double*)malloc((size_t)(M * N) * sizeof(double));
+        double* V = (double*)malloc((size_t)(M * P) * sizeof(double));
+        double* ell = (double*)malloc((size_t)M * sizeof(double));
+        double* gw = (double*)malloc((size_t)M * sizeof(double));
+        double* R = (double*)malloc((size_t)P * sizeof(double));
+        double* dqbar = (double*)malloc((size_t)N * sizeof(double));
+        double* debar = (double*)malloc((size_t)P * sizeof(double));
+        for (i64 h = 0; h < H; ++h) {
+            i64 g = group_of(h, H, G);
+            const double* mem0 = dHm + ((b * M) * H + h) * NP;
+            double* dmem0 = dMem + ((b * M) * H + h) * NP;
+            for (i64 j = 0; j < M; ++j) {
+                const double* D = mem0 + j * H * NP;
+                for (i64 n = 0; n < N; ++n) {
+                    double ss = 0.0;
+                    for (i64 p = 0; p < P; ++p) ss += D[n * P + p] * D[n * P + p];
+                    r[j * N + n] = 1.0 / sqrt(ss / (double)P + eps);
+                }
+            }
+            for (i64 t = 0; t < L; ++t) {
+                i64 nh = t / S;
+                if (nh == 0) continue;  /* R = 0: no gradient reaches this token's inputs */
+                const double* q = Q + ((b * L + t) * G + g) * N;
+                const double* c = Cm + ((b * L + t) * G + g) * N;
+                const double* e = E + ((b * L + t) * G + g) * P;
+                const double* dYt = dY + ((b * L + t) * H + h) * P;
+                rmsnorm(q, N, eps, qbar);
+                rmsnorm(e, P, eps, ebar);
+                /* forward: Kraw, l, V, two-pass softmax, R */
+                for (i64 j = 0; j < nh; ++j) {
+                    const double* D = mem0 + j * H * NP;
+                    double l = 0.0;
+                    for (i64 n = 0; n < N; ++n) {
+                        double ke = 0.0;
+                        for (i64 p = 0; p < P; ++p) ke += D[n * P + p] * ebar[p];
+                        Kraw[j * N + n] = ke;
+                        l += qbar[n] * r[j * N + n] * ke;
+                    }
+                    ell[j] = l * rsn;
+                    for (i64 p = 0; p < P; ++p) {
+                        double v = 0.0;
+                        for (i64 n = 0; n < N; ++n) v += c[n] * D[n * P + p];
+                        V[j * P + p] = v;
+                    }
+                }
+                double m = ell[0];
+                for (i64 j = 1; j < nh; ++j) if (ell[j] > m) m = ell[j];
+                double sum = 0.0;
+                for (i64 j = 0; j < nh; ++j) sum += exp(ell[j] - m);
+                for (i64 p = 0; p < P; ++p) R[p] = 0.0;
+                for (i64 j = 0; j < nh; ++j) {
+                    gw[j] = exp(ell[j] - m) / sum;
+                    for (i64 p = 0; p < P; ++p) R[p] += gw[j] * V[j * P + p];
+                }
+                /* merge: Y = Y_ssd + SiLU(z) R */
+                double zz = z[(b * L + t) * H + h];
+                double sg = 1.0 / (1.0 + exp(-zz));
+                double gate = zz * sg;
+                double dyr = 0.0;
+                for (i64 p = 0; p < P; ++p) dyr += dYt[p] * R[p];
+                dz[(b * L + t) * H + h] = dyr * sg * (1.0 + zz * (1.0 - sg));
+                /* softmax and readouts */
+                double Dt = gate * dyr;  /* dR . R */
+                for (i64 n = 0; n < N; ++n) dqbar[n] = 0.0;
+                for (i64 p = 0; p < P; ++p) debar[p] = 0.0;
+                double* dCt = dC + ((b * L + t) * G + g) * N;
+                for (i64 j = 0; j < nh; ++j) {
+                    const double* D = mem0 + j * H * NP;
+                    double* dD = dmem0 + j * H * NP;
+                    double drv = 0.0;
+                    for (i64 p = 0; p < P; ++p) drv += gate * dYt[p] * V[j * P + p];
+                    double dl = gw[j] * (drv - Dt);
+                    for (i64 n = 0; n < N; ++n) {
+                        double rn = r[j * N + n];
+                        double dkr = rsn * dl * qbar[n] * rn;          /* d Kraw[n] */
+                        double dr = rsn * dl * qbar[n] * Kraw[j * N + n]; /* d r[n] */
+                        dqbar[n] += rsn * dl * rn * Kraw[j * N + n];
+                        double acc = 0.0;
+                        for (i64 p = 0; p < P; ++p) {
+                            double dv = gw[j] * gate * dYt[p];
+                            acc += D[n * P + p] * dv;
+                            dD[n * P + p] += c[n] * dv + dkr * ebar[p]
+                                             - dr * rn * rn * rn * D[n * P + p] / (double)P;
+                            debar[p] += D[n * P + p] * dkr;
+                        }
+                        dCt[n] += acc;
+                    }
+                }
+                /* unit-weight RMSNorm backward: dx = s (dxbar - xbar (dxbar . xbar) / n) */
+                double sq = 0.0, se = 0.0, dq_dot = 0.0, de_dot = 0.0;
+                for (i64 n = 0; n < N; ++n) { sq += q[n] * q[n]; dq_dot += dqbar[n] * qbar[n]; }
+                for (i64 p = 0; p < P; ++p) { se += e[p] * e[p]; de_dot += debar[p] * ebar[p]; }
+                double s_q = 1.0 / sqrt(sq / (double)N + eps), s_e = 1.0 / sqrt(se / (double)P + eps);
+                double* dQt = dQ + ((b * L + t) * G + g) * N;
+                double* dEt = dE + ((b * L + t) * G + g) * P;
+                for (i64 n = 0; n < N; ++n) dQt[n] += s_q * (dqbar[n] - qbar[n] * dq_dot / (double)N);
+                for (i64 p = 0; p < P; ++p) dEt[p] += s_e * (debar[p] - ebar[p] * de_dot / (double)P);
+            }
+        }
+        free(qbar); free(ebar); free(r); free(Kraw); free(V); free(ell); free(gw); free(R);
+        free(dqbar); free(debar);
+    }
+}
