@@ -14,6 +14,10 @@
  *                     Y = Y_ssd + SiLU(z) R (Sec. 3).
  *   dart_decode_step  one autoregressive token over the chunk-memory cache
  *                     and the running state (Sec. 4 "Inference Cache").
+ *   dart_sma_backward, dart_chunk_scan_backward
+ *                     gradients of the two prefill calls for training (the
+ *                     paper trains the layer end to end but prints no
+ *                     backward; these are the chain rule on the forms above).
  *
  * Conventions shared by every entry point
  *   - Every tensor pointer is a DEVICE pointer owned by the caller, 16-byte
@@ -87,7 +91,9 @@ typedef struct {
 typedef enum {
     DART_OP_CHUNK_SCAN = 0,
     DART_OP_SMA_FORWARD = 1,
-    DART_OP_DECODE_STEP = 2
+    DART_OP_DECODE_STEP = 2,
+    DART_OP_SMA_BACKWARD = 3,
+    DART_OP_SCAN_BACKWARD = 4
 } dart_op;
 
 /* Human-readable name of a status code (static storage, never NULL). */
@@ -135,8 +141,8 @@ dart_status dart_chunk_scan(const dart_dims* dims, const void* X, const float* d
  *          lse (Bsz, L, H) fp32 or NULL.
  * Workspace: dart_workspace_size(dims, DART_OP_SMA_FORWARD) bytes. Always
  *          needed on the tensor-core path (bf16 inputs, P = 64, N = 128,
- *          S % 128 == 0, H / G a multiple of 4), where it holds each memory's
- *          MMA operands (48 KiB per memory and head); elsewhere only when rM is
+ *          S % 128 == 0, H / G even), where it holds each memory's MMA
+ *          operands (48 KiB per memory and head); elsewhere only when rM is
  *          NULL (for r).
  */
 dart_status dart_sma_forward(const dart_dims* dims, const void* M, const float* rM,
@@ -167,6 +173,57 @@ dart_status dart_decode_step(const dart_dims* dims, int64_t pos, int64_t m_cap, 
                              const float* A, const void* b, const void* c, const void* q,
                              const void* e, const void* z, void* y, float* lse,
                              void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * Backward of dart_sma_forward (training). Chain rule on the forward above,
+ * with the saved lse as the softmax normaliser: per token t with history and
+ * memory j,
+ *   dR_t = SiLU(z_t) dY_t,  g_{t,j} = exp(l_{t,j} - lse_t),
+ *   dl_{t,j} = g_{t,j} (dR_t . V_{t,j} - dR_t . R_t),  dV_{t,j} = g_{t,j} dR_t,
+ * then through V = C M_j, l = Qbar (r_j (.) M_j Ebar) / sqrt(N), r_j(M_j) and
+ * the unit-weight RMSNorms to dM, dQ, dC, dE; dz_t = (dY_t . R_t) SiLU'(z_t).
+ * The gradient w.r.t. Y_ssd is dY itself and is not written.
+ * Inputs:  M, rM (or NULL), Q, Cm, E, z as for dart_sma_forward (rM, when
+ *          given, must be the one the forward used); lse (Bsz, L, H) fp32 as
+ *          written by dart_sma_forward; dY (Bsz, L, H, P) in_dtype.
+ * Outputs: fp32, overwritten: dM (Bsz, M, H, N, P); dQ, dC (Bsz, L, G, N);
+ *          dE (Bsz, L, G, P); dz (Bsz, L, H). dQ, dC and dE are summed over
+ *          the heads of a group with fp32 atomics, so their low bits vary from
+ *          run to run.
+ * Workspace: dart_workspace_size(dims, DART_OP_SMA_BACKWARD): the weights g and
+ *          logit gradients dl of every (memory, token) pair, 2 x Bsz x H x M x L
+ *          fp32, plus r when rM is NULL.
+ */
+dart_status dart_sma_backward(const dart_dims* dims, const void* M, const float* rM,
+                              const void* Q, const void* Cm, const void* E, const void* z,
+                              const float* lse, const void* dY, float* dM, float* dQ, float* dC,
+                              float* dE, float* dz, void* workspace, size_t workspace_bytes,
+                              void* stream);
+
+/*
+ * Backward of dart_chunk_scan (training): gradients of a loss that depends on
+ * Y_ssd (through dY) and on the chunk memories (through dM, e.g. the output of
+ * dart_sma_backward). Chain rule on the chunked forms of App. A: the states
+ * entering each chunk are recomputed, the adjoint of the inter-chunk state runs
+ * backwards over the chunks, and each chunk's intra-chunk, inter-chunk and
+ * memory terms give dX, dB, dC and the gradient of the within-chunk decay,
+ * which a reverse cumulative sum turns into d(dt) and dA.
+ * Inputs:  X, dt, A, Bm, Cm as for dart_chunk_scan; dY (Bsz, L, H, P) in_dtype;
+ *          dM (Bsz, M, H, N, P) fp32 or NULL (no memory gradient).
+ * Outputs: fp32. Overwritten: dX (Bsz, L, H, P), ddt (Bsz, L, H), dA (H),
+ *          dB (Bsz, L, G, N). ACCUMULATED: dC (Bsz, L, G, N) gets the scan's
+ *          part added, so the SMA part from dart_sma_backward can be passed in
+ *          (zero it first otherwise). dA, dB and dC are sums over heads or
+ *          tokens taken with fp32 atomics.
+ * Workspace: dart_workspace_size(dims, DART_OP_SCAN_BACKWARD): the within-chunk
+ *          cumulative decay, the state entering each chunk and the memory
+ *          adjoints (2 x Bsz x M x H x N x P fp32).
+ */
+dart_status dart_chunk_scan_backward(const dart_dims* dims, const void* X, const float* dt,
+                                     const float* A, const void* Bm, const void* Cm,
+                                     const void* dY, const float* dM, float* dX, float* ddt,
+                                     float* dA, float* dB, float* dC, void* workspace,
+                                     size_t workspace_bytes, void* stream);
 
 /*
  * dart_sma_forward_noalloc: dart_sma_forward with rM = NULL, for callers that

@@ -97,3 +97,61 @@ def decode_step(cache, state, partial, x, dt, A, b, c, q, e, z, pos: int, chunk:
     lse = torch.empty(Bsz, H, dtype=torch.float32, device=x.device)
     B.dart_decode_step(dims, pos, m_cap, cache, state, partial, x, dt, A, b, c, q, e, z, y, lse)
     return y, lse
+
+
+@dataclass
+class LayerGrads:
+    dX: torch.Tensor    # (Bsz, L, H, P) fp32
+    ddt: torch.Tensor   # (Bsz, L, H) fp32
+    dA: torch.Tensor    # (H,) fp32
+    dB: torch.Tensor    # (Bsz, L, G, N) fp32
+    dC: torch.Tensor    # (Bsz, L, G, N) fp32, SSD + SMA parts
+    dQ: torch.Tensor    # (Bsz, L, G, N) fp32
+    dE: torch.Tensor    # (Bsz, L, G, P) fp32
+    dz: torch.Tensor    # (Bsz, L, H) fp32
+    dM: torch.Tensor    # (Bsz, M, H, N, P) fp32 gradient of the chunk memories
+
+
+def sma_backward(Mem, rM, Q, Cm, E, z, lse, dY, chunk: int, eps: float = 1e-6,
+                 workspace: torch.Tensor | None = None):
+    """Backward of ``sma_forward`` (``dart_sma_backward``): (dM, dQ, dC, dE, dz), all fp32."""
+    Bsz, L, H, P = dY.shape
+    G, N = Q.shape[2], Q.shape[3]
+    dims = B.make_dims(Bsz, L, H, G, P, N, chunk, _dtype_code(Q), _dtype_code(Mem),
+                       B.DART_F32, eps=eps)
+    dev = dY.device
+    f32 = dict(dtype=torch.float32, device=dev)
+    dM = torch.empty(Mem.shape, **f32)
+    dQ, dC, dE = torch.empty(Q.shape, **f32), torch.empty(Cm.shape, **f32), torch.empty(E.shape, **f32)
+    dz = torch.empty(Bsz, L, H, **f32)
+    ws = workspace if workspace is not None else _workspace(dims, B.DART_OP_SMA_BACKWARD, dev)
+    B.dart_sma_backward(dims, Mem, rM, Q, Cm, E, z, lse, dY, dM, dQ, dC, dE, dz, ws)
+    return dM, dQ, dC, dE, dz
+
+
+def chunk_scan_backward(X, dt, A, Bm, Cm, dY, dM, chunk: int, dC=None, eps: float = 1e-6,
+                        workspace: torch.Tensor | None = None):
+    """Backward of ``chunk_scan`` (``dart_chunk_scan_backward``): (dX, ddt, dA, dB, dC), fp32.
+
+    ``dC``, when given (fp32), is accumulated into (e.g. the SMA part); else it starts at zero.
+    """
+    Bsz, L, H, P = X.shape
+    G, N = Bm.shape[2], Bm.shape[3]
+    dims = B.make_dims(Bsz, L, H, G, P, N, chunk, _dtype_code(X), B.DART_F32, B.DART_F32, eps=eps)
+    dev = X.device
+    f32 = dict(dtype=torch.float32, device=dev)
+    dX, ddt, dA = torch.empty(X.shape, **f32), torch.empty(dt.shape, **f32), torch.empty(A.shape, **f32)
+    dB = torch.empty(Bm.shape, **f32)
+    dC = torch.zeros(Cm.shape, **f32) if dC is None else dC
+    ws = workspace if workspace is not None else _workspace(dims, B.DART_OP_SCAN_BACKWARD, dev)
+    B.dart_chunk_scan_backward(dims, X, dt, A, Bm, Cm, dY, dM, dX, ddt, dA, dB, dC, ws)
+    return dX, ddt, dA, dB, dC
+
+
+def layer_backward(X, dt, A, Bm, Cm, Q, E, z, dY, scan: ScanOut, sma: SmaOut, chunk: int,
+                   eps: float = 1e-6) -> LayerGrads:
+    """Backward of ``prefill_forward`` for a loss gradient dY on Y: SMA backward, whose
+    memory gradient and dC feed the scan backward."""
+    dM, dQ, dC, dE, dz = sma_backward(scan.M, scan.rM, Q, Cm, E, z, sma.lse, dY, chunk, eps)
+    dX, ddt, dA, dB, dC = chunk_scan_backward(X, dt, A, Bm, Cm, dY, dM, chunk, dC=dC, eps=eps)
+    return LayerGrads(dX, ddt, dA, dB, dC, dQ, dE, dz, dM)

@@ -20,6 +20,7 @@ LIB_PATH = os.path.join(_PKG, "libdart.so")
 DART_OK = 0
 DART_F32, DART_BF16 = 0, 1
 DART_OP_CHUNK_SCAN, DART_OP_SMA_FORWARD, DART_OP_DECODE_STEP = 0, 1, 2
+DART_OP_SMA_BACKWARD, DART_OP_SCAN_BACKWARD = 3, 4
 STATUS_NAMES = {0: "DART_OK", 1: "DART_ERR_INVALID_ARG", 2: "DART_ERR_UNSUPPORTED",
                 3: "DART_ERR_WORKSPACE", 4: "DART_ERR_CUDA", 5: "DART_ERR_TIMEOUT",
                 6: "DART_ERR_TOO_LARGE"}
@@ -29,7 +30,8 @@ DART_DTYPE = {torch.float32: DART_F32, torch.bfloat16: DART_BF16}
 
 EXPORTED = ("dart_status_string", "dart_last_cuda_error", "dart_workspace_size",
             "dart_chunk_scan", "dart_sma_forward", "dart_decode_step", "dart_sma_forward_noalloc",
-            "dart_launch_count", "dart_set_wait_limit_ns", "dart_get_device_status")
+            "dart_launch_count", "dart_set_wait_limit_ns", "dart_get_device_status",
+            "dart_sma_backward", "dart_chunk_scan_backward")
 
 
 class DartError(RuntimeError):
@@ -93,6 +95,11 @@ def lib() -> ctypes.CDLL:
         L.dart_set_wait_limit_ns.argtypes = [ctypes.c_uint64]
         L.dart_get_device_status.restype = ctypes.c_int
         L.dart_get_device_status.argtypes = [_vp]
+        L.dart_get_device_status.restype = ctypes.c_int
+        L.dart_sma_backward.argtypes = [dp] + [_vp] * 14 + [ctypes.c_size_t, _vp]
+        L.dart_sma_backward.restype = ctypes.c_int
+        L.dart_chunk_scan_backward.argtypes = [dp] + [_vp] * 13 + [ctypes.c_size_t, _vp]
+        L.dart_chunk_scan_backward.restype = ctypes.c_int
         _lib = L
     return _lib
 
@@ -170,6 +177,24 @@ def dart_decode_step(dims, pos, m_cap, cache, state, partial, x, dt, A, b, c, q,
         _ptr(partial, "partial"), _ptr(x, "x"), _ptr(dt, "dt"), _ptr(A, "A"), _ptr(b, "b"),
         _ptr(c, "c"), _ptr(q, "q"), _ptr(e, "e"), _ptr(z, "z"), _ptr(y, "y"), _ptr(lse, "lse"),
         w, nb, _stream(stream)))
+
+
+def dart_sma_backward(dims, M, rM, Q, Cm, E, z, lse, dY, dM, dQ, dC, dE, dz, workspace=None,
+                      stream=None) -> None:
+    w, nb = _ws(workspace)
+    _check("dart_sma_backward", lib().dart_sma_backward(
+        ctypes.byref(dims), _ptr(M, "M"), _ptr(rM, "rM"), _ptr(Q, "Q"), _ptr(Cm, "Cm"),
+        _ptr(E, "E"), _ptr(z, "z"), _ptr(lse, "lse"), _ptr(dY, "dY"), _ptr(dM, "dM"),
+        _ptr(dQ, "dQ"), _ptr(dC, "dC"), _ptr(dE, "dE"), _ptr(dz, "dz"), w, nb, _stream(stream)))
+
+
+def dart_chunk_scan_backward(dims, X, dt, A, Bm, Cm, dY, dM, dX, ddt, dA, dB, dC, workspace=None,
+                             stream=None) -> None:
+    w, nb = _ws(workspace)
+    _check("dart_chunk_scan_backward", lib().dart_chunk_scan_backward(
+        ctypes.byref(dims), _ptr(X, "X"), _ptr(dt, "dt"), _ptr(A, "A"), _ptr(Bm, "Bm"),
+        _ptr(Cm, "Cm"), _ptr(dY, "dY"), _ptr(dM, "dM"), _ptr(dX, "dX"), _ptr(ddt, "ddt"),
+        _ptr(dA, "dA"), _ptr(dB, "dB"), _ptr(dC, "dC"), w, nb, _stream(stream)))
 
 
 def dart_get_device_status(stream=None) -> None:

@@ -165,6 +165,14 @@ size_t dart_workspace_size(const dart_dims* d, int op) {
             return sma_ws(d);
         case DART_OP_DECODE_STEP:
             return 0;
+        case DART_OP_SMA_BACKWARD:
+            if (check_dims(d, true) != DART_OK) return 0;
+            return align256(dart::sma_bwd_workspace(d->batch, d->seqlen, d->nheads,
+                                                    d->seqlen / d->chunk, d->dstate));
+        case DART_OP_SCAN_BACKWARD:
+            if (check_dims(d, true) != DART_OK) return 0;
+            return align256(dart::scan_bwd_workspace(d->batch, d->seqlen, d->nheads, d->dstate,
+                                                     d->headdim, d->chunk));
     }
     return 0;
 }
@@ -283,6 +291,68 @@ dart_status dart_decode_step(const dart_dims* d, int64_t pos, int64_t m_cap, voi
     cudaStream_t s = (cudaStream_t)stream;
     cudaError_t err = dispatch<DecodeL>(d, a, s);
     return err == cudaSuccess ? DART_OK : cuda_fail(err);
+}
+
+dart_status dart_sma_backward(const dart_dims* d, const void* M, const float* rM, const void* Q,
+                              const void* Cm, const void* E, const void* z, const float* lse,
+                              const void* dY, float* dM, float* dQ, float* dC, float* dE,
+                              float* dz, void* ws, size_t ws_bytes, void* stream) {
+    dart_status st = check_dims(d, true);
+    if (st != DART_OK) return st;
+    const void* req[] = {M, Q, Cm, E, z, lse, dY, dM, dQ, dC, dE, dz};
+    for (const void* p : req)
+        if (p == nullptr || !aligned16(p)) return DART_ERR_INVALID_ARG;
+    if (rM != nullptr && !aligned16(rM)) return DART_ERR_INVALID_ARG;
+    const size_t need = dart_workspace_size(d, DART_OP_SMA_BACKWARD);
+    if (ws == nullptr || ((uintptr_t)ws & 255u) != 0 || ws_bytes < need) return DART_ERR_WORKSPACE;
+    dart::SmaBwdArgs a;
+    a.B = d->batch; a.L = d->seqlen; a.H = d->nheads; a.G = d->ngroups;
+    a.P = d->headdim; a.N = d->dstate; a.S = d->chunk; a.eps = d->eps;
+    a.M = M; a.rM = rM; a.Q = Q; a.Cm = Cm; a.E = E; a.z = z; a.lse = lse; a.dY = dY;
+    a.dM = dM; a.dQ = dQ; a.dC = dC; a.dE = dE; a.dz = dz;
+    cudaStream_t s = (cudaStream_t)stream;
+    typedef __nv_bfloat16 bf;
+    cudaError_t e;
+    if (d->in_dtype == DART_F32 && d->mem_dtype == DART_F32)
+        e = dart::launch_sma_backward<float, float>(a, ws, s);
+    else if (d->in_dtype == DART_BF16 && d->mem_dtype == DART_F32)
+        e = dart::launch_sma_backward<bf, float>(a, ws, s);
+    else if (d->in_dtype == DART_BF16 && d->mem_dtype == DART_BF16)
+        e = dart::launch_sma_backward<bf, bf>(a, ws, s);
+    else
+        return DART_ERR_UNSUPPORTED;
+    return e == cudaSuccess ? DART_OK : cuda_fail(e);
+}
+
+dart_status dart_chunk_scan_backward(const dart_dims* d, const void* X, const float* dt,
+                                     const float* A, const void* Bm, const void* Cm,
+                                     const void* dY, const float* dM, float* dX, float* ddt,
+                                     float* dA, float* dB, float* dC, void* ws, size_t ws_bytes,
+                                     void* stream) {
+    dart_status st = check_dims(d, true);
+    if (st != DART_OK) return st;
+    const void* req[] = {X, dt, A, Bm, Cm, dY, dX, ddt, dA, dB, dC};
+    for (const void* p : req)
+        if (p == nullptr || !aligned16(p)) return DART_ERR_INVALID_ARG;
+    if (dM != nullptr && !aligned16(dM)) return DART_ERR_INVALID_ARG;
+    const size_t need = dart_workspace_size(d, DART_OP_SCAN_BACKWARD);
+    if (ws == nullptr || ((uintptr_t)ws & 255u) != 0 || ws_bytes < need) return DART_ERR_WORKSPACE;
+    dart::ScanBwdArgs a{};
+    dart::ScanArgs& f = a.fwd;
+    f.B = d->batch; f.L = d->seqlen; f.H = d->nheads; f.G = d->ngroups;
+    f.P = d->headdim; f.N = d->dstate; f.S = d->chunk; f.eps = d->eps;
+    f.X = X; f.dt = dt; f.A = A; f.Bm = Bm; f.Cm = Cm;
+    a.dY = dY; a.dM = dM; a.dX = dX; a.ddt = ddt; a.dA = dA; a.dB = dB; a.dC = dC;
+    a.accumulate_dC = true;
+    cudaStream_t s = (cudaStream_t)stream;
+    cudaError_t e;
+    if (d->in_dtype == DART_F32)
+        e = dart::launch_chunk_scan_backward<float>(a, ws, s);
+    else if (d->in_dtype == DART_BF16)
+        e = dart::launch_chunk_scan_backward<__nv_bfloat16>(a, ws, s);
+    else
+        return DART_ERR_UNSUPPORTED;
+    return e == cudaSuccess ? DART_OK : cuda_fail(e);
 }
 
 dart_status dart_get_device_status(void* stream) {

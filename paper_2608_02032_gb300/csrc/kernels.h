@@ -65,6 +65,52 @@ struct DecodeArgs {
     float* lse;
 };
 
+// Backward of SMA + merge (sma_bwd.cu). Gradients are fp32.
+struct SmaBwdArgs {
+    int64_t B, L, H, G, P, N, S;
+    float eps;
+    const void* M;
+    const float* rM;  // nullptr: recomputed into the workspace
+    const void* Q;
+    const void* Cm;
+    const void* E;
+    const void* z;
+    const float* lse;
+    const void* dY;
+    float* dM;  // B x Mc x H x N x P (overwritten)
+    float* dQ;  // B x L x G x N (overwritten)
+    float* dC;  // B x L x G x N (overwritten)
+    float* dE;  // B x L x G x P (overwritten)
+    float* dz;  // B x L x H (overwritten)
+};
+
+// Backward of the chunked scan (scan_bwd.cu). Gradients are fp32.
+struct ScanBwdArgs {
+    ScanArgs fwd;      // sizes and the forward inputs X, dt, A, Bm, Cm
+    const void* dY;    // gradient w.r.t. Y_ssd, input dtype
+    const float* dM;   // gradient w.r.t. the chunk memories (fp32) or nullptr
+    float* dX;         // B x L x H x P (overwritten)
+    float* ddt;        // B x L x H (overwritten)
+    float* dA;         // H (overwritten)
+    float* dB;         // B x L x G x N (overwritten)
+    float* dC;         // B x L x G x N (accumulated into when accumulate_dC)
+    bool accumulate_dC;
+};
+
+size_t sma_bwd_workspace(int64_t B, int64_t L, int64_t H, int64_t Mc, int64_t N);
+template <typename Tin, typename Tmem>
+cudaError_t launch_sma_backward(const SmaBwdArgs& a, void* ws, cudaStream_t stream);
+
+size_t scan_bwd_workspace(int64_t B, int64_t L, int64_t H, int64_t N, int64_t P, int64_t S);
+template <typename Tin>
+cudaError_t launch_chunk_scan_backward(const ScanBwdArgs& a, void* ws, cudaStream_t stream);
+// Forward steps 1-3 of the scan (cumsum, chunk states, state passing) for the
+// backward: cum and the states entering each chunk, with scratch (fp32, the
+// size of the memories) for the chunk-state kernel's memory output.
+template <typename Tin>
+cudaError_t launch_scan_states(const ScanArgs& a, float* cum, float* Hprev, float* scratch,
+                               cudaStream_t stream);
+
 // Kernels launched by the library (read by dart_launch_count()).
 void note_launches(int n);
 

@@ -130,7 +130,7 @@ chunk_state_kernel(const Tin* __restrict__ X, const float* __restrict__ dt,
             for (int i = tid; i < 64; i += 256) {
                 const int n = nt + i;
                 if (n < N)
-                    rM[(((i64)b * M + c) * H + h) * N + n] = rsqrtf(sSq[i] / (float)P + eps);
+                    rM[(((i64)b * M + c) * H + h) * N + n] = __frsqrt_rn(sSq[i] / (float)P + eps);
             }
         }
         __syncthreads();
@@ -342,7 +342,29 @@ cudaError_t launch_chunk_scan_simt(const ScanArgs& a, cudaStream_t stream) {
     return cudaGetLastError();
 }
 
+template <typename Tin>
+cudaError_t launch_scan_states(const ScanArgs& a0, float* cum, float* Hprev, float* scratch,
+                               cudaStream_t stream) {
+    ScanArgs a = a0;
+    a.cum = cum;
+    a.dH32 = Hprev;
+    a.M = scratch;
+    a.rM = nullptr;
+    a.final_state = nullptr;
+    const int L = (int)a.L, H = (int)a.H, G = (int)a.G, P = (int)a.P, N = (int)a.N,
+              S = (int)a.S, M = L / S;
+    cudaError_t e = launch_chunk_cumsum(a, stream);
+    if (e != cudaSuccess) return e;
+    chunk_state_kernel<Tin, float><<<dim3(M, H, (int)a.B), 256, 0, stream>>>(
+        (const Tin*)a.X, a.dt, a.cum, (const Tin*)a.Bm, a.dH32, scratch, nullptr, L, H, G, P, N, S,
+        M, a.eps);
+    note_launches(1);
+    return launch_state_passing(a, stream);
+}
+
 typedef __nv_bfloat16 bf16;
+template cudaError_t launch_scan_states<float>(const ScanArgs&, float*, float*, float*, cudaStream_t);
+template cudaError_t launch_scan_states<bf16>(const ScanArgs&, float*, float*, float*, cudaStream_t);
 template cudaError_t launch_chunk_scan_simt<float, float, float>(const ScanArgs&, cudaStream_t);
 template cudaError_t launch_chunk_scan_simt<bf16, float, float>(const ScanArgs&, cudaStream_t);
 template cudaError_t launch_chunk_scan_simt<bf16, bf16, float>(const ScanArgs&, cudaStream_t);

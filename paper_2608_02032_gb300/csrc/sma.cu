@@ -31,7 +31,7 @@ __global__ void memory_rms_kernel(const Tmem* __restrict__ M, float* __restrict_
         ss = fmaf(v, v, ss);
     }
     for (int off = 16; off > 0; off >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, off);
-    if (lane == 0) rM[row] = rsqrtf(ss / (float)P + eps);
+    if (lane == 0) rM[row] = __frsqrt_rn(ss / (float)P + eps);
 }
 
 template <typename Tmem>
@@ -94,8 +94,8 @@ sma_forward_simt_kernel(const Tmem* __restrict__ Mem, const float* __restrict__ 
             ssq += __shfl_xor_sync(0xffffffffu, ssq, off);
             sse += __shfl_xor_sync(0xffffffffu, sse, off);
         }
-        const float iq = rsqrtf(ssq / (float)N + eps);
-        const float ie = rsqrtf(sse / (float)P + eps);
+        const float iq = __frsqrt_rn(ssq / (float)N + eps);
+        const float ie = __frsqrt_rn(sse / (float)P + eps);
         for (int n = lane; n < N; n += 32) {
             sQt[n * kTT + r] = ok ? ld_f32(q + n) * iq : 0.0f;
             sCt[n * kTT + r] = ok ? ld_f32(c + n) : 0.0f;
@@ -107,7 +107,7 @@ sma_forward_simt_kernel(const Tmem* __restrict__ Mem, const float* __restrict__ 
 #pragma unroll
     for (int i = 0; i < 4; ++i) nh[i] = (t0 + ty * 4 + i) / S;  // memories each row attends to
     const int nh_max = (t0 + ntok - 1) / S;
-    const float inv_sqrt_n = rsqrtf((float)N);
+    const float inv_sqrt_n = __frsqrt_rn((float)N);
 
     float O[4][4] = {}, m[4], d[4];
 #pragma unroll

@@ -105,6 +105,13 @@ def prefill_inputs(w: Workload, with_grad: bool = False) -> dict:
     return out
 
 
+def memory_grad_input(w: Workload, scale: float = 0.1) -> torch.Tensor:
+    """Seeded gradient w.r.t. the chunk memories, ``B x M x H x N x P`` fp32 ~ N(0, scale^2)
+    (drawn from its own generator, seed + 7919, after nothing else)."""
+    g = torch.Generator().manual_seed(w.seed + 7919)
+    return scale * torch.randn(w.batch, w.nchunks, w.heads, w.dstate, w.headdim, generator=g)
+
+
 def decode_token_inputs(w: Workload) -> dict:
     """Seeded per-token decode inputs: x, dt, A, b, c, q, e, z (CPU fp32)."""
     g = torch.Generator().manual_seed(w.seed)

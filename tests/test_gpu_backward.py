@@ -1,0 +1,106 @@
+"""Parity of the backward entry points (dart_chunk_scan_backward,
+dart_sma_backward) against the fp64 oracle's hand-derived backward, which the
+CPU tests pin by finite differences. Inputs come from the seeded generators;
+expected values from the oracle on the same (bf16-rounded) inputs."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from helpers import TOL, dev, host, rel_err
+from paper_2608_02032_gb300 import api
+from paper_2608_02032_gb300.workloads import WORKLOADS, Workload, memory_grad_input, prefill_inputs
+
+pytestmark = pytest.mark.gpu
+
+CASES = [
+    WORKLOADS["tiny_fp32"],
+    Workload("bwd_f32_s32_g2", 1, 4, 256, 32, 32, 32, groups=2, dtype="f32", seed=2101),
+    Workload("bwd_f32_s16", 2, 2, 128, 16, 16, 16, dtype="f32", seed=2102),
+    Workload("bwd_bf16_s128", 1, 4, 512, 64, 128, 128, seed=2103),
+    Workload("bwd_bf16_s256", 2, 4, 1024, 64, 128, 256, seed=2104),
+]
+
+
+def _tol(w):
+    return TOL[w.dtype]
+
+
+@pytest.mark.parametrize("w", CASES, ids=lambda w: w.name)
+def test_scan_backward_matches_oracle(w):
+    inp = prefill_inputs(w, with_grad=True)
+    dMem = memory_grad_input(w)
+    ref = oracle.ssd_backward(inp["X"], inp["dt"], inp["A"], inp["Bm"], inp["Cm"], inp["dY"],
+                              dMem, w.chunk)
+    X, Bm, Cm, dY = (dev(inp[k], w.dtype) for k in ("X", "Bm", "Cm", "dY"))
+    dt, A = dev(inp["dt"], torch.float32), dev(inp["A"], torch.float32)
+    got = api.chunk_scan_backward(X, dt, A, Bm, Cm, dY, dev(dMem, torch.float32), w.chunk, eps=w.eps)
+    torch.cuda.synchronize()
+    errs = {name: rel_err(host(g), r) for name, g, r in zip(["dX", "ddt", "dA", "dB", "dC"], got, ref)}
+    print(w.name, {k: f"{v:.2e}" for k, v in errs.items()})
+    for name, err in errs.items():
+        assert err <= _tol(w), f"{name}: {err:.3e}"
+
+
+def test_scan_backward_accumulates_into_dC_and_takes_no_memory_gradient():
+    w = WORKLOADS["tiny_fp32"]
+    inp = prefill_inputs(w, with_grad=True)
+    ref = oracle.ssd_backward(inp["X"], inp["dt"], inp["A"], inp["Bm"], inp["Cm"], inp["dY"],
+                              None, w.chunk)
+    X, Bm, Cm, dY = (dev(inp[k], "f32") for k in ("X", "Bm", "Cm", "dY"))
+    dt, A = dev(inp["dt"], torch.float32), dev(inp["A"], torch.float32)
+    base = torch.full(Cm.shape, 0.25, dtype=torch.float32, device="cuda")
+    got = api.chunk_scan_backward(X, dt, A, Bm, Cm, dY, None, w.chunk, dC=base.clone())
+    torch.cuda.synchronize()
+    assert rel_err(host(got[4]) - 0.25, ref[4]) <= TOL["f32"]
+    assert rel_err(host(got[0]), ref[0]) <= TOL["f32"]
+
+
+@pytest.mark.parametrize("w", CASES, ids=lambda w: w.name)
+def test_sma_backward_matches_oracle(w):
+    """Memories and lse from the oracle, so the check covers the backward alone."""
+    inp = prefill_inputs(w, with_grad=True)
+    D = oracle.chunk_memories(inp["X"], inp["dt"], inp["A"], inp["Bm"], w.chunk)
+    _, lse = oracle.sma(D, inp["Q"], inp["Cm"], inp["E"], w.chunk, w.eps)
+    ref = oracle.sma_backward(D, inp["Q"], inp["Cm"], inp["E"], inp["z"], inp["dY"], w.chunk, w.eps)
+    Q, Cm, E, z, dY = (dev(inp[k], w.dtype) for k in ("Q", "Cm", "E", "z", "dY"))
+    Mem = dev(torch.from_numpy(D).float(), torch.float32)
+    got = api.sma_backward(Mem, None, Q, Cm, E, z, dev(torch.from_numpy(lse).float(), torch.float32),
+                           dY, w.chunk, w.eps)
+    torch.cuda.synchronize()
+    errs = {name: rel_err(host(g), r) for name, g, r in zip(["dM", "dQ", "dC", "dE", "dz"], got, ref)}
+    print(w.name, {k: f"{v:.2e}" for k, v in errs.items()})
+    for name, err in errs.items():
+        assert err <= _tol(w), f"{name}: {err:.3e}"
+
+
+@pytest.mark.parametrize("w", [CASES[0], CASES[3]], ids=lambda w: w.name)
+def test_layer_backward_matches_oracle(w):
+    """Forward through the library, then the layer backward: SMA backward's dM and
+    dC feed the scan backward."""
+    inp = prefill_inputs(w, with_grad=True)
+    ref = oracle.backward(inp["X"], inp["dt"], inp["A"], inp["Bm"], inp["Cm"], inp["Q"], inp["E"],
+                          inp["z"], inp["dY"], w.chunk, w.eps)
+    X, Bm, Cm, Q, E, z, dY = (dev(inp[k], w.dtype) for k in ("X", "Bm", "Cm", "Q", "E", "z", "dY"))
+    dt, A = dev(inp["dt"], torch.float32), dev(inp["A"], torch.float32)
+    s, o = api.prefill_forward(X, dt, A, Bm, Cm, Q, E, z, w.chunk, w.eps)
+    gr = api.layer_backward(X, dt, A, Bm, Cm, Q, E, z, dY, s, o, w.chunk, w.eps)
+    torch.cuda.synchronize()
+    got = [gr.dX, gr.ddt, gr.dA, gr.dB, gr.dC, gr.dQ, gr.dE, gr.dz]
+    errs = {n: rel_err(host(g), r) for n, g, r in zip(["dX", "ddt", "dA", "dB", "dC", "dQ", "dE", "dz"], got, ref)}
+    print(w.name, {k: f"{v:.2e}" for k, v in errs.items()})
+    for name, err in errs.items():
+        assert err <= _tol(w), f"{name}: {err:.3e}"
+
+
+def test_backward_single_chunk_has_no_sma_gradient():
+    """S = L: no token has history, so the SMA gradients are exactly zero."""
+    w = Workload("bwd_one_chunk", 1, 2, 128, 32, 16, 128, dtype="f32", seed=2105)
+    inp = prefill_inputs(w, with_grad=True)
+    X, Bm, Cm, Q, E, z, dY = (dev(inp[k], "f32") for k in ("X", "Bm", "Cm", "Q", "E", "z", "dY"))
+    dt, A = dev(inp["dt"], torch.float32), dev(inp["A"], torch.float32)
+    s, o = api.prefill_forward(X, dt, A, Bm, Cm, Q, E, z, w.chunk, w.eps)
+    dM, dQ, dC, dE, dz = api.sma_backward(s.M, s.rM, Q, Cm, E, z, o.lse, dY, w.chunk, w.eps)
+    torch.cuda.synchronize()
+    for t in (dM, dQ, dC, dE, dz):
+        assert torch.count_nonzero(t).item() == 0
