@@ -342,6 +342,10 @@ def run_dart(args) -> None:
         dec = bench_decode(args, dev, world, peaks, Bd, WORKLOADS[DECODE], decode_cache_slab,
                            decode_state_slab, decode_token_inputs)
     del flush
+    # ---- training step (forward + backward)
+    train = None
+    if not args.no_train:
+        train = bench_train(args, dev, world, peaks, Bd, WORKLOADS[args.train_workload], prefill_inputs)
 
     # ---- CPU oracle on a bounded sample (rank 0, N = 1 only)
     cpu = None
@@ -374,6 +378,7 @@ def run_dart(args) -> None:
                     "d2h_bytes_per_step": d2h, "ms_per_step": e2e_avg},
             "gpu_launches": launches, "clocks": clocks, "wall_s_timed": t_wall,
             "decode": dec,
+            "train": train,
         }
         print(json.dumps(line), flush=True)
     if world > 1:
@@ -430,6 +435,78 @@ def bench_decode(args, dev, world, peaks, Bd, w, cache_slab, state_slab, token_i
                          "peak_source": f"{peaks['source']} copy bandwidth", "traffic": None}}
 
 
+def bench_train(args, dev, world, peaks, Bd, w, prefill_inputs):
+    """One training step of the layer: forward (scan, SMA + merge) and backward
+    (SMA, scan) on the training workload, inputs resident in HBM."""
+    import torch
+
+    inp = prefill_inputs(w, with_grad=True)
+    tdt = torch.bfloat16
+    Bsz, L, H, G, P, N, S = w.batch, w.seqlen, w.heads, w.groups, w.headdim, w.dstate, w.chunk
+    M = w.nchunks
+    d = {k: inp[k].to(dev, tdt).contiguous() for k in ("X", "Bm", "Cm", "Q", "E", "z", "dY")}
+    d["dt"], d["A"] = inp["dt"].to(dev).contiguous(), inp["A"].to(dev).contiguous()
+    dims = Bd.make_dims(Bsz, L, H, G, P, N, S, Bd.DART_BF16, eps=w.eps)
+    f32 = dict(dtype=torch.float32, device=dev)
+    Yssd, Y = torch.empty(Bsz, L, H, P, **f32), torch.empty(Bsz, L, H, P, **f32)
+    Mem, rM = torch.empty(Bsz, M, H, N, P, **f32), torch.empty(Bsz, M, H, N, **f32)
+    lse = torch.empty(Bsz, L, H, **f32)
+    dM = torch.empty(Bsz, M, H, N, P, **f32)
+    dQ, dC = torch.empty(Bsz, L, G, N, **f32), torch.empty(Bsz, L, G, N, **f32)
+    dE, dz = torch.empty(Bsz, L, G, P, **f32), torch.empty(Bsz, L, H, **f32)
+    dX, ddt = torch.empty(Bsz, L, H, P, **f32), torch.empty(Bsz, L, H, **f32)
+    dA, dB = torch.empty(H, **f32), torch.empty(Bsz, L, G, N, **f32)
+    wsz = lambda op: torch.empty(max(Bd.dart_workspace_size(dims, op), 256), dtype=torch.uint8, device=dev)
+    ws_scan, ws_sma = wsz(Bd.DART_OP_CHUNK_SCAN), wsz(Bd.DART_OP_SMA_FORWARD)
+    ws_sbwd, ws_cbwd = wsz(Bd.DART_OP_SMA_BACKWARD), wsz(Bd.DART_OP_SCAN_BACKWARD)
+    stream = torch.cuda.current_stream(dev)
+
+    def step(evs=None):
+        def mark():
+            if evs is not None:
+                evs.append(torch.cuda.Event(enable_timing=True))
+                evs[-1].record(stream)
+
+        mark()
+        Bd.dart_chunk_scan(dims, d["X"], d["dt"], d["A"], d["Bm"], d["Cm"], Yssd, Mem, rM, None, ws_scan,
+                           stream)
+        mark()
+        Bd.dart_sma_forward(dims, Mem, rM, d["Q"], d["Cm"], d["E"], d["z"], Yssd, Y, None, lse, ws_sma,
+                            stream)
+        mark()
+        Bd.dart_sma_backward(dims, Mem, rM, d["Q"], d["Cm"], d["E"], d["z"], lse, d["dY"], dM, dQ, dC,
+                             dE, dz, ws_sbwd, stream)
+        mark()
+        Bd.dart_chunk_scan_backward(dims, d["X"], d["dt"], d["A"], d["Bm"], d["Cm"], d["dY"], dM, dX,
+                                    ddt, dA, dB, dC, ws_cbwd, stream)
+        mark()
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    barrier(world)
+    runs = []
+    for _ in range(args.steps):  # every step reads and writes far more than L2
+        evs = []
+        step(evs)
+        runs.append(evs)
+    torch.cuda.synchronize()
+    phase = [sum(r[i].elapsed_time(r[i + 1]) for r in runs) / len(runs) for i in range(4)]
+    ms = max_over_ranks(sum(phase), world, dev)
+    flops = 4 * sma_flops(w) + 3 * scan_flops(w)
+    tf = flops / (ms / 1e3) / 1e12
+    return {"workload": f"{w.name}: {w.notes}", "tokens_per_s": world * w.tokens / (ms / 1e3),
+            "ms_per_step": ms,
+            "phase_ms": {"scan_fwd": phase[0], "sma_fwd": phase[1], "sma_bwd": phase[2],
+                         "scan_bwd": phase[3]},
+            "roofline": {"kernel": "layer fwd+bwd", "bound": "tensor", "achieved": tf,
+                         "peak": peaks["bf16_sus"], "unit": "TFLOP/s", "frac": tf / peaks["bf16_sus"],
+                         "peak_source": f"{peaks['source']} bf16 dense (sustained)",
+                         "algorithmic_flops_per_step": flops,
+                         "flops_model": "4 x SMA forward + 3 x scan forward (backward ~3x / 2x)",
+                         "traffic": None}}
+
+
 def _traffic_from_profiles():
     """DRAM bytes per SMA launch from the committed ncu summary, when it still
     describes the current kernel (else null)."""
@@ -451,6 +528,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=("dart", "reference"), default="dart")
     ap.add_argument("--no-decode", action="store_true")
+    ap.add_argument("--no-train", action="store_true")
+    ap.add_argument("--train-workload", default="train_b8_l4k_s256")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-heads", type=int, default=4, help="heads in the oracle CPU sample")
     ap.add_argument("--ref-heads", type=int, default=1, help="heads per reference-arm step")
