@@ -265,13 +265,29 @@ struct OutSmem {
     uint8_t x_src[256 * 128];      // X_h of the sources as fp16, MN-major (rows s)
     uint8_t h_prev[2][kN * 128];   // H_[c-1] of head h, bf16 hi | lo, MN-major (rows n)
     float c2[256];                 // cum * log2(e) of the sources
-    float dts[256];
+    float e2[256];                 // c2 - log2(dt): exp2(c2_t - e2_s) = exp(cum_t - cum_s) dt_s
+    float wpart[2][kT];            // row maxima of |W| over each half of the sources
     uint64_t bar;
     uint32_t tmem_base;
 };
 
+constexpr int kOutThreads = 256;  // two threads per token row
+
+__device__ __forceinline__ float ex2_approx(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+// Next head's inputs, loaded into registers while the current head computes.
+struct HeadRegs {
+    uint4 xv[8];    // X rows of the sources (bf16), 16-byte pieces i = tid + 256 k
+    float4 hv[8];   // H_[c-1] (fp32), pieces i = tid + 256 k (two float4 per 8-wide piece)
+    float c2, dtv;  // source tid (tid < ns)
+};
+
 template <typename Tout>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(kOutThreads, 1)
 chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restrict__ dt,
                        const float* __restrict__ cum, const __nv_bfloat16* __restrict__ Bm,
                        const __nv_bfloat16* __restrict__ Cm, const float* __restrict__ Hin,
@@ -284,12 +300,14 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
     const int c = blockIdx.y / (H / kHeadsPerCta);
     const int hg = blockIdx.y % (H / kHeadsPerCta);
     const int b = blockIdx.z;
-    const int tid = threadIdx.x, warp = tid >> 5;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int row = tid & (kT - 1), half = tid >> 7;  // token row, half of the sources / columns
     const int h0 = hg * kHeadsPerCta;
     const int g = h0 / (H / G);
     const int ns = (tt + 1) * kT;  // sources 0 .. ns-1 of the chunk
     const i64 tok0 = (i64)b * L + (i64)c * S;
-    const uint32_t lane_addr = (uint32_t)(32 * warp) << 16;
+    const uint32_t lane_addr = (uint32_t)(32 * (warp & 3)) << 16;
+    const bool has_prev = c > 0;
     constexpr uint32_t kColSc = 0, kColW = 256, kColIn = 384, kColEx = 448;
 
     if (tid == 0) {
@@ -301,13 +319,13 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
         tc::tmem_relinquish();
     }
     // C of the tile: row t, K-major, two K blocks of 64 (16-byte chunks, swizzled)
-    for (int i = tid; i < kT * 16; i += kThreads) {
+    for (int i = tid; i < kT * 16; i += kOutThreads) {
         const int t = i / 16, q = i % 16;
         const uint4 v = reinterpret_cast<const uint4*>(Cm + ((tok0 + tt * kT + t) * G + g) * kN)[q];
         *reinterpret_cast<uint4*>(sm.c_tile[q / 8] + sw128((uint32_t)t, (uint32_t)(q % 8) * 16u)) = v;
     }
     // B of the sources: row s, K-major
-    for (int i = tid; i < ns * 16; i += kThreads) {
+    for (int i = tid; i < ns * 16; i += kOutThreads) {
         const int s = i / 16, q = i % 16;
         const uint4 v = reinterpret_cast<const uint4*>(Bm + ((tok0 + s) * G + g) * kN)[q];
         *reinterpret_cast<uint4*>(sm.b_src[q / 8] + sw128((uint32_t)s, (uint32_t)(q % 8) * 16u)) = v;
@@ -318,7 +336,7 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
     tc::tc_fence_after();
     const uint32_t tmem = sm.tmem_base;
     uint32_t phase = 0;
-    // scores = C_tile B_src^T (M 128, N ns, K 128)
+    // scores = C_tile B_src^T (M 128, N ns, K 128), shared by the CTA's heads
     if (tid == 0) {
         const uint32_t idesc = tc::idesc_f16(1, false, kT, (uint32_t)ns);
         for (int ks = 0; ks < kN / 16; ++ks) {
@@ -327,61 +345,63 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
             mma_f16_ss(tmem + kColSc, ad, bd, idesc, ks > 0 ? 1u : 0u);
         }
     }
+
+    // register prefetch of a head's sources (X rows, H_[c-1], cum, dt)
+    const int xiters = ns * 8 / kOutThreads;  // 4 or 8 pieces of 16 bytes
+    HeadRegs nx;
+    auto load_head = [&](int h) {
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            if (k < xiters) {
+                const int i = tid + k * kOutThreads, sidx = i / 8, q = i % 8;
+                nx.xv[k] = reinterpret_cast<const uint4*>(X + ((tok0 + sidx) * H + h) * kP)[q];
+            }
+        }
+        if (has_prev) {
+            const float* Hh = Hin + (((i64)b * Mc + c) * H + h) * (i64)(kN * kP);
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                const int i = tid + k * kOutThreads, n = i / 8, q = i % 8;
+                nx.hv[2 * k] = reinterpret_cast<const float4*>(Hh + n * kP)[2 * q];
+                nx.hv[2 * k + 1] = reinterpret_cast<const float4*>(Hh + n * kP)[2 * q + 1];
+            }
+        }
+        if (tid < ns) {
+            nx.c2 = cum[(((i64)b * H + h) * Mc + c) * S + tid] * kLog2e;
+            nx.dtv = dt[(tok0 + tid) * H + h];
+        }
+    };
+    load_head(h0);
     bool ok = commit_and_wait(&sm.bar, phase, wait_limit_ns, 2);
     phase ^= 1u;
 
-    const int tl = tt * kT + tid;  // this thread's token inside the chunk
+    const int tl = tt * kT + row;  // this thread's token inside the chunk
     const i64 tok = tok0 + tl;
+    const int tl_warp_max = tt * kT + 32 * (warp & 3) + 31;
+    const int s_lo = half * (ns / 2), s_hi = s_lo + ns / 2;
     for (int hh = 0; hh < kHeadsPerCta && ok; ++hh) {
         const int h = h0 + hh;
-        const float* cumc = cum + (((i64)b * H + h) * Mc + c) * S;
-        for (int s = tid; s < ns; s += kThreads) {
-            sm.c2[s] = cumc[s] * kLog2e;
-            sm.dts[s] = dt[(tok0 + s) * H + h];
-        }
-        // X_h of the sources as fp16, rows s (MN-major B operand of the intra MMA);
-        // all of a thread's 16-byte loads are issued before any is used
-        {
-            const int iters = ns * 8 / kThreads;  // 8 or 16
-            uint4 xv[16];
+        // prefetched sources into shared memory (the previous head's MMAs are done)
 #pragma unroll
-            for (int k = 0; k < 16; ++k) {
-                if (k < iters) {
-                    const int i = tid + k * kThreads, s = i / 8, q = i % 8;
-                    xv[k] = reinterpret_cast<const uint4*>(X + ((tok0 + s) * H + h) * kP)[q];
+        for (int k = 0; k < 8; ++k) {
+            if (k < xiters) {
+                const int i = tid + k * kOutThreads, sidx = i / 8, q = i % 8;
+                const uint32_t xw[4] = {nx.xv[k].x, nx.xv[k].y, nx.xv[k].z, nx.xv[k].w};
+                uint32_t f[4];
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const float2 v = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&xw[e]));
+                    f[e] = pack_f16(v.x, v.y);
                 }
-            }
-#pragma unroll
-            for (int k = 0; k < 16; ++k) {
-                if (k < iters) {
-                    const int i = tid + k * kThreads, s = i / 8, q = i % 8;
-                    const uint32_t xw[4] = {xv[k].x, xv[k].y, xv[k].z, xv[k].w};
-                    uint32_t f[4];
-#pragma unroll
-                    for (int e = 0; e < 4; ++e) {
-                        const float2 v = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&xw[e]));
-                        f[e] = pack_f16(v.x, v.y);
-                    }
-                    *reinterpret_cast<uint4*>(sm.x_src + sw128((uint32_t)s, (uint32_t)q * 16u)) =
-                        make_uint4(f[0], f[1], f[2], f[3]);
-                }
+                *reinterpret_cast<uint4*>(sm.x_src + sw128((uint32_t)sidx, (uint32_t)q * 16u)) =
+                    make_uint4(f[0], f[1], f[2], f[3]);
             }
         }
-        // H_[c-1] of head h as bf16 hi | lo, rows n (zero state before chunk 0)
-        const bool has_prev = c > 0;
         if (has_prev) {
-            const float* Hh = Hin + (((i64)b * Mc + c) * H + h) * (i64)(kN * kP);
-            float4 hv4[16];
 #pragma unroll
-            for (int k = 0; k < 8; ++k) {
-                const int i = tid + k * kThreads, n = i / 8, q = i % 8;
-                hv4[2 * k] = reinterpret_cast<const float4*>(Hh + n * kP)[2 * q];
-                hv4[2 * k + 1] = reinterpret_cast<const float4*>(Hh + n * kP)[2 * q + 1];
-            }
-#pragma unroll
-            for (int k = 0; k < 8; ++k) {
-                const int i = tid + k * kThreads, n = i / 8, q = i % 8;
-                const float4 a = hv4[2 * k], bb = hv4[2 * k + 1];
+            for (int k = 0; k < 4; ++k) {
+                const int i = tid + k * kOutThreads, n = i / 8, q = i % 8;
+                const float4 a = nx.hv[2 * k], bb = nx.hv[2 * k + 1];
                 const float vals[8] = {a.x, a.y, a.z, a.w, bb.x, bb.y, bb.z, bb.w};
                 uint32_t hi[4], lo[4];
 #pragma unroll
@@ -396,31 +416,46 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
                 *reinterpret_cast<uint4*>(sm.h_prev[1] + o) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
             }
         }
+        if (tid < ns) {
+            sm.c2[tid] = nx.c2;
+            sm.e2[tid] = nx.c2 - log2f(nx.dtv);  // dt = 0 gives +inf: a zero weight
+        }
         __syncthreads();
-        // W_h row of this thread: two passes over the scores (max, then scale + fp16)
+        if (hh + 1 < kHeadsPerCta) load_head(h + 1);  // lands while this head computes
+
+        // W row of this thread over its half of the sources: max pass, then scale + fp16
         const float c2t = sm.c2[tl];
         float wmax = 0.0f;
-        for (int s0 = 0; s0 < ns; s0 += 32) {
+        for (int s0 = s_lo; s0 < s_hi; s0 += 32) {
+            if (s0 > tl_warp_max) break;  // every row of the warp is before these sources
             float v[32];
             tmem_ld32(tmem + lane_addr + kColSc + (uint32_t)s0, v);
 #pragma unroll
             for (int i = 0; i < 32; ++i) {
-                const int s = s0 + i;
-                const float wv = s <= tl ? v[i] * exp2f(c2t - sm.c2[s]) * sm.dts[s] : 0.0f;
+                const int sidx = s0 + i;
+                const float wv = sidx <= tl ? v[i] * ex2_approx(c2t - sm.e2[sidx]) : 0.0f;
                 wmax = fmaxf(wmax, fabsf(wv));
             }
         }
+        sm.wpart[half][row] = wmax;
+        __syncthreads();
+        wmax = fmaxf(sm.wpart[0][row], sm.wpart[1][row]);
         const float rscale = wmax > 0.0f ? 1.0f / wmax : 1.0f;
-        for (int s0 = 0; s0 < ns; s0 += 32) {
-            float v[32];
-            tmem_ld32(tmem + lane_addr + kColSc + (uint32_t)s0, v);
+        for (int s0 = s_lo; s0 < s_hi; s0 += 32) {
             uint32_t pk[16];
+            if (s0 > tl_warp_max) {
 #pragma unroll
-            for (int i = 0; i < 16; ++i) {
-                const int s = s0 + 2 * i;
-                const float w0 = s <= tl ? v[2 * i] * exp2f(c2t - sm.c2[s]) * sm.dts[s] : 0.0f;
-                const float w1 = s + 1 <= tl ? v[2 * i + 1] * exp2f(c2t - sm.c2[s + 1]) * sm.dts[s + 1] : 0.0f;
-                pk[i] = pack_f16(w0 * rscale, w1 * rscale);
+                for (int i = 0; i < 16; ++i) pk[i] = 0u;
+            } else {
+                float v[32];
+                tmem_ld32(tmem + lane_addr + kColSc + (uint32_t)s0, v);
+#pragma unroll
+                for (int i = 0; i < 16; ++i) {
+                    const int sidx = s0 + 2 * i;
+                    const float w0 = sidx <= tl ? v[2 * i] * ex2_approx(c2t - sm.e2[sidx]) : 0.0f;
+                    const float w1 = sidx + 1 <= tl ? v[2 * i + 1] * ex2_approx(c2t - sm.e2[sidx + 1]) : 0.0f;
+                    pk[i] = pack_f16(w0 * rscale, w1 * rscale);
+                }
             }
             tc::tmem_st16(tmem + lane_addr + kColW + (uint32_t)(s0 / 2), pk);
         }
@@ -451,24 +486,20 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
         ok = commit_and_wait(&sm.bar, phase, wait_limit_ns, 3);
         phase ^= 1u;
         if (!ok) break;
-        // Y_t = wmax * (W~ X)_t + exp(cum_t) (C H)_t
+        // Y_t = wmax * (W~ X)_t + exp(cum_t) (C H)_t, columns 32 half .. 32 half + 31
         {
             const float dec = exp2f(c2t);
-            Tout* yrow = Y + (tok * H + h) * kP;
+            float vi[32], ve[32];
+            tmem_ld32(tmem + lane_addr + kColIn + 32u * half, vi);
+            if (has_prev) {
+                tmem_ld32(tmem + lane_addr + kColEx + 32u * half, ve);
+            } else {
 #pragma unroll
-            for (int half = 0; half < 2; ++half) {
-                float vi[32], ve[32];
-                tmem_ld32(tmem + lane_addr + kColIn + 32u * half, vi);
-                if (has_prev) {
-                    tmem_ld32(tmem + lane_addr + kColEx + 32u * half, ve);
-                } else {
-#pragma unroll
-                    for (int i = 0; i < 32; ++i) ve[i] = 0.0f;
-                }
-#pragma unroll
-                for (int i = 0; i < 32; ++i) vi[i] = fmaf(wmax, vi[i], dec * ve[i]);
-                store_row32(yrow + 32 * half, vi);
+                for (int i = 0; i < 32; ++i) ve[i] = 0.0f;
             }
+#pragma unroll
+            for (int i = 0; i < 32; ++i) vi[i] = fmaf(wmax, vi[i], dec * ve[i]);
+            store_row32(Y + (tok * H + h) * kP + 32 * half, vi);
         }
         tc::tc_fence_before();
         __syncthreads();  // shared staging and TMEM are reused by the next head
@@ -515,7 +546,7 @@ cudaError_t launch_chunk_scan_tc(const ScanArgs& a, unsigned long long wait_limi
         const size_t smem = sizeof(OutSmem) + 1024;
         cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
-        kern<<<dim3(S / kT, M * (H / kHeadsPerCta), B), kThreads, smem, stream>>>(
+        kern<<<dim3(S / kT, M * (H / kHeadsPerCta), B), kOutThreads, smem, stream>>>(
             (const __nv_bfloat16*)a.X, a.dt, a.cum, (const __nv_bfloat16*)a.Bm,
             (const __nv_bfloat16*)a.Cm, a.dH32, (Tout*)a.Y, L, H, G, S, M, wait_limit_ns);
     }
