@@ -271,6 +271,16 @@ uint64_t dart_launch_count(void);
 void dart_set_wait_limit_ns(uint64_t limit_ns);
 
 /*
+ * Test hook for the failure path of the tensor-core kernels (no counterpart in
+ * the paper): while on, tensor-core dart_sma_forward launches issue none of
+ * their operand copies, so their pipeline waits can only run out (each bounded
+ * by dart_set_wait_limit_ns); the call then reports DART_ERR_TIMEOUT through
+ * dart_get_device_status and its outputs are undefined. Process-wide; 0 (the
+ * default) turns it off. For tests only.
+ */
+void dart_test_withhold_copies(int on);
+
+/*
  * Synchronises `stream`, then reports and clears the device status word that
  * kernels set when a bounded device-side wait gives up: DART_ERR_TIMEOUT if
  * one did since the last call, DART_ERR_CUDA if the synchronisation failed,

@@ -31,7 +31,7 @@ DART_DTYPE = {torch.float32: DART_F32, torch.bfloat16: DART_BF16}
 EXPORTED = ("dart_status_string", "dart_last_cuda_error", "dart_workspace_size",
             "dart_chunk_scan", "dart_sma_forward", "dart_decode_step", "dart_sma_forward_noalloc",
             "dart_launch_count", "dart_set_wait_limit_ns", "dart_get_device_status",
-            "dart_sma_backward", "dart_chunk_scan_backward")
+            "dart_sma_backward", "dart_chunk_scan_backward", "dart_test_withhold_copies")
 
 
 class DartError(RuntimeError):
@@ -96,6 +96,8 @@ def lib() -> ctypes.CDLL:
         L.dart_get_device_status.restype = ctypes.c_int
         L.dart_get_device_status.argtypes = [_vp]
         L.dart_get_device_status.restype = ctypes.c_int
+        L.dart_test_withhold_copies.argtypes = [ctypes.c_int]
+        L.dart_test_withhold_copies.restype = None
         L.dart_sma_backward.argtypes = [dp] + [_vp] * 14 + [ctypes.c_size_t, _vp]
         L.dart_sma_backward.restype = ctypes.c_int
         L.dart_chunk_scan_backward.argtypes = [dp] + [_vp] * 13 + [ctypes.c_size_t, _vp]
@@ -204,6 +206,11 @@ def dart_get_device_status(stream=None) -> None:
 def dart_launch_count() -> int:
     """Kernels the library has launched in this process."""
     return int(lib().dart_launch_count())
+
+
+def dart_test_withhold_copies(on: bool) -> None:
+    """Failure-path test hook: tensor-core SMA launches issue no operand copies while on."""
+    lib().dart_test_withhold_copies(1 if on else 0)
 
 
 def dart_set_wait_limit_ns(limit_ns: int) -> None:

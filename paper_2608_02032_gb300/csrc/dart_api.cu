@@ -123,6 +123,7 @@ size_t sma_ws(const dart_dims* d) {
 }
 
 std::atomic<unsigned long long> g_wait_limit_ns{2000000000ull};
+std::atomic<int> g_test_withhold{0};
 
 std::atomic<uint64_t> g_launches{0};
 
@@ -236,6 +237,7 @@ dart_status dart_sma_forward(const dart_dims* d, const void* M, const float* rM,
         dart::SmaArgs a = sma_args(d);
         a.M = M; a.rM = rM; a.Q = Q; a.Cm = Cm; a.E = E; a.z = z; a.Yssd = Y_ssd; a.Y = Y;
         a.R = R; a.lse = lse;
+        a.test_withhold = g_test_withhold.load();
         const unsigned long long lim = g_wait_limit_ns.load();
         typedef __nv_bfloat16 bf;
         cudaError_t e;
@@ -363,6 +365,8 @@ dart_status dart_get_device_status(void* stream) {
     if (code < 0 || code2 < 0) return cuda_fail(cudaGetLastError());
     return (code != 0 || code2 != 0) ? DART_ERR_TIMEOUT : DART_OK;
 }
+
+void dart_test_withhold_copies(int on) { g_test_withhold.store(on != 0 ? 1 : 0); }
 
 void dart_set_wait_limit_ns(uint64_t limit_ns) {
     g_wait_limit_ns.store(limit_ns == 0 ? 2000000000ull : (unsigned long long)limit_ns);

@@ -45,6 +45,7 @@ struct SmaArgs {
     void* Y;
     void* R;
     float* lse;
+    int test_withhold;  // tensor-core path: issue no operand copies (failure-path test hook)
 };
 
 struct DecodeArgs {

@@ -302,7 +302,7 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
               const __nv_bfloat16* __restrict__ E, const __nv_bfloat16* __restrict__ z,
               const Tout* __restrict__ Yssd, Tout* __restrict__ Y, Tout* __restrict__ R,
               float* __restrict__ lse, int Bsz, int L, int H, int G, int S, int Mc, float eps,
-              unsigned long long wait_limit_ns) {
+              unsigned long long wait_limit_ns, int withhold) {
     extern __shared__ uint8_t smem_raw[];
     TcSmem& sm = *reinterpret_cast<TcSmem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                             ~(uintptr_t)1023);
@@ -358,7 +358,8 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
             const i64 job_stride = (i64)hpairs * kPair;
             bool ok = true;
             int njobs = 0;  // jobs whose copy was issued
-            for (int j = 0; j < nj; ++j) {
+            // (withhold: the failure-path test hook; every wait on the operands then runs out)
+            for (int j = 0; j < (withhold ? 0 : nj); ++j) {
                 const int ub = j & 1;
                 // stages 3..5 hold the epilogue's row staging until the operands are in TMEM;
                 // stages 3b .. 3b+2 were last used by job j - 2: wait for its U and V
@@ -664,7 +665,7 @@ cudaError_t launch_sma_forward_tc(const SmaArgs& a, void* ws, unsigned long long
                                             (const __nv_bfloat16*)a.Cm, (const __nv_bfloat16*)a.E,
                                             (const __nv_bfloat16*)a.z, (const Tout*)a.Yssd,
                                             (Tout*)a.Y, (Tout*)a.R, a.lse, Bsz, L, H, (int)a.G,
-                                            (int)a.S, Mc, a.eps, wait_limit_ns);
+                                            (int)a.S, Mc, a.eps, wait_limit_ns, a.test_withhold);
     note_launches(1);
     return cudaGetLastError();
 }
