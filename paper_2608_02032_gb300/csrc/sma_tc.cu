@@ -34,7 +34,7 @@
 // already in the 128-byte-swizzled shared-memory layout, so each part is one
 // bulk copy.
 // Kernel 2 (sma_tc_kernel), one CTA per (batch, 128-token tile, 2 heads),
-// heaviest tiles first:
+// grouped by (batch, head pair), heaviest tiles first inside a group:
 //   warp 0      producer: bulk copies of the parts into a 6-stage ring
 //   warp 1      TMEM allocation; one thread issues the MMAs
 //   warps 2, 3  idle (they complete warpgroup 0 for the register split)
@@ -308,14 +308,16 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
                                             ~(uintptr_t)1023);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
-    // work item: heaviest token tiles first
+    // work item: (batch, head pair) major, heaviest token tiles first inside it, so the
+    // CTAs resident at one time stream the operands of one or two head pairs (a few MB
+    // that stay in L2) rather than of all of them
     const int tiles = L / kRows;
     const int hpairs = H / kHeadsPerCta;
     const int item = blockIdx.x;
-    const int tt = tiles - 1 - item / (Bsz * hpairs);
-    const int rem = item % (Bsz * hpairs);
-    const int b = rem / hpairs;
-    const int hp = rem % hpairs;
+    const int grp = item / tiles;
+    const int tt = tiles - 1 - item % tiles;
+    const int b = grp / hpairs;
+    const int hp = grp % hpairs;
     const int h0 = hp * kHeadsPerCta;
     const int t0 = tt * kRows;
     // S is a multiple of the tile height, so every token of the tile lies in
