@@ -339,7 +339,7 @@ def run_dart(args) -> None:
     # ---- decode step (HBM bound)
     dec = None
     if not args.no_decode:
-        dec = bench_decode(args, dev, world, peaks, Bd, WORKLOADS[DECODE], decode_cache_slab,
+        dec = bench_decode(args, dev, world, peaks, Bd, WORKLOADS[args.decode_workload], decode_cache_slab,
                            decode_state_slab, decode_token_inputs)
     del flush
     # ---- training step (forward + backward)
@@ -529,6 +529,7 @@ def main():
     ap.add_argument("--impl", choices=("dart", "reference"), default="dart")
     ap.add_argument("--no-decode", action="store_true")
     ap.add_argument("--no-train", action="store_true")
+    ap.add_argument("--decode-workload", default=DECODE, help="decode workload (a smaller one for profiling)")
     ap.add_argument("--train-workload", default="train_b8_l4k_s256")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-heads", type=int, default=4, help="heads in the oracle CPU sample")

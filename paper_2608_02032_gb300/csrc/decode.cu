@@ -22,11 +22,15 @@ namespace dart {
 constexpr int kDecThreads = 256;
 constexpr int kDecWarps = kDecThreads / 32;
 
+// 16-byte pieces of a memory row: raw load (streamed once) and unpack to fp32.
 template <typename T> struct Vec16;
 template <> struct Vec16<__nv_bfloat16> {
     static constexpr int n = 8;
-    __device__ static void load(const __nv_bfloat16* p, float* out) {
-        const uint4 u = __ldcs(reinterpret_cast<const uint4*>(p));  // streamed once
+    typedef uint4 raw_t;
+    __device__ static raw_t load(const __nv_bfloat16* p) {
+        return __ldcs(reinterpret_cast<const uint4*>(p));
+    }
+    __device__ static void unpack(const raw_t& u, float* out) {
         const __nv_bfloat162* h2 = reinterpret_cast<const __nv_bfloat162*>(&u);
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
@@ -38,11 +42,14 @@ template <> struct Vec16<__nv_bfloat16> {
 };
 template <> struct Vec16<float> {
     static constexpr int n = 4;
-    __device__ static void load(const float* p, float* out) {
-        const float4 f = __ldcs(reinterpret_cast<const float4*>(p));
+    typedef float4 raw_t;
+    __device__ static raw_t load(const float* p) { return __ldcs(reinterpret_cast<const float4*>(p)); }
+    __device__ static void unpack(const raw_t& f, float* out) {
         out[0] = f.x; out[1] = f.y; out[2] = f.z; out[3] = f.w;
     }
 };
+
+constexpr int kBatch = 8;  // row steps whose loads a lane issues before using any
 
 template <typename Tin, typename Tmem, typename Tout, int P>
 __global__ void __launch_bounds__(kDecThreads)
@@ -59,7 +66,7 @@ decode_step_kernel(long long pos, int m_cap, Tmem* __restrict__ cache, float* __
     static_assert(LPR >= 1 && LPR <= 32 && (32 % LPR) == 0, "unsupported P");
 
     __shared__ float sx[P], se[P], sb[128], sc[128], sq[128];
-    __shared__ float sY[kDecThreads];
+    __shared__ float sY[4 * kDecThreads];  // per (row group, column) partial y_ssd
     __shared__ float sWm[kDecWarps], sWd[kDecWarps], sWO[kDecWarps][P];
     __shared__ float sRed[2];
 
@@ -102,22 +109,55 @@ decode_step_kernel(long long pos, int m_cap, Tmem* __restrict__ cache, float* __
     float* Pt = partial + bh * NP;
     Tmem* slot = (chunk_end && ichunk < m_cap) ? cache + (((i64)b * m_cap + ichunk) * H + h) * NP
                                                : nullptr;
-    // thread owns columns p = tid % P (kDecThreads % P == 0) and rows n = tid / P + k * rstep
-    static_assert(kDecThreads % P == 0, "P must divide the block");
-    const int p_own = tid % P;
-    const int rstep = kDecThreads / P;
-    float yp = 0.0f;
-    for (int n = tid / P; n < N; n += rstep) {
-        const int e = n * P + p_own;
-        const float w = d * sb[n] * sx[p_own];
-        const float hn = fmaf(a, St[e], w);
-        const float pn = chunk_start ? w : fmaf(a, Pt[e], w);
-        St[e] = hn;
-        Pt[e] = pn;
-        if (slot != nullptr) slot[e] = cvt_from_f32<Tmem>(pn);
-        yp = fmaf(sc[n], hn, yp);
+    // thread owns columns 4 q .. 4 q + 3 (q = tid % (P / 4)) of rows n = tid / (P / 4) + k rstep;
+    // the loads of all its rows are issued before any is used
+    constexpr int QP = P / 4;
+    static_assert(kDecThreads % QP == 0, "P / 4 must divide the block");
+    const int q_own = tid % QP;
+    const int rstep = kDecThreads / QP;
+    constexpr int kRowBatch = 4;  // rows whose loads are issued together
+    float yp[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+    for (int k0 = 0; tid / QP + k0 * rstep < N; k0 += kRowBatch) {
+    float4 s4[kRowBatch], p4[kRowBatch];
+#pragma unroll
+    for (int k = 0; k < kRowBatch; ++k) {
+        const int n = tid / QP + (k0 + k) * rstep;
+        if (n < N) {
+            s4[k] = reinterpret_cast<const float4*>(St + n * P)[q_own];
+            if (!chunk_start) p4[k] = reinterpret_cast<const float4*>(Pt + n * P)[q_own];
+        }
     }
-    sY[tid] = yp;
+#pragma unroll
+    for (int k = 0; k < kRowBatch; ++k) {
+        const int n = tid / QP + (k0 + k) * rstep;
+        if (n >= N) continue;
+        const float bd = d * sb[n];
+        const float4 xs = make_float4(sx[4 * q_own], sx[4 * q_own + 1], sx[4 * q_own + 2], sx[4 * q_own + 3]);
+        const float w[4] = {bd * xs.x, bd * xs.y, bd * xs.z, bd * xs.w};
+        const float so[4] = {s4[k].x, s4[k].y, s4[k].z, s4[k].w};
+        float hn[4], pn[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) hn[i] = fmaf(a, so[i], w[i]);
+        if (chunk_start) {
+#pragma unroll
+            for (int i = 0; i < 4; ++i) pn[i] = w[i];
+        } else {
+            const float po[4] = {p4[k].x, p4[k].y, p4[k].z, p4[k].w};
+#pragma unroll
+            for (int i = 0; i < 4; ++i) pn[i] = fmaf(a, po[i], w[i]);
+        }
+        reinterpret_cast<float4*>(St + n * P)[q_own] = make_float4(hn[0], hn[1], hn[2], hn[3]);
+        reinterpret_cast<float4*>(Pt + n * P)[q_own] = make_float4(pn[0], pn[1], pn[2], pn[3]);
+        if (slot != nullptr) {
+#pragma unroll
+            for (int i = 0; i < 4; ++i) slot[n * P + 4 * q_own + i] = cvt_from_f32<Tmem>(pn[i]);
+        }
+#pragma unroll
+        for (int i = 0; i < 4; ++i) yp[i] = fmaf(sc[n], hn[i], yp[i]);
+    }
+    }
+#pragma unroll
+    for (int i = 0; i < 4; ++i) sY[(tid / QP) * P + 4 * q_own + i] = yp[i];
 
     // phase 2: sweep the completed memories
     const int nhist = (int)(ichunk < (i64)m_cap ? ichunk : (i64)m_cap);
@@ -136,26 +176,36 @@ decode_step_kernel(long long pos, int m_cap, Tmem* __restrict__ cache, float* __
         float lacc = 0.0f, vacc[VEC];
 #pragma unroll
         for (int v = 0; v < VEC; ++v) vacc[v] = 0.0f;
-#pragma unroll 4
-        for (int n = r0; n < N; n += RPW) {
-            float val[VEC];
-            Vec16<Tmem>::load(Mj + (i64)n * P + p0, val);
-            float dot = 0.0f, ssq = 0.0f;
+        for (int n0 = r0; n0 < N; n0 += kBatch * RPW) {
+            typename Vec16<Tmem>::raw_t raw[kBatch];
 #pragma unroll
-            for (int v = 0; v < VEC; ++v) {
-                dot = fmaf(val[v], ev_reg[v], dot);
-                ssq = fmaf(val[v], val[v], ssq);
+            for (int u = 0; u < kBatch; ++u) {
+                const int n = n0 + u * RPW;
+                if (n < N) raw[u] = Vec16<Tmem>::load(Mj + (i64)n * P + p0);
             }
 #pragma unroll
-            for (int off = 1; off < LPR; off <<= 1) {
-                dot += __shfl_xor_sync(0xffffffffu, dot, off);
-                ssq += __shfl_xor_sync(0xffffffffu, ssq, off);
-            }
-            const float rn = rsqrtf(ssq / (float)P + eps);
-            lacc = fmaf(sq[n], rn * dot, lacc);
-            const float cn = sc[n];
+            for (int u = 0; u < kBatch; ++u) {
+                const int n = n0 + u * RPW;
+                if (n >= N) break;  // N is a multiple of RPW: every lane leaves at the same u
+                float val[VEC];
+                Vec16<Tmem>::unpack(raw[u], val);
+                float dot = 0.0f, ssq = 0.0f;
 #pragma unroll
-            for (int v = 0; v < VEC; ++v) vacc[v] = fmaf(cn, val[v], vacc[v]);
+                for (int v = 0; v < VEC; ++v) {
+                    dot = fmaf(val[v], ev_reg[v], dot);
+                    ssq = fmaf(val[v], val[v], ssq);
+                }
+#pragma unroll
+                for (int off = 1; off < LPR; off <<= 1) {
+                    dot += __shfl_xor_sync(0xffffffffu, dot, off);
+                    ssq += __shfl_xor_sync(0xffffffffu, ssq, off);
+                }
+                const float rn = rsqrtf(ssq / (float)P + eps);
+                lacc = fmaf(sq[n], rn * dot, lacc);
+                const float cn = sc[n];
+#pragma unroll
+                for (int v = 0; v < VEC; ++v) vacc[v] = fmaf(cn, val[v], vacc[v]);
+            }
         }
         // logit: one copy of each row's term lives in the LPR lanes of its group
         float l = (lane % LPR) == 0 ? lacc : 0.0f;
@@ -187,7 +237,7 @@ decode_step_kernel(long long pos, int m_cap, Tmem* __restrict__ cache, float* __
     // phase 3: merge the warps' partial softmaxes, gate, write y
     if (tid < P) {
         float yssd = 0.0f;
-        for (int k = tid; k < kDecThreads; k += P) yssd += sY[k];
+        for (int k = 0; k < kDecThreads / (P / 4); ++k) yssd += sY[k * P + tid];
         float mx = -INFINITY;
         for (int w = 0; w < kDecWarps; ++w) mx = fmaxf(mx, sWm[w]);
         float den = 0.0f, num = 0.0f;

@@ -71,6 +71,8 @@ WORKLOADS = {
                             notes="B1 H32 L8192 P64 N128 S256, bf16 (profiling size)"),
     "decode_b64": Workload("decode_b64", 64, 32, 1, 64, 128, 256, seed=1003, mem=64, pos=16384,
                            notes="B64 H32 P64 N128 S256, 64 cached memories, pos 16384"),
+    "decode_b16": Workload("decode_b16", 16, 32, 1, 64, 128, 256, seed=1007, mem=64, pos=16384,
+                           notes="B16 H32 P64 N128 S256, 64 cached memories (profiling size)"),
     "train_b8_l4k_s128": Workload("train_b8_l4k_s128", 8, 24, 4096, 64, 128, 128, seed=1004,
                                   notes="B8 H24 L4096 P64 N128 S128, bf16"),
     "train_b8_l4k_s256": Workload("train_b8_l4k_s256", 8, 24, 4096, 64, 128, 256, seed=1005,
