@@ -19,7 +19,9 @@ of the same workload; it is the only other place this file runs the oracle.
 from __future__ import annotations
 
 import argparse
+import hashlib
 import json
+import re
 import math
 import os
 import statistics
@@ -508,17 +510,22 @@ def bench_train(args, dev, world, peaks, Bd, w, prefill_inputs):
 
 
 def _traffic_from_profiles():
-    """DRAM bytes per SMA launch from the committed ncu summary, when it still
-    describes the current kernel (else null)."""
-    path = os.path.join(ROOT, "profiles", "sma_forward_prefill_l16k.json")
-    if not os.path.exists(path):
-        return None
+    """DRAM bytes per SMA launch from the committed ncu summary, while the
+    source hash recorded there matches the current kernel source (else null)."""
+    path = os.path.join(ROOT, "profiles", "sma_forward_prefill_l16k.md")
+    src = os.path.join(ROOT, "paper_2608_02032_gb300", "csrc", "sma_tc.cu")
     try:
         with open(path) as f:
-            d = json.load(f)
-        return d.get("dram_bytes_per_launch") if d.get("current", False) else None
-    except (OSError, ValueError):
+            text = f.read()
+        with open(src, "rb") as f:
+            digest = hashlib.sha256(f.read()).hexdigest()
+    except OSError:
         return None
+    mb = re.search(r"^dram_bytes_per_launch: (\d+)$", text, re.M)
+    mh = re.search(r"^source_sha256: ([0-9a-f]{64})$", text, re.M)
+    if mb is None or mh is None or mh.group(1) != digest:
+        return None
+    return int(mb.group(1))
 
 
 def main():

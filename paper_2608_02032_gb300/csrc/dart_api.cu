@@ -90,16 +90,26 @@ dart_status check_dims(const dart_dims* d, bool need_seqlen) {
 }
 
 struct ScanWs {
-    size_t cum_off, dh_off, total;
+    size_t cum_off, dh_off, hops_off, total;
 };
+
+bool scan_uses_tc(const dart_dims* d) {
+    dart::ScanArgs a{};
+    a.B = d->batch; a.L = d->seqlen; a.H = d->nheads; a.G = d->ngroups;
+    a.P = d->headdim; a.N = d->dstate; a.S = d->chunk;
+    return d->in_dtype == DART_BF16 && dart::scan_tc_supported(a);
+}
 
 ScanWs scan_ws(const dart_dims* d) {
     const i64 M = d->seqlen / d->chunk;
+    const size_t states = align256((size_t)(d->batch * M * d->nheads * d->dstate * d->headdim) *
+                                   sizeof(float));
     ScanWs w;
     w.cum_off = 0;
     w.dh_off = align256((size_t)(d->batch * d->nheads * M * d->chunk) * sizeof(float));
-    w.total = w.dh_off +
-              align256((size_t)(d->batch * M * d->nheads * d->dstate * d->headdim) * sizeof(float));
+    w.hops_off = w.dh_off + states;
+    // tensor-core path: the chunk-entry states also as bf16 hi | lo operand tiles (same bytes)
+    w.total = w.hops_off + (scan_uses_tc(d) ? states : 0);
     return w;
 }
 
@@ -192,7 +202,7 @@ dart_status dart_chunk_scan(const dart_dims* d, const void* X, const float* dt, 
     if (ws == nullptr || ((uintptr_t)ws & 255u) != 0 || ws_bytes < w.total)
         return DART_ERR_WORKSPACE;
 
-    dart::ScanArgs a;
+    dart::ScanArgs a{};
     a.B = d->batch; a.L = d->seqlen; a.H = d->nheads; a.G = d->ngroups;
     a.P = d->headdim; a.N = d->dstate; a.S = d->chunk; a.eps = d->eps;
     a.X = X; a.dt = dt; a.A = A; a.Bm = Bm; a.Cm = Cm; a.Y = Y_ssd; a.M = M; a.rM = rM;
@@ -201,7 +211,8 @@ dart_status dart_chunk_scan(const dart_dims* d, const void* X, const float* dt, 
     a.dH32 = (float*)((char*)ws + w.dh_off);
     cudaStream_t s = (cudaStream_t)stream;
     cudaError_t e;
-    if (d->in_dtype == DART_BF16 && dart::scan_tc_supported(a)) {
+    if (scan_uses_tc(d)) {
+        a.Hops = (uint8_t*)ws + w.hops_off;
         typedef __nv_bfloat16 bf;
         const unsigned long long lim = g_wait_limit_ns.load();
         if (d->mem_dtype == DART_F32)

@@ -30,6 +30,9 @@ struct ScanArgs {
     // workspace
     float* cum;   // B x H x M x S
     float* dH32;  // B x M x H x N x P (fp32 memories, then states entering each chunk)
+    // optional (tensor-core path): the states entering each chunk as bf16 hi | lo
+    // tiles in the 128-byte-swizzled shared-memory layout, 32 KiB per (b, c, h)
+    uint8_t* Hops;
 };
 
 struct SmaArgs {

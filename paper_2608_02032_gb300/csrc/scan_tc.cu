@@ -10,7 +10,7 @@
 //   per head as bf16 hi + lo (two MMAs, ~2^-16 relative) in the 128-byte
 //   swizzled MN-major layout. The epilogue (thread n = row n) writes the
 //   memory, its inverse RMS r (App. B.1) and the fp32 copy for state passing.
-// chunk_output_tc_kernel, one CTA (128 threads) per (128-token tile, chunk, head group, b):
+// chunk_output_tc_kernel, one CTA (256 threads) per (128-token tile, chunk, head group, b):
 //   scores = C_tile B_src^T                  (once, shared by the heads: G = 1)
 //   W_h[t,s] = scores[t,s] exp(cum_t - cum_s) dt_s  for s <= t, else 0
 //   Y_t = W_h X_h + exp(cum_t) C_t H_[c-1]   (App. A intra + inter terms)
@@ -18,7 +18,8 @@
 //   max_s |W_h[t,s]| (the decay is at most 1), and stored fp16 in TMEM as the
 //   A operand (fp16 keeps 11 bits; the row scale keeps small decayed weights
 //   out of the subnormal range, and the bound needs no pass over the row);
-//   H_[c-1] is split bf16 hi + lo. A CPU emulation against the oracle gives
+//   H_[c-1] arrives split bf16 hi + lo, already swizzled by the state passing
+//   (one 32 KiB bulk copy per head, double-buffered). A CPU emulation against the oracle gives
 //   max|err|/RMS(Y) = 2.1e-3 with the exact row maximum as the scale (5.4e-3
 //   without a row scale, 4.2e-2 with plain bf16).
 // TMEM of the output kernel: scores [0, 256), W [256, 384), intra accumulator
@@ -77,6 +78,37 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
     for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+// tcgen05.ld of 32 + 32 fp32 columns (two addresses) of this thread's lane, one wait.
+__device__ __forceinline__ void tmem_ld32x2(uint32_t ta, uint32_t tb, float (&va)[32], float (&vb)[32]) {
+    uint32_t r[64];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%64];\n\t"
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+        "{%32,%33,%34,%35,%36,%37,%38,%39,%40,%41,%42,%43,%44,%45,%46,%47,"
+        "%48,%49,%50,%51,%52,%53,%54,%55,%56,%57,%58,%59,%60,%61,%62,%63}, [%65];\n\t"
+        "tcgen05.wait::ld.sync.aligned;"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+          "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),
+          "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),
+          "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31]),
+          "=r"(r[32]), "=r"(r[33]), "=r"(r[34]), "=r"(r[35]), "=r"(r[36]), "=r"(r[37]),
+          "=r"(r[38]), "=r"(r[39]), "=r"(r[40]), "=r"(r[41]), "=r"(r[42]), "=r"(r[43]),
+          "=r"(r[44]), "=r"(r[45]), "=r"(r[46]), "=r"(r[47]), "=r"(r[48]), "=r"(r[49]),
+          "=r"(r[50]), "=r"(r[51]), "=r"(r[52]), "=r"(r[53]), "=r"(r[54]), "=r"(r[55]),
+          "=r"(r[56]), "=r"(r[57]), "=r"(r[58]), "=r"(r[59]), "=r"(r[60]), "=r"(r[61]),
+          "=r"(r[62]), "=r"(r[63])
+        : "r"(ta), "r"(tb)
+        : "memory");
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+        va[i] = __uint_as_float(r[i]);
+        vb[i] = __uint_as_float(r[32 + i]);
+    }
+}
+
 // D[tmem] (+)= A[smem] * B[smem]
 __device__ __forceinline__ void mma_f16_ss(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
                                            uint32_t idesc, uint32_t accumulate) {
@@ -92,9 +124,10 @@ __device__ __forceinline__ void mma_f16_ss(uint32_t d_tmem, uint64_t a_desc, uin
 // timeout set the status and return false (the caller stops; the final drain
 // waits for the MMAs in flight with the long bound).
 __device__ __forceinline__ bool commit_and_wait(uint64_t* bar, uint32_t parity,
-                                                unsigned long long limit_ns, int code) {
+                                                unsigned long long limit_ns, int code,
+                                                bool pre_ok = true) {
     if (threadIdx.x == 0) tc::mma_commit(bar);
-    const bool ok = tc::mbar_wait(bar, parity, limit_ns, nullptr);
+    const bool ok = tc::mbar_wait(bar, parity, limit_ns, nullptr) && pre_ok;
     if (!ok) atomicCAS(&g_scan_tc_status, 0, code);
     const bool all_ok = __syncthreads_and(ok ? 1 : 0) != 0;
     tc::tc_fence_after();
@@ -265,7 +298,8 @@ struct OutSmem {
     uint8_t c_tile[2][kT * 128];   // C of the tile, K-major, two 64-wide K blocks
     uint8_t b_src[2][256 * 128];   // B of the sources, K-major (rows s), two K blocks
     uint8_t x_src[256 * 128];      // X_h of the sources as fp16, MN-major (rows s)
-    uint8_t h_prev[2][kN * 128];   // H_[c-1] of head h, bf16 hi | lo, MN-major (rows n)
+    uint8_t h_prev[2][kN * 128];   // H_[c-1] of a head, bf16 hi | lo, MN-major (rows n); the
+                                   // second buffer of the pair is b_src, free after the scores
     float c2[256];                 // cum * log2(e) of the sources
     float e2[256];                 // c2 - log2(dt): exp2(c2_t - e2_s) = exp(cum_t - cum_s) dt_s
     float bfac[256];               // exp2(c2_r - e2_s), r = last source of s's group of 32
@@ -273,6 +307,7 @@ struct OutSmem {
     float cnorm[kT];               // |C_t| of the tile's rows
     uint32_t bdmax[2];             // max_s |B_s| dt_s of a head (float bits), by head parity
     uint64_t bar;
+    uint64_t hbar[2];              // H_[c-1] tile copy into buffer 0 / 1 landed
     uint32_t tmem_base;
 };
 
@@ -287,7 +322,6 @@ __device__ __forceinline__ float ex2_approx(float x) {
 // Next head's inputs, loaded into registers while the current head computes.
 struct HeadRegs {
     uint4 xv[8];    // X rows of the sources (bf16), 16-byte pieces i = tid + 256 k
-    float4 hv[8];   // H_[c-1] (fp32), pieces i = tid + 256 k (two float4 per 8-wide piece)
     float c2, dtv;  // source tid (tid < ns)
 };
 
@@ -295,7 +329,7 @@ template <typename Tout>
 __global__ void __launch_bounds__(kOutThreads, 1)
 chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restrict__ dt,
                        const float* __restrict__ cum, const __nv_bfloat16* __restrict__ Bm,
-                       const __nv_bfloat16* __restrict__ Cm, const float* __restrict__ Hin,
+                       const __nv_bfloat16* __restrict__ Cm, const uint8_t* __restrict__ Hops,
                        Tout* __restrict__ Y, int L, int H, int G, int S, int Mc,
                        unsigned long long wait_limit_ns) {
     extern __shared__ uint8_t smem_raw[];
@@ -317,12 +351,27 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
 
     if (tid == 0) {
         tc::mbar_init(&sm.bar, 1);
+        tc::mbar_init(&sm.hbar[0], 1);
+        tc::mbar_init(&sm.hbar[1], 1);
         tc::fence_barrier_init();
     }
     if (warp == 0) {
         tc::tmem_alloc(&sm.tmem_base, 512);
         tc::tmem_relinquish();
     }
+    // H_[c-1] tiles (bf16 hi | lo, 32 KiB per head, written swizzled by the state passing):
+    // head hh's copy goes to buffer hh & 1; only thread 0 issues, waits and drains them
+    auto hbuf = [&](int bi) -> uint8_t* { return bi ? sm.b_src[0] : sm.h_prev[0]; };
+    int hissued = 0;  // copies issued (thread 0)
+    auto issue_h = [&](int hh) {
+        const int bi = hh & 1;
+        const uint8_t* src = Hops + (((i64)b * Mc + c) * H + h0 + hh) * 32768;
+        tc::mbar_arrive_expect_tx(&sm.hbar[bi], 32768u);
+        tc::bulk_g2s(hbuf(bi), src, 32768u, &sm.hbar[bi]);
+        ++hissued;
+    };
+    __syncthreads();  // barriers initialised before any copy
+    if (tid == 0 && has_prev) issue_h(0);
     // C of the tile: row t, K-major, two K blocks of 64 (16-byte chunks, swizzled)
     for (int i = tid; i < kT * 16; i += kOutThreads) {
         const int t = i / 16, q = i % 16;
@@ -394,15 +443,6 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
                 nx.xv[k] = reinterpret_cast<const uint4*>(X + ((tok0 + sidx) * H + h) * kP)[q];
             }
         }
-        if (has_prev) {
-            const float* Hh = Hin + (((i64)b * Mc + c) * H + h) * (i64)(kN * kP);
-#pragma unroll
-            for (int k = 0; k < 4; ++k) {
-                const int i = tid + k * kOutThreads, n = i / 8, q = i % 8;
-                nx.hv[2 * k] = reinterpret_cast<const float4*>(Hh + n * kP)[2 * q];
-                nx.hv[2 * k + 1] = reinterpret_cast<const float4*>(Hh + n * kP)[2 * q + 1];
-            }
-        }
         if (tid < ns) {
             nx.c2 = cum[(((i64)b * H + h) * Mc + c) * S + tid] * kLog2e;
             nx.dtv = dt[(tok0 + tid) * H + h];
@@ -434,25 +474,6 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
                     make_uint4(f[0], f[1], f[2], f[3]);
             }
         }
-        if (has_prev) {
-#pragma unroll
-            for (int k = 0; k < 4; ++k) {
-                const int i = tid + k * kOutThreads, n = i / 8, q = i % 8;
-                const float4 a = nx.hv[2 * k], bb = nx.hv[2 * k + 1];
-                const float vals[8] = {a.x, a.y, a.z, a.w, bb.x, bb.y, bb.z, bb.w};
-                uint32_t hi[4], lo[4];
-#pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    const __nv_bfloat162 hv = __floats2bfloat162_rn(vals[2 * e], vals[2 * e + 1]);
-                    const float2 hf = __bfloat1622float2(hv);
-                    hi[e] = *reinterpret_cast<const uint32_t*>(&hv);
-                    lo[e] = pack_bf16(vals[2 * e] - hf.x, vals[2 * e + 1] - hf.y);
-                }
-                const uint32_t o = sw128((uint32_t)n, (uint32_t)q * 16u);
-                *reinterpret_cast<uint4*>(sm.h_prev[0] + o) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
-                *reinterpret_cast<uint4*>(sm.h_prev[1] + o) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
-            }
-        }
         if (tid < ns) {
             sm.c2[tid] = nx.c2;
             sm.e2[tid] = nx.c2 - log2f(nx.dtv);  // dt = 0 gives +inf: a zero weight
@@ -465,7 +486,11 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
         // sources ending at r; both factors are at most 1 (cum never rises) when r <= t
         if (tid < ns) sm.bfac[tid] = ex2_approx(sm.c2[tid | 31] - sm.e2[tid]);
         __syncthreads();
-        if (hh + 1 < kHeadsPerCta) load_head(h + 1);  // lands while this head computes
+        if (hh + 1 < kHeadsPerCta) {  // lands while this head computes
+            load_head(h + 1);
+            // buffer (hh + 1) & 1 was last read by head hh - 1's MMAs (or the scores), both done
+            if (tid == 0 && has_prev) issue_h(hh + 1);
+        }
 
         // W row of this thread over its half of the sources, scaled by the bound
         // 1 / (|C_t| max_s |B_s| dt_s) and stored fp16 in one pass
@@ -473,58 +498,69 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
         const float bound = sm.cnorm[row] * __uint_as_float(sm.bdmax[hh & 1]);
         const float wmax = bound > 0.0f ? bound : 1.0f;  // undone on the intra accumulator
         const float rscale = 1.0f / wmax;
-        for (int s0 = s_lo; s0 < s_hi; s0 += 32) {
+        // groups of 32 sources in pairs: both TMEM loads issued before one wait
+        auto w_group = [&](int s0, const float (&v)[32], bool live) {
             uint32_t pk[16];
-            if (s0 > tl_warp_max) {  // every row of the warp is before these sources
+            if (!live) {  // every row of the warp is before these sources
 #pragma unroll
                 for (int i = 0; i < 16; ++i) pk[i] = 0u;
-            } else {
-                float v[32];
-                tmem_ld32(tmem + lane_addr + kColSc + (uint32_t)s0, v);
-                if (s0 + 31 <= tl) {  // the whole group is at or before t: factored decay
-                    const float a = ex2_approx(c2t - sm.c2[s0 + 31]) * rscale;
+            } else if (s0 + 31 <= tl) {  // the whole group is at or before t: factored decay
+                const float a = ex2_approx(c2t - sm.c2[s0 + 31]) * rscale;
 #pragma unroll
-                    for (int i = 0; i < 16; ++i) {
-                        const float2 bf = *reinterpret_cast<const float2*>(&sm.bfac[s0 + 2 * i]);
-                        pk[i] = pack_f16(v[2 * i] * bf.x * a, v[2 * i + 1] * bf.y * a);
-                    }
-                } else {  // the group holding t: masked, one exp per element
+                for (int i = 0; i < 16; ++i) {
+                    const float2 bf = *reinterpret_cast<const float2*>(&sm.bfac[s0 + 2 * i]);
+                    pk[i] = pack_f16(v[2 * i] * bf.x * a, v[2 * i + 1] * bf.y * a);
+                }
+            } else {  // the group holding t: masked, one exp per element
 #pragma unroll
-                    for (int i = 0; i < 16; ++i) {
-                        const int sidx = s0 + 2 * i;
-                        const float w0 = sidx <= tl ? v[2 * i] * ex2_approx(c2t - sm.e2[sidx]) : 0.0f;
-                        const float w1 = sidx + 1 <= tl ? v[2 * i + 1] * ex2_approx(c2t - sm.e2[sidx + 1]) : 0.0f;
-                        pk[i] = pack_f16(w0 * rscale, w1 * rscale);
-                    }
+                for (int i = 0; i < 16; ++i) {
+                    const int sidx = s0 + 2 * i;
+                    const float w0 = sidx <= tl ? v[2 * i] * ex2_approx(c2t - sm.e2[sidx]) : 0.0f;
+                    const float w1 = sidx + 1 <= tl ? v[2 * i + 1] * ex2_approx(c2t - sm.e2[sidx + 1]) : 0.0f;
+                    pk[i] = pack_f16(w0 * rscale, w1 * rscale);
                 }
             }
             tc::tmem_st16(tmem + lane_addr + kColW + (uint32_t)(s0 / 2), pk);
+        };
+        for (int s0 = s_lo; s0 < s_hi; s0 += 64) {  // s_hi - s_lo is 64 or 128
+            const bool live0 = s0 <= tl_warp_max, live1 = s0 + 32 <= tl_warp_max;
+            float v0[32], v1[32];
+            if (live1)
+                tmem_ld32x2(tmem + lane_addr + kColSc + (uint32_t)s0,
+                            tmem + lane_addr + kColSc + (uint32_t)(s0 + 32), v0, v1);
+            else if (live0)
+                tmem_ld32(tmem + lane_addr + kColSc + (uint32_t)s0, v0);
+            w_group(s0, v0, live0);
+            w_group(s0 + 32, v1, live1);
         }
         asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
         tc::fence_proxy_async_shared();
         tc::tc_fence_before();
         __syncthreads();
+        bool hok = true;
         if (tid == 0) {
             tc::tc_fence_after();
+            if (has_prev) hok = tc::mbar_wait(&sm.hbar[hh & 1], (uint32_t)((hh >> 1) & 1), wait_limit_ns, nullptr);
             const uint32_t id16 = tc::idesc_f16(0, true, kT, kP);
             for (int ks = 0; ks < ns / 16; ++ks) {
                 const uint64_t bd = tc::smem_desc_sw128(tc::smem_u32(sm.x_src) + 2048u * ks, 1024u, 1024u);
                 tc::mma_f16_ts(tmem + kColIn, tmem + kColW + 8u * ks, bd, id16, ks > 0 ? 1u : 0u);
             }
-            if (has_prev) {
+            if (has_prev && hok) {
                 const uint32_t idb = tc::idesc_f16(1, true, kT, kP);
                 for (int part = 0; part < 2; ++part) {
                     for (int ks = 0; ks < kN / 16; ++ks) {
                         const uint64_t ad = tc::smem_desc_sw128(
                             tc::smem_u32(sm.c_tile[ks / 4]) + 32u * (ks % 4), 16u, 1024u);
                         const uint64_t bd = tc::smem_desc_sw128(
-                            tc::smem_u32(sm.h_prev[part]) + 2048u * ks, 1024u, 1024u);
+                            tc::smem_u32(hbuf(hh & 1) + 16384 * part) + 2048u * ks, 1024u, 1024u);
                         mma_f16_ss(tmem + kColEx, ad, bd, idb, (part > 0 || ks > 0) ? 1u : 0u);
                     }
                 }
             }
+            if (!hok) atomicCAS(&g_scan_tc_status, 0, 11);
         }
-        ok = commit_and_wait(&sm.bar, phase, wait_limit_ns, 3);
+        ok = commit_and_wait(&sm.bar, phase, wait_limit_ns, 3, hok);
         phase ^= 1u;
         if (!ok) break;
         // Y_t = wmax * (W~ X)_t + exp(cum_t) (C H)_t, columns 32 half .. 32 half + 31
@@ -548,6 +584,12 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
     if (!ok) {
         if (!tc::mbar_wait(&sm.bar, phase ^ 1u, kDrainLimitNs, nullptr))
             atomicCAS(&g_scan_tc_status, 0, 10);
+    }
+    // never leave an H copy in flight behind: wait for the last one into each buffer
+    if (tid == 0) {
+        for (int k = hissued - 1; k >= 0 && k >= hissued - 2; --k)
+            if (!tc::mbar_wait(&sm.hbar[k & 1], (uint32_t)((k >> 1) & 1), kDrainLimitNs, nullptr))
+                atomicCAS(&g_scan_tc_status, 0, 12);
     }
     tc::tc_fence_before();
     __syncthreads();
@@ -589,7 +631,7 @@ cudaError_t launch_chunk_scan_tc(const ScanArgs& a, unsigned long long wait_limi
         if (e != cudaSuccess) return e;
         kern<<<dim3(S / kT, M * (H / kHeadsPerCta), B), kOutThreads, smem, stream>>>(
             (const __nv_bfloat16*)a.X, a.dt, a.cum, (const __nv_bfloat16*)a.Bm,
-            (const __nv_bfloat16*)a.Cm, a.dH32, (Tout*)a.Y, L, H, G, S, M, wait_limit_ns);
+            (const __nv_bfloat16*)a.Cm, a.Hops, (Tout*)a.Y, L, H, G, S, M, wait_limit_ns);
     }
     note_launches(2);
     return cudaGetLastError();
