@@ -4,13 +4,15 @@
 // chunk-output kernels; the within-chunk cumsum and the inter-chunk state
 // passing stay as they are (scan.cu).
 //
-// chunk_state_tc_kernel, one CTA (128 threads) per (chunk c, head group, b):
+// chunk_state_tc_kernel, one CTA (256 threads) per (chunk c, head group, b):
 //   M_c = B_c^T (w (.) X_c),  w_s = exp(cum_end - cum_s) dt_s      (App. A)
 //   A = B_c^T sits in TMEM (lane n, K = s); the B operand w (.) X_c is staged
 //   per head as bf16 hi + lo (two MMAs, ~2^-16 relative) in the 128-byte
-//   swizzled MN-major layout. The epilogue (thread n = row n) writes the
-//   memory, its inverse RMS r (App. B.1) and the fp32 copy for state passing.
-// chunk_output_tc_kernel, one CTA (256 threads) per (128-token tile, chunk, head group, b):
+//   swizzled MN-major layout, from X rows prefetched into registers while the
+//   previous head computes. The epilogue (two threads per row n) writes the
+//   memory, its inverse RMS r (App. B.1) and, for bf16 memories, an fp32 copy
+//   for the state passing (fp32 memories are read by it directly).
+// chunk_output_tc_kernel, one CTA (512 threads) per (128-token tile, chunk, head group, b):
 //   scores = C_tile B_src^T                  (once, shared by the heads: G = 1)
 //   W_h[t,s] = scores[t,s] exp(cum_t - cum_s) dt_s  for s <= t, else 0
 //   Y_t = W_h X_h + exp(cum_t) C_t H_[c-1]   (App. A intra + inter terms)
@@ -25,6 +27,8 @@
 // TMEM of the output kernel: scores [0, 256), W [256, 384), intra accumulator
 // [384, 448), inter accumulator [448, 512).
 #include <math.h>
+
+#include <type_traits>
 
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
@@ -41,7 +45,6 @@ __device__ int g_scan_tc_status;  // first timeout code since the last read (0 =
 constexpr int kP = 64;
 constexpr int kN = 128;
 constexpr int kT = 128;  // tokens per output tile
-constexpr int kThreads = 128;
 constexpr int kHeadsPerCta = 8;
 constexpr uint64_t kDrainLimitNs = 2000000000ull;
 constexpr float kLog2e = 1.4426950408889634f;
@@ -78,35 +81,19 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
     for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
 
-// tcgen05.ld of 32 + 32 fp32 columns (two addresses) of this thread's lane, one wait.
-__device__ __forceinline__ void tmem_ld32x2(uint32_t ta, uint32_t tb, float (&va)[32], float (&vb)[32]) {
-    uint32_t r[64];
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
+    uint32_t r[16];
     asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
-        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
-        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%64];\n\t"
-        "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
-        "{%32,%33,%34,%35,%36,%37,%38,%39,%40,%41,%42,%43,%44,%45,%46,%47,"
-        "%48,%49,%50,%51,%52,%53,%54,%55,%56,%57,%58,%59,%60,%61,%62,%63}, [%65];\n\t"
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];\n\t"
         "tcgen05.wait::ld.sync.aligned;"
         : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
           "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
-          "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),
-          "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),
-          "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31]),
-          "=r"(r[32]), "=r"(r[33]), "=r"(r[34]), "=r"(r[35]), "=r"(r[36]), "=r"(r[37]),
-          "=r"(r[38]), "=r"(r[39]), "=r"(r[40]), "=r"(r[41]), "=r"(r[42]), "=r"(r[43]),
-          "=r"(r[44]), "=r"(r[45]), "=r"(r[46]), "=r"(r[47]), "=r"(r[48]), "=r"(r[49]),
-          "=r"(r[50]), "=r"(r[51]), "=r"(r[52]), "=r"(r[53]), "=r"(r[54]), "=r"(r[55]),
-          "=r"(r[56]), "=r"(r[57]), "=r"(r[58]), "=r"(r[59]), "=r"(r[60]), "=r"(r[61]),
-          "=r"(r[62]), "=r"(r[63])
-        : "r"(ta), "r"(tb)
+          "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr)
         : "memory");
 #pragma unroll
-    for (int i = 0; i < 32; ++i) {
-        va[i] = __uint_as_float(r[i]);
-        vb[i] = __uint_as_float(r[32 + i]);
-    }
+    for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
 }
 
 // D[tmem] (+)= A[smem] * B[smem]
@@ -135,18 +122,27 @@ __device__ __forceinline__ bool commit_and_wait(uint64_t* bar, uint32_t parity,
 }
 
 // ------------------------------------------------------------ chunk state
+constexpr int kStateThreads = 256;  // two threads per chunk row s and per memory row n
+
 struct StateSmem {
     union {
         uint8_t wx[2][256 * 128];        // (w (.) X) hi | lo: S rows x 128 bytes, swizzled
         __nv_bfloat16 b_rows[256 * kN];  // the chunk's B rows (only while building A)
     };
     float w[256];
+    float ssq[kN];  // sum of squares of the second half of each memory row
     uint64_t bar;
     uint32_t tmem_base;
 };
 
+// Next head's inputs, loaded into registers while the current head computes.
+struct StateRegs {
+    uint4 xv[8];           // X pieces i = tid + 256 k: row i / 8, 16-byte piece i % 8
+    float cumv, cend, dtv;  // cum of source tid and of the chunk's last token, dt of tid
+};
+
 template <typename Tmem>
-__global__ void __launch_bounds__(kThreads)
+__global__ void __launch_bounds__(kStateThreads, 2)
 chunk_state_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restrict__ dt,
                       const float* __restrict__ cum, const __nv_bfloat16* __restrict__ Bm,
                       float* __restrict__ dH32, Tmem* __restrict__ Mout, float* __restrict__ rM,
@@ -157,10 +153,11 @@ chunk_state_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restri
                                                   ~(uintptr_t)1023);
     const int c = blockIdx.x, hg = blockIdx.y, b = blockIdx.z;
     const int tid = threadIdx.x, warp = tid >> 5;
+    const int n = tid & (kN - 1), half = tid >> 7;  // memory row (TMEM lane) and column half
     const int h0 = hg * kHeadsPerCta;
     const int g = h0 / (H / G);
     const i64 tok0 = (i64)b * L + (i64)c * S;
-    const uint32_t lane_addr = (uint32_t)(32 * warp) << 16;
+    const uint32_t lane_addr = (uint32_t)(32 * (warp & 3)) << 16;
 
     if (tid == 0) {
         tc::mbar_init(&sm.bar, 1);
@@ -170,11 +167,30 @@ chunk_state_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restri
         tc::tmem_alloc(&sm.tmem_base, 256);
         tc::tmem_relinquish();
     }
+    // register prefetch of a head's sources
+    const int xiters = S * 8 / kStateThreads;  // 4 or 8 pieces of 16 bytes
+    StateRegs nx;
+    auto load_head = [&](int h) {
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            if (k < xiters) {
+                const int i = tid + k * kStateThreads, s = i / 8, q = i % 8;
+                nx.xv[k] = reinterpret_cast<const uint4*>(X + ((tok0 + s) * H + h) * kP)[q];
+            }
+        }
+        if (tid < S) {
+            const float* cumc = cum + (((i64)b * H + h) * Mc + c) * S;
+            nx.cumv = cumc[tid];
+            nx.cend = cumc[S - 1];
+            nx.dtv = dt[(tok0 + tid) * H + h];
+        }
+    };
+    load_head(h0);
     // the chunk's B rows into shared memory (16-byte loads)
     {
         uint4* dst = reinterpret_cast<uint4*>(sm.b_rows);
         const int per_row = kN * 2 / 16;  // 16
-        for (int i = tid; i < S * per_row; i += kThreads) {
+        for (int i = tid; i < S * per_row; i += kStateThreads) {
             const int s = i / per_row, q = i % per_row;
             dst[i] = reinterpret_cast<const uint4*>(Bm + ((tok0 + s) * G + g) * kN)[q];
         }
@@ -183,10 +199,11 @@ chunk_state_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restri
     __syncthreads();
     tc::tc_fence_after();
     const uint32_t tmem = sm.tmem_base;
-    // A = B^T into TMEM: lane n, columns s / 2 (bf16 pairs)
+    // A = B^T into TMEM: lane n, columns s / 2 (bf16 pairs); each half of the threads
+    // writes half of the columns
     {
-        const int n = tid;
-        for (int c0 = 0; c0 < S / 2; c0 += 16) {
+        const int cw = S / 4;  // 64 or 32 columns per half
+        for (int c0 = half * cw; c0 < (half + 1) * cw; c0 += 16) {
             uint32_t r[16];
 #pragma unroll
             for (int i = 0; i < 16; ++i) {
@@ -207,22 +224,15 @@ chunk_state_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restri
     bool ok = true;
     for (int hh = 0; hh < kHeadsPerCta && ok; ++hh) {
         const int h = h0 + hh;
-        const float* cumc = cum + (((i64)b * H + h) * Mc + c) * S;
-        const float cum_end = cumc[S - 1];
-        for (int s = tid; s < S; s += kThreads)
-            sm.w[s] = expf(cum_end - cumc[s]) * dt[(tok0 + s) * H + h];
+        if (tid < S) sm.w[tid] = expf(nx.cend - nx.cumv) * nx.dtv;
         __syncthreads();
         // stage (w (.) X_h) as bf16 hi / lo, rows s, 128-byte swizzle
-        for (int s = tid; s < S; s += kThreads) {
-            const uint4* xr = reinterpret_cast<const uint4*>(X + ((tok0 + s) * H + h) * kP);
-            const float ws = sm.w[s];
-            uint4 xrow[8];
 #pragma unroll
-            for (int q = 0; q < 8; ++q) xrow[q] = xr[q];
-#pragma unroll
-            for (int q = 0; q < 8; ++q) {  // 8 bf16 per 16-byte chunk
-                const uint4 xv = xrow[q];
-                const uint32_t xw[4] = {xv.x, xv.y, xv.z, xv.w};
+        for (int k = 0; k < 8; ++k) {
+            if (k < xiters) {
+                const int i = tid + k * kStateThreads, s = i / 8, q = i % 8;
+                const float ws = sm.w[s];
+                const uint32_t xw[4] = {nx.xv[k].x, nx.xv[k].y, nx.xv[k].z, nx.xv[k].w};
                 uint32_t hi[4], lo[4];
 #pragma unroll
                 for (int e = 0; e < 4; ++e) {
@@ -238,6 +248,7 @@ chunk_state_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restri
                 *reinterpret_cast<uint4*>(sm.wx[1] + o) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
             }
         }
+        if (hh + 1 < kHeadsPerCta) load_head(h + 1);  // lands while this head computes
         tc::fence_proxy_async_shared();
         tc::tc_fence_before();
         __syncthreads();
@@ -255,30 +266,29 @@ chunk_state_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restri
         ok = commit_and_wait(&sm.bar, phase, wait_limit_ns, 1);
         phase ^= 1u;
         if (!ok) break;
-        // epilogue: thread n = memory row n
+        // epilogue: row n of the memory, columns 32 half .. 32 half + 31
+        const i64 mrow = ((((i64)b * Mc + c) * H + h) * kN + n);
+        float ss = 0.0f;
         {
-            const int n = tid;
-            const i64 mrow = ((((i64)b * Mc + c) * H + h) * kN + n);
             float v[32];
-            float ss = 0.0f;
-#pragma unroll
-            for (int half = 0; half < 2; ++half) {
-                tmem_ld32(tmem + lane_addr + d_col + 32u * half, v);
+            tmem_ld32(tmem + lane_addr + d_col + 32u * half, v);
+            if (dH32 != nullptr) {
                 float4* d32 = reinterpret_cast<float4*>(dH32 + mrow * kP + 32 * half);
 #pragma unroll
                 for (int q = 0; q < 8; ++q)
                     d32[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
-                store_row32(Mout + mrow * kP + 32 * half, v);
-#pragma unroll
-                for (int i = 0; i < 32; ++i) {
-                    const float sv = stored_value<Tmem>(v[i]);
-                    ss = fmaf(sv, sv, ss);
-                }
             }
-            if (rM != nullptr) rM[mrow] = rsqrtf(ss / (float)kP + eps);
+            store_row32(Mout + mrow * kP + 32 * half, v);
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+                const float sv = stored_value<Tmem>(v[i]);
+                ss = fmaf(sv, sv, ss);
+            }
         }
+        if (half == 1) sm.ssq[n] = ss;
         tc::tc_fence_before();
         __syncthreads();  // the accumulator and the staging buffers are reused
+        if (half == 0 && rM != nullptr) rM[mrow] = rsqrtf((ss + sm.ssq[n]) / (float)kP + eps);
     }
     if (!ok) {  // a wait ran out: let the MMAs in flight finish before freeing TMEM
         if (!tc::mbar_wait(&sm.bar, phase ^ 1u, kDrainLimitNs, nullptr))
@@ -311,7 +321,7 @@ struct OutSmem {
     uint32_t tmem_base;
 };
 
-constexpr int kOutThreads = 256;  // two threads per token row
+constexpr int kOutThreads = 512;  // four threads per token row
 
 __device__ __forceinline__ float ex2_approx(float x) {
     float y;
@@ -321,7 +331,7 @@ __device__ __forceinline__ float ex2_approx(float x) {
 
 // Next head's inputs, loaded into registers while the current head computes.
 struct HeadRegs {
-    uint4 xv[8];    // X rows of the sources (bf16), 16-byte pieces i = tid + 256 k
+    uint4 xv[4];    // X rows of the sources (bf16), 16-byte pieces i = tid + 512 k
     float c2, dtv;  // source tid (tid < ns)
 };
 
@@ -339,8 +349,8 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
     const int c = blockIdx.y / (H / kHeadsPerCta);
     const int hg = blockIdx.y % (H / kHeadsPerCta);
     const int b = blockIdx.z;
-    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int row = tid & (kT - 1), half = tid >> 7;  // token row, half of the sources / columns
+    const int tid = threadIdx.x, warp = tid >> 5;
+    const int row = tid & (kT - 1), quarter = tid >> 7;  // token row, quarter of the sources / columns
     const int h0 = hg * kHeadsPerCta;
     const int g = h0 / (H / G);
     const int ns = (tt + 1) * kT;  // sources 0 .. ns-1 of the chunk
@@ -433,11 +443,11 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
     }
 
     // register prefetch of a head's sources (X rows, H_[c-1], cum, dt)
-    const int xiters = ns * 8 / kOutThreads;  // 4 or 8 pieces of 16 bytes
+    const int xiters = ns * 8 / kOutThreads;  // 2 or 4 pieces of 16 bytes
     HeadRegs nx;
     auto load_head = [&](int h) {
 #pragma unroll
-        for (int k = 0; k < 8; ++k) {
+        for (int k = 0; k < 4; ++k) {
             if (k < xiters) {
                 const int i = tid + k * kOutThreads, sidx = i / 8, q = i % 8;
                 nx.xv[k] = reinterpret_cast<const uint4*>(X + ((tok0 + sidx) * H + h) * kP)[q];
@@ -455,12 +465,12 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
     const int tl = tt * kT + row;  // this thread's token inside the chunk
     const i64 tok = tok0 + tl;
     const int tl_warp_max = tt * kT + 32 * (warp & 3) + 31;
-    const int s_lo = half * (ns / 2), s_hi = s_lo + ns / 2;
+    const int s_lo = quarter * (ns / 4), s_hi = s_lo + ns / 4;  // 32 or 64 sources
     for (int hh = 0; hh < kHeadsPerCta && ok; ++hh) {
         const int h = h0 + hh;
         // prefetched sources into shared memory (the previous head's MMAs are done)
 #pragma unroll
-        for (int k = 0; k < 8; ++k) {
+        for (int k = 0; k < 4; ++k) {
             if (k < xiters) {
                 const int i = tid + k * kOutThreads, sidx = i / 8, q = i % 8;
                 const uint32_t xw[4] = {nx.xv[k].x, nx.xv[k].y, nx.xv[k].z, nx.xv[k].w};
@@ -492,13 +502,12 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
             if (tid == 0 && has_prev) issue_h(hh + 1);
         }
 
-        // W row of this thread over its half of the sources, scaled by the bound
+        // W row of this thread over its quarter of the sources, scaled by the bound
         // 1 / (|C_t| max_s |B_s| dt_s) and stored fp16 in one pass
         const float c2t = sm.c2[tl];
         const float bound = sm.cnorm[row] * __uint_as_float(sm.bdmax[hh & 1]);
         const float wmax = bound > 0.0f ? bound : 1.0f;  // undone on the intra accumulator
         const float rscale = 1.0f / wmax;
-        // groups of 32 sources in pairs: both TMEM loads issued before one wait
         auto w_group = [&](int s0, const float (&v)[32], bool live) {
             uint32_t pk[16];
             if (!live) {  // every row of the warp is before these sources
@@ -522,16 +531,11 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
             }
             tc::tmem_st16(tmem + lane_addr + kColW + (uint32_t)(s0 / 2), pk);
         };
-        for (int s0 = s_lo; s0 < s_hi; s0 += 64) {  // s_hi - s_lo is 64 or 128
-            const bool live0 = s0 <= tl_warp_max, live1 = s0 + 32 <= tl_warp_max;
-            float v0[32], v1[32];
-            if (live1)
-                tmem_ld32x2(tmem + lane_addr + kColSc + (uint32_t)s0,
-                            tmem + lane_addr + kColSc + (uint32_t)(s0 + 32), v0, v1);
-            else if (live0)
-                tmem_ld32(tmem + lane_addr + kColSc + (uint32_t)s0, v0);
-            w_group(s0, v0, live0);
-            w_group(s0 + 32, v1, live1);
+        for (int s0 = s_lo; s0 < s_hi; s0 += 32) {  // s_hi - s_lo is 32 or 64
+            const bool live = s0 <= tl_warp_max;
+            float v[32];
+            if (live) tmem_ld32(tmem + lane_addr + kColSc + (uint32_t)s0, v);
+            w_group(s0, v, live);
         }
         asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
         tc::fence_proxy_async_shared();
@@ -563,20 +567,20 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
         ok = commit_and_wait(&sm.bar, phase, wait_limit_ns, 3, hok);
         phase ^= 1u;
         if (!ok) break;
-        // Y_t = wmax * (W~ X)_t + exp(cum_t) (C H)_t, columns 32 half .. 32 half + 31
+        // Y_t = wmax * (W~ X)_t + exp(cum_t) (C H)_t, columns 16 quarter .. 16 quarter + 15
         {
             const float dec = exp2f(c2t);
-            float vi[32], ve[32];
-            tmem_ld32(tmem + lane_addr + kColIn + 32u * half, vi);
+            float vi[16], ve[16];
+            tmem_ld16(tmem + lane_addr + kColIn + 16u * quarter, vi);
             if (has_prev) {
-                tmem_ld32(tmem + lane_addr + kColEx + 32u * half, ve);
+                tmem_ld16(tmem + lane_addr + kColEx + 16u * quarter, ve);
             } else {
 #pragma unroll
-                for (int i = 0; i < 32; ++i) ve[i] = 0.0f;
+                for (int i = 0; i < 16; ++i) ve[i] = 0.0f;
             }
 #pragma unroll
-            for (int i = 0; i < 32; ++i) vi[i] = fmaf(wmax, vi[i], dec * ve[i]);
-            store_row32(Y + (tok * H + h) * kP + 32 * half, vi);
+            for (int i = 0; i < 16; ++i) vi[i] = fmaf(wmax, vi[i], dec * ve[i]);
+            store_row16(Y + (tok * H + h) * kP + 16 * quarter, vi);
         }
         tc::tc_fence_before();
         __syncthreads();  // shared staging and TMEM are reused by the next head
@@ -611,6 +615,8 @@ template <typename Tmem, typename Tout>
 cudaError_t launch_chunk_scan_tc(const ScanArgs& a, unsigned long long wait_limit_ns,
                                  cudaStream_t stream) {
     const int B = (int)a.B, L = (int)a.L, H = (int)a.H, G = (int)a.G, S = (int)a.S, M = L / S;
+    constexpr bool mem_is_f32 = std::is_same<Tmem, float>::value;
+    if (a.Hops == nullptr) return cudaErrorInvalidValue;  // the output kernel's H_[c-1] tiles
     cudaError_t e0 = launch_chunk_cumsum(a, stream);
     if (e0 != cudaSuccess) return e0;
     {
@@ -618,11 +624,17 @@ cudaError_t launch_chunk_scan_tc(const ScanArgs& a, unsigned long long wait_limi
         const size_t smem = sizeof(StateSmem) + 1024;
         cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
-        kern<<<dim3(M, H / kHeadsPerCta, B), kThreads, smem, stream>>>(
-            (const __nv_bfloat16*)a.X, a.dt, a.cum, (const __nv_bfloat16*)a.Bm, a.dH32, (Tmem*)a.M,
-            a.rM, L, H, G, S, M, a.eps, wait_limit_ns);
+        kern<<<dim3(M, H / kHeadsPerCta, B), kStateThreads, smem, stream>>>(
+            (const __nv_bfloat16*)a.X, a.dt, a.cum, (const __nv_bfloat16*)a.Bm,
+            mem_is_f32 ? nullptr : a.dH32, (Tmem*)a.M, a.rM, L, H, G, S, M, a.eps, wait_limit_ns);
     }
-    e0 = launch_state_passing(a, stream);
+    {
+        // fp32 memories are the chunk states themselves: the state passing reads them
+        // (it writes only the operand tiles on this path, never its input)
+        ScanArgs sp = a;
+        if (mem_is_f32) sp.dH32 = (float*)a.M;
+        e0 = launch_state_passing(sp, stream);
+    }
     if (e0 != cudaSuccess) return e0;
     {
         auto kern = chunk_output_tc_kernel<Tout>;
