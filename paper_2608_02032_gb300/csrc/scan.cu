@@ -139,26 +139,14 @@ chunk_state_kernel(const Tin* __restrict__ X, const float* __restrict__ dt,
 
 // --------------------------------------------------------- 3. state passing
 // One thread per state element (n, p) of one (b, h); loops over chunks.
-// Byte offset of element (n, p) of a 128-row x 128-byte bf16 tile, 128-byte swizzle.
-__device__ __forceinline__ uint32_t sw128_elem(int n, int p) {
-    const uint32_t o = (uint32_t)n * 128u + (uint32_t)p * 2u;
-    return o ^ (((uint32_t)n & 7u) << 4);
-}
-
-__global__ void __launch_bounds__(256, 4)
-state_passing_kernel(float* __restrict__ dH32, const float* __restrict__ cum,
-                     float* __restrict__ final_state, uint8_t* __restrict__ Hops,
-                     int H, int M, int S, int P, int NP) {
+__global__ void state_passing_kernel(float* __restrict__ dH32, const float* __restrict__ cum,
+                                     float* __restrict__ final_state, int H, int M, int S, int NP) {
     const int e = blockIdx.x * blockDim.x + threadIdx.x;
     const int h = blockIdx.y, b = blockIdx.z;
     if (e >= NP) return;
     const float* cumh = cum + ((i64)b * H + h) * M * S;
     const i64 stride = (i64)H * NP;  // between chunk slots of the same element
     float* base = dH32 + ((i64)b * M * H + h) * NP + e;
-    // operand tiles: element (n, p) of chunk c's tile, hi at +0 and lo at +16 KiB
-    uint8_t* hop = Hops == nullptr ? nullptr
-                                   : Hops + ((i64)b * M * H + h) * 32768 + sw128_elem(e / P, e % P);
-    const i64 hstride = (i64)H * 32768;
     float st = 0.0f;
     // groups of 16 chunks: issue the independent loads first, then the chain
     for (int c0 = 0; c0 < M; c0 += 16) {
@@ -174,15 +162,7 @@ state_passing_kernel(float* __restrict__ dH32, const float* __restrict__ cum,
 #pragma unroll
         for (int k = 0; k < 16; ++k) {
             if (k < n) {
-                if (Hops == nullptr) {  // state entering chunk c0 + k
-                    base[(i64)(c0 + k) * stride] = st;
-                } else {  // the same state only as a bf16 hi | lo operand tile (P = 64)
-                    uint8_t* t = hop + (i64)(c0 + k) * hstride;
-                    const __nv_bfloat16 hi = __float2bfloat16_rn(st);
-                    *reinterpret_cast<__nv_bfloat16*>(t) = hi;
-                    *reinterpret_cast<__nv_bfloat16*>(t + 16384) =
-                        __float2bfloat16_rn(st - __bfloat162float(hi));
-                }
+                base[(i64)(c0 + k) * stride] = st;  // state entering chunk c0 + k
                 st = fmaf(dec[k], st, d[k]);
             }
         }
@@ -337,7 +317,7 @@ cudaError_t launch_state_passing(const ScanArgs& a, cudaStream_t stream) {
     const int B = (int)a.B, H = (int)a.H, S = (int)a.S, M = (int)(a.L / a.S);
     const int NP = (int)(a.N * a.P);
     state_passing_kernel<<<dim3((NP + 255) / 256, H, B), 256, 0, stream>>>(
-        a.dH32, a.cum, a.final_state, a.Hops, H, M, S, (int)a.P, NP);
+        a.dH32, a.cum, a.final_state, H, M, S, NP);
     note_launches(1);
     return cudaGetLastError();
 }
@@ -370,7 +350,6 @@ cudaError_t launch_scan_states(const ScanArgs& a0, float* cum, float* Hprev, flo
     a.M = scratch;
     a.rM = nullptr;
     a.final_state = nullptr;
-    a.Hops = nullptr;
     const int L = (int)a.L, H = (int)a.H, G = (int)a.G, P = (int)a.P, N = (int)a.N,
               S = (int)a.S, M = L / S;
     cudaError_t e = launch_chunk_cumsum(a, stream);

@@ -1,8 +1,9 @@
 // Chunked SSD scan on the 5th-generation tensor cores for bf16 token inputs,
 // P = 64, N = 128, S in {128, 256} (Sec. 2; Sec. 3 "Chunk State Memories";
-// App. A chunked scan). Two kernels replace the FFMA chunk-state and
-// chunk-output kernels; the within-chunk cumsum and the inter-chunk state
-// passing stay as they are (scan.cu).
+// App. A chunked scan). The chunk-state and chunk-output kernels run on the
+// tensor cores, the state passing streams the chunk states through shared
+// memory with bulk copies; the within-chunk cumsum is shared with the FFMA
+// path (scan.cu).
 //
 // chunk_state_tc_kernel, one CTA (256 threads) per (chunk c, head group, b):
 //   M_c = B_c^T (w (.) X_c),  w_s = exp(cum_end - cum_s) dt_s      (App. A)
@@ -301,6 +302,104 @@ chunk_state_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restri
         tc::tc_fence_after();
         tc::tmem_dealloc(tmem, 256);
     }
+}
+
+// ----------------------------------------------------------- state passing
+// H_[c] = exp(cum_end_c) H_[c-1] + dH_c over the chunks (App. A), written as the
+// output kernel's operand tiles: for each (b, c, h) the state entering chunk c
+// as bf16 hi | lo, 128-byte swizzled, 32 KiB. One CTA per (1024-element slab
+// of the N x P state, h, b); the slabs of successive chunks stream through a
+// ring of shared-memory stages filled by 4 KiB bulk copies, so the loads stay
+// in flight independently of the per-thread recurrence.
+constexpr int kSpThreads = 256;
+constexpr int kSpElems = 4;                     // consecutive (n, p) elements per thread
+constexpr int kSpSlab = kSpThreads * kSpElems;  // 1024 elements, 4 KiB per chunk
+constexpr int kSpStages = 8;
+constexpr int kSpDec = 1024;                    // chunk decays staged per block of chunks
+
+struct SpSmem {
+    float slab[kSpStages][kSpSlab];
+    float dec[kSpDec];
+    uint64_t full[kSpStages];
+};
+
+__global__ void __launch_bounds__(kSpThreads)
+state_passing_tc_kernel(const float* __restrict__ dH, const float* __restrict__ cum,
+                        float* __restrict__ final_state, uint8_t* __restrict__ Hops,
+                        int H, int M, int S, unsigned long long wait_limit_ns) {
+    __shared__ __align__(128) SpSmem sm;
+    constexpr int NP = kN * kP;
+    const int slab = blockIdx.x, h = blockIdx.y, b = blockIdx.z, tid = threadIdx.x;
+    const int e0 = slab * kSpSlab + tid * kSpElems;  // this thread's first element (n, p)
+    const int n = e0 / kP, p = e0 % kP;
+    const i64 cstride = (i64)H * NP;  // floats between the chunk slots of one (b, h)
+    const float* src = dH + ((i64)b * M * H + h) * NP + (i64)slab * kSpSlab;
+    uint8_t* hop = Hops + ((i64)b * M * H + h) * 32768 + sw128((uint32_t)n, (uint32_t)p * 2u);
+    const i64 hstride = (i64)H * 32768;
+    const float* cumh = cum + ((i64)b * H + h) * (i64)M * S;
+
+    if (tid == 0) {
+        for (int k = 0; k < kSpStages; ++k) tc::mbar_init(&sm.full[k], 1);
+        tc::fence_barrier_init();
+    }
+    __syncthreads();
+    int issued = 0;  // chunks whose copy thread 0 has issued
+    auto issue = [&](int c) {
+        const int stg = c % kSpStages;
+        tc::mbar_arrive_expect_tx(&sm.full[stg], (uint32_t)(kSpSlab * 4));
+        tc::bulk_g2s(sm.slab[stg], src + (i64)c * cstride, (uint32_t)(kSpSlab * 4), &sm.full[stg]);
+        ++issued;
+    };
+    if (tid == 0)
+        for (int c = 0; c < min(kSpStages, M); ++c) issue(c);
+    float st[kSpElems] = {0.0f, 0.0f, 0.0f, 0.0f};
+    bool ok = true;
+    int c = 0;
+    for (; c < M; ++c) {
+        if (c % kSpDec == 0) {
+            for (int i = tid; i < min(kSpDec, M - c); i += kSpThreads)
+                sm.dec[i] = expf(cumh[(i64)(c + i) * S + S - 1]);
+            __syncthreads();
+        }
+        const int stg = c % kSpStages;
+        const bool got = tc::mbar_wait(&sm.full[stg], (uint32_t)((c / kSpStages) & 1), wait_limit_ns, nullptr);
+        if (got) {
+            const float4 d = *reinterpret_cast<const float4*>(&sm.slab[stg][tid * kSpElems]);
+            // the state entering chunk c, as the split operand
+            uint32_t hi[2], lo[2];
+#pragma unroll
+            for (int k = 0; k < 2; ++k) {
+                const __nv_bfloat162 hv = __floats2bfloat162_rn(st[2 * k], st[2 * k + 1]);
+                const float2 hf = __bfloat1622float2(hv);
+                hi[k] = *reinterpret_cast<const uint32_t*>(&hv);
+                lo[k] = pack_bf16(st[2 * k] - hf.x, st[2 * k + 1] - hf.y);
+            }
+            uint8_t* t = hop + (i64)c * hstride;
+            *reinterpret_cast<uint2*>(t) = make_uint2(hi[0], hi[1]);
+            *reinterpret_cast<uint2*>(t + 16384) = make_uint2(lo[0], lo[1]);
+            const float a = sm.dec[c % kSpDec];
+            st[0] = fmaf(a, st[0], d.x);
+            st[1] = fmaf(a, st[1], d.y);
+            st[2] = fmaf(a, st[2], d.z);
+            st[3] = fmaf(a, st[3], d.w);
+        } else {
+            atomicCAS(&g_scan_tc_status, 0, 13);
+        }
+        // every thread has read the stage (and the decays) before it is refilled
+        ok = __syncthreads_and(got ? 1 : 0) != 0;
+        if (!ok) break;
+        if (tid == 0 && c + kSpStages < M) issue(c + kSpStages);
+    }
+    if (!ok && tid == 0) {  // let the copies in flight land before the CTA exits
+        for (int k = c; k < issued; ++k)
+            if (!tc::mbar_wait(&sm.full[k % kSpStages], (uint32_t)((k / kSpStages) & 1), kDrainLimitNs, nullptr)) {
+                atomicCAS(&g_scan_tc_status, 0, 14);
+                break;
+            }
+    }
+    if (ok && final_state != nullptr)
+        *reinterpret_cast<float4*>(final_state + ((i64)b * H + h) * NP + e0) =
+            make_float4(st[0], st[1], st[2], st[3]);
 }
 
 // ----------------------------------------------------------- chunk output
@@ -628,14 +727,10 @@ cudaError_t launch_chunk_scan_tc(const ScanArgs& a, unsigned long long wait_limi
             (const __nv_bfloat16*)a.X, a.dt, a.cum, (const __nv_bfloat16*)a.Bm,
             mem_is_f32 ? nullptr : a.dH32, (Tmem*)a.M, a.rM, L, H, G, S, M, a.eps, wait_limit_ns);
     }
-    {
-        // fp32 memories are the chunk states themselves: the state passing reads them
-        // (it writes only the operand tiles on this path, never its input)
-        ScanArgs sp = a;
-        if (mem_is_f32) sp.dH32 = (float*)a.M;
-        e0 = launch_state_passing(sp, stream);
-    }
-    if (e0 != cudaSuccess) return e0;
+    // fp32 memories are the chunk states themselves: the state passing reads them
+    state_passing_tc_kernel<<<dim3(kN * kP / kSpSlab, H, B), kSpThreads, 0, stream>>>(
+        mem_is_f32 ? (const float*)a.M : a.dH32, a.cum, a.final_state, a.Hops, H, M, S,
+        wait_limit_ns);
     {
         auto kern = chunk_output_tc_kernel<Tout>;
         const size_t smem = sizeof(OutSmem) + 1024;
@@ -645,7 +740,7 @@ cudaError_t launch_chunk_scan_tc(const ScanArgs& a, unsigned long long wait_limi
             (const __nv_bfloat16*)a.X, a.dt, a.cum, (const __nv_bfloat16*)a.Bm,
             (const __nv_bfloat16*)a.Cm, a.Hops, (Tout*)a.Y, L, H, G, S, M, wait_limit_ns);
     }
-    note_launches(2);
+    note_launches(3);
     return cudaGetLastError();
 }
 
