@@ -107,5 +107,10 @@ __device__ __forceinline__ void store_row16(__nv_bfloat16* dst, const float* v) 
 
 // SiLU(z) = z * sigmoid(z), the SMA residual gate (Sec. 3).
 __device__ __forceinline__ float silu_f32(float z) { return z / (1.0f + expf(-z)); }
+// d SiLU / dz = s (1 + z (1 - s)), s = sigmoid(z)
+__device__ __forceinline__ float silu_grad_f32(float z) {
+    const float s = 1.0f / (1.0f + expf(-z));
+    return s * (1.0f + z * (1.0f - s));
+}
 
 }  // namespace dart

@@ -126,6 +126,17 @@ bool sma_uses_tc(const dart_dims* d) {
     return d->in_dtype == DART_BF16 && dart::sma_tc_supported(sma_args(d));
 }
 
+// The tensor-core SMA backward serves bf16 token inputs at its tile shape with G = 1.
+dart::SmaBwdArgs sma_bwd_args(const dart_dims* d) {
+    dart::SmaBwdArgs a{};
+    a.B = d->batch; a.L = d->seqlen; a.H = d->nheads; a.G = d->ngroups;
+    a.P = d->headdim; a.N = d->dstate; a.S = d->chunk; a.eps = d->eps;
+    return a;
+}
+bool sma_bwd_uses_tc(const dart_dims* d) {
+    return d->in_dtype == DART_BF16 && dart::sma_bwd_tc_supported(sma_bwd_args(d));
+}
+
 size_t sma_ws(const dart_dims* d) {
     const i64 M = d->seqlen / d->chunk;
     if (sma_uses_tc(d)) return align256(dart::sma_tc_workspace(d->batch, M, d->nheads));
@@ -178,6 +189,9 @@ size_t dart_workspace_size(const dart_dims* d, int op) {
             return 0;
         case DART_OP_SMA_BACKWARD:
             if (check_dims(d, true) != DART_OK) return 0;
+            if (sma_bwd_uses_tc(d))
+                return align256(dart::sma_bwd_tc_workspace(d->batch, d->seqlen, d->nheads,
+                                                           d->seqlen / d->chunk, d->dstate));
             return align256(dart::sma_bwd_workspace(d->batch, d->seqlen, d->nheads,
                                                     d->seqlen / d->chunk, d->dstate));
         case DART_OP_SCAN_BACKWARD:
@@ -318,15 +332,19 @@ dart_status dart_sma_backward(const dart_dims* d, const void* M, const float* rM
     if (rM != nullptr && !aligned16(rM)) return DART_ERR_INVALID_ARG;
     const size_t need = dart_workspace_size(d, DART_OP_SMA_BACKWARD);
     if (ws == nullptr || ((uintptr_t)ws & 255u) != 0 || ws_bytes < need) return DART_ERR_WORKSPACE;
-    dart::SmaBwdArgs a;
-    a.B = d->batch; a.L = d->seqlen; a.H = d->nheads; a.G = d->ngroups;
-    a.P = d->headdim; a.N = d->dstate; a.S = d->chunk; a.eps = d->eps;
+    dart::SmaBwdArgs a = sma_bwd_args(d);
     a.M = M; a.rM = rM; a.Q = Q; a.Cm = Cm; a.E = E; a.z = z; a.lse = lse; a.dY = dY;
     a.dM = dM; a.dQ = dQ; a.dC = dC; a.dE = dE; a.dz = dz;
     cudaStream_t s = (cudaStream_t)stream;
     typedef __nv_bfloat16 bf;
     cudaError_t e;
-    if (d->in_dtype == DART_F32 && d->mem_dtype == DART_F32)
+    if (sma_bwd_uses_tc(d)) {
+        const unsigned long long lim = g_wait_limit_ns.load();
+        if (d->mem_dtype == DART_F32)
+            e = dart::launch_sma_backward_tc<float>(a, ws, lim, s);
+        else
+            e = dart::launch_sma_backward_tc<bf>(a, ws, lim, s);
+    } else if (d->in_dtype == DART_F32 && d->mem_dtype == DART_F32)
         e = dart::launch_sma_backward<float, float>(a, ws, s);
     else if (d->in_dtype == DART_BF16 && d->mem_dtype == DART_F32)
         e = dart::launch_sma_backward<bf, float>(a, ws, s);
@@ -373,8 +391,9 @@ dart_status dart_get_device_status(void* stream) {
     if (e != cudaSuccess) return cuda_fail(e);
     const int code = dart::take_tc_status();
     const int code2 = dart::take_scan_tc_status();
-    if (code < 0 || code2 < 0) return cuda_fail(cudaGetLastError());
-    return (code != 0 || code2 != 0) ? DART_ERR_TIMEOUT : DART_OK;
+    const int code3 = dart::take_bwd_tc_status();
+    if (code < 0 || code2 < 0 || code3 < 0) return cuda_fail(cudaGetLastError());
+    return (code != 0 || code2 != 0 || code3 != 0) ? DART_ERR_TIMEOUT : DART_OK;
 }
 
 void dart_test_withhold_copies(int on) { g_test_withhold.store(on != 0 ? 1 : 0); }

@@ -150,4 +150,16 @@ cudaError_t launch_sma_forward_tc(const SmaArgs& a, void* ws, unsigned long long
 // Reads and clears the tensor-core kernels' timeout code (0 = none, -1 = read failed).
 int take_tc_status();
 
+// Tensor-core SMA backward (sma_bwd_tc.cu; statistics pass in sma_tc.cu).
+template <typename Tmem>
+cudaError_t launch_sma_bwd_stats_tc(const SmaBwdArgs& a, const float* rM, uint8_t* ops,
+                                    int pair_bytes, float* scale, float* g, float2* gd,
+                                    unsigned long long wait_limit_ns, cudaStream_t stream);
+bool sma_bwd_tc_supported(const SmaBwdArgs& a);
+size_t sma_bwd_tc_workspace(int64_t B, int64_t L, int64_t H, int64_t Mc, int64_t N);
+template <typename Tmem>
+cudaError_t launch_sma_backward_tc(const SmaBwdArgs& a, void* ws, unsigned long long wait_limit_ns,
+                                   cudaStream_t stream);
+int take_bwd_tc_status();
+
 }  // namespace dart

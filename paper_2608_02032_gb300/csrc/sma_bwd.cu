@@ -30,11 +30,6 @@ namespace {
 constexpr int kBT = 64;  // tokens per tile
 constexpr int kPad = 65; // padded row of 64 floats (conflict-free column walks)
 
-__device__ __forceinline__ float silu_grad(float z) {
-    const float s = 1.0f / (1.0f + expf(-z));
-    return s * (1.0f + z * (1.0f - s));
-}
-
 // Warp lanes 16 apart hold the same token row of a 16-wide tx group: sums
 // over the 16 lanes of a half-warp.
 __device__ __forceinline__ float sum16(float v) {
@@ -191,7 +186,7 @@ sma_bwd_rows_kernel(const Tmem* __restrict__ Mem, const float* __restrict__ rM,
         }
         Dt[i] = sum16(dr);
         dyr = sum16(dyr);
-        if (tx == 0 && tl < ntok) dz[row] = nh[i] > 0 ? dyr * silu_grad(ld_f32(z + row)) : 0.0f;
+        if (tx == 0 && tl < ntok) dz[row] = nh[i] > 0 ? dyr * silu_grad_f32(ld_f32(z + row)) : 0.0f;
     }
 
     // ---- pass 2: dl, dEbar (t x p layout), dQbar and dC (t x n layout: n = tx + 16 k)

@@ -112,21 +112,23 @@ __device__ __forceinline__ uint32_t sw128(int n, int p) {
 // ------------------------------------------------------------ kernel 1
 // One block of 256 threads per (j, h, b) memory. Warp w owns rows n = w + 8k;
 // lane owns columns p = lane, lane + 32. Head h = 2 hp + x writes its tile x
-// of each of the three parts of ops + ((b Mc + j) (H/2) + hp) kPair.
+// of each part of ops + ((b Mc + j) (H/2) + hp) pair_bytes: W_hi, W_lo, M16
+// and, when pair_bytes holds five parts (the backward), M split bf16 hi + lo.
 template <typename Tmem>
 __global__ void __launch_bounds__(256)
 sma_operands_kernel(const Tmem* __restrict__ M, const float* __restrict__ rM,
                     uint8_t* __restrict__ ops, float* __restrict__ scale, int Mc, int H,
-                    float eps) {
+                    float eps, int pair_bytes) {
     const int j = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const i64 mem = ((i64)b * Mc + j) * H + h;
     const Tmem* src = M + mem * (kN * kP);
     const i64 pair = ((i64)b * Mc + j) * (H / kHeadsPerCta) + h / kHeadsPerCta;
     const int x = h % kHeadsPerCta;
-    uint8_t* dst_hi = ops + pair * kPair + x * kTile;
+    uint8_t* dst_hi = ops + pair * pair_bytes + x * kTile;
     uint8_t* dst_lo = dst_hi + kPart;
     uint8_t* dst_v = dst_hi + 2 * kPart;
+    uint8_t* dst_mb = pair_bytes > kPair ? dst_hi + 3 * kPart : nullptr;  // then + kPart: lo
     __shared__ float s_max[8];
 
     float v0[16], v1[16], rr[16];
@@ -166,6 +168,11 @@ sma_operands_kernel(const Tmem* __restrict__ M, const float* __restrict__ rM,
             *reinterpret_cast<__nv_bfloat16*>(dst_hi + o) = hi;
             *reinterpret_cast<__nv_bfloat16*>(dst_lo + o) = lo;
             *reinterpret_cast<__half*>(dst_v + o) = m16;
+            if (dst_mb != nullptr) {
+                const __nv_bfloat16 mh = __float2bfloat16_rn(v);
+                *reinterpret_cast<__nv_bfloat16*>(dst_mb + o) = mh;
+                *reinterpret_cast<__nv_bfloat16*>(dst_mb + kPart + o) = __float2bfloat16_rn(v - __bfloat162float(mh));
+            }
         }
     }
 }
@@ -295,14 +302,23 @@ __device__ __forceinline__ void issue_part(uint32_t d_tmem, uint32_t a_tmem, uin
         tc::mma_f16_ts(d_tmem, a_tmem + 8u * ks, b_desc + 128u * ks, kIdesc, ks > 0 ? 1u : first_acc);
 }
 
-template <typename Tout>
+// What the backward-statistics variant (kStats) writes instead of the merge:
+// the softmax weights g_{t,j} = exp(l_{t,j} - lse_t) (lse from the forward)
+// and their sum G1_t. It runs the U half of each job only (parts W_hi, W_lo;
+// no value chain).
+struct SmaStats {
+    float* g;    // B x H x Mc x L
+    float2* gd;  // B x L x H: (G1, -) -- the second field is written later
+};
+
+template <typename Tout, bool kStats>
 __global__ void __launch_bounds__(kThreads, 1)
 sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
               const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* __restrict__ Cm,
               const __nv_bfloat16* __restrict__ E, const __nv_bfloat16* __restrict__ z,
               const Tout* __restrict__ Yssd, Tout* __restrict__ Y, Tout* __restrict__ R,
               float* __restrict__ lse, int Bsz, int L, int H, int G, int S, int Mc, float eps,
-              unsigned long long wait_limit_ns, int withhold) {
+              unsigned long long wait_limit_ns, int withhold, int pair_bytes, SmaStats st) {
     extern __shared__ uint8_t smem_raw[];
     TcSmem& sm = *reinterpret_cast<TcSmem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                             ~(uintptr_t)1023);
@@ -356,8 +372,8 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
         // ------------------------------------------------------- producer
         // one 96 KiB copy per job: part p of job j lands in stage 3 (j & 1) + p
         if (lane == 0) {
-            const uint8_t* src = ops + ((i64)b * Mc * hpairs + hp) * (i64)kPair;
-            const i64 job_stride = (i64)hpairs * kPair;
+            const uint8_t* src = ops + ((i64)b * Mc * hpairs + hp) * (i64)pair_bytes;
+            const i64 job_stride = (i64)hpairs * pair_bytes;
             bool ok = true;
             int njobs = 0;  // jobs whose copy was issued
             // (withhold: the failure-path test hook; every wait on the operands then runs out)
@@ -368,14 +384,15 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
                 const uint32_t par = (uint32_t)((j >> 1) & 1) ^ 1u;
                 ok = (j != 1 || tc::mbar_wait(&sm.a_ready, 0, wait_limit_ns, abort)) &&
                      tc::mbar_wait(&sm.uready[ub], par, wait_limit_ns, abort) &&
-                     tc::mbar_wait(&sm.vready[ub], par, wait_limit_ns, abort);
+                     (kStats || tc::mbar_wait(&sm.vready[ub], par, wait_limit_ns, abort));
                 if (!ok) {
                     fail(abort, 1);
                     break;
                 }
                 // the job's hi, lo and value parts are contiguous in global and in the ring
-                tc::mbar_arrive_expect_tx(&sm.full[ub], (uint32_t)kPair);
-                tc::bulk_g2s(sm.stage[kPartsPerJob * ub], src + j * job_stride, (uint32_t)kPair, &sm.full[ub]);
+                constexpr uint32_t bytes = kStats ? 2 * kPart : kPair;
+                tc::mbar_arrive_expect_tx(&sm.full[ub], bytes);
+                tc::bulk_g2s(sm.stage[kPartsPerJob * ub], src + j * job_stride, bytes, &sm.full[ub]);
                 ++njobs;
             }
             // never leave a copy in flight behind: wait for the last copy into each half
@@ -398,16 +415,18 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
                 const uint32_t par = (uint32_t)((j >> 1) & 1);
                 const uint64_t bd = desc0 + (uint64_t)((s0 * kPart) >> 4);
                 ok = tc::mbar_wait(&sm.u_free, (uint32_t)ub ^ 1u, wait_limit_ns, abort) &&
-                     tc::mbar_wait(&sm.v_free[ub], par ^ 1u, wait_limit_ns, abort);
+                     (kStats || tc::mbar_wait(&sm.v_free[ub], par ^ 1u, wait_limit_ns, abort));
                 tc::tc_fence_after();
                 ok = ok && tc::mbar_wait(&sm.full[ub], par, wait_limit_ns, abort);
                 if (!ok) break;
                 issue_part<kIdescU, 0u>(tmem + kColU, tmem + kColQ, bd);
                 issue_part<kIdescU, 1u>(tmem + kColU, tmem + kColQ, bd + (uint64_t)(kPart >> 4));
                 tc::mma_commit(&sm.uready[ub]);
-                issue_part<kIdescV, 0u>(tmem + kColV + 128u * (uint32_t)ub, tmem + kColC,
-                                        bd + (uint64_t)((2 * kPart) >> 4));
-                tc::mma_commit(&sm.vready[ub]);
+                if (!kStats) {
+                    issue_part<kIdescV, 0u>(tmem + kColV + 128u * (uint32_t)ub, tmem + kColC,
+                                            bd + (uint64_t)((2 * kPart) >> 4));
+                    tc::mma_commit(&sm.vready[ub]);
+                }
                 issued = true;
             }
             if (!ok) fail(abort, 3);
@@ -516,112 +535,149 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
         const float lfac = sm.lq[row];
         const float cdown = sm.cdown[row];
 
-        uint64_t O[kP / 2];  // running sum of w_j V_j as fp32 pairs
-#pragma unroll
-        for (int i = 0; i < kP / 2; ++i) O[i] = 0ull;
-        float m = -INFINITY, dsum = 0.0f;
-        bool ok = true;
-        const float* scl = scale + (i64)b * Mc * H + h;  // scale of memory j at scl[j H]
-        float s_next = nj > 0 ? __ldg(scl) : 0.0f;
-        const uint32_t ua = tmem + lane_addr + kColU + (uint32_t)(kP * wg);
-        const uint32_t va = tmem + lane_addr + kColV + (uint32_t)(kP * wg);  // + 128 per V buffer
-        // the merge's Y_ssd row and gate come from L2 if fetched a few jobs ahead
-        const i64 rowo_pf = tok * H + h;
-        const int pf_job = nj > 4 ? nj - 4 : 0;
-        if (nj == 0) prefetch_row<kP * (int)sizeof(Tout)>(Yssd + rowo_pf * kP, z + rowo_pf);
-        for (int j = 0; j < nj; ++j) {
-            const int ub = j & 1;
-            const float s_j = s_next;
-            if (j == pf_job) prefetch_row<kP * (int)sizeof(Tout)>(Yssd + rowo_pf * kP, z + rowo_pf);
-            if (j + 1 < nj) s_next = __ldg(scl + (i64)(j + 1) * H);  // one job ahead
-            if (!warp_wait(&sm.uready[ub], (uint32_t)((j >> 1) & 1), wait_limit_ns, abort)) {
-                fail(abort, 4);
-                ok = false;
-                break;
-            }
-            tc::tc_fence_after();
-            float l;
-            {
-                uint64_t acc = 0ull, v[16];
-                tmem_ld32p(ua, v);
-#pragma unroll
-                for (int i = 0; i < 16; ++i) acc = f2_fma(v[i], eb[i], acc);
-                tmem_ld32p(ua + 32u, v);
-                warp_release(&sm.u_free);
-#pragma unroll
-                for (int i = 0; i < 16; ++i) acc = f2_fma(v[i], eb[16 + i], acc);
-                float lx, ly;
-                f2_unpack(acc, lx, ly);
-                l = (lx + ly) * lfac;
-            }
-            // online softmax; the running sums are rescaled only when the maximum moves
-            if (l > m) {
-                const float sc = expf(m - l);
-                const uint64_t sc2 = f2_pack(sc, sc);
-#pragma unroll
-                for (int i = 0; i < kP / 2; ++i) O[i] = f2_mul(O[i], sc2);
-                dsum *= sc;
-                m = l;
-            }
-            const float pe = expf(l - m);
-            dsum += pe;
-            const float w = pe * s_j;
-            const uint64_t w2 = f2_pack(w, w);
-            if (!warp_wait(&sm.vready[ub], (uint32_t)((j >> 1) & 1), wait_limit_ns, abort)) {
-                fail(abort, 4);
-                ok = false;
-                break;
-            }
-            tc::tc_fence_after();
-            {
-                uint64_t v[16];
-                tmem_ld32p(va + 128u * ub, v);
-#pragma unroll
-                for (int i = 0; i < 16; ++i) O[i] = f2_fma(w2, v[i], O[i]);
-                tmem_ld32p(va + 128u * ub + 32u, v);
-                warp_release(&sm.v_free[ub]);
-#pragma unroll
-                for (int i = 0; i < 16; ++i) O[16 + i] = f2_fma(w2, v[i], O[16 + i]);
-            }
-        }
-        if (ok) {
-            // R = O / d (C's row scale undone), lse, gated merge. Every MMA is done
-            // (the last job's V was read, or there were no jobs), so the ring is free
-            // for the row transposes: Y_ssd in, Y and R out.
-            constexpr int kRowB = kP * (int)sizeof(Tout);
+        if constexpr (kStats) {
+            // backward statistics: g_{t,j} = exp(l_{t,j} - lse_t) and G1_t = sum_j g
             const i64 rowo = tok * H + h;
-            const i64 row0 = tok0 * H + h;  // this warp's first output row
-            uint8_t* yslots = sm.stage[0] + (warp - 4) * 2 * kSlots;
-            uint8_t* rslots = yslots + kSlots;
-            const i64 rstride = (i64)H * kRowB;
-            const bool has = nj > 0;
-            const float inv_d = has ? cdown / dsum : 0.0f;
-            const float gate = silu_f32(__bfloat162float(z[rowo]));
-            rows_to_slots<kRowB>(yslots, reinterpret_cast<const uint8_t*>(Yssd + row0 * kP), rstride, lane);
-            float r[kP];
+            const float lse_t = lse[rowo];
+            float G1 = 0.0f;
+            bool ok = true;
+            const uint32_t ua = tmem + lane_addr + kColU + (uint32_t)(kP * wg);
+            float* gp = st.g + ((i64)b * H + h) * Mc * L + t;  // + j L
+            for (int j = 0; j < nj; ++j) {
+                const int ub = j & 1;
+                if (!warp_wait(&sm.uready[ub], (uint32_t)((j >> 1) & 1), wait_limit_ns, abort)) {
+                    fail(abort, 4);
+                    ok = false;
+                    break;
+                }
+                tc::tc_fence_after();
+                float l;
+                {
+                    uint64_t acc = 0ull, v[16];
+                    tmem_ld32p(ua, v);
 #pragma unroll
-            for (int i = 0; i < kP / 2; ++i) {
-                f2_unpack(O[i], r[2 * i], r[2 * i + 1]);
-                r[2 * i] *= inv_d;
-                r[2 * i + 1] *= inv_d;
+                    for (int i = 0; i < 16; ++i) acc = f2_fma(v[i], eb[i], acc);
+                    tmem_ld32p(ua + 32u, v);
+                    warp_release(&sm.u_free);
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) acc = f2_fma(v[i], eb[16 + i], acc);
+                    float lx, ly;
+                    f2_unpack(acc, lx, ly);
+                    l = (lx + ly) * lfac;
+                }
+                const float gw = expf(l - lse_t);
+                G1 += gw;
+                gp[(i64)j * L] = gw;
             }
-            Tout* rs = reinterpret_cast<Tout*>(rslots + lane * (kRowB + 16));
-            Tout* ys = reinterpret_cast<Tout*>(yslots + lane * (kRowB + 16));
-#pragma unroll
-            for (int c = 0; c < 4; ++c) store_row16(rs + 16 * c, r + 16 * c);
-            if (lse != nullptr) lse[rowo] = has ? m + logf(dsum) : -INFINITY;
-            __syncwarp();
-#pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                float y[16];
-                load_row16(ys + 16 * c, y);
-#pragma unroll
-                for (int i = 0; i < 16; ++i) y[i] = fmaf(gate, r[16 * c + i], y[i]);
-                store_row16(ys + 16 * c, y);
+            if (ok) st.gd[rowo] = make_float2(G1, 0.0f);
+        } else {
+            uint64_t O[kP / 2];  // running sum of w_j V_j as fp32 pairs
+    #pragma unroll
+            for (int i = 0; i < kP / 2; ++i) O[i] = 0ull;
+            float m = -INFINITY, dsum = 0.0f;
+            bool ok = true;
+            const float* scl = scale + (i64)b * Mc * H + h;  // scale of memory j at scl[j H]
+            float s_next = nj > 0 ? __ldg(scl) : 0.0f;
+            const uint32_t ua = tmem + lane_addr + kColU + (uint32_t)(kP * wg);
+            const uint32_t va = tmem + lane_addr + kColV + (uint32_t)(kP * wg);  // + 128 per V buffer
+            // the merge's Y_ssd row and gate come from L2 if fetched a few jobs ahead
+            const i64 rowo_pf = tok * H + h;
+            const int pf_job = nj > 4 ? nj - 4 : 0;
+            if (nj == 0) prefetch_row<kP * (int)sizeof(Tout)>(Yssd + rowo_pf * kP, z + rowo_pf);
+            for (int j = 0; j < nj; ++j) {
+                const int ub = j & 1;
+                const float s_j = s_next;
+                if (j == pf_job) prefetch_row<kP * (int)sizeof(Tout)>(Yssd + rowo_pf * kP, z + rowo_pf);
+                if (j + 1 < nj) s_next = __ldg(scl + (i64)(j + 1) * H);  // one job ahead
+                if (!warp_wait(&sm.uready[ub], (uint32_t)((j >> 1) & 1), wait_limit_ns, abort)) {
+                    fail(abort, 4);
+                    ok = false;
+                    break;
+                }
+                tc::tc_fence_after();
+                float l;
+                {
+                    uint64_t acc = 0ull, v[16];
+                    tmem_ld32p(ua, v);
+    #pragma unroll
+                    for (int i = 0; i < 16; ++i) acc = f2_fma(v[i], eb[i], acc);
+                    tmem_ld32p(ua + 32u, v);
+                    warp_release(&sm.u_free);
+    #pragma unroll
+                    for (int i = 0; i < 16; ++i) acc = f2_fma(v[i], eb[16 + i], acc);
+                    float lx, ly;
+                    f2_unpack(acc, lx, ly);
+                    l = (lx + ly) * lfac;
+                }
+                // online softmax; the running sums are rescaled only when the maximum moves
+                if (l > m) {
+                    const float sc = expf(m - l);
+                    const uint64_t sc2 = f2_pack(sc, sc);
+    #pragma unroll
+                    for (int i = 0; i < kP / 2; ++i) O[i] = f2_mul(O[i], sc2);
+                    dsum *= sc;
+                    m = l;
+                }
+                const float pe = expf(l - m);
+                dsum += pe;
+                const float w = pe * s_j;
+                const uint64_t w2 = f2_pack(w, w);
+                if (!warp_wait(&sm.vready[ub], (uint32_t)((j >> 1) & 1), wait_limit_ns, abort)) {
+                    fail(abort, 4);
+                    ok = false;
+                    break;
+                }
+                tc::tc_fence_after();
+                {
+                    uint64_t v[16];
+                    tmem_ld32p(va + 128u * ub, v);
+    #pragma unroll
+                    for (int i = 0; i < 16; ++i) O[i] = f2_fma(w2, v[i], O[i]);
+                    tmem_ld32p(va + 128u * ub + 32u, v);
+                    warp_release(&sm.v_free[ub]);
+    #pragma unroll
+                    for (int i = 0; i < 16; ++i) O[16 + i] = f2_fma(w2, v[i], O[16 + i]);
+                }
             }
-            __syncwarp();
-            slots_to_rows<kRowB>(reinterpret_cast<uint8_t*>(Y + row0 * kP), rstride, yslots, lane);
-            if (R != nullptr) slots_to_rows<kRowB>(reinterpret_cast<uint8_t*>(R + row0 * kP), rstride, rslots, lane);
+            if (ok) {
+                // R = O / d (C's row scale undone), lse, gated merge. Every MMA is done
+                // (the last job's V was read, or there were no jobs), so the ring is free
+                // for the row transposes: Y_ssd in, Y and R out.
+                constexpr int kRowB = kP * (int)sizeof(Tout);
+                const i64 rowo = tok * H + h;
+                const i64 row0 = tok0 * H + h;  // this warp's first output row
+                uint8_t* yslots = sm.stage[0] + (warp - 4) * 2 * kSlots;
+                uint8_t* rslots = yslots + kSlots;
+                const i64 rstride = (i64)H * kRowB;
+                const bool has = nj > 0;
+                const float inv_d = has ? cdown / dsum : 0.0f;
+                const float gate = silu_f32(__bfloat162float(z[rowo]));
+                rows_to_slots<kRowB>(yslots, reinterpret_cast<const uint8_t*>(Yssd + row0 * kP), rstride, lane);
+                float r[kP];
+    #pragma unroll
+                for (int i = 0; i < kP / 2; ++i) {
+                    f2_unpack(O[i], r[2 * i], r[2 * i + 1]);
+                    r[2 * i] *= inv_d;
+                    r[2 * i + 1] *= inv_d;
+                }
+                Tout* rs = reinterpret_cast<Tout*>(rslots + lane * (kRowB + 16));
+                Tout* ys = reinterpret_cast<Tout*>(yslots + lane * (kRowB + 16));
+    #pragma unroll
+                for (int c = 0; c < 4; ++c) store_row16(rs + 16 * c, r + 16 * c);
+                if (lse != nullptr) lse[rowo] = has ? m + logf(dsum) : -INFINITY;
+                __syncwarp();
+    #pragma unroll
+                for (int c = 0; c < 4; ++c) {
+                    float y[16];
+                    load_row16(ys + 16 * c, y);
+    #pragma unroll
+                    for (int i = 0; i < 16; ++i) y[i] = fmaf(gate, r[16 * c + i], y[i]);
+                    store_row16(ys + 16 * c, y);
+                }
+                __syncwarp();
+                slots_to_rows<kRowB>(reinterpret_cast<uint8_t*>(Y + row0 * kP), rstride, yslots, lane);
+                if (R != nullptr) slots_to_rows<kRowB>(reinterpret_cast<uint8_t*>(R + row0 * kP), rstride, rslots, lane);
+            }
         }
     }
 
@@ -655,11 +711,11 @@ cudaError_t launch_sma_forward_tc(const SmaArgs& a, void* ws, unsigned long long
     float* scale = (float*)(ops + (size_t)(a.B * Mc * (H / kHeadsPerCta)) * kPair);
     if (Mc > 1) {
         sma_operands_kernel<Tmem><<<dim3(Mc - 1, H, Bsz), 256, 0, stream>>>(
-            (const Tmem*)a.M, a.rM, ops, scale, Mc, H, a.eps);
+            (const Tmem*)a.M, a.rM, ops, scale, Mc, H, a.eps, kPair);
         note_launches(1);
     }
     const size_t smem = sizeof(TcSmem) + 1024;
-    auto kern = sma_tc_kernel<Tout>;
+    auto kern = sma_tc_kernel<Tout, false>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     const int items = (L / kRows) * Bsz * (H / kHeadsPerCta);
@@ -667,10 +723,42 @@ cudaError_t launch_sma_forward_tc(const SmaArgs& a, void* ws, unsigned long long
                                             (const __nv_bfloat16*)a.Cm, (const __nv_bfloat16*)a.E,
                                             (const __nv_bfloat16*)a.z, (const Tout*)a.Yssd,
                                             (Tout*)a.Y, (Tout*)a.R, a.lse, Bsz, L, H, (int)a.G,
-                                            (int)a.S, Mc, a.eps, wait_limit_ns, a.test_withhold);
+                                            (int)a.S, Mc, a.eps, wait_limit_ns, a.test_withhold,
+                                            kPair, SmaStats{});
     note_launches(1);
     return cudaGetLastError();
 }
+
+template <typename Tmem>
+cudaError_t launch_sma_bwd_stats_tc(const SmaBwdArgs& a, const float* rM, uint8_t* ops,
+                                    int pair_bytes, float* scale, float* g, float2* gd,
+                                    unsigned long long wait_limit_ns, cudaStream_t stream) {
+    const int Bsz = (int)a.B, L = (int)a.L, H = (int)a.H, Mc = (int)(a.L / a.S);
+    if (Mc > 1) {
+        sma_operands_kernel<Tmem><<<dim3(Mc - 1, H, Bsz), 256, 0, stream>>>(
+            (const Tmem*)a.M, rM, ops, scale, Mc, H, a.eps, pair_bytes);
+        note_launches(1);
+    }
+    const size_t smem = sizeof(TcSmem) + 1024;
+    auto kern = sma_tc_kernel<float, true>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    const int items = (L / kRows) * Bsz * (H / kHeadsPerCta);
+    SmaStats st{g, gd};
+    kern<<<items, kThreads, smem, stream>>>(ops, scale, (const __nv_bfloat16*)a.Q,
+                                            (const __nv_bfloat16*)a.Cm, (const __nv_bfloat16*)a.E,
+                                            (const __nv_bfloat16*)a.z, nullptr, nullptr, nullptr,
+                                            const_cast<float*>(a.lse), Bsz, L, H, (int)a.G,
+                                            (int)a.S, Mc, a.eps, wait_limit_ns, 0, pair_bytes, st);
+    note_launches(1);
+    return cudaGetLastError();
+}
+template cudaError_t launch_sma_bwd_stats_tc<float>(const SmaBwdArgs&, const float*, uint8_t*, int,
+                                                    float*, float*, float2*, unsigned long long,
+                                                    cudaStream_t);
+template cudaError_t launch_sma_bwd_stats_tc<__nv_bfloat16>(const SmaBwdArgs&, const float*, uint8_t*,
+                                                            int, float*, float*, float2*,
+                                                            unsigned long long, cudaStream_t);
 
 typedef __nv_bfloat16 bf16;
 template cudaError_t launch_sma_forward_tc<float, float>(const SmaArgs&, void*, unsigned long long,

@@ -19,6 +19,8 @@ CASES = [
     Workload("bwd_f32_s16", 2, 2, 128, 16, 16, 16, dtype="f32", seed=2102),
     Workload("bwd_bf16_s128", 1, 4, 512, 64, 128, 128, seed=2103),
     Workload("bwd_bf16_s256", 2, 4, 1024, 64, 128, 256, seed=2104),
+    # three head pairs and seven memories: many jobs per tile through the two-stage rings
+    Workload("bwd_bf16_h6_s128", 1, 6, 1024, 64, 128, 128, seed=2106),
 ]
 
 
