@@ -378,9 +378,9 @@ dart_status dart_chunk_scan_backward(const dart_dims* d, const void* X, const fl
     cudaStream_t s = (cudaStream_t)stream;
     cudaError_t e;
     if (d->in_dtype == DART_F32)
-        e = dart::launch_chunk_scan_backward<float>(a, ws, s);
+        e = dart::launch_chunk_scan_backward<float>(a, ws, g_wait_limit_ns.load(), s);
     else if (d->in_dtype == DART_BF16)
-        e = dart::launch_chunk_scan_backward<__nv_bfloat16>(a, ws, s);
+        e = dart::launch_chunk_scan_backward<__nv_bfloat16>(a, ws, g_wait_limit_ns.load(), s);
     else
         return DART_ERR_UNSUPPORTED;
     return e == cudaSuccess ? DART_OK : cuda_fail(e);

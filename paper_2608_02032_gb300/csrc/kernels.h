@@ -107,7 +107,8 @@ cudaError_t launch_sma_backward(const SmaBwdArgs& a, void* ws, cudaStream_t stre
 
 size_t scan_bwd_workspace(int64_t B, int64_t L, int64_t H, int64_t N, int64_t P, int64_t S);
 template <typename Tin>
-cudaError_t launch_chunk_scan_backward(const ScanBwdArgs& a, void* ws, cudaStream_t stream);
+cudaError_t launch_chunk_scan_backward(const ScanBwdArgs& a, void* ws, unsigned long long wait_limit_ns,
+                                       cudaStream_t stream);
 // Forward steps 1-3 of the scan (cumsum, chunk states, state passing) for the
 // backward: cum and the states entering each chunk, with scratch (fp32, the
 // size of the memories) for the chunk-state kernel's memory output.
@@ -130,6 +131,10 @@ template <typename Tmem, typename Tout>
 cudaError_t launch_chunk_scan_tc(const ScanArgs& a, unsigned long long wait_limit_ns,
                                  cudaStream_t stream);
 int take_scan_tc_status();
+cudaError_t launch_scan_states_tc(const ScanArgs& a, float* cum, float* Hprev,
+                                  unsigned long long wait_limit_ns, cudaStream_t stream);
+cudaError_t launch_scan_bwd_inter_tc(const ScanArgs& a, const float* cum, const void* dY, float* Z,
+                                     unsigned long long wait_limit_ns, cudaStream_t stream);
 
 template <typename Tmem>
 cudaError_t launch_memory_rms(const void* M, float* rM, int64_t rows, int64_t P, float eps,

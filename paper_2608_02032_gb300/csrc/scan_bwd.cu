@@ -355,7 +355,8 @@ size_t scan_bwd_workspace(int64_t B, int64_t L, int64_t H, int64_t N, int64_t P,
 }
 
 template <typename Tin>
-cudaError_t launch_chunk_scan_backward(const ScanBwdArgs& a, void* ws, cudaStream_t stream) {
+cudaError_t launch_chunk_scan_backward(const ScanBwdArgs& a, void* ws, unsigned long long wait_limit_ns,
+                                       cudaStream_t stream) {
     const ScanArgs& f = a.fwd;
     const int B = (int)f.B, L = (int)f.L, H = (int)f.H, G = (int)f.G, P = (int)f.P,
               N = (int)f.N, S = (int)f.S, Mc = L / S, NP = N * P;
@@ -369,8 +370,11 @@ cudaError_t launch_chunk_scan_backward(const ScanBwdArgs& a, void* ws, cudaStrea
     w += al((size_t)(f.B * Mc * f.H) * NP * sizeof(float));
     float* dcum_end = (float*)w;
 
+    // bf16 inputs at the tensor-core shapes: the state recompute and Z_c on the tensor cores
+    const bool tc = sizeof(Tin) == 2 && scan_tc_supported(f);
     // recompute cum and the state entering every chunk (forward kernels)
-    cudaError_t e = launch_scan_states<Tin>(a.fwd, cum, Hprev, ZD, stream);
+    cudaError_t e = tc ? launch_scan_states_tc(a.fwd, cum, Hprev, wait_limit_ns, stream)
+                       : launch_scan_states<Tin>(a.fwd, cum, Hprev, ZD, stream);
     if (e != cudaSuccess) return e;
     if ((e = cudaMemsetAsync(dcum_end, 0, (size_t)(f.B * f.H * Mc) * sizeof(float), stream)) != cudaSuccess)
         return e;
@@ -380,8 +384,13 @@ cudaError_t launch_chunk_scan_backward(const ScanBwdArgs& a, void* ws, cudaStrea
     if (!a.accumulate_dC &&
         (e = cudaMemsetAsync(a.dC, 0, (size_t)(f.B * f.L * f.G * f.N) * sizeof(float), stream)) != cudaSuccess)
         return e;
-    scan_bwd_inter_kernel<Tin><<<dim3(Mc, H, B), 256, 0, stream>>>(
-        (const Tin*)a.fwd.Cm, (const Tin*)a.dY, cum, ZD, L, H, G, P, N, S, Mc);
+    if (tc) {
+        if ((e = launch_scan_bwd_inter_tc(f, cum, a.dY, ZD, wait_limit_ns, stream)) != cudaSuccess) return e;
+    } else {
+        scan_bwd_inter_kernel<Tin><<<dim3(Mc, H, B), 256, 0, stream>>>(
+            (const Tin*)a.fwd.Cm, (const Tin*)a.dY, cum, ZD, L, H, G, P, N, S, Mc);
+        note_launches(1);
+    }
     scan_bwd_passing_kernel<<<dim3((NP + 255) / 256, H, B), 256, 0, stream>>>(
         ZD, a.dM, Hprev, cum, dcum_end, H, S, Mc, NP);
     const size_t smem = (size_t)(N * 65 + 2 * kTB * 129 + 2 * kTB * 65 + 3 * kTB * 33 + 3 * S + kTB) *
@@ -393,12 +402,14 @@ cudaError_t launch_chunk_scan_backward(const ScanBwdArgs& a, void* ws, cudaStrea
         (const Tin*)a.fwd.X, a.fwd.dt, a.fwd.A, (const Tin*)a.fwd.Bm, (const Tin*)a.fwd.Cm,
         (const Tin*)a.dY, cum, Hprev, ZD, dcum_end, a.dX, a.ddt, a.dA, a.dB, a.dC, L, H, G, P, N, S,
         Mc);
-    note_launches(3);
+    note_launches(2);
     return cudaGetLastError();
 }
 
 typedef __nv_bfloat16 bf16;
-template cudaError_t launch_chunk_scan_backward<float>(const ScanBwdArgs&, void*, cudaStream_t);
-template cudaError_t launch_chunk_scan_backward<bf16>(const ScanBwdArgs&, void*, cudaStream_t);
+template cudaError_t launch_chunk_scan_backward<float>(const ScanBwdArgs&, void*, unsigned long long,
+                                                       cudaStream_t);
+template cudaError_t launch_chunk_scan_backward<bf16>(const ScanBwdArgs&, void*, unsigned long long,
+                                                      cudaStream_t);
 
 }  // namespace dart

@@ -142,7 +142,9 @@ struct StateRegs {
     float cumv, cend, dtv;  // cum of source tid and of the chunk's last token, dt of tid
 };
 
-template <typename Tmem>
+// kZ: the backward's inter-chunk term Z_c = sum_{t in c} exp(cum_t) C_t^T dY_t
+// with the same kernel: Bm <- C, X <- dY, w_t = exp(cum_t), only the fp32 output.
+template <typename Tmem, bool kZ = false>
 __global__ void __launch_bounds__(kStateThreads, 2)
 chunk_state_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restrict__ dt,
                       const float* __restrict__ cum, const __nv_bfloat16* __restrict__ Bm,
@@ -225,7 +227,7 @@ chunk_state_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restri
     bool ok = true;
     for (int hh = 0; hh < kHeadsPerCta && ok; ++hh) {
         const int h = h0 + hh;
-        if (tid < S) sm.w[tid] = expf(nx.cend - nx.cumv) * nx.dtv;
+        if (tid < S) sm.w[tid] = kZ ? expf(nx.cumv) : expf(nx.cend - nx.cumv) * nx.dtv;
         __syncthreads();
         // stage (w (.) X_h) as bf16 hi / lo, rows s, 128-byte swizzle
 #pragma unroll
@@ -279,17 +281,19 @@ chunk_state_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restri
                 for (int q = 0; q < 8; ++q)
                     d32[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
             }
-            store_row32(Mout + mrow * kP + 32 * half, v);
+            if (!kZ) {
+                store_row32(Mout + mrow * kP + 32 * half, v);
 #pragma unroll
-            for (int i = 0; i < 32; ++i) {
-                const float sv = stored_value<Tmem>(v[i]);
-                ss = fmaf(sv, sv, ss);
+                for (int i = 0; i < 32; ++i) {
+                    const float sv = stored_value<Tmem>(v[i]);
+                    ss = fmaf(sv, sv, ss);
+                }
             }
         }
         if (half == 1) sm.ssq[n] = ss;
         tc::tc_fence_before();
         __syncthreads();  // the accumulator and the staging buffers are reused
-        if (half == 0 && rM != nullptr) rM[mrow] = rsqrtf((ss + sm.ssq[n]) / (float)kP + eps);
+        if (!kZ && half == 0 && rM != nullptr) rM[mrow] = rsqrtf((ss + sm.ssq[n]) / (float)kP + eps);
     }
     if (!ok) {  // a wait ran out: let the MMAs in flight finish before freeing TMEM
         if (!tc::mbar_wait(&sm.bar, phase ^ 1u, kDrainLimitNs, nullptr))
@@ -741,6 +745,44 @@ cudaError_t launch_chunk_scan_tc(const ScanArgs& a, unsigned long long wait_limi
             (const __nv_bfloat16*)a.Cm, a.Hops, (Tout*)a.Y, L, H, G, S, M, wait_limit_ns);
     }
     note_launches(3);
+    return cudaGetLastError();
+}
+
+// Backward helpers on the tensor-core path (bf16 inputs, the same shapes).
+// States: cum and the fp32 state entering every chunk (in Hprev), i.e. the
+// forward's chunk states followed by the in-place fp32 state passing.
+cudaError_t launch_scan_states_tc(const ScanArgs& a0, float* cum, float* Hprev,
+                                  unsigned long long wait_limit_ns, cudaStream_t stream) {
+    ScanArgs a = a0;
+    a.cum = cum;
+    const int B = (int)a.B, L = (int)a.L, H = (int)a.H, G = (int)a.G, S = (int)a.S, M = L / S;
+    cudaError_t e = launch_chunk_cumsum(a, stream);
+    if (e != cudaSuccess) return e;
+    auto kern = chunk_state_tc_kernel<float, false>;
+    const size_t smem = sizeof(StateSmem) + 1024;
+    if ((e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) != cudaSuccess)
+        return e;
+    kern<<<dim3(M, H / kHeadsPerCta, B), kStateThreads, smem, stream>>>(
+        (const __nv_bfloat16*)a.X, a.dt, a.cum, (const __nv_bfloat16*)a.Bm, nullptr, Hprev, nullptr,
+        L, H, G, S, M, a.eps, wait_limit_ns);
+    note_launches(1);
+    a.dH32 = Hprev;  // chunk states in, entering states out (in place)
+    a.final_state = nullptr;
+    return launch_state_passing(a, stream);
+}
+
+// Z_c = sum_{t in c} exp(cum_t) C_t^T dY_t for every chunk (fp32, B x Mc x H x N x P).
+cudaError_t launch_scan_bwd_inter_tc(const ScanArgs& a, const float* cum, const void* dY, float* Z,
+                                     unsigned long long wait_limit_ns, cudaStream_t stream) {
+    const int B = (int)a.B, L = (int)a.L, H = (int)a.H, G = (int)a.G, S = (int)a.S, M = L / S;
+    auto kern = chunk_state_tc_kernel<float, true>;
+    const size_t smem = sizeof(StateSmem) + 1024;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    kern<<<dim3(M, H / kHeadsPerCta, B), kStateThreads, smem, stream>>>(
+        (const __nv_bfloat16*)dY, a.dt, cum, (const __nv_bfloat16*)a.Cm, Z, nullptr, nullptr, L, H, G,
+        S, M, a.eps, wait_limit_ns);
+    note_launches(1);
     return cudaGetLastError();
 }
 

@@ -21,6 +21,9 @@ CASES = [
     Workload("bwd_bf16_s256", 2, 4, 1024, 64, 128, 256, seed=2104),
     # three head pairs and seven memories: many jobs per tile through the two-stage rings
     Workload("bwd_bf16_h6_s128", 1, 6, 1024, 64, 128, 128, seed=2106),
+    # eight heads: the tensor-core scan backward (head groups of 8)
+    Workload("bwd_bf16_h8_s256", 1, 8, 1024, 64, 128, 256, seed=2107),
+    Workload("bwd_bf16_h8_s128", 2, 8, 512, 64, 128, 128, seed=2108),
 ]
 
 
