@@ -194,10 +194,16 @@ size_t dart_workspace_size(const dart_dims* d, int op) {
                                                            d->seqlen / d->chunk, d->dstate));
             return align256(dart::sma_bwd_workspace(d->batch, d->seqlen, d->nheads,
                                                     d->seqlen / d->chunk, d->dstate));
-        case DART_OP_SCAN_BACKWARD:
+        case DART_OP_SCAN_BACKWARD: {
             if (check_dims(d, true) != DART_OK) return 0;
+            dart::ScanArgs a{};
+            a.B = d->batch; a.L = d->seqlen; a.H = d->nheads; a.G = d->ngroups;
+            a.P = d->headdim; a.N = d->dstate; a.S = d->chunk;
+            if (d->in_dtype == DART_BF16 && dart::scan_bwd_tc_supported(a))
+                return align256(dart::scan_bwd_tc_workspace(d->batch, d->seqlen, d->nheads, d->chunk));
             return align256(dart::scan_bwd_workspace(d->batch, d->seqlen, d->nheads, d->dstate,
                                                      d->headdim, d->chunk));
+        }
     }
     return 0;
 }
@@ -392,8 +398,9 @@ dart_status dart_get_device_status(void* stream) {
     const int code = dart::take_tc_status();
     const int code2 = dart::take_scan_tc_status();
     const int code3 = dart::take_bwd_tc_status();
-    if (code < 0 || code2 < 0 || code3 < 0) return cuda_fail(cudaGetLastError());
-    return (code != 0 || code2 != 0 || code3 != 0) ? DART_ERR_TIMEOUT : DART_OK;
+    const int code4 = dart::take_scan_bwd_tc_status();
+    if (code < 0 || code2 < 0 || code3 < 0 || code4 < 0) return cuda_fail(cudaGetLastError());
+    return (code != 0 || code2 != 0 || code3 != 0 || code4 != 0) ? DART_ERR_TIMEOUT : DART_OK;
 }
 
 void dart_test_withhold_copies(int on) { g_test_withhold.store(on != 0 ? 1 : 0); }

@@ -131,10 +131,22 @@ template <typename Tmem, typename Tout>
 cudaError_t launch_chunk_scan_tc(const ScanArgs& a, unsigned long long wait_limit_ns,
                                  cudaStream_t stream);
 int take_scan_tc_status();
-cudaError_t launch_scan_states_tc(const ScanArgs& a, float* cum, float* Hprev,
+cudaError_t launch_scan_states_tc(const ScanArgs& a, float* cum, float* Hprev, uint8_t* Hops,
                                   unsigned long long wait_limit_ns, cudaStream_t stream);
 cudaError_t launch_scan_bwd_inter_tc(const ScanArgs& a, const float* cum, const void* dY, float* Z,
                                      unsigned long long wait_limit_ns, cudaStream_t stream);
+cudaError_t launch_scan_bwd_output_tc(const ScanArgs& a, const float* cum, const uint8_t* Hops,
+                                      const uint8_t* Dops, const void* dY, float* rowI,
+                                      float* dX, float* xi, unsigned long long wait_limit_ns,
+                                      cudaStream_t stream);
+size_t scan_bwd_tc_workspace(int64_t B, int64_t L, int64_t H, int64_t S);
+cudaError_t launch_chunk_scan_backward_tc(const ScanBwdArgs& a, void* ws,
+                                          unsigned long long wait_limit_ns, cudaStream_t stream);
+int take_scan_bwd_tc_status();
+cudaError_t launch_scan_bwd_passing(float* ZD, const float* dM, const float* Hprev, const float* cum,
+                                    float* dcum_end, uint8_t* Dops, int B, int H, int S, int Mc,
+                                    int NP, cudaStream_t stream);
+bool scan_bwd_tc_supported(const ScanArgs& f);
 
 template <typename Tmem>
 cudaError_t launch_memory_rms(const void* M, float* rM, int64_t rows, int64_t P, float eps,

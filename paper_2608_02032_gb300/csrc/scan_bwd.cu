@@ -75,12 +75,14 @@ scan_bwd_inter_kernel(const Tin* __restrict__ Cm, const Tin* __restrict__ dY,
 }
 
 // Reverse pass over chunks for each (b, h, element): ZD holds Z on entry and
-// d(dH_c) on exit. dcum_end[b,h,c] += exp(cum_end) <A_c, H_[c-1]>.
+// d(dH_c) on exit. dcum_end[b,h,c] += exp(cum_end) <A_c, H_[c-1]>. With Dops
+// (P = 64), d(dH_c) is also written as bf16 hi | lo tiles in the 128-byte
+// swizzled layout of the tensor-core kernels (32 KiB per (b, c, h)).
 __global__ void scan_bwd_passing_kernel(float* __restrict__ ZD, const float* __restrict__ dM,
                                         const float* __restrict__ Hprev,
                                         const float* __restrict__ cum,
-                                        float* __restrict__ dcum_end, int H, int S, int Mc,
-                                        int NP) {
+                                        float* __restrict__ dcum_end, uint8_t* __restrict__ Dops,
+                                        int H, int S, int Mc, int NP) {
     const int e = blockIdx.x * blockDim.x + threadIdx.x;
     const int h = blockIdx.y, b = blockIdx.z;
     const float* cumh = cum + ((i64)b * H + h) * Mc * S;
@@ -93,7 +95,16 @@ __global__ void scan_bwd_passing_kernel(float* __restrict__ ZD, const float* __r
             const float z = ZD[idx];
             const float dmv = dM != nullptr ? dM[idx] : 0.0f;
             part = dec * adj * Hprev[idx];
-            ZD[idx] = adj + dmv;
+            const float dd = adj + dmv;
+            ZD[idx] = dd;
+            if (Dops != nullptr) {
+                const int n = e >> 6, p = e & 63;
+                const uint32_t o = ((uint32_t)n * 128u + (uint32_t)p * 2u) ^ (((uint32_t)n & 7u) << 4);
+                uint8_t* tile = Dops + (((i64)b * Mc + c) * H + h) * 32768;
+                const __nv_bfloat16 hi = __float2bfloat16_rn(dd);
+                *reinterpret_cast<__nv_bfloat16*>(tile + o) = hi;
+                *reinterpret_cast<__nv_bfloat16*>(tile + 16384 + o) = __float2bfloat16_rn(dd - __bfloat162float(hi));
+            }
             adj = fmaf(dec, adj, z);
         }
         for (int off = 16; off > 0; off >>= 1) part += __shfl_xor_sync(0xffffffffu, part, off);
@@ -354,6 +365,17 @@ size_t scan_bwd_workspace(int64_t B, int64_t L, int64_t H, int64_t N, int64_t P,
            + al((size_t)(B * H * M) * sizeof(float));           // d(cum_end)
 }
 
+cudaError_t launch_scan_bwd_passing(float* ZD, const float* dM, const float* Hprev, const float* cum,
+                                    float* dcum_end, uint8_t* Dops, int B, int H, int S, int Mc,
+                                    int NP, cudaStream_t stream) {
+    scan_bwd_passing_kernel<<<dim3((NP + 255) / 256, H, B), 256, 0, stream>>>(
+        ZD, dM, Hprev, cum, dcum_end, Dops, H, S, Mc, NP);
+    note_launches(1);
+    return cudaGetLastError();
+}
+
+bool scan_bwd_tc_supported(const ScanArgs& f) { return f.G == 1 && scan_tc_supported(f); }
+
 template <typename Tin>
 cudaError_t launch_chunk_scan_backward(const ScanBwdArgs& a, void* ws, unsigned long long wait_limit_ns,
                                        cudaStream_t stream) {
@@ -370,10 +392,13 @@ cudaError_t launch_chunk_scan_backward(const ScanBwdArgs& a, void* ws, unsigned 
     w += al((size_t)(f.B * Mc * f.H) * NP * sizeof(float));
     float* dcum_end = (float*)w;
 
-    // bf16 inputs at the tensor-core shapes: the state recompute and Z_c on the tensor cores
+    // bf16 inputs at the tensor-core shapes with G = 1: the whole backward on the tensor
+    // cores; other bf16 inputs at those shapes: the state recompute and Z_c there
+    if (sizeof(Tin) == 2 && scan_bwd_tc_supported(f))
+        return launch_chunk_scan_backward_tc(a, ws, wait_limit_ns, stream);
     const bool tc = sizeof(Tin) == 2 && scan_tc_supported(f);
     // recompute cum and the state entering every chunk (forward kernels)
-    cudaError_t e = tc ? launch_scan_states_tc(a.fwd, cum, Hprev, wait_limit_ns, stream)
+    cudaError_t e = tc ? launch_scan_states_tc(a.fwd, cum, Hprev, nullptr, wait_limit_ns, stream)
                        : launch_scan_states<Tin>(a.fwd, cum, Hprev, ZD, stream);
     if (e != cudaSuccess) return e;
     if ((e = cudaMemsetAsync(dcum_end, 0, (size_t)(f.B * f.H * Mc) * sizeof(float), stream)) != cudaSuccess)
@@ -392,7 +417,7 @@ cudaError_t launch_chunk_scan_backward(const ScanBwdArgs& a, void* ws, unsigned 
         note_launches(1);
     }
     scan_bwd_passing_kernel<<<dim3((NP + 255) / 256, H, B), 256, 0, stream>>>(
-        ZD, a.dM, Hprev, cum, dcum_end, H, S, Mc, NP);
+        ZD, a.dM, Hprev, cum, dcum_end, nullptr, H, S, Mc, NP);
     const size_t smem = (size_t)(N * 65 + 2 * kTB * 129 + 2 * kTB * 65 + 3 * kTB * 33 + 3 * S + kTB) *
                         sizeof(float);
     auto k3 = scan_bwd_chunk_kernel<Tin>;

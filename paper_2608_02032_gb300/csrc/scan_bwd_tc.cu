@@ -1,0 +1,671 @@
+// Backward of the chunked SSD scan on the tensor cores, for bf16 inputs with
+// P = 64, N = 128, G = 1, S in {128, 256} (the chain rule on the chunked
+// forms of App. A; the paper prints no backward). With cum the within-chunk
+// cumsum of dt A, L[t,s] = exp(cum_t - cum_s) (s <= t in one chunk), the
+// chunk-entry states H_[c-1] and the adjoint d(dH_c) of each chunk state:
+//   dX_s   = dt_s Y'_s,  Y'_s = sum_{t >= s} L[t,s] (B_s . C_t) dY_t
+//                               + exp(cum_end - cum_s) B_s d(dH_c)
+//            (the output kernel in reversed time, scan_tc.cu);
+//   dC_t  += sum_s Psi[t,s] B_s + sum_h exp(cum_t) dY_t H_[c-1]^T,
+//   dB_s   = sum_t Psi[t,s] C_t + sum_h exp(cum_end - cum_s) dt_s X_s d(dH_c)^T,
+//            Psi[t,s] = sum_h L[t,s] dt_s (dY_t . X_s): with B and C shared by
+//            the heads (G = 1) the intra-chunk terms need only this head sum;
+//   d(cum_t) = dY_t . Y_t - dt_t X_t . Y'_t, plus at the chunk end
+//            sum_s kappa_s (kappa_s = dt_s X_s . (exp(cum_end - cum_s) B_s d(dH_c)))
+//            and exp(cum_end) <adjoint of H_c, H_[c-1]> (passing kernel);
+//   d(dt_u) = X_u . Y'_u + A_h sum_{k >= u} d(cum_k),  dA_h = sum_u dt_u sum_{k >= u} d(cum_k).
+// Kernels here: psi_kernel (Psi, per chunk and 128-row tile, summed over the
+// heads from one tensor-core score tile dY X^T per head), dcdb_kernel (dC and
+// dB as MMA chains over K units: Psi blocks against B or C rows, then one unit
+// per head for the inter-chunk term), finalize_kernel (the d(cum) reverse sums).
+// Operands that are not exact bf16 inputs are split bf16 hi + lo.
+#include <math.h>
+
+#include <cuda_bf16.h>
+
+#include "common.cuh"
+#include "kernels.h"
+#include "tc_ptx.cuh"
+
+namespace dart {
+namespace {
+
+__device__ int g_sbwd_tc_status;  // first timeout code since the last read (0 = none)
+
+constexpr int kP = 64;
+constexpr int kN = 128;
+constexpr int kT = 128;
+constexpr uint64_t kDrainLimitNs = 2000000000ull;
+constexpr float kLog2e = 1.4426950408889634f;
+
+__device__ __forceinline__ uint32_t sw128(uint32_t row, uint32_t byte_in_row) {
+    const uint32_t o = row * 128u + byte_in_row;
+    return o ^ ((row & 7u) << 4);
+}
+__device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
+    const __nv_bfloat162 v = __floats2bfloat162_rn(a, b);
+    return *reinterpret_cast<const uint32_t*>(&v);
+}
+__device__ __forceinline__ float bf_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf_hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
+__device__ __forceinline__ float ex2_approx(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+// Splits 8 floats into bf16 hi and lo words (4 + 4).
+__device__ __forceinline__ void split8(const float* v, uint4& hi, uint4& lo) {
+    uint32_t h[4], l[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+        const __nv_bfloat162 hv = __floats2bfloat162_rn(v[2 * e], v[2 * e + 1]);
+        const float2 hf = __bfloat1622float2(hv);
+        h[e] = *reinterpret_cast<const uint32_t*>(&hv);
+        l[e] = pack_bf16(v[2 * e] - hf.x, v[2 * e + 1] - hf.y);
+    }
+    hi = make_uint4(h[0], h[1], h[2], h[3]);
+    lo = make_uint4(l[0], l[1], l[2], l[3]);
+}
+
+__host__ __device__ constexpr uint32_t idesc_bf16(bool a_mn, bool b_mn, uint32_t M, uint32_t N) {
+    return (1u << 4) | (1u << 7) | (1u << 10) | ((a_mn ? 1u : 0u) << 15) | ((b_mn ? 1u : 0u) << 16) |
+           ((N >> 3) << 17) | ((M >> 4) << 24);
+}
+__device__ __forceinline__ void mma_ss(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
+                                       uint32_t idesc, uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}"
+        ::"r"(d_tmem), "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
+    uint32_t r[32];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];\n\t"
+        "tcgen05.wait::ld.sync.aligned;"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+          "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),
+          "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),
+          "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+        : "r"(taddr)
+        : "memory");
+#pragma unroll
+    for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// Bounded wait by every thread of the CTA, then a CTA-wide AND of the outcome.
+__device__ __forceinline__ bool cta_wait(uint64_t* bar, uint32_t parity, uint64_t limit_ns, int code) {
+    const bool got = tc::mbar_wait(bar, parity, limit_ns, nullptr);
+    if (!got) atomicCAS(&g_sbwd_tc_status, 0, code);
+    const bool all = __syncthreads_and(got ? 1 : 0) != 0;
+    tc::tc_fence_after();
+    return all;
+}
+
+// Psi layout, per (b, c): two parts (hi, lo) of S / 64 column blocks, each
+// block S rows x 128 bytes in the 128-byte swizzle (row t, bytes 2 (s % 64)).
+// A block read K-major (rows t, K = s) and one read MN-major (M = s, K = t)
+// have this same layout.
+__host__ __device__ inline int64_t psi_chunk_bytes(int S) { return 2LL * S * S * 2; }
+
+// ---------------------------------------------------------------- psi / phi
+// One CTA of 512 threads (four per row, a quarter of the sources each) per
+// (128-token tile, chunk, b), looping over the heads; per head one MMA chain
+// gives the score tile dY X^T (rows t, columns s <= t of the chunk).
+//   !kPhi: Psi[t,s] = sum_h L[t,s] dt_s (dY_t . X_s), kept in registers, written
+//          split hi + lo in the Psi layout;
+//   kPhi:  Phi_h[t,s] = L[t,s] dt_s (C_t . B_s)(dY_t . X_s) with C B^T from one
+//          more MMA chain (shared by the heads), reduced to its row sums
+//          (phi_row, per (t, h)) and column sums (phi_col, per (s, h); two tiles
+//          add to the columns of the first, so phi_col is accumulated).
+constexpr int kPsiThreads = 512;
+
+struct PsiSmem {
+    uint8_t yt[kT * 128];         // dY rows of the tile: A (rows t, K = p), K-major
+    uint8_t xs[256 * 128];        // X rows of the sources: B (rows s, K = p), K-major
+    uint8_t ct[2][kT * 128];      // kPhi: C rows of the tile, K-major A (two K blocks)
+    uint8_t bs[2][256 * 128];     // kPhi: B rows of the sources, K-major B (two K blocks)
+    float c2[256];                // cum log2(e) of tokens 0 .. ns - 1
+    float e2[256];                // c2 - log2(dt): exp2(c2_t - e2_s) = L[t,s] dt_s
+    float bfac[256];              // exp2(c2_r - e2_s), r = last token of s's group of 32
+    float rowacc[kT];             // kPhi: row sums of the head
+    float colacc[256];            // kPhi: column sums of the head
+    uint64_t bar;
+    uint32_t tmem_base;
+};
+
+// Sums v[i] over the 32 lanes for i = 0..31; lane l returns the sum of v[l].
+__device__ __forceinline__ float warp_colsum32(float (&v)[32], int lane) {
+#pragma unroll
+    for (int off = 16; off >= 1; off >>= 1) {
+        const bool upper = (lane & off) != 0;
+#pragma unroll
+        for (int i = 0; i < off; ++i) {
+            const float send = upper ? v[i] : v[i + off];
+            const float keep = upper ? v[i + off] : v[i];
+            v[i] = keep + __shfl_xor_sync(0xffffffffu, send, off);
+        }
+    }
+    return v[0];
+}
+
+template <bool kPhi>
+__global__ void __launch_bounds__(kPsiThreads, 1)
+psi_kernel(const __nv_bfloat16* __restrict__ X, const float* __restrict__ dt,
+           const float* __restrict__ cum, const __nv_bfloat16* __restrict__ dY,
+           const __nv_bfloat16* __restrict__ Bm, const __nv_bfloat16* __restrict__ Cm,
+           uint8_t* __restrict__ psi, float* __restrict__ phi_row, float* __restrict__ phi_col,
+           int L, int H, int S, int Mc, unsigned long long wait_limit_ns) {
+    extern __shared__ uint8_t smem_raw[];
+    PsiSmem& sm = *reinterpret_cast<PsiSmem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                              ~(uintptr_t)1023);
+    const int tt = blockIdx.x, c = blockIdx.y, b = blockIdx.z;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int row = tid & (kT - 1), quarter = tid >> 7;
+    const int ns = (tt + 1) * kT;
+    const i64 tok0 = (i64)b * L + (i64)c * S;
+    const uint32_t lane_addr = (uint32_t)(32 * (warp & 3)) << 16;
+    const int tl = tt * kT + row;
+    const int tl_warp_max = tt * kT + 32 * (warp & 3) + 31;
+    const int sq = ns / 4, s_lo = quarter * sq;  // 32 or 64 sources of this thread
+    constexpr uint32_t kColCB = 256;
+
+    if (tid == 0) {
+        tc::mbar_init(&sm.bar, 1);
+        tc::fence_barrier_init();
+    }
+    if (warp == 0) {
+        tc::tmem_alloc(&sm.tmem_base, kPhi ? 512 : 256);
+        tc::tmem_relinquish();
+    }
+    if (kPhi) {
+        for (int i = tid; i < kT * 16; i += kPsiThreads) {
+            const int r = i / 16, q = i % 16;
+            *reinterpret_cast<uint4*>(sm.ct[q / 8] + sw128((uint32_t)r, (uint32_t)(q % 8) * 16u)) =
+                reinterpret_cast<const uint4*>(Cm + (tok0 + tt * kT + r) * kN)[q];
+        }
+        for (int i = tid; i < ns * 16; i += kPsiThreads) {
+            const int r = i / 16, q = i % 16;
+            *reinterpret_cast<uint4*>(sm.bs[q / 8] + sw128((uint32_t)r, (uint32_t)(q % 8) * 16u)) =
+                reinterpret_cast<const uint4*>(Bm + (tok0 + r) * kN)[q];
+        }
+        for (int i = tid; i < kT; i += kPsiThreads) sm.rowacc[i] = 0.0f;
+        for (int i = tid; i < 256; i += kPsiThreads) sm.colacc[i] = 0.0f;
+        tc::fence_proxy_async_shared();
+    }
+    tc::tc_fence_before();
+    __syncthreads();
+    tc::tc_fence_after();
+    const uint32_t tmem = sm.tmem_base;
+    if (kPhi && tid == 0) {  // C B^T of the tile, committed with the first head's scores
+        const uint32_t id = idesc_bf16(false, false, kT, (uint32_t)ns);
+        for (int ks = 0; ks < kN / 16; ++ks) {
+            const uint64_t ad = tc::smem_desc_sw128(tc::smem_u32(sm.ct[ks / 4]) + 32u * (ks % 4), 16u, 1024u);
+            const uint64_t bd = tc::smem_desc_sw128(tc::smem_u32(sm.bs[ks / 4]) + 32u * (ks % 4), 16u, 1024u);
+            mma_ss(tmem + kColCB, ad, bd, id, ks > 0 ? 1u : 0u);
+        }
+    }
+    float acc[kPhi ? 1 : 64];
+#pragma unroll
+    for (int i = 0; i < (kPhi ? 1 : 64); ++i) acc[i] = 0.0f;
+    uint32_t phase = 0;
+    bool ok = true;
+    for (int h = 0; h < H && ok; ++h) {
+        // the head's dY rows of the tile and X rows of the sources (the previous head's
+        // MMA and TMEM reads are done)
+        for (int i = tid; i < kT * 8; i += kPsiThreads) {
+            const int r = i / 8, q = i % 8;
+            *reinterpret_cast<uint4*>(sm.yt + sw128((uint32_t)r, (uint32_t)q * 16u)) =
+                reinterpret_cast<const uint4*>(dY + ((tok0 + tt * kT + r) * H + h) * kP)[q];
+        }
+        for (int i = tid; i < ns * 8; i += kPsiThreads) {
+            const int s = i / 8, q = i % 8;
+            *reinterpret_cast<uint4*>(sm.xs + sw128((uint32_t)s, (uint32_t)q * 16u)) =
+                reinterpret_cast<const uint4*>(X + ((tok0 + s) * H + h) * kP)[q];
+        }
+        if (tid < ns) {
+            const float c2 = cum[(((i64)b * H + h) * Mc + c) * S + tid] * kLog2e;
+            sm.c2[tid] = c2;
+            sm.e2[tid] = c2 - log2f(dt[(tok0 + tid) * H + h]);  // dt = 0 gives +inf: a zero weight
+        }
+        tc::fence_proxy_async_shared();
+        tc::tc_fence_before();
+        __syncthreads();
+        if (tid == 0) {
+            tc::tc_fence_after();
+            const uint32_t id = idesc_bf16(false, false, kT, (uint32_t)ns);
+            for (int ks = 0; ks < kP / 16; ++ks) {
+                const uint64_t ad = tc::smem_desc_sw128(tc::smem_u32(sm.yt) + 32u * ks, 16u, 1024u);
+                const uint64_t bd = tc::smem_desc_sw128(tc::smem_u32(sm.xs) + 32u * ks, 16u, 1024u);
+                mma_ss(tmem, ad, bd, id, ks > 0 ? 1u : 0u);
+            }
+            tc::mma_commit(&sm.bar);
+        }
+        if (tid < ns) sm.bfac[tid] = ex2_approx(sm.c2[tid | 31] - sm.e2[tid]);
+        ok = cta_wait(&sm.bar, phase, wait_limit_ns, 41);
+        phase ^= 1u;
+        if (!ok) break;
+        const float c2t = sm.c2[tl];
+        float rsum = 0.0f;
+#pragma unroll
+        for (int g0 = 0; g0 < 64; g0 += 32) {
+            const int s0 = s_lo + g0;
+            if (g0 >= sq || s0 > tl_warp_max) continue;  // warp-uniform
+            float v[32];
+            tmem_ld32(tmem + lane_addr + (uint32_t)s0, v);
+            // v <- L[t,s] dt_s scores[t,s] (zero for s > t)
+            if (s0 + 31 <= tl) {  // the whole group at or before t: factored decay
+                const float a = ex2_approx(c2t - sm.c2[s0 + 31]);
+#pragma unroll
+                for (int i = 0; i < 32; ++i) v[i] *= sm.bfac[s0 + i] * a;
+            } else {
+#pragma unroll
+                for (int i = 0; i < 32; ++i) v[i] = s0 + i <= tl ? v[i] * ex2_approx(c2t - sm.e2[s0 + i]) : 0.0f;
+            }
+            if constexpr (kPhi) {
+                float w[32];
+                tmem_ld32(tmem + lane_addr + kColCB + (uint32_t)s0, w);
+#pragma unroll
+                for (int i = 0; i < 32; ++i) {
+                    v[i] *= w[i];
+                    rsum += v[i];
+                }
+                const float cs = warp_colsum32(v, lane);  // this warp's rows, column s0 + lane
+                atomicAdd(&sm.colacc[s0 + lane], cs);
+            } else {
+#pragma unroll
+                for (int i = 0; i < 32; ++i) acc[g0 + i] += v[i];
+            }
+        }
+        if constexpr (kPhi) {
+            atomicAdd(&sm.rowacc[row], rsum);
+            __syncthreads();
+            for (int i = tid; i < kT; i += kPsiThreads) {
+                phi_row[(tok0 + tt * kT + i) * H + h] = sm.rowacc[i];
+                sm.rowacc[i] = 0.0f;
+            }
+            for (int i = tid; i < ns; i += kPsiThreads) {
+                atomicAdd(phi_col + (tok0 + i) * H + h, sm.colacc[i]);
+                sm.colacc[i] = 0.0f;
+            }
+        }
+        tc::tc_fence_before();
+        __syncthreads();  // shared tiles, sums and TMEM are reused by the next head
+    }
+    if (!ok) {  // the MMA chain in flight finishes before TMEM is freed
+        if (!tc::mbar_wait(&sm.bar, phase ^ 1u, kDrainLimitNs, nullptr)) atomicCAS(&g_sbwd_tc_status, 0, 42);
+    }
+    if (!kPhi && ok) {
+        uint8_t* base = psi + (i64)(b * Mc + c) * psi_chunk_bytes(S);
+        const i64 part = (i64)(S / 64) * S * 128;
+#pragma unroll
+        for (int g8 = 0; g8 < 64; g8 += 8) {
+            if (g8 >= sq) continue;
+            const int s = s_lo + g8;
+            uint4 hi, lo;
+            split8(acc + g8, hi, lo);
+            const i64 o = (i64)(s / 64) * S * 128 + sw128((uint32_t)tl, (uint32_t)(s % 64) * 2u);
+            *reinterpret_cast<uint4*>(base + o) = hi;
+            *reinterpret_cast<uint4*>(base + part + o) = lo;
+        }
+        // the tile's rows beyond its sources are zero
+        const int zc = (S - ns) / 8;  // 16-byte chunks per row
+        for (int i = tid; i < kT * zc; i += kPsiThreads) {
+            const int r = i / zc, s = ns + 8 * (i % zc);
+            const i64 o = (i64)(s / 64) * S * 128 + sw128((uint32_t)(tt * kT + r), (uint32_t)(s % 64) * 2u);
+            *reinterpret_cast<uint4*>(base + o) = make_uint4(0, 0, 0, 0);
+            *reinterpret_cast<uint4*>(base + part + o) = make_uint4(0, 0, 0, 0);
+        }
+    }
+    tc::tc_fence_before();
+    __syncthreads();
+    if (warp == 0) {
+        __syncwarp();
+        tc::tc_fence_after();
+        tc::tmem_dealloc(tmem, kPhi ? 512 : 256);
+    }
+}
+
+// ---------------------------------------------------------------- dC / dB
+constexpr int kDcThreads = 256;
+constexpr int kUnit = 16384;  // one operand slot
+
+struct DcSmem {
+    uint8_t slot[2][4][kUnit];  // per buffer: A hi, A lo, B (or B hi), B lo
+    uint64_t mma_done[2];
+    uint64_t drain;
+    uint32_t tmem_base;
+};
+
+// kind 0: dC rows of a 128-token tile (accumulated into dC); kind 1: dB rows.
+__global__ void __launch_bounds__(kDcThreads, 1)
+dcdb_kernel(const __nv_bfloat16* __restrict__ X, const float* __restrict__ dt,
+            const float* __restrict__ cum, const __nv_bfloat16* __restrict__ Bm,
+            const __nv_bfloat16* __restrict__ Cm, const __nv_bfloat16* __restrict__ dY,
+            const uint8_t* __restrict__ psi, const uint8_t* __restrict__ Hops,
+            const uint8_t* __restrict__ Dops, float* __restrict__ dC, float* __restrict__ dB, int L,
+            int H, int S, int Mc, unsigned long long wait_limit_ns) {
+    extern __shared__ uint8_t smem_raw[];
+    DcSmem& sm = *reinterpret_cast<DcSmem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                            ~(uintptr_t)1023);
+    const int tiles = S / kT;
+    const int kind = (int)blockIdx.x / tiles, tt = (int)blockIdx.x % tiles;
+    const int c = blockIdx.y, b = blockIdx.z;
+    const int tid = threadIdx.x, warp = tid >> 5;
+    const i64 tok0 = (i64)b * L + (i64)c * S;
+    const uint8_t* pbase = psi + (i64)(b * Mc + c) * psi_chunk_bytes(S);
+    const i64 ppart = (i64)(S / 64) * S * 128;
+    // K units: intra blocks of 64 tokens, then one per head (dC: only after chunk 0)
+    const int nintra = kind == 0 ? (tt + 1) * kT / 64 : (S - tt * kT) / 64;
+    const int ninter = (kind == 0 && c == 0) ? 0 : H;
+    const int nunits = nintra + ninter;
+
+    if (tid == 0) {
+        tc::mbar_init(&sm.mma_done[0], 1);
+        tc::mbar_init(&sm.mma_done[1], 1);
+        tc::mbar_init(&sm.drain, 1);
+        tc::fence_barrier_init();
+    }
+    if (warp == 0) {
+        tc::tmem_alloc(&sm.tmem_base, 128);
+        tc::tmem_relinquish();
+    }
+    tc::tc_fence_before();
+    __syncthreads();
+    tc::tc_fence_after();
+    const uint32_t tmem = sm.tmem_base;
+    const float* cumb = cum + (i64)b * H * Mc * S;  // + (h Mc + c) S + t
+
+    bool ok = true;
+    int issued = 0;
+    for (int u = 0; u < nunits; ++u) {
+        const int bi = u & 1;
+        if (u >= 2) {
+            ok = cta_wait(&sm.mma_done[bi], (uint32_t)(((u - 2) >> 1) & 1), wait_limit_ns, 43);
+            if (!ok) break;
+        }
+        uint8_t* a_hi = sm.slot[bi][0];
+        uint8_t* a_lo = sm.slot[bi][1];
+        uint8_t* b0 = sm.slot[bi][2];
+        uint8_t* b1 = sm.slot[bi][3];
+        const bool intra = u < nintra;
+        if (intra) {
+            if (kind == 0) {
+                // A: Psi rows of the tile, column block u (K = 64 sources), K-major
+                for (int i = tid; i < 2 * kT * 8; i += kDcThreads) {
+                    const int part = i / (kT * 8), j = i % (kT * 8);
+                    const uint4 v = reinterpret_cast<const uint4*>(
+                        pbase + part * ppart + (i64)u * S * 128 + (i64)tt * kT * 128)[j];
+                    *reinterpret_cast<uint4*>((part ? a_lo : a_hi) + j * 16) = v;
+                }
+            } else {
+                // A: Psi^T, M = the tile's 128 sources (column blocks 2 tt, 2 tt + 1), K = 64
+                // target rows from tt * 128 + 64 u, MN-major: [block][64 rows][128 bytes]
+                const int t0u = tt * kT + 64 * u;
+                for (int i = tid; i < 2 * 2 * 64 * 8; i += kDcThreads) {
+                    const int part = i / (2 * 64 * 8), j = i % (2 * 64 * 8);
+                    const int blk = j / (64 * 8), jj = j % (64 * 8);
+                    const uint4 v = reinterpret_cast<const uint4*>(
+                        pbase + part * ppart + (i64)(2 * tt + blk) * S * 128 + (i64)t0u * 128)[jj];
+                    *reinterpret_cast<uint4*>((part ? a_lo : a_hi) + blk * 8192 + jj * 16) = v;
+                }
+            }
+            // B: 64 token rows of B (dC) or C (dB), MN-major N = 128: [n block][64 rows][128 bytes]
+            const int r0 = kind == 0 ? 64 * u : tt * kT + 64 * u;
+            const __nv_bfloat16* src = kind == 0 ? Bm : Cm;
+            for (int i = tid; i < 64 * 16; i += kDcThreads) {
+                const int r = i / 16, q = i % 16;
+                const uint4 v = reinterpret_cast<const uint4*>(src + (tok0 + r0 + r) * kN)[q];
+                *reinterpret_cast<uint4*>(b0 + (q / 8) * 8192 + sw128((uint32_t)r, (uint32_t)(q % 8) * 16u)) = v;
+            }
+        } else {
+            const int h = u - nintra;
+            // A: exp(cum_t) dY_t (dC) or exp(cum_end - cum_s) dt_s X_s (dB) of head h, K = p, split
+            const float* cumh = cumb + ((i64)h * Mc + c) * S;
+            const float cend = cumh[S - 1];
+            for (int i = tid; i < kT * 8; i += kDcThreads) {
+                const int r = i / 8, q = i % 8;
+                const int t = tt * kT + r;
+                const i64 tok = tok0 + t;
+                float f;
+                uint4 w;
+                if (kind == 0) {
+                    f = expf(cumh[t]);
+                    w = reinterpret_cast<const uint4*>(dY + (tok * H + h) * kP)[q];
+                } else {
+                    f = expf(cend - cumh[t]) * dt[tok * H + h];
+                    w = reinterpret_cast<const uint4*>(X + (tok * H + h) * kP)[q];
+                }
+                const uint32_t ww[4] = {w.x, w.y, w.z, w.w};
+                float v[8];
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    v[2 * e] = bf_lo(ww[e]) * f;
+                    v[2 * e + 1] = bf_hi(ww[e]) * f;
+                }
+                uint4 hi, lo;
+                split8(v, hi, lo);
+                const uint32_t o = sw128((uint32_t)r, (uint32_t)q * 16u);
+                *reinterpret_cast<uint4*>(a_hi + o) = hi;
+                *reinterpret_cast<uint4*>(a_lo + o) = lo;
+            }
+            // B: H_[c-1] (dC) or d(dH_c) (dB) of head h, [n][p] hi | lo: K-major (rows n, K = p)
+            const uint8_t* tile = (kind == 0 ? Hops : Dops) + (((i64)b * Mc + c) * H + h) * 32768;
+            for (int i = tid; i < 2048; i += kDcThreads)
+                *reinterpret_cast<uint4*>(b0 + i * 16) = reinterpret_cast<const uint4*>(tile)[i];
+        }
+        tc::fence_proxy_async_shared();
+        tc::tc_fence_before();
+        __syncthreads();
+        if (tid == 0) {
+            tc::tc_fence_after();
+            const uint32_t sa_hi = tc::smem_u32(a_hi), sa_lo = tc::smem_u32(a_lo);
+            const uint32_t sb0 = tc::smem_u32(b0), sb1 = tc::smem_u32(b1);
+            if (intra) {
+                const uint32_t id = idesc_bf16(kind == 1, true, kT, kN);
+                for (int part = 0; part < 2; ++part) {
+                    const uint32_t sa = part ? sa_lo : sa_hi;
+                    for (int ks = 0; ks < 4; ++ks) {
+                        const uint64_t ad = kind == 0 ? tc::smem_desc_sw128(sa + 32u * ks, 16u, 1024u)
+                                                      : tc::smem_desc_sw128(sa + 2048u * ks, 8192u, 1024u);
+                        const uint64_t bd = tc::smem_desc_sw128(sb0 + 2048u * ks, 8192u, 1024u);
+                        mma_ss(tmem, ad, bd, id, (u > 0 || part > 0 || ks > 0) ? 1u : 0u);
+                    }
+                }
+            } else {
+                const uint32_t id = idesc_bf16(false, false, kT, kN);
+                for (int term = 0; term < 3; ++term) {  // a_hi b_hi, a_lo b_hi, a_hi b_lo
+                    const uint32_t sa = term == 1 ? sa_lo : sa_hi;
+                    const uint32_t sb = term == 2 ? sb1 : sb0;
+                    for (int ks = 0; ks < 4; ++ks) {
+                        const uint64_t ad = tc::smem_desc_sw128(sa + 32u * ks, 16u, 1024u);
+                        const uint64_t bd = tc::smem_desc_sw128(sb + 32u * ks, 16u, 1024u);
+                        mma_ss(tmem, ad, bd, id, (u > 0 || term > 0 || ks > 0) ? 1u : 0u);
+                    }
+                }
+            }
+            tc::mma_commit(&sm.mma_done[bi]);
+        }
+        issued = u + 1;
+    }
+    if (ok && nunits > 0) {
+        const int last = nunits - 1;
+        ok = cta_wait(&sm.mma_done[last & 1], (uint32_t)((last >> 1) & 1), wait_limit_ns, 44);
+    }
+    if (!ok && issued > 0 && tid == 0) {
+        tc::mma_commit(&sm.drain);
+        if (!tc::mbar_wait(&sm.drain, 0, kDrainLimitNs, nullptr)) atomicCAS(&g_sbwd_tc_status, 0, 45);
+    }
+    tc::tc_fence_after();
+    if (ok) {
+        // thread (row, half): 64 columns of its token row
+        const int r = tid & (kT - 1), half = tid >> 7;
+        const uint32_t lane_addr = (uint32_t)(32 * (warp & 3)) << 16;
+        const i64 tok = tok0 + tt * kT + r;
+        float* dst = (kind == 0 ? dC : dB) + tok * kN + 64 * half;
+        for (int cc = 0; cc < 2; ++cc) {
+            float v[32];
+            tmem_ld32(tmem + lane_addr + (uint32_t)(64 * half + 32 * cc), v);
+            float4* d4 = reinterpret_cast<float4*>(dst + 32 * cc);
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+                float4 o = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+                if (kind == 0) {
+                    const float4 p = d4[q];
+                    o.x += p.x; o.y += p.y; o.z += p.z; o.w += p.w;
+                }
+                d4[q] = o;
+            }
+        }
+    }
+    tc::tc_fence_before();
+    __syncthreads();
+    if (warp == 0) {
+        __syncwarp();
+        tc::tc_fence_after();
+        tc::tmem_dealloc(tmem, 128);
+    }
+}
+
+// ------------------------------------------------------------- finalize
+// One CTA of S threads per (c, h, b): d(cum) of the chunk,
+//   d(cum_t) = phi_row_t + rowI_t - phi_col_t - kappa_t,  kappa_t = dt_t xi_t,
+// plus sum_s kappa_s and the passing term at the chunk's last token; then the
+// reverse sums, d(dt) and the chunk's share of dA_h.
+__global__ void finalize_kernel(const float* __restrict__ dt, const float* __restrict__ A,
+                                const float* __restrict__ phi_row, const float* __restrict__ phi_col,
+                                const float* __restrict__ rowI, const float* __restrict__ xi,
+                                const float* __restrict__ dcum_end, float* __restrict__ ddt,
+                                float* __restrict__ dA, int L, int H, int S, int Mc) {
+    __shared__ float sv[256];
+    __shared__ float red[8];
+    const int c = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
+    const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+    const i64 idx = ((i64)b * L + (i64)c * S + t) * H + h;
+    const float dtv = dt[idx];
+    const float pc = phi_col[idx], xv = xi[idx];
+    const float kap = dtv * xv;
+    float dcum = phi_row[idx] + rowI[idx] - pc - kap;
+    float k = kap;
+    for (int off = 16; off > 0; off >>= 1) k += __shfl_xor_sync(0xffffffffu, k, off);
+    if (lane == 0) red[warp] = k;
+    __syncthreads();
+    if (t == S - 1) {
+        float ks = 0.0f;
+        for (int w = 0; w < S / 32; ++w) ks += red[w];
+        dcum += ks + dcum_end[((i64)b * H + h) * Mc + c];
+    }
+    // reverse inclusive scan: run_t = sum_{k >= t} dcum_k
+    sv[t] = dcum;
+    __syncthreads();
+    for (int off = 1; off < S; off <<= 1) {
+        const float add = t + off < S ? sv[t + off] : 0.0f;
+        __syncthreads();
+        sv[t] += add;
+        __syncthreads();
+    }
+    const float run = sv[t];
+    // d(dt) direct part: X_t . Y'_t = phi_col_t / dt_t + xi_t
+    ddt[idx] = (dtv != 0.0f ? pc / dtv : 0.0f) + xv + A[h] * run;
+    float da = dtv * run;
+    for (int off = 16; off > 0; off >>= 1) da += __shfl_xor_sync(0xffffffffu, da, off);
+    __syncthreads();
+    if (lane == 0) red[warp] = da;
+    __syncthreads();
+    if (t == 0) {
+        float s = 0.0f;
+        for (int w = 0; w < S / 32; ++w) s += red[w];
+        atomicAdd(dA + h, s);
+    }
+}
+
+}  // namespace
+
+// Workspace of the tensor-core scan backward.
+size_t scan_bwd_tc_workspace(int64_t B, int64_t L, int64_t H, int64_t S) {
+    const int64_t M = L / S;
+    auto al = [](size_t x) { return (x + 255) & ~(size_t)255; };
+    const size_t states = (size_t)(B * M * H) * kN * kP * 4;
+    return al((size_t)(B * H * M * S) * 4)        // cum
+           + 2 * al(states)                        // H_[c-1] fp32; Z, then d(dH_c)
+           + al((size_t)(B * H * M) * 4)           // d(cum_end)
+           + 2 * al((size_t)(B * M * H) * 32768)   // Hops, Dops
+           + 4 * al((size_t)(B * L * H) * 4)       // rowI, xi, phi_row, phi_col
+           + al((size_t)(B * M) * psi_chunk_bytes((int)S));  // Psi
+}
+
+cudaError_t launch_chunk_scan_backward_tc(const ScanBwdArgs& a, void* ws,
+                                          unsigned long long wait_limit_ns, cudaStream_t stream) {
+    const ScanArgs& f = a.fwd;
+    const int B = (int)f.B, L = (int)f.L, H = (int)f.H, S = (int)f.S, Mc = L / S, NP = kN * kP;
+    auto al = [](size_t x) { return (x + 255) & ~(size_t)255; };
+    const size_t states = (size_t)(f.B * Mc * f.H) * NP * 4;
+    uint8_t* w = (uint8_t*)ws;
+    float* cum = (float*)w;            w += al((size_t)(f.B * f.H * Mc * S) * 4);
+    float* Hprev = (float*)w;          w += al(states);
+    float* ZD = (float*)w;             w += al(states);
+    float* dcum_end = (float*)w;       w += al((size_t)(f.B * f.H * Mc) * 4);
+    uint8_t* Hops = w;                 w += al((size_t)(f.B * Mc * f.H) * 32768);
+    uint8_t* Dops = w;                 w += al((size_t)(f.B * Mc * f.H) * 32768);
+    const size_t tokh = al((size_t)(f.B * f.L * f.H) * 4);
+    float* rowI = (float*)w;           w += tokh;
+    float* xi = (float*)w;             w += tokh;
+    float* phi_row = (float*)w;        w += tokh;
+    float* phi_col = (float*)w;        w += tokh;
+    uint8_t* psi = w;
+
+    cudaError_t e = launch_scan_states_tc(f, cum, Hprev, Hops, wait_limit_ns, stream);
+    if (e != cudaSuccess) return e;
+    if ((e = cudaMemsetAsync(dcum_end, 0, (size_t)(f.B * f.H * Mc) * 4, stream)) != cudaSuccess) return e;
+    if ((e = cudaMemsetAsync(a.dA, 0, (size_t)f.H * 4, stream)) != cudaSuccess) return e;
+    if (!a.accumulate_dC &&
+        (e = cudaMemsetAsync(a.dC, 0, (size_t)(f.B * f.L) * kN * 4, stream)) != cudaSuccess)
+        return e;
+    if ((e = launch_scan_bwd_inter_tc(f, cum, a.dY, ZD, wait_limit_ns, stream)) != cudaSuccess) return e;
+    if ((e = launch_scan_bwd_passing(ZD, a.dM, Hprev, cum, dcum_end, Dops, B, H, S, Mc, NP, stream)) !=
+        cudaSuccess)
+        return e;
+    if ((e = launch_scan_bwd_output_tc(f, cum, Hops, Dops, a.dY, rowI, a.dX, xi, wait_limit_ns,
+                                       stream)) != cudaSuccess)
+        return e;
+    if ((e = cudaMemsetAsync(phi_col, 0, (size_t)(f.B * f.L * f.H) * 4, stream)) != cudaSuccess) return e;
+    for (int phi = 0; phi < 2; ++phi) {
+        const size_t smem = sizeof(PsiSmem) + 1024;
+        auto k = phi ? psi_kernel<true> : psi_kernel<false>;
+        if ((e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) != cudaSuccess)
+            return e;
+        k<<<dim3(S / kT, Mc, B), kPsiThreads, smem, stream>>>(
+            (const __nv_bfloat16*)f.X, f.dt, cum, (const __nv_bfloat16*)a.dY, (const __nv_bfloat16*)f.Bm,
+            (const __nv_bfloat16*)f.Cm, psi, phi_row, phi_col, L, H, S, Mc, wait_limit_ns);
+    }
+    {
+        const size_t smem = sizeof(DcSmem) + 1024;
+        if ((e = cudaFuncSetAttribute(dcdb_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) !=
+            cudaSuccess)
+            return e;
+        dcdb_kernel<<<dim3(2 * (S / kT), Mc, B), kDcThreads, smem, stream>>>(
+            (const __nv_bfloat16*)f.X, f.dt, cum, (const __nv_bfloat16*)f.Bm, (const __nv_bfloat16*)f.Cm,
+            (const __nv_bfloat16*)a.dY, psi, Hops, Dops, a.dC, a.dB, L, H, S, Mc, wait_limit_ns);
+    }
+    finalize_kernel<<<dim3(Mc, H, B), S, 0, stream>>>(f.dt, f.A, phi_row, phi_col, rowI, xi, dcum_end,
+                                                      a.ddt, a.dA, L, H, S, Mc);
+    note_launches(4);
+    return cudaGetLastError();
+}
+
+int take_scan_bwd_tc_status() {
+    int v = 0;
+    if (cudaMemcpyFromSymbol(&v, g_sbwd_tc_status, sizeof(int)) != cudaSuccess) return -1;
+    if (v != 0) {
+        const int zero = 0;
+        cudaMemcpyToSymbol(g_sbwd_tc_status, &zero, sizeof(int));
+    }
+    return v;
+}
+
+}  // namespace dart

@@ -330,7 +330,8 @@ struct SpSmem {
 __global__ void __launch_bounds__(kSpThreads)
 state_passing_tc_kernel(const float* __restrict__ dH, const float* __restrict__ cum,
                         float* __restrict__ final_state, uint8_t* __restrict__ Hops,
-                        int H, int M, int S, unsigned long long wait_limit_ns) {
+                        float* __restrict__ Hout, int H, int M, int S,
+                        unsigned long long wait_limit_ns) {
     __shared__ __align__(128) SpSmem sm;
     constexpr int NP = kN * kP;
     const int slab = blockIdx.x, h = blockIdx.y, b = blockIdx.z, tid = threadIdx.x;
@@ -338,7 +339,7 @@ state_passing_tc_kernel(const float* __restrict__ dH, const float* __restrict__ 
     const int n = e0 / kP, p = e0 % kP;
     const i64 cstride = (i64)H * NP;  // floats between the chunk slots of one (b, h)
     const float* src = dH + ((i64)b * M * H + h) * NP + (i64)slab * kSpSlab;
-    uint8_t* hop = Hops + ((i64)b * M * H + h) * 32768 + sw128((uint32_t)n, (uint32_t)p * 2u);
+    uint8_t* hop = Hops == nullptr ? nullptr : Hops + ((i64)b * M * H + h) * 32768 + sw128((uint32_t)n, (uint32_t)p * 2u);
     const i64 hstride = (i64)H * 32768;
     const float* cumh = cum + ((i64)b * H + h) * (i64)M * S;
 
@@ -378,9 +379,15 @@ state_passing_tc_kernel(const float* __restrict__ dH, const float* __restrict__ 
                 hi[k] = *reinterpret_cast<const uint32_t*>(&hv);
                 lo[k] = pack_bf16(st[2 * k] - hf.x, st[2 * k + 1] - hf.y);
             }
-            uint8_t* t = hop + (i64)c * hstride;
-            *reinterpret_cast<uint2*>(t) = make_uint2(hi[0], hi[1]);
-            *reinterpret_cast<uint2*>(t + 16384) = make_uint2(lo[0], lo[1]);
+            if (hop != nullptr) {
+                uint8_t* t = hop + (i64)c * hstride;
+                *reinterpret_cast<uint2*>(t) = make_uint2(hi[0], hi[1]);
+                *reinterpret_cast<uint2*>(t + 16384) = make_uint2(lo[0], lo[1]);
+            }
+            if (Hout != nullptr)  // also fp32 (may be dH itself: chunk c's slab is already read)
+                *reinterpret_cast<float4*>(Hout + ((i64)b * M * H + h) * NP + (i64)slab * kSpSlab +
+                                           (i64)c * cstride + tid * kSpElems) =
+                    make_float4(st[0], st[1], st[2], st[3]);
             const float a = sm.dec[c % kSpDec];
             st[0] = fmaf(a, st[0], d.x);
             st[1] = fmaf(a, st[1], d.y);
@@ -419,12 +426,23 @@ struct OutSmem {
     float bnorm[256];              // |B_s| of the sources
     float cnorm[kT];               // |C_t| of the tile's rows
     uint32_t bdmax[2];             // max_s |B_s| dt_s of a head (float bits), by head parity
+    float dacc[8][kT][2];          // backward modes: per (head, row) dot product
     uint64_t bar;
     uint64_t hbar[2];              // H_[c-1] tile copy into buffer 0 / 1 landed
     uint32_t tmem_base;
 };
 
 constexpr int kOutThreads = 512;  // four threads per token row
+
+// Modes of the output kernel. kOutY: the forward, Y. kOutDot: for the
+// backward, only the inter-chunk part of the forward (no intra work), writing
+// dY_t . exp(cum_t) C_t H_[c-1] per (t, h). kOutRev: the backward's dX as the
+// same computation in reversed time inside each chunk (target s, sources
+// t >= s; C <- B, B <- C, X <- dY, dt <- 1, cum' = cum_end - cum,
+// H_[c-1] <- d(dH_c)):
+//   Y'_s = sum_{t >= s} e^{cum_t - cum_s} (B_s . C_t) dY_t + e^{cum_end - cum_s} B_s d(dH_c),
+// writing dX_s = dt_s Y'_s and per (s, h) X_s . (its inter-chunk part).
+constexpr int kOutY = 0, kOutDot = 1, kOutRev = 2;
 
 __device__ __forceinline__ float ex2_approx(float x) {
     float y;
@@ -438,13 +456,14 @@ struct HeadRegs {
     float c2, dtv;  // source tid (tid < ns)
 };
 
-template <typename Tout>
+template <typename Tout, int kMode = kOutY>
 __global__ void __launch_bounds__(kOutThreads, 1)
 chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restrict__ dt,
                        const float* __restrict__ cum, const __nv_bfloat16* __restrict__ Bm,
                        const __nv_bfloat16* __restrict__ Cm, const uint8_t* __restrict__ Hops,
                        Tout* __restrict__ Y, int L, int H, int G, int S, int Mc,
-                       unsigned long long wait_limit_ns) {
+                       unsigned long long wait_limit_ns,
+                       const __nv_bfloat16* __restrict__ Zd = nullptr, float* __restrict__ dots = nullptr) {
     extern __shared__ uint8_t smem_raw[];
     OutSmem& sm = *reinterpret_cast<OutSmem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                               ~(uintptr_t)1023);
@@ -459,8 +478,13 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
     const int ns = (tt + 1) * kT;  // sources 0 .. ns-1 of the chunk
     const i64 tok0 = (i64)b * L + (i64)c * S;
     const uint32_t lane_addr = (uint32_t)(32 * (warp & 3)) << 16;
-    const bool has_prev = c > 0;
+    const bool has_prev = kMode == kOutRev || c > 0;
     constexpr uint32_t kColSc = 0, kColW = 256, kColIn = 384, kColEx = 448;
+    // chunk position of the kernel's token k (reversed inside the chunk for kOutRev)
+    auto pos = [&](int k) { return kMode == kOutRev ? S - 1 - k : k; };
+    constexpr bool kIntra = kMode != kOutDot;
+    if (kMode != kOutY)
+        for (int i = tid; i < kHeadsPerCta * kT * 2; i += kOutThreads) (&sm.dacc[0][0][0])[i] = 0.0f;
 
     if (tid == 0) {
         tc::mbar_init(&sm.bar, 1);
@@ -488,18 +512,18 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
     // C of the tile: row t, K-major, two K blocks of 64 (16-byte chunks, swizzled)
     for (int i = tid; i < kT * 16; i += kOutThreads) {
         const int t = i / 16, q = i % 16;
-        const uint4 v = reinterpret_cast<const uint4*>(Cm + ((tok0 + tt * kT + t) * G + g) * kN)[q];
+        const uint4 v = reinterpret_cast<const uint4*>(Cm + ((tok0 + pos(tt * kT + t)) * G + g) * kN)[q];
         *reinterpret_cast<uint4*>(sm.c_tile[q / 8] + sw128((uint32_t)t, (uint32_t)(q % 8) * 16u)) = v;
     }
     // B of the sources: row s, K-major
-    for (int i = tid; i < ns * 16; i += kOutThreads) {
+    for (int i = tid; kIntra && i < ns * 16; i += kOutThreads) {
         const int s = i / 16, q = i % 16;
-        const uint4 v = reinterpret_cast<const uint4*>(Bm + ((tok0 + s) * G + g) * kN)[q];
+        const uint4 v = reinterpret_cast<const uint4*>(Bm + ((tok0 + pos(s)) * G + g) * kN)[q];
         *reinterpret_cast<uint4*>(sm.b_src[q / 8] + sw128((uint32_t)s, (uint32_t)(q % 8) * 16u)) = v;
     }
     // row norms for the W scale bound: thread tid < ns takes |B_tid|, tid < kT takes |C_tid|
-    if (tid < ns) {
-        const uint4* brow = reinterpret_cast<const uint4*>(Bm + ((tok0 + tid) * G + g) * kN);
+    if (kIntra && tid < ns) {
+        const uint4* brow = reinterpret_cast<const uint4*>(Bm + ((tok0 + pos(tid)) * G + g) * kN);
         float ss = 0.0f;
 #pragma unroll 4
         for (int q = 0; q < 16; ++q) {
@@ -514,7 +538,7 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
         sm.bnorm[tid] = sqrtf(ss);
     }
     if (tid < kT) {
-        const uint4* crow = reinterpret_cast<const uint4*>(Cm + ((tok0 + tt * kT + tid) * G + g) * kN);
+        const uint4* crow = reinterpret_cast<const uint4*>(Cm + ((tok0 + pos(tt * kT + tid)) * G + g) * kN);
         float ss = 0.0f;
 #pragma unroll 4
         for (int q = 0; q < 16; ++q) {
@@ -536,7 +560,7 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
     const uint32_t tmem = sm.tmem_base;
     uint32_t phase = 0;
     // scores = C_tile B_src^T (M 128, N ns, K 128), shared by the CTA's heads
-    if (tid == 0) {
+    if (kIntra && tid == 0) {
         const uint32_t idesc = tc::idesc_f16(1, false, kT, (uint32_t)ns);
         for (int ks = 0; ks < kN / 16; ++ks) {
             const uint64_t ad = tc::smem_desc_sw128(tc::smem_u32(sm.c_tile[ks / 4]) + 32u * (ks % 4), 16u, 1024u);
@@ -551,22 +575,28 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
     auto load_head = [&](int h) {
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
-            if (k < xiters) {
+            if (kIntra && k < xiters) {
                 const int i = tid + k * kOutThreads, sidx = i / 8, q = i % 8;
-                nx.xv[k] = reinterpret_cast<const uint4*>(X + ((tok0 + sidx) * H + h) * kP)[q];
+                nx.xv[k] = reinterpret_cast<const uint4*>(X + ((tok0 + pos(sidx)) * H + h) * kP)[q];
             }
         }
         if (tid < ns) {
-            nx.c2 = cum[(((i64)b * H + h) * Mc + c) * S + tid] * kLog2e;
-            nx.dtv = dt[(tok0 + tid) * H + h];
+            const float* cumc = cum + (((i64)b * H + h) * Mc + c) * S;
+            if (kMode == kOutRev) {  // cum' = cum_end - cum (reversed), dt' = 1
+                nx.c2 = (cumc[S - 1] - cumc[pos(tid)]) * kLog2e;
+                nx.dtv = 1.0f;
+            } else {
+                nx.c2 = cumc[tid] * kLog2e;
+                nx.dtv = dt[(tok0 + tid) * H + h];
+            }
         }
     };
     load_head(h0);
     bool ok = commit_and_wait(&sm.bar, phase, wait_limit_ns, 2);
     phase ^= 1u;
 
-    const int tl = tt * kT + row;  // this thread's token inside the chunk
-    const i64 tok = tok0 + tl;
+    const int tl = tt * kT + row;  // this thread's token inside the chunk (kernel order)
+    const i64 tok = tok0 + pos(tl);
     const int tl_warp_max = tt * kT + 32 * (warp & 3) + 31;
     const int s_lo = quarter * (ns / 4), s_hi = s_lo + ns / 4;  // 32 or 64 sources
     for (int hh = 0; hh < kHeadsPerCta && ok; ++hh) {
@@ -574,7 +604,7 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
         // prefetched sources into shared memory (the previous head's MMAs are done)
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
-            if (k < xiters) {
+            if (kIntra && k < xiters) {
                 const int i = tid + k * kOutThreads, sidx = i / 8, q = i % 8;
                 const uint32_t xw[4] = {nx.xv[k].x, nx.xv[k].y, nx.xv[k].z, nx.xv[k].w};
                 uint32_t f[4];
@@ -634,7 +664,7 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
             }
             tc::tmem_st16(tmem + lane_addr + kColW + (uint32_t)(s0 / 2), pk);
         };
-        for (int s0 = s_lo; s0 < s_hi; s0 += 32) {  // s_hi - s_lo is 32 or 64
+        for (int s0 = s_lo; kIntra && s0 < s_hi; s0 += 32) {  // s_hi - s_lo is 32 or 64
             const bool live = s0 <= tl_warp_max;
             float v[32];
             if (live) tmem_ld32(tmem + lane_addr + kColSc + (uint32_t)s0, v);
@@ -649,7 +679,7 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
             tc::tc_fence_after();
             if (has_prev) hok = tc::mbar_wait(&sm.hbar[hh & 1], (uint32_t)((hh >> 1) & 1), wait_limit_ns, nullptr);
             const uint32_t id16 = tc::idesc_f16(0, true, kT, kP);
-            for (int ks = 0; ks < ns / 16; ++ks) {
+            for (int ks = 0; kIntra && ks < ns / 16; ++ks) {
                 const uint64_t bd = tc::smem_desc_sw128(tc::smem_u32(sm.x_src) + 2048u * ks, 1024u, 1024u);
                 tc::mma_f16_ts(tmem + kColIn, tmem + kColW + 8u * ks, bd, id16, ks > 0 ? 1u : 0u);
             }
@@ -674,16 +704,46 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
         {
             const float dec = exp2f(c2t);
             float vi[16], ve[16];
-            tmem_ld16(tmem + lane_addr + kColIn + 16u * quarter, vi);
+            if (kIntra) {
+                tmem_ld16(tmem + lane_addr + kColIn + 16u * quarter, vi);
+            } else {
+#pragma unroll
+                for (int i = 0; i < 16; ++i) vi[i] = 0.0f;
+            }
             if (has_prev) {
                 tmem_ld16(tmem + lane_addr + kColEx + 16u * quarter, ve);
             } else {
 #pragma unroll
                 for (int i = 0; i < 16; ++i) ve[i] = 0.0f;
             }
+            if (kMode == kOutRev) {
+                // dX = dt Y', and X . (inter part of Y')
+                const float dts = dt[tok * H + h];
+                float zv[16];
+                load_row16(Zd + (tok * H + h) * kP + 16 * quarter, zv);
+                float d2 = 0.0f;
 #pragma unroll
-            for (int i = 0; i < 16; ++i) vi[i] = fmaf(wmax, vi[i], dec * ve[i]);
-            store_row16(Y + (tok * H + h) * kP + 16 * quarter, vi);
+                for (int i = 0; i < 16; ++i) {
+                    const float inter = dec * ve[i];
+                    vi[i] = fmaf(wmax, vi[i], inter) * dts;
+                    d2 = fmaf(zv[i], inter, d2);
+                }
+                store_row16(Y + (tok * H + h) * kP + 16 * quarter, vi);
+                atomicAdd(&sm.dacc[hh][row][0], d2);
+            } else {
+#pragma unroll
+                for (int i = 0; i < 16; ++i) vi[i] = fmaf(wmax, vi[i], dec * ve[i]);
+                if (kMode == kOutY) {
+                    store_row16(Y + (tok * H + h) * kP + 16 * quarter, vi);
+                } else {  // dY . (inter part of Y); vi holds only that part here
+                    float zv[16];
+                    load_row16(Zd + (tok * H + h) * kP + 16 * quarter, zv);
+                    float d1 = 0.0f;
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) d1 = fmaf(zv[i], vi[i], d1);
+                    atomicAdd(&sm.dacc[hh][row][0], d1);
+                }
+            }
         }
         tc::tc_fence_before();
         __syncthreads();  // shared staging and TMEM are reused by the next head
@@ -700,6 +760,13 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
     }
     tc::tc_fence_before();
     __syncthreads();
+    if (kMode != kOutY && ok) {  // the per (token, head) dots
+        for (int i = tid; i < kHeadsPerCta * kT; i += kOutThreads) {
+            const int hh = i / kT, r = i % kT;
+            const i64 tk = tok0 + pos(tt * kT + r);
+            dots[tk * H + h0 + hh] = sm.dacc[hh][r][0];
+        }
+    }
     if (warp == 0) {
         __syncwarp();
         tc::tc_fence_after();
@@ -733,7 +800,7 @@ cudaError_t launch_chunk_scan_tc(const ScanArgs& a, unsigned long long wait_limi
     }
     // fp32 memories are the chunk states themselves: the state passing reads them
     state_passing_tc_kernel<<<dim3(kN * kP / kSpSlab, H, B), kSpThreads, 0, stream>>>(
-        mem_is_f32 ? (const float*)a.M : a.dH32, a.cum, a.final_state, a.Hops, H, M, S,
+        mem_is_f32 ? (const float*)a.M : a.dH32, a.cum, a.final_state, a.Hops, nullptr, H, M, S,
         wait_limit_ns);
     {
         auto kern = chunk_output_tc_kernel<Tout>;
@@ -742,16 +809,18 @@ cudaError_t launch_chunk_scan_tc(const ScanArgs& a, unsigned long long wait_limi
         if (e != cudaSuccess) return e;
         kern<<<dim3(S / kT, M * (H / kHeadsPerCta), B), kOutThreads, smem, stream>>>(
             (const __nv_bfloat16*)a.X, a.dt, a.cum, (const __nv_bfloat16*)a.Bm,
-            (const __nv_bfloat16*)a.Cm, a.Hops, (Tout*)a.Y, L, H, G, S, M, wait_limit_ns);
+            (const __nv_bfloat16*)a.Cm, a.Hops, (Tout*)a.Y, L, H, G, S, M, wait_limit_ns, nullptr,
+            nullptr);
     }
     note_launches(3);
     return cudaGetLastError();
 }
 
 // Backward helpers on the tensor-core path (bf16 inputs, the same shapes).
-// States: cum and the fp32 state entering every chunk (in Hprev), i.e. the
-// forward's chunk states followed by the in-place fp32 state passing.
-cudaError_t launch_scan_states_tc(const ScanArgs& a0, float* cum, float* Hprev,
+// States: cum and the state entering every chunk, fp32 (in Hprev) and as the
+// split operand tiles (Hops), i.e. the forward's chunk states followed by the
+// state passing.
+cudaError_t launch_scan_states_tc(const ScanArgs& a0, float* cum, float* Hprev, uint8_t* Hops,
                                   unsigned long long wait_limit_ns, cudaStream_t stream) {
     ScanArgs a = a0;
     a.cum = cum;
@@ -765,10 +834,10 @@ cudaError_t launch_scan_states_tc(const ScanArgs& a0, float* cum, float* Hprev,
     kern<<<dim3(M, H / kHeadsPerCta, B), kStateThreads, smem, stream>>>(
         (const __nv_bfloat16*)a.X, a.dt, a.cum, (const __nv_bfloat16*)a.Bm, nullptr, Hprev, nullptr,
         L, H, G, S, M, a.eps, wait_limit_ns);
-    note_launches(1);
-    a.dH32 = Hprev;  // chunk states in, entering states out (in place)
-    a.final_state = nullptr;
-    return launch_state_passing(a, stream);
+    state_passing_tc_kernel<<<dim3(kN * kP / kSpSlab, H, B), kSpThreads, 0, stream>>>(
+        Hprev, a.cum, nullptr, Hops, Hprev, H, M, S, wait_limit_ns);
+    note_launches(2);
+    return cudaGetLastError();
 }
 
 // Z_c = sum_{t in c} exp(cum_t) C_t^T dY_t for every chunk (fp32, B x Mc x H x N x P).
@@ -783,6 +852,39 @@ cudaError_t launch_scan_bwd_inter_tc(const ScanArgs& a, const float* cum, const 
         (const __nv_bfloat16*)dY, a.dt, cum, (const __nv_bfloat16*)a.Cm, Z, nullptr, nullptr, L, H, G,
         S, M, a.eps, wait_limit_ns);
     note_launches(1);
+    return cudaGetLastError();
+}
+
+// The output kernel's backward modes. rowI (B x L x H): dY_t . exp(cum_t) C_t
+// H_[c-1], from the forward operand tiles Hops. dX (B x L x H x P, fp32) and
+// xi (B x L x H): X_s . exp(cum_end - cum_s) B_s d(dH_c), from the reversed
+// computation with Dops (d(dH_c)) as the state operand.
+cudaError_t launch_scan_bwd_output_tc(const ScanArgs& a, const float* cum, const uint8_t* Hops,
+                                      const uint8_t* Dops, const void* dY, float* rowI,
+                                      float* dX, float* xi, unsigned long long wait_limit_ns,
+                                      cudaStream_t stream) {
+    const int B = (int)a.B, L = (int)a.L, H = (int)a.H, G = (int)a.G, S = (int)a.S, M = L / S;
+    typedef __nv_bfloat16 bf;
+    const size_t smem = sizeof(OutSmem) + 1024;
+    const dim3 grid(S / kT, M * (H / kHeadsPerCta), B);
+    {
+        auto kern = chunk_output_tc_kernel<float, kOutDot>;
+        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+        kern<<<grid, kOutThreads, smem, stream>>>((const bf*)a.X, a.dt, cum, (const bf*)a.Bm,
+                                                  (const bf*)a.Cm, Hops, nullptr, L, H, G, S, M,
+                                                  wait_limit_ns, (const bf*)dY, rowI);
+    }
+    {
+        auto kern = chunk_output_tc_kernel<float, kOutRev>;
+        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+        // sources X <- dY, B <- C, C <- B; the dots take X
+        kern<<<grid, kOutThreads, smem, stream>>>((const bf*)dY, a.dt, cum, (const bf*)a.Cm,
+                                                  (const bf*)a.Bm, Dops, dX, L, H, G, S, M,
+                                                  wait_limit_ns, (const bf*)a.X, xi);
+    }
+    note_launches(2);
     return cudaGetLastError();
 }
 

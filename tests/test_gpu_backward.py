@@ -79,7 +79,7 @@ def test_sma_backward_matches_oracle(w):
         assert err <= _tol(w), f"{name}: {err:.3e}"
 
 
-@pytest.mark.parametrize("w", [CASES[0], CASES[3]], ids=lambda w: w.name)
+@pytest.mark.parametrize("w", [CASES[0], CASES[3], CASES[6]], ids=lambda w: w.name)
 def test_layer_backward_matches_oracle(w):
     """Forward through the library, then the layer backward: SMA backward's dM and
     dC feed the scan backward."""
