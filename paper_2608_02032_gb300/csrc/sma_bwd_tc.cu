@@ -110,6 +110,29 @@ __device__ __forceinline__ void warp_arrive(uint64_t* bar) {
     if ((threadIdx.x & 31) == 0) tc::mbar_arrive(bar);
 }
 
+// Bounded wait by every thread of the CTA, then a CTA-wide AND of the outcome.
+__device__ __forceinline__ bool cta_and_wait(uint64_t* bar, uint32_t parity, uint64_t limit_ns, int code) {
+    const bool got = tc::mbar_wait(bar, parity, limit_ns, nullptr);
+    if (!got) atomicCAS(&g_bwd_tc_status, 0, code);
+    const bool all = __syncthreads_and(got ? 1 : 0) != 0;
+    tc::tc_fence_after();
+    return all;
+}
+
+// Splits 8 floats into bf16 hi and lo words.
+__device__ __forceinline__ void split_bf16x8(const float* v, uint4& hi, uint4& lo) {
+    uint32_t hw[4], lw[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+        const __nv_bfloat162 h2 = __floats2bfloat162_rn(v[2 * e], v[2 * e + 1]);
+        const float2 hf = __bfloat1622float2(h2);
+        hw[e] = *reinterpret_cast<const uint32_t*>(&h2);
+        lw[e] = pack_bf16(v[2 * e] - hf.x, v[2 * e + 1] - hf.y);
+    }
+    hi = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+    lo = make_uint4(lw[0], lw[1], lw[2], lw[3]);
+}
+
 // AND of v over the 256 threads of named barrier 1 (the epilogue warpgroups).
 __device__ __forceinline__ bool epi_and(bool v) {
     uint32_t r;
@@ -586,7 +609,7 @@ sma_bwd_rows_kernel(const uint8_t* __restrict__ ops, const __nv_bfloat16* __rest
 // buffered: T += C^T (c_hi + c_lo), G += Q^T (a_hi + a_lo) with C and Q exact
 // (bf16 inputs, MN-major A) and the scaled B rows split hi + lo:
 // c = g SiLU(z) dY, a = iq dl Ebar / sqrt(N) (Qbar's scale moved onto B).
-constexpr int kMemThreads = 256;
+constexpr int kMemThreads = 512;
 constexpr int kMT = 64;          // tokens per staged tile (K of one MMA chain: 4 steps)
 constexpr int kBlk = kMT * 128;  // one 64-column MN block of kMT rows
 
@@ -594,11 +617,18 @@ struct MemSmem {
     // per buffer: C^T, Q^T (two 64-row blocks of n each), then c_hi, c_lo, a_hi, a_lo
     // (one 64-column block per head each)
     uint8_t buf[2][6][2 * kBlk];
-    float sg[2][kMT];  // g SiLU(z) per head x and token
-    float sd[2][kMT];  // iq dl ie / sqrt(N) per head x and token
     uint64_t mma_done[2];
     uint64_t drain;
     uint32_t tmem_base;
+};
+
+// One tile's global data for one thread, prefetched into registers while the
+// previous tile's MMAs run: rows r = (tid >> 4) + 32 k of C and Q (16-byte
+// piece tid & 15), and row tid >> 3 of dY (both heads) and E (piece tid & 7)
+// with the per (token, head) factors of c and a.
+struct MemRegs {
+    uint4 cv[2], qv[2], dv[2], ev;
+    float fg[2], fd[2];
 };
 
 template <typename Tmem>
@@ -629,6 +659,29 @@ sma_bwd_mem_kernel(const Tmem* __restrict__ Mem, const float* __restrict__ rM,
         tc::tmem_alloc(&sm.tmem_base, 256);
         tc::tmem_relinquish();
     }
+    const int cr = tid >> 4, cq = tid & 15;  // C / Q rows cr, cr + 32; piece cq
+    const int er = tid >> 3, eq = tid & 7;   // dY / E row er; piece eq
+    MemRegs nx;
+    auto prefetch = [&](int it) {
+        const i64 tok0 = (i64)b * L + first + it * kMT;
+#pragma unroll
+        for (int k = 0; k < 2; ++k) {
+            nx.cv[k] = reinterpret_cast<const uint4*>(Cm + (tok0 + cr + 32 * k) * kN)[cq];
+            nx.qv[k] = reinterpret_cast<const uint4*>(Q + (tok0 + cr + 32 * k) * kN)[cq];
+        }
+        const i64 tok = tok0 + er;
+        const float2 q = rs[tok];
+#pragma unroll
+        for (int x = 0; x < 2; ++x) {
+            const int h = 2 * hp + x;
+            nx.dv[x] = reinterpret_cast<const uint4*>(dY + (tok * H + h) * kP)[eq];
+            const i64 sidx = (((i64)b * H + h) * Mc + j) * L + first + it * kMT + er;
+            nx.fg[x] = gbuf[sidx] * silu_f32(__bfloat162float(z[tok * H + h]));
+            nx.fd[x] = dlbuf[sidx] * q.x * q.y * rsn;
+        }
+        nx.ev = reinterpret_cast<const uint4*>(E + tok * kP)[eq];
+    };
+    if (ntiles > 0) prefetch(0);
     tc::tc_fence_before();
     __syncthreads();
     tc::tc_fence_after();
@@ -639,64 +692,43 @@ sma_bwd_mem_kernel(const Tmem* __restrict__ Mem, const float* __restrict__ rM,
     int issued = 0;  // tiles whose MMAs were issued
     for (int it = 0; it < ntiles; ++it) {
         const int bi = it & 1;
-        const int tb = first + it * kMT;
-        const i64 tok0 = (i64)b * L + tb;
         // buffer bi was read by the MMAs of tile it - 2
         if (it >= 2) {
-            const bool got = tc::mbar_wait(&sm.mma_done[bi], (uint32_t)(((it - 2) >> 1) & 1), wait_limit_ns, nullptr);
-            if (!got) atomicCAS(&g_bwd_tc_status, 0, 31);
-            ok = __syncthreads_and(got ? 1 : 0) != 0;
+            ok = cta_and_wait(&sm.mma_done[bi], (uint32_t)(((it - 2) >> 1) & 1), wait_limit_ns, 31);
             if (!ok) break;
-            tc::tc_fence_after();
         }
-        // per (head, token) scalars
-        {
-            const int x = (tid >> 6) & 1, r = tid & 63;  // tid < 128: sg; 128 .. 255: sd
-            const int h = 2 * hp + x;
-            const i64 sidx = (((i64)b * H + h) * Mc + j) * L + tb + r;
-            if (tid < 128) {
-                sm.sg[x][r] = gbuf[sidx] * silu_f32(__bfloat162float(z[(tok0 + r) * H + h]));
-            } else {
-                const float2 q = rs[tok0 + r];
-                sm.sd[x][r] = dlbuf[sidx] * q.x * q.y * rsn;
-            }
-        }
-        __syncthreads();
         uint8_t* bc = sm.buf[bi][0];
         uint8_t* bq = sm.buf[bi][1];
         // C and Q rows: token r, columns n -> block n / 64, row r, bytes 2 (n % 64)
-        for (int i = tid; i < kMT * 16; i += kMemThreads) {
-            const int r = i >> 4, c = i & 15;
-            const uint32_t o = (uint32_t)(c >> 3) * kBlk + sw128((uint32_t)r, (uint32_t)(c & 7) * 16u);
-            *reinterpret_cast<uint4*>(bc + o) = reinterpret_cast<const uint4*>(Cm + (tok0 + r) * kN)[c];
-            *reinterpret_cast<uint4*>(bq + o) = reinterpret_cast<const uint4*>(Q + (tok0 + r) * kN)[c];
+#pragma unroll
+        for (int k = 0; k < 2; ++k) {
+            const uint32_t o = (uint32_t)(cq >> 3) * kBlk + sw128((uint32_t)(cr + 32 * k), (uint32_t)(cq & 7) * 16u);
+            *reinterpret_cast<uint4*>(bc + o) = nx.cv[k];
+            *reinterpret_cast<uint4*>(bq + o) = nx.qv[k];
         }
         // c and a rows split hi / lo: token r, head x, columns p -> block x, row r, bytes 2 p
-        for (int i = tid; i < 2 * kMT * 8; i += kMemThreads) {
-            const int x = i / (kMT * 8), r = (i >> 3) % kMT, c = i & 7;
-            const int h = 2 * hp + x;
-            const uint32_t o = (uint32_t)x * kBlk + sw128((uint32_t)r, (uint32_t)c * 16u);
-            const uint4 dv = reinterpret_cast<const uint4*>(dY + ((tok0 + r) * H + h) * kP)[c];
-            const uint4 ev = reinterpret_cast<const uint4*>(E + (tok0 + r) * kP)[c];
-            const float fg = sm.sg[x][r], fd = sm.sd[x][r];
-            const uint32_t dw[4] = {dv.x, dv.y, dv.z, dv.w}, ew[4] = {ev.x, ev.y, ev.z, ev.w};
-            uint32_t gh[4], gl[4], eh[4], el[4];
+        {
+            const uint32_t ew[4] = {nx.ev.x, nx.ev.y, nx.ev.z, nx.ev.w};
 #pragma unroll
-            for (int e = 0; e < 4; ++e) {
-                const float g0 = bf_lo(dw[e]) * fg, g1 = bf_hi(dw[e]) * fg;
-                const float e0 = bf_lo(ew[e]) * fd, e1 = bf_hi(ew[e]) * fd;
-                const __nv_bfloat162 gv = __floats2bfloat162_rn(g0, g1);
-                const __nv_bfloat162 evh = __floats2bfloat162_rn(e0, e1);
-                const float2 gf = __bfloat1622float2(gv), ef = __bfloat1622float2(evh);
-                gh[e] = *reinterpret_cast<const uint32_t*>(&gv);
-                eh[e] = *reinterpret_cast<const uint32_t*>(&evh);
-                gl[e] = pack_bf16(g0 - gf.x, g1 - gf.y);
-                el[e] = pack_bf16(e0 - ef.x, e1 - ef.y);
+            for (int x = 0; x < 2; ++x) {
+                const uint32_t o = (uint32_t)x * kBlk + sw128((uint32_t)er, (uint32_t)eq * 16u);
+                const uint32_t dw[4] = {nx.dv[x].x, nx.dv[x].y, nx.dv[x].z, nx.dv[x].w};
+                float gv[8], av[8];
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    gv[2 * e] = bf_lo(dw[e]) * nx.fg[x];
+                    gv[2 * e + 1] = bf_hi(dw[e]) * nx.fg[x];
+                    av[2 * e] = bf_lo(ew[e]) * nx.fd[x];
+                    av[2 * e + 1] = bf_hi(ew[e]) * nx.fd[x];
+                }
+                uint4 hi, lo;
+                split_bf16x8(gv, hi, lo);
+                *reinterpret_cast<uint4*>(sm.buf[bi][2] + o) = hi;
+                *reinterpret_cast<uint4*>(sm.buf[bi][3] + o) = lo;
+                split_bf16x8(av, hi, lo);
+                *reinterpret_cast<uint4*>(sm.buf[bi][4] + o) = hi;
+                *reinterpret_cast<uint4*>(sm.buf[bi][5] + o) = lo;
             }
-            *reinterpret_cast<uint4*>(sm.buf[bi][2] + o) = make_uint4(gh[0], gh[1], gh[2], gh[3]);
-            *reinterpret_cast<uint4*>(sm.buf[bi][3] + o) = make_uint4(gl[0], gl[1], gl[2], gl[3]);
-            *reinterpret_cast<uint4*>(sm.buf[bi][4] + o) = make_uint4(eh[0], eh[1], eh[2], eh[3]);
-            *reinterpret_cast<uint4*>(sm.buf[bi][5] + o) = make_uint4(el[0], el[1], el[2], el[3]);
         }
         tc::fence_proxy_async_shared();
         tc::tc_fence_before();
@@ -718,21 +750,20 @@ sma_bwd_mem_kernel(const Tmem* __restrict__ Mem, const float* __restrict__ rM,
             tc::mma_commit(&sm.mma_done[bi]);
         }
         issued = it + 1;
+        if (it + 1 < ntiles) prefetch(it + 1);  // lands while these MMAs run
     }
     // the last tile's MMAs (and with them every earlier one) are done
     if (ok && ntiles > 0) {
         const int last = ntiles - 1;
-        const bool got = tc::mbar_wait(&sm.mma_done[last & 1], (uint32_t)((last >> 1) & 1), wait_limit_ns, nullptr);
-        if (!got) atomicCAS(&g_bwd_tc_status, 0, 32);
-        ok = __syncthreads_and(got ? 1 : 0) != 0;
+        ok = cta_and_wait(&sm.mma_done[last & 1], (uint32_t)((last >> 1) & 1), wait_limit_ns, 32);
     }
     if (!ok && issued > 0 && tid == 0) {  // let the MMAs in flight finish before TMEM is freed
         tc::mma_commit(&sm.drain);
         if (!tc::mbar_wait(&sm.drain, 0, kDrainLimitNs, nullptr)) atomicCAS(&g_bwd_tc_status, 0, 33);
     }
     tc::tc_fence_after();
-    if (ok) {
-        // thread (n, x): row n of T and G for head 2 hp + x
+    if (ok && tid < 256) {
+        // thread (n, x): row n of T and G for head 2 hp + x, in 16-column sweeps
         const int n = tid & 127, x = tid >> 7;
         const int h = 2 * hp + x;
         const uint32_t lane_addr = (uint32_t)(32 * (warp & 3)) << 16;
@@ -740,32 +771,34 @@ sma_bwd_mem_kernel(const Tmem* __restrict__ Mem, const float* __restrict__ rM,
         const Tmem* Mj = Mem + (mbase * kN + n) * kP;
         float* dMj = dM + (mbase * kN + n) * kP;
         const float rn = rM[mbase * kN + n];
-        float tv[kP], gv[kP], mv[kP];
+        auto sweep = [&](int c, float (&tv)[16], float (&gv)[16], float (&mv)[16]) {
 #pragma unroll
-        for (int p = 0; p < kP; ++p) mv[p] = ld_f32(Mj + p);
-        if (ntiles > 0) {
+            for (int i = 0; i < 16; ++i) mv[i] = ld_f32(Mj + 16 * c + i);
+            if (ntiles > 0) {
+                tmem_ld16(tmem + lane_addr + (uint32_t)(kP * x + 16 * c), tv);
+                tmem_ld16(tmem + lane_addr + 128u + (uint32_t)(kP * x + 16 * c), gv);
+            } else {
 #pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                float v[16];
-                tmem_ld16(tmem + lane_addr + (uint32_t)(kP * x + 16 * c), v);
-#pragma unroll
-                for (int i = 0; i < 16; ++i) tv[16 * c + i] = v[i];
-                tmem_ld16(tmem + lane_addr + 128u + (uint32_t)(kP * x + 16 * c), v);
-#pragma unroll
-                for (int i = 0; i < 16; ++i) gv[16 * c + i] = v[i];
+                for (int i = 0; i < 16; ++i) { tv[i] = 0.0f; gv[i] = 0.0f; }
             }
-        } else {
-#pragma unroll
-            for (int p = 0; p < kP; ++p) { tv[p] = 0.0f; gv[p] = 0.0f; }
-        }
+        };
         float dr = 0.0f;
 #pragma unroll
-        for (int p = 0; p < kP; ++p) dr = fmaf(mv[p], gv[p], dr);
+        for (int c = 0; c < 4; ++c) {
+            float tv[16], gv[16], mv[16];
+            sweep(c, tv, gv, mv);
+#pragma unroll
+            for (int i = 0; i < 16; ++i) dr = fmaf(mv[i], gv[i], dr);
+        }
         const float c3 = dr * rn * rn * rn / (float)kP;
 #pragma unroll
-        for (int p = 0; p < kP; ++p) tv[p] = tv[p] + rn * gv[p] - c3 * mv[p];
-        store_row32(dMj, tv);
-        store_row32(dMj + 32, tv + 32);
+        for (int c = 0; c < 4; ++c) {
+            float tv[16], gv[16], mv[16];
+            sweep(c, tv, gv, mv);
+#pragma unroll
+            for (int i = 0; i < 16; ++i) tv[i] = tv[i] + rn * gv[i] - c3 * mv[i];
+            store_row16(dMj + 16 * c, tv);
+        }
     }
     tc::tc_fence_before();
     __syncthreads();
