@@ -610,25 +610,28 @@ sma_bwd_rows_kernel(const uint8_t* __restrict__ ops, const __nv_bfloat16* __rest
 // (bf16 inputs, MN-major A) and the scaled B rows split hi + lo:
 // c = g SiLU(z) dY, a = iq dl Ebar / sqrt(N) (Qbar's scale moved onto B).
 constexpr int kMemThreads = 512;
-constexpr int kMT = 64;          // tokens per staged tile (K of one MMA chain: 4 steps)
+constexpr int kMT = 32;          // tokens per staged tile (K of one MMA chain: 2 steps)
 constexpr int kBlk = kMT * 128;  // one 64-column MN block of kMT rows
+constexpr int kMemPerCta = 2;    // memories per CTA, sharing the staged C and Q rows
 
 struct MemSmem {
-    // per buffer: C^T, Q^T (two 64-row blocks of n each), then c_hi, c_lo, a_hi, a_lo
-    // (one 64-column block per head each)
-    uint8_t buf[2][6][2 * kBlk];
+    // per buffer: C^T, Q^T (two 64-row blocks of n each); per memory c_hi, c_lo, a_hi,
+    // a_lo (one 64-column block per head each)
+    uint8_t bc[2][2 * kBlk];
+    uint8_t bq[2][2 * kBlk];
+    uint8_t bm[2][kMemPerCta][4][2 * kBlk];
     uint64_t mma_done[2];
     uint64_t drain;
     uint32_t tmem_base;
 };
 
 // One tile's global data for one thread, prefetched into registers while the
-// previous tile's MMAs run: rows r = (tid >> 4) + 32 k of C and Q (16-byte
-// piece tid & 15), and row tid >> 3 of dY (both heads) and E (piece tid & 7)
-// with the per (token, head) factors of c and a.
+// previous tile's MMAs run: row tid >> 4 of C and Q (16-byte piece tid & 15),
+// and for head x = tid >> 8, row (tid >> 3) & 31: dY and E (piece tid & 7)
+// with the factors of c and a for both memories.
 struct MemRegs {
-    uint4 cv[2], qv[2], dv[2], ev;
-    float fg[2], fd[2];
+    uint4 cv, qv, dv, ev;
+    float fg[kMemPerCta], fd[kMemPerCta];
 };
 
 template <typename Tmem>
@@ -643,9 +646,10 @@ sma_bwd_mem_kernel(const Tmem* __restrict__ Mem, const float* __restrict__ rM,
     extern __shared__ uint8_t smem_raw[];
     MemSmem& sm = *reinterpret_cast<MemSmem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                               ~(uintptr_t)1023);
-    const int j = blockIdx.x, hp = blockIdx.y, b = blockIdx.z;
+    const int j0 = blockIdx.x * kMemPerCta, hp = blockIdx.y, b = blockIdx.z;
     const int tid = threadIdx.x, warp = tid >> 5;
-    const int first = (j + 1) * S;  // tokens of the later chunks
+    const int nm = min(kMemPerCta, Mc - j0);  // memories of this CTA
+    const int first = (j0 + 1) * S;           // tokens of the chunks after memory j0
     const int ntiles = (L - first) / kMT;
     const float rsn = rsqrtf((float)kN);
 
@@ -656,30 +660,32 @@ sma_bwd_mem_kernel(const Tmem* __restrict__ Mem, const float* __restrict__ rM,
         tc::fence_barrier_init();
     }
     if (warp == 0) {
-        tc::tmem_alloc(&sm.tmem_base, 256);
+        tc::tmem_alloc(&sm.tmem_base, 512);
         tc::tmem_relinquish();
     }
-    const int cr = tid >> 4, cq = tid & 15;  // C / Q rows cr, cr + 32; piece cq
-    const int er = tid >> 3, eq = tid & 7;   // dY / E row er; piece eq
+    const int cr = tid >> 4, cq = tid & 15;                      // C / Q row, piece
+    const int ex = tid >> 8, er = (tid >> 3) & 31, eq = tid & 7;  // head, dY / E row, piece
+    const int eh = 2 * hp + ex;
     MemRegs nx;
     auto prefetch = [&](int it) {
         const i64 tok0 = (i64)b * L + first + it * kMT;
-#pragma unroll
-        for (int k = 0; k < 2; ++k) {
-            nx.cv[k] = reinterpret_cast<const uint4*>(Cm + (tok0 + cr + 32 * k) * kN)[cq];
-            nx.qv[k] = reinterpret_cast<const uint4*>(Q + (tok0 + cr + 32 * k) * kN)[cq];
-        }
+        nx.cv = reinterpret_cast<const uint4*>(Cm + (tok0 + cr) * kN)[cq];
+        nx.qv = reinterpret_cast<const uint4*>(Q + (tok0 + cr) * kN)[cq];
         const i64 tok = tok0 + er;
         const float2 q = rs[tok];
-#pragma unroll
-        for (int x = 0; x < 2; ++x) {
-            const int h = 2 * hp + x;
-            nx.dv[x] = reinterpret_cast<const uint4*>(dY + (tok * H + h) * kP)[eq];
-            const i64 sidx = (((i64)b * H + h) * Mc + j) * L + first + it * kMT + er;
-            nx.fg[x] = gbuf[sidx] * silu_f32(__bfloat162float(z[tok * H + h]));
-            nx.fd[x] = dlbuf[sidx] * q.x * q.y * rsn;
-        }
+        nx.dv = reinterpret_cast<const uint4*>(dY + (tok * H + eh) * kP)[eq];
         nx.ev = reinterpret_cast<const uint4*>(E + tok * kP)[eq];
+        const float gate = silu_f32(__bfloat162float(z[tok * H + eh]));
+        const int t = first + it * kMT + er;  // position in the sequence
+#pragma unroll
+        for (int m = 0; m < kMemPerCta; ++m) {
+            const int j = j0 + m;
+            // memory j sees tokens of later chunks only (its factors are zero before)
+            const bool live = m < nm && t >= (j + 1) * S;
+            const i64 sidx = (((i64)b * H + eh) * Mc + j) * L + t;
+            nx.fg[m] = live ? gbuf[sidx] * gate : 0.0f;
+            nx.fd[m] = live ? dlbuf[sidx] * q.x * q.y * rsn : 0.0f;
+        }
     };
     if (ntiles > 0) prefetch(0);
     tc::tc_fence_before();
@@ -697,37 +703,34 @@ sma_bwd_mem_kernel(const Tmem* __restrict__ Mem, const float* __restrict__ rM,
             ok = cta_and_wait(&sm.mma_done[bi], (uint32_t)(((it - 2) >> 1) & 1), wait_limit_ns, 31);
             if (!ok) break;
         }
-        uint8_t* bc = sm.buf[bi][0];
-        uint8_t* bq = sm.buf[bi][1];
         // C and Q rows: token r, columns n -> block n / 64, row r, bytes 2 (n % 64)
-#pragma unroll
-        for (int k = 0; k < 2; ++k) {
-            const uint32_t o = (uint32_t)(cq >> 3) * kBlk + sw128((uint32_t)(cr + 32 * k), (uint32_t)(cq & 7) * 16u);
-            *reinterpret_cast<uint4*>(bc + o) = nx.cv[k];
-            *reinterpret_cast<uint4*>(bq + o) = nx.qv[k];
-        }
-        // c and a rows split hi / lo: token r, head x, columns p -> block x, row r, bytes 2 p
         {
+            const uint32_t o = (uint32_t)(cq >> 3) * kBlk + sw128((uint32_t)cr, (uint32_t)(cq & 7) * 16u);
+            *reinterpret_cast<uint4*>(sm.bc[bi] + o) = nx.cv;
+            *reinterpret_cast<uint4*>(sm.bq[bi] + o) = nx.qv;
+        }
+        // c and a rows split hi / lo: memory m, token r, head x, columns p -> block x, row r
+        {
+            const uint32_t o = (uint32_t)ex * kBlk + sw128((uint32_t)er, (uint32_t)eq * 16u);
+            const uint32_t dw[4] = {nx.dv.x, nx.dv.y, nx.dv.z, nx.dv.w};
             const uint32_t ew[4] = {nx.ev.x, nx.ev.y, nx.ev.z, nx.ev.w};
 #pragma unroll
-            for (int x = 0; x < 2; ++x) {
-                const uint32_t o = (uint32_t)x * kBlk + sw128((uint32_t)er, (uint32_t)eq * 16u);
-                const uint32_t dw[4] = {nx.dv[x].x, nx.dv[x].y, nx.dv[x].z, nx.dv[x].w};
+            for (int m = 0; m < kMemPerCta; ++m) {
                 float gv[8], av[8];
 #pragma unroll
                 for (int e = 0; e < 4; ++e) {
-                    gv[2 * e] = bf_lo(dw[e]) * nx.fg[x];
-                    gv[2 * e + 1] = bf_hi(dw[e]) * nx.fg[x];
-                    av[2 * e] = bf_lo(ew[e]) * nx.fd[x];
-                    av[2 * e + 1] = bf_hi(ew[e]) * nx.fd[x];
+                    gv[2 * e] = bf_lo(dw[e]) * nx.fg[m];
+                    gv[2 * e + 1] = bf_hi(dw[e]) * nx.fg[m];
+                    av[2 * e] = bf_lo(ew[e]) * nx.fd[m];
+                    av[2 * e + 1] = bf_hi(ew[e]) * nx.fd[m];
                 }
                 uint4 hi, lo;
                 split_bf16x8(gv, hi, lo);
-                *reinterpret_cast<uint4*>(sm.buf[bi][2] + o) = hi;
-                *reinterpret_cast<uint4*>(sm.buf[bi][3] + o) = lo;
+                *reinterpret_cast<uint4*>(sm.bm[bi][m][0] + o) = hi;
+                *reinterpret_cast<uint4*>(sm.bm[bi][m][1] + o) = lo;
                 split_bf16x8(av, hi, lo);
-                *reinterpret_cast<uint4*>(sm.buf[bi][4] + o) = hi;
-                *reinterpret_cast<uint4*>(sm.buf[bi][5] + o) = lo;
+                *reinterpret_cast<uint4*>(sm.bm[bi][m][2] + o) = hi;
+                *reinterpret_cast<uint4*>(sm.bm[bi][m][3] + o) = lo;
             }
         }
         tc::fence_proxy_async_shared();
@@ -735,18 +738,25 @@ sma_bwd_mem_kernel(const Tmem* __restrict__ Mem, const float* __restrict__ rM,
         __syncthreads();
         if (tid == 0) {
             tc::tc_fence_after();
-            for (int part = 0; part < 2; ++part)
-                for (int ks = 0; ks < kMT / 16; ++ks) {
-                    const uint32_t acc = (it > 0 || part > 0 || ks > 0) ? 1u : 0u;
-                    const uint64_t ac = tc::smem_desc_sw128(tc::smem_u32(bc) + 2048u * ks, (uint32_t)kBlk, 1024u);
-                    const uint64_t bgd = tc::smem_desc_sw128(tc::smem_u32(sm.buf[bi][2 + part]) + 2048u * ks,
-                                                             (uint32_t)kBlk, 1024u);
-                    mma_ss(tmem, ac, bgd, idM, acc);
-                    const uint64_t aq = tc::smem_desc_sw128(tc::smem_u32(bq) + 2048u * ks, (uint32_t)kBlk, 1024u);
-                    const uint64_t bdd = tc::smem_desc_sw128(tc::smem_u32(sm.buf[bi][4 + part]) + 2048u * ks,
-                                                             (uint32_t)kBlk, 1024u);
-                    mma_ss(tmem + 128u, aq, bdd, idM, acc);
-                }
+            const int tb = first + it * kMT;
+            for (int m = 0; m < nm; ++m) {
+                const int jfirst = (j0 + m + 1) * S;  // memory m's first token
+                if (tb < jfirst) continue;             // nothing of memory m in this tile
+                const bool fresh = tb == jfirst;       // its first tile starts the sums
+                const uint32_t d = tmem + 256u * (uint32_t)m;
+                for (int part = 0; part < 2; ++part)
+                    for (int ks = 0; ks < kMT / 16; ++ks) {
+                        const uint32_t acc = (!fresh || part > 0 || ks > 0) ? 1u : 0u;
+                        const uint64_t ac = tc::smem_desc_sw128(tc::smem_u32(sm.bc[bi]) + 2048u * ks, (uint32_t)kBlk, 1024u);
+                        const uint64_t bgd = tc::smem_desc_sw128(tc::smem_u32(sm.bm[bi][m][part]) + 2048u * ks,
+                                                                 (uint32_t)kBlk, 1024u);
+                        mma_ss(d, ac, bgd, idM, acc);
+                        const uint64_t aq = tc::smem_desc_sw128(tc::smem_u32(sm.bq[bi]) + 2048u * ks, (uint32_t)kBlk, 1024u);
+                        const uint64_t bdd = tc::smem_desc_sw128(tc::smem_u32(sm.bm[bi][m][2 + part]) + 2048u * ks,
+                                                                 (uint32_t)kBlk, 1024u);
+                        mma_ss(d + 128u, aq, bdd, idM, acc);
+                    }
+            }
             tc::mma_commit(&sm.mma_done[bi]);
         }
         issued = it + 1;
@@ -762,11 +772,14 @@ sma_bwd_mem_kernel(const Tmem* __restrict__ Mem, const float* __restrict__ rM,
         if (!tc::mbar_wait(&sm.drain, 0, kDrainLimitNs, nullptr)) atomicCAS(&g_bwd_tc_status, 0, 33);
     }
     tc::tc_fence_after();
-    if (ok && tid < 256) {
-        // thread (n, x): row n of T and G for head 2 hp + x, in 16-column sweeps
-        const int n = tid & 127, x = tid >> 7;
-        const int h = 2 * hp + x;
+    const int m = tid >> 8;
+    if (ok && m < nm) {
+        // thread (n, x, m): row n of T and G for head 2 hp + x of memory j0 + m
+        const int n = tid & 127, x = (tid >> 7) & 1;
+        const int j = j0 + m, h = 2 * hp + x;
+        const bool any = (j + 1) * S < L;  // the memory has later tokens
         const uint32_t lane_addr = (uint32_t)(32 * (warp & 3)) << 16;
+        const uint32_t col = 256u * (uint32_t)m + (uint32_t)(kP * x);
         const i64 mbase = ((i64)b * Mc + j) * H + h;
         const Tmem* Mj = Mem + (mbase * kN + n) * kP;
         float* dMj = dM + (mbase * kN + n) * kP;
@@ -774,9 +787,9 @@ sma_bwd_mem_kernel(const Tmem* __restrict__ Mem, const float* __restrict__ rM,
         auto sweep = [&](int c, float (&tv)[16], float (&gv)[16], float (&mv)[16]) {
 #pragma unroll
             for (int i = 0; i < 16; ++i) mv[i] = ld_f32(Mj + 16 * c + i);
-            if (ntiles > 0) {
-                tmem_ld16(tmem + lane_addr + (uint32_t)(kP * x + 16 * c), tv);
-                tmem_ld16(tmem + lane_addr + 128u + (uint32_t)(kP * x + 16 * c), gv);
+            if (any) {
+                tmem_ld16(tmem + lane_addr + col + (uint32_t)(16 * c), tv);
+                tmem_ld16(tmem + lane_addr + col + 128u + (uint32_t)(16 * c), gv);
             } else {
 #pragma unroll
                 for (int i = 0; i < 16; ++i) { tv[i] = 0.0f; gv[i] = 0.0f; }
@@ -805,7 +818,7 @@ sma_bwd_mem_kernel(const Tmem* __restrict__ Mem, const float* __restrict__ rM,
     if (warp == 0) {
         __syncwarp();
         tc::tc_fence_after();
-        tc::tmem_dealloc(tmem, 256);
+        tc::tmem_dealloc(tmem, 512);
     }
 }
 
@@ -863,7 +876,7 @@ cudaError_t launch_sma_backward_tc(const SmaBwdArgs& a, void* ws, unsigned long 
         auto k = sma_bwd_mem_kernel<Tmem>;
         if ((e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) != cudaSuccess)
             return e;
-        k<<<dim3(Mc, H / 2, Bsz), kMemThreads, smem, stream>>>(
+        k<<<dim3((Mc + kMemPerCta - 1) / kMemPerCta, H / 2, Bsz), kMemThreads, smem, stream>>>(
             (const Tmem*)a.M, rM, (const __nv_bfloat16*)a.Q, (const __nv_bfloat16*)a.Cm,
             (const __nv_bfloat16*)a.E, (const __nv_bfloat16*)a.z, (const __nv_bfloat16*)a.dY, gbuf, sdl,
             rs, a.dM, L, H, S, Mc, wait_limit_ns);
