@@ -109,3 +109,27 @@ def test_backward_single_chunk_has_no_sma_gradient():
     torch.cuda.synchronize()
     for t in (dM, dQ, dC, dE, dz):
         assert torch.count_nonzero(t).item() == 0
+
+
+@pytest.mark.parametrize("name", ["train_b8_l4k_s256", "train_b8_l4k_s128"])
+def test_training_step_full_size_on_one_batch(name):
+    """The training workload at full size (B8 H24 L4096), forward and layer backward
+    through the library exactly as the bench's training step runs them; the oracle
+    computes batch 0 (batches are independent) and every per-batch gradient is
+    compared there. dA sums over the batch, so it is checked on the small cases."""
+    w = WORKLOADS[name]
+    inp = prefill_inputs(w, with_grad=True)
+    X, Bm, Cm, Q, E, z, dY = (dev(inp[k], w.dtype) for k in ("X", "Bm", "Cm", "Q", "E", "z", "dY"))
+    dt, A = dev(inp["dt"], torch.float32), dev(inp["A"], torch.float32)
+    s, o = api.prefill_forward(X, dt, A, Bm, Cm, Q, E, z, w.chunk, w.eps)
+    gr = api.layer_backward(X, dt, A, Bm, Cm, Q, E, z, dY, s, o, w.chunk, w.eps)
+    torch.cuda.synchronize()
+    one = {k: inp[k][:1] for k in ("X", "dt", "Bm", "Cm", "Q", "E", "z", "dY")}
+    ref = oracle.backward(one["X"], one["dt"], inp["A"], one["Bm"], one["Cm"], one["Q"], one["E"],
+                          one["z"], one["dY"], w.chunk, w.eps)
+    got = [gr.dX, gr.ddt, None, gr.dB, gr.dC, gr.dQ, gr.dE, gr.dz]
+    names = ["dX", "ddt", "dA", "dB", "dC", "dQ", "dE", "dz"]
+    errs = {n: rel_err(host(g[:1]), r) for n, g, r in zip(names, got, ref) if g is not None}
+    print(name, {k: f"{v:.2e}" for k, v in errs.items()})
+    for n, err in errs.items():
+        assert err <= _tol(w), f"{n}: {err:.3e}"
