@@ -170,6 +170,19 @@ constexpr int kRegsLow = 64, kRegsHigh = 216;
 constexpr uint32_t kColU = 0, kColAcc = 256;  // U buffer b at kColU + 128 b (kDQ)
 constexpr int kSlotB = 2 * kN + 16;           // one staged 256-byte row, padded
 constexpr int kPairB = 5 * kPart;             // W_hi, W_lo, M16, M_hi, M_lo per (memory, head pair)
+// Each (b, tile) is split over kRowSplit CTAs by head pairs, so the uneven
+// per-tile work (nj memories) balances over more, smaller CTAs; the partial
+// dQ, dC, dE (linear in the head sums) are added into zeroed outputs.
+constexpr int kRowSplit = 2;
+
+// dst[0..15] += v[0..15] (16-byte aligned), four vector reductions.
+__device__ __forceinline__ void red_add16(float* dst, const float* v) {
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+        asm volatile("red.global.add.v4.f32 [%0], {%1, %2, %3, %4};" ::"l"(dst + 4 * q), "f"(v[4 * q]),
+                     "f"(v[4 * q + 1]), "f"(v[4 * q + 2]), "f"(v[4 * q + 3])
+                     : "memory");
+}
 
 struct RowsSmem {
     uint8_t q[2][kRows * 128];     // Q (raw bf16), K-major A of U: two 64-wide K blocks (kDQ)
@@ -203,12 +216,14 @@ sma_bwd_rows_kernel(const uint8_t* __restrict__ ops, const __nv_bfloat16* __rest
                                                 ~(uintptr_t)1023);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int tiles = L / kRows;
-    const int tt = tiles - 1 - (int)blockIdx.x / Bsz;  // heaviest tiles first
-    const int b = (int)blockIdx.x % Bsz;
+    const int split = (int)blockIdx.x % kRowSplit, rest = (int)blockIdx.x / kRowSplit;
+    const int tt = tiles - 1 - rest / Bsz;  // heaviest tiles first
+    const int b = rest % Bsz;
     const int t0 = tt * kRows;
     const int nj = t0 / S;  // memories seen by every token of the tile
     const int hpairs = H / 2;
-    const int njobs = hpairs * nj;  // job k = (head pair k / nj, memory k % nj)
+    const int hp_lo = split * hpairs / kRowSplit, hp_hi = (split + 1) * hpairs / kRowSplit;
+    const int njobs = (hp_hi - hp_lo) * nj;  // job k = (head pair hp_lo + k / nj, memory k % nj)
     volatile int* abort = &sm.abort;
 
     if (threadIdx.x == 0) {
@@ -242,7 +257,7 @@ sma_bwd_rows_kernel(const uint8_t* __restrict__ ops, const __nv_bfloat16* __rest
             int issued = 0;
             const int part0 = kDQ ? 0 : 3;  // W_hi, W_lo or M_hi, M_lo (contiguous)
             for (int k = 0; k < njobs; ++k) {
-                const int sb = k & 1, hp = k / nj, j = k % nj;
+                const int sb = k & 1, hp = hp_lo + k / nj, j = k % nj;
                 const uint32_t par = (uint32_t)((k >> 1) & 1) ^ 1u;
                 // stage 1 and the A buffers hold the prologue's row staging until a_ready
                 ok = (k != 1 || tc::mbar_wait(&sm.a_ready, 0, wait_limit_ns, abort)) &&
@@ -383,14 +398,14 @@ sma_bwd_rows_kernel(const uint8_t* __restrict__ ops, const __nv_bfloat16* __rest
         asm volatile("bar.sync 1, 256;" ::: "memory");  // lq visible; slots free for the A tiles
         if constexpr (kDQ) {
             lfac = sm.lq[row];
-            if (x == 0) rs[tok] = make_float2(lfac * sqrtf((float)kN), ie);
+            if (x == 0 && split == 0) rs[tok] = make_float2(lfac * sqrtf((float)kN), ie);
         }
 
         float de[kDQ ? kP : 1];  // dEbar partial over this warpgroup's heads
 #pragma unroll
         for (int i = 0; i < (kDQ ? kP : 1); ++i) de[i] = 0.0f;
         bool ok = true;
-        for (int hp = 0; hp < hpairs && ok && nj > 0; ++hp) {
+        for (int hp = hp_lo; hp < hp_hi && ok && nj > 0; ++hp) {
             const int h = 2 * hp + x;
             const i64 rowo = tok * H + h;
             const float gate = silu_f32(__bfloat162float(z[rowo]));
@@ -408,7 +423,7 @@ sma_bwd_rows_kernel(const uint8_t* __restrict__ ops, const __nv_bfloat16* __rest
             const i64 sidx = ((i64)b * H + h) * Mc * L + t;  // + j L
             float g_next = gbuf[sidx], s_next = kDQ ? sdl[sidx] : 0.0f;  // s (!kDQ writes it)
             for (int j = 0; j < nj; ++j) {
-                const int k = hp * nj + j, ub = k & 1;
+                const int k = (hp - hp_lo) * nj + j, ub = k & 1;
                 const float gw = g_next, sv = s_next;
                 if (j + 1 < nj) {
                     g_next = gbuf[sidx + (i64)(j + 1) * L];
@@ -491,7 +506,7 @@ sma_bwd_rows_kernel(const uint8_t* __restrict__ ops, const __nv_bfloat16* __rest
             }
         }
         if (!kDQ && nj == 0) {  // no history: the gate's gradient is zero
-            for (int hp = 0; hp < hpairs; ++hp) dz[tok * H + 2 * hp + x] = 0.0f;
+            for (int hp = hp_lo; hp < hp_hi; ++hp) dz[tok * H + 2 * hp + x] = 0.0f;
         }
         if (ok && nj > 0 && !warp_wait(&sm.done, 0, wait_limit_ns, abort)) {
             fail(abort, 28);
@@ -499,7 +514,7 @@ sma_bwd_rows_kernel(const uint8_t* __restrict__ ops, const __nv_bfloat16* __rest
         }
         tc::tc_fence_after();
         ok = epi_and(ok);  // every epilogue thread takes the same branch below (named barriers)
-        if (ok) {
+        if (ok && nj > 0) {  // (no history: the zeroed outputs stay zero)
             const i64 grow = tok;  // G = 1: one group row per token
             if constexpr (!kDQ) {
                 // dC over this warpgroup's 64 columns
@@ -512,7 +527,7 @@ sma_bwd_rows_kernel(const uint8_t* __restrict__ ops, const __nv_bfloat16* __rest
 #pragma unroll
                         for (int i = 0; i < 16; ++i) v[i] = 0.0f;
                     }
-                    store_row16(dQC + grow * kN + kP * x + 16 * c, v);
+                    red_add16(dQC + grow * kN + kP * x + 16 * c, v);
                 }
             } else {
                 // dQ = iq (dQbar - Qbar (Qbar . dQbar) / N) over this warpgroup's 64 columns,
@@ -559,7 +574,7 @@ sma_bwd_rows_kernel(const uint8_t* __restrict__ ops, const __nv_bfloat16* __rest
                     qbar16(c, qb);
 #pragma unroll
                     for (int i = 0; i < 16; ++i) v[i] = iq * (v[i] - qb[i] * qdq);
-                    store_row16(dQC + grow * kN + kP * x + 16 * c, v);
+                    red_add16(dQC + grow * kN + kP * x + 16 * c, v);
                 }
                 // dE = ie (dEbar - Ebar (Ebar . dEbar) / P), the two warpgroups' partials
                 // summed through the (now idle) stage buffers
@@ -588,8 +603,8 @@ sma_bwd_rows_kernel(const uint8_t* __restrict__ ops, const __nv_bfloat16* __rest
                         de[2 * i] = ie * (de[2 * i] - bf_lo(ew[i]) * ie * ed);
                         de[2 * i + 1] = ie * (de[2 * i + 1] - bf_hi(ew[i]) * ie * ed);
                     }
-                    store_row32(dE + grow * kP, de);
-                    store_row32(dE + grow * kP + 32, de + 32);
+#pragma unroll
+                    for (int c = 0; c < 4; ++c) red_add16(dE + grow * kP + 16 * c, de + 16 * c);
                 }
             }
         }
@@ -859,12 +874,17 @@ cudaError_t launch_sma_backward_tc(const SmaBwdArgs& a, void* ws, unsigned long 
     }
     e = launch_sma_bwd_stats_tc<Tmem>(a, rM, ops, kPairB, scale, gbuf, gd, wait_limit_ns, stream);
     if (e != cudaSuccess) return e;
+    // the row kernels add their head-pair halves into these
+    const size_t rows = (size_t)(a.B * a.L);
+    if ((e = cudaMemsetAsync(a.dQ, 0, rows * kN * sizeof(float), stream)) != cudaSuccess) return e;
+    if ((e = cudaMemsetAsync(a.dC, 0, rows * kN * sizeof(float), stream)) != cudaSuccess) return e;
+    if ((e = cudaMemsetAsync(a.dE, 0, rows * kP * sizeof(float), stream)) != cudaSuccess) return e;
     const size_t smem_rows = sizeof(RowsSmem) + 1024;
     for (int pass = 0; pass < 2; ++pass) {  // dC, s, D, dz first; then dQ, dE, dl
         auto k = pass == 0 ? sma_bwd_rows_kernel<false> : sma_bwd_rows_kernel<true>;
         if ((e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_rows)) != cudaSuccess)
             return e;
-        k<<<Bsz * (L / kRows), kRowsThreads, smem_rows, stream>>>(
+        k<<<Bsz * (L / kRows) * kRowSplit, kRowsThreads, smem_rows, stream>>>(
             ops, (const __nv_bfloat16*)a.Q, (const __nv_bfloat16*)a.E, (const __nv_bfloat16*)a.z,
             (const __nv_bfloat16*)a.dY, gbuf, sdl, gd, rs, pass == 0 ? a.dC : a.dQ, a.dE, a.dz,
             (const __nv_bfloat16*)a.Cm, Bsz, L, H, S, Mc, a.eps, wait_limit_ns);
