@@ -532,6 +532,126 @@ dcdb_kernel(const __nv_bfloat16* __restrict__ X, const float* __restrict__ dt,
     }
 }
 
+// ------------------------------------------------------------- passing
+// Reverse pass over the chunks for one (1024-element slab of the N x P state,
+// h, b): with adj the adjoint of H_c (zero after the last chunk),
+//   d(dH_c) = adj + dM_c   (written as split operand tiles),
+//   d(cum_end_c) += exp(cum_end_c) <adj, H_[c-1]>,
+//   adj <- exp(cum_end_c) adj + Z_c.
+// The slabs of Z, dM and H_[c-1] stream through a ring of shared-memory
+// stages filled by 4 KiB bulk copies, chunks in reverse order.
+constexpr int kBpThreads = 256;
+constexpr int kBpElems = 4;
+constexpr int kBpSlab = kBpThreads * kBpElems;  // 1024 elements
+constexpr int kBpStages = 6;
+
+struct BpSmem {
+    float z[kBpStages][kBpSlab];
+    float m[kBpStages][kBpSlab];
+    float hp[kBpStages][kBpSlab];
+    float red[kBpThreads / 32];
+    uint64_t full[kBpStages];
+};
+
+__global__ void __launch_bounds__(kBpThreads)
+bwd_passing_tc_kernel(const float* __restrict__ Z, const float* __restrict__ dM,
+                      const float* __restrict__ Hprev, const float* __restrict__ cum,
+                      float* __restrict__ dcum_end, uint8_t* __restrict__ Dops, int H, int S, int Mc,
+                      unsigned long long wait_limit_ns) {
+    extern __shared__ uint8_t smem_raw[];
+    BpSmem& sm = *reinterpret_cast<BpSmem*>((reinterpret_cast<uintptr_t>(smem_raw) + 127) & ~(uintptr_t)127);
+    constexpr int NP = kN * kP;
+    const int slab = blockIdx.x, h = blockIdx.y, b = blockIdx.z, tid = threadIdx.x;
+    const int lane = tid & 31, warp = tid >> 5;
+    const int e0 = slab * kBpSlab + tid * kBpElems;
+    const int n = e0 / kP, p = e0 % kP;
+    const i64 cstride = (i64)H * NP;
+    const i64 base = ((i64)b * Mc * H + h) * NP + (i64)slab * kBpSlab;  // + c cstride
+    uint8_t* dop = Dops + ((i64)b * Mc * H + h) * 32768 + sw128((uint32_t)n, (uint32_t)p * 2u);
+    const i64 dstride = (i64)H * 32768;
+    const float* cumh = cum + ((i64)b * H + h) * (i64)Mc * S;
+    const uint32_t bytes = (uint32_t)(kBpSlab * 4) * (dM != nullptr ? 3u : 2u);
+
+    if (tid == 0) {
+        for (int k = 0; k < kBpStages; ++k) tc::mbar_init(&sm.full[k], 1);
+        tc::fence_barrier_init();
+    }
+    __syncthreads();
+    int issued = 0;  // reverse-order steps whose copies thread 0 issued
+    auto issue = [&](int k) {  // step k = chunk Mc - 1 - k
+        const int c = Mc - 1 - k, stg = k % kBpStages;
+        const i64 off = base + (i64)c * cstride;
+        tc::mbar_arrive_expect_tx(&sm.full[stg], bytes);
+        tc::bulk_g2s(sm.z[stg], Z + off, (uint32_t)(kBpSlab * 4), &sm.full[stg]);
+        tc::bulk_g2s(sm.hp[stg], Hprev + off, (uint32_t)(kBpSlab * 4), &sm.full[stg]);
+        if (dM != nullptr) tc::bulk_g2s(sm.m[stg], dM + off, (uint32_t)(kBpSlab * 4), &sm.full[stg]);
+        ++issued;
+    };
+    if (tid == 0)
+        for (int k = 0; k < min(kBpStages, Mc); ++k) issue(k);
+    float adj[kBpElems] = {0.0f, 0.0f, 0.0f, 0.0f};
+    bool ok = true;
+    int k = 0;
+    for (; k < Mc; ++k) {
+        const int c = Mc - 1 - k, stg = k % kBpStages;
+        const bool got = tc::mbar_wait(&sm.full[stg], (uint32_t)((k / kBpStages) & 1), wait_limit_ns, nullptr);
+        float part = 0.0f;
+        if (got) {
+            const float dec = expf(cumh[(i64)c * S + S - 1]);
+            const float4 zv = *reinterpret_cast<const float4*>(&sm.z[stg][tid * kBpElems]);
+            const float4 hv = *reinterpret_cast<const float4*>(&sm.hp[stg][tid * kBpElems]);
+            float4 mv = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+            if (dM != nullptr) mv = *reinterpret_cast<const float4*>(&sm.m[stg][tid * kBpElems]);
+            const float zz[4] = {zv.x, zv.y, zv.z, zv.w}, hh[4] = {hv.x, hv.y, hv.z, hv.w};
+            const float mm[4] = {mv.x, mv.y, mv.z, mv.w};
+            float dd[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                part = fmaf(dec * adj[i], hh[i], part);
+                dd[i] = adj[i] + mm[i];
+                adj[i] = fmaf(dec, adj[i], zz[i]);
+            }
+            uint4 hi, lo;
+            {
+                uint32_t hw[2], lw[2];
+#pragma unroll
+                for (int e = 0; e < 2; ++e) {
+                    const __nv_bfloat162 h2 = __floats2bfloat162_rn(dd[2 * e], dd[2 * e + 1]);
+                    const float2 hf = __bfloat1622float2(h2);
+                    hw[e] = *reinterpret_cast<const uint32_t*>(&h2);
+                    lw[e] = pack_bf16(dd[2 * e] - hf.x, dd[2 * e + 1] - hf.y);
+                }
+                hi = make_uint4(hw[0], hw[1], 0, 0);
+                lo = make_uint4(lw[0], lw[1], 0, 0);
+            }
+            uint8_t* t = dop + (i64)c * dstride;
+            *reinterpret_cast<uint2*>(t) = make_uint2(hi.x, hi.y);
+            *reinterpret_cast<uint2*>(t + 16384) = make_uint2(lo.x, lo.y);
+        } else {
+            atomicCAS(&g_sbwd_tc_status, 0, 46);
+        }
+        for (int off = 16; off > 0; off >>= 1) part += __shfl_xor_sync(0xffffffffu, part, off);
+        if (lane == 0) sm.red[warp] = part;
+        // every thread has read the stage before it is refilled; the partial sums are in
+        ok = __syncthreads_and(got ? 1 : 0) != 0;
+        if (!ok) break;
+        if (tid == 0) {
+            float sum = 0.0f;
+            for (int w = 0; w < kBpThreads / 32; ++w) sum += sm.red[w];
+            atomicAdd(dcum_end + ((i64)b * H + h) * Mc + c, sum);
+            if (k + kBpStages < Mc) issue(k + kBpStages);
+        }
+        __syncthreads();  // red is reused by the next step
+    }
+    if (!ok && tid == 0) {  // the copies in flight land before the CTA exits
+        for (int kk = k; kk < issued; ++kk)
+            if (!tc::mbar_wait(&sm.full[kk % kBpStages], (uint32_t)((kk / kBpStages) & 1), kDrainLimitNs, nullptr)) {
+                atomicCAS(&g_sbwd_tc_status, 0, 47);
+                break;
+            }
+    }
+}
+
 // ------------------------------------------------------------- finalize
 // One CTA of S threads per (c, h, b): d(cum) of the chunk,
 //   d(cum_t) = phi_row_t + rowI_t - phi_col_t - kappa_t,  kappa_t = dt_t xi_t,
@@ -627,9 +747,15 @@ cudaError_t launch_chunk_scan_backward_tc(const ScanBwdArgs& a, void* ws,
         (e = cudaMemsetAsync(a.dC, 0, (size_t)(f.B * f.L) * kN * 4, stream)) != cudaSuccess)
         return e;
     if ((e = launch_scan_bwd_inter_tc(f, cum, a.dY, ZD, wait_limit_ns, stream)) != cudaSuccess) return e;
-    if ((e = launch_scan_bwd_passing(ZD, a.dM, Hprev, cum, dcum_end, Dops, B, H, S, Mc, NP, stream)) !=
-        cudaSuccess)
-        return e;
+    {
+        const size_t smem = sizeof(BpSmem) + 128;
+        if ((e = cudaFuncSetAttribute(bwd_passing_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                      (int)smem)) != cudaSuccess)
+            return e;
+        bwd_passing_tc_kernel<<<dim3(NP / kBpSlab, H, B), kBpThreads, smem, stream>>>(
+            ZD, a.dM, Hprev, cum, dcum_end, Dops, H, S, Mc, wait_limit_ns);
+        note_launches(1);
+    }
     if ((e = launch_scan_bwd_output_tc(f, cum, Hops, Dops, a.dY, rowI, a.dX, xi, wait_limit_ns,
                                        stream)) != cudaSuccess)
         return e;
