@@ -124,6 +124,9 @@ __device__ __forceinline__ bool commit_and_wait(uint64_t* bar, uint32_t parity,
 
 // ------------------------------------------------------------ chunk state
 constexpr int kStateThreads = 256;  // two threads per chunk row s and per memory row n
+// Heads per CTA of the chunk-state kernel (B^T in TMEM is shared by them): four,
+// so that batches of many chunks fill the SMs in more, shorter waves.
+constexpr int kStateHeads = 4;
 
 struct StateSmem {
     union {
@@ -157,7 +160,7 @@ chunk_state_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restri
     const int c = blockIdx.x, hg = blockIdx.y, b = blockIdx.z;
     const int tid = threadIdx.x, warp = tid >> 5;
     const int n = tid & (kN - 1), half = tid >> 7;  // memory row (TMEM lane) and column half
-    const int h0 = hg * kHeadsPerCta;
+    const int h0 = hg * kStateHeads;
     const int g = h0 / (H / G);
     const i64 tok0 = (i64)b * L + (i64)c * S;
     const uint32_t lane_addr = (uint32_t)(32 * (warp & 3)) << 16;
@@ -225,7 +228,7 @@ chunk_state_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restri
     constexpr uint32_t idesc = tc::idesc_f16(1, true, kN, kP);
     uint32_t phase = 0;
     bool ok = true;
-    for (int hh = 0; hh < kHeadsPerCta && ok; ++hh) {
+    for (int hh = 0; hh < kStateHeads && ok; ++hh) {
         const int h = h0 + hh;
         if (tid < S) sm.w[tid] = kZ ? expf(nx.cumv) : expf(nx.cend - nx.cumv) * nx.dtv;
         __syncthreads();
@@ -251,7 +254,7 @@ chunk_state_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restri
                 *reinterpret_cast<uint4*>(sm.wx[1] + o) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
             }
         }
-        if (hh + 1 < kHeadsPerCta) load_head(h + 1);  // lands while this head computes
+        if (hh + 1 < kStateHeads) load_head(h + 1);  // lands while this head computes
         tc::fence_proxy_async_shared();
         tc::tc_fence_before();
         __syncthreads();
@@ -794,7 +797,7 @@ cudaError_t launch_chunk_scan_tc(const ScanArgs& a, unsigned long long wait_limi
         const size_t smem = sizeof(StateSmem) + 1024;
         cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
-        kern<<<dim3(M, H / kHeadsPerCta, B), kStateThreads, smem, stream>>>(
+        kern<<<dim3(M, H / kStateHeads, B), kStateThreads, smem, stream>>>(
             (const __nv_bfloat16*)a.X, a.dt, a.cum, (const __nv_bfloat16*)a.Bm,
             mem_is_f32 ? nullptr : a.dH32, (Tmem*)a.M, a.rM, L, H, G, S, M, a.eps, wait_limit_ns);
     }
@@ -831,7 +834,7 @@ cudaError_t launch_scan_states_tc(const ScanArgs& a0, float* cum, float* Hprev, 
     const size_t smem = sizeof(StateSmem) + 1024;
     if ((e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) != cudaSuccess)
         return e;
-    kern<<<dim3(M, H / kHeadsPerCta, B), kStateThreads, smem, stream>>>(
+    kern<<<dim3(M, H / kStateHeads, B), kStateThreads, smem, stream>>>(
         (const __nv_bfloat16*)a.X, a.dt, a.cum, (const __nv_bfloat16*)a.Bm, nullptr, Hprev, nullptr,
         L, H, G, S, M, a.eps, wait_limit_ns);
     state_passing_tc_kernel<<<dim3(kN * kP / kSpSlab, H, B), kSpThreads, 0, stream>>>(
@@ -848,7 +851,7 @@ cudaError_t launch_scan_bwd_inter_tc(const ScanArgs& a, const float* cum, const 
     const size_t smem = sizeof(StateSmem) + 1024;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    kern<<<dim3(M, H / kHeadsPerCta, B), kStateThreads, smem, stream>>>(
+    kern<<<dim3(M, H / kStateHeads, B), kStateThreads, smem, stream>>>(
         (const __nv_bfloat16*)dY, a.dt, cum, (const __nv_bfloat16*)a.Cm, Z, nullptr, nullptr, L, H, G,
         S, M, a.eps, wait_limit_ns);
     note_launches(1);
