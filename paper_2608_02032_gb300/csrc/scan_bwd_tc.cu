@@ -332,11 +332,12 @@ psi_kernel(const __nv_bfloat16* __restrict__ X, const float* __restrict__ dt,
 }
 
 // ---------------------------------------------------------------- dC / dB
-constexpr int kDcThreads = 256;
+constexpr int kDcThreads = 512;
 constexpr int kUnit = 16384;  // one operand slot
 
 struct DcSmem {
     uint8_t slot[2][4][kUnit];  // per buffer: A hi, A lo, B (or B hi), B lo
+    uint64_t full[2];           // the unit's 32 KiB bulk-copied part landed in buffer 0 / 1
     uint64_t mma_done[2];
     uint64_t drain;
     uint32_t tmem_base;
@@ -366,8 +367,10 @@ dcdb_kernel(const __nv_bfloat16* __restrict__ X, const float* __restrict__ dt,
     const int nunits = nintra + ninter;
 
     if (tid == 0) {
-        tc::mbar_init(&sm.mma_done[0], 1);
-        tc::mbar_init(&sm.mma_done[1], 1);
+        for (int u = 0; u < 2; ++u) {
+            tc::mbar_init(&sm.full[u], 1);
+            tc::mbar_init(&sm.mma_done[u], 1);
+        }
         tc::mbar_init(&sm.drain, 1);
         tc::fence_barrier_init();
     }
@@ -382,7 +385,8 @@ dcdb_kernel(const __nv_bfloat16* __restrict__ X, const float* __restrict__ dt,
     const float* cumb = cum + (i64)b * H * Mc * S;  // + (h Mc + c) S + t
 
     bool ok = true;
-    int issued = 0;
+    int issued = 0;   // units whose MMAs were issued
+    int copied = 0;   // units whose bulk copy was issued (thread 0)
     for (int u = 0; u < nunits; ++u) {
         const int bi = u & 1;
         if (u >= 2) {
@@ -394,27 +398,34 @@ dcdb_kernel(const __nv_bfloat16* __restrict__ X, const float* __restrict__ dt,
         uint8_t* b0 = sm.slot[bi][2];
         uint8_t* b1 = sm.slot[bi][3];
         const bool intra = u < nintra;
-        if (intra) {
-            if (kind == 0) {
+        // Every unit has one 32 KiB part that is already laid out in global memory: the
+        // Psi blocks (intra) or the H / d(dH) operand tile (per head); bulk copies bring
+        // it in while the threads stage the rest.
+        if (tid == 0) {
+            tc::mbar_arrive_expect_tx(&sm.full[bi], 32768u);
+            if (!intra) {
+                const int h = u - nintra;
+                const uint8_t* tile = (kind == 0 ? Hops : Dops) + (((i64)b * Mc + c) * H + h) * 32768;
+                tc::bulk_g2s(b0, tile, 32768u, &sm.full[bi]);  // into b0 and b1
+            } else if (kind == 0) {
                 // A: Psi rows of the tile, column block u (K = 64 sources), K-major
-                for (int i = tid; i < 2 * kT * 8; i += kDcThreads) {
-                    const int part = i / (kT * 8), j = i % (kT * 8);
-                    const uint4 v = reinterpret_cast<const uint4*>(
-                        pbase + part * ppart + (i64)u * S * 128 + (i64)tt * kT * 128)[j];
-                    *reinterpret_cast<uint4*>((part ? a_lo : a_hi) + j * 16) = v;
-                }
+                for (int part = 0; part < 2; ++part)
+                    tc::bulk_g2s(part ? a_lo : a_hi,
+                                 pbase + part * ppart + (i64)u * S * 128 + (i64)tt * kT * 128,
+                                 (uint32_t)(kT * 128), &sm.full[bi]);
             } else {
                 // A: Psi^T, M = the tile's 128 sources (column blocks 2 tt, 2 tt + 1), K = 64
                 // target rows from tt * 128 + 64 u, MN-major: [block][64 rows][128 bytes]
                 const int t0u = tt * kT + 64 * u;
-                for (int i = tid; i < 2 * 2 * 64 * 8; i += kDcThreads) {
-                    const int part = i / (2 * 64 * 8), j = i % (2 * 64 * 8);
-                    const int blk = j / (64 * 8), jj = j % (64 * 8);
-                    const uint4 v = reinterpret_cast<const uint4*>(
-                        pbase + part * ppart + (i64)(2 * tt + blk) * S * 128 + (i64)t0u * 128)[jj];
-                    *reinterpret_cast<uint4*>((part ? a_lo : a_hi) + blk * 8192 + jj * 16) = v;
-                }
+                for (int part = 0; part < 2; ++part)
+                    for (int blk = 0; blk < 2; ++blk)
+                        tc::bulk_g2s((part ? a_lo : a_hi) + blk * 8192,
+                                     pbase + part * ppart + (i64)(2 * tt + blk) * S * 128 + (i64)t0u * 128,
+                                     8192u, &sm.full[bi]);
             }
+            copied = u + 1;
+        }
+        if (intra) {
             // B: 64 token rows of B (dC) or C (dB), MN-major N = 128: [n block][64 rows][128 bytes]
             const int r0 = kind == 0 ? 64 * u : tt * kT + 64 * u;
             const __nv_bfloat16* src = kind == 0 ? Bm : Cm;
@@ -454,15 +465,16 @@ dcdb_kernel(const __nv_bfloat16* __restrict__ X, const float* __restrict__ dt,
                 *reinterpret_cast<uint4*>(a_hi + o) = hi;
                 *reinterpret_cast<uint4*>(a_lo + o) = lo;
             }
-            // B: H_[c-1] (dC) or d(dH_c) (dB) of head h, [n][p] hi | lo: K-major (rows n, K = p)
-            const uint8_t* tile = (kind == 0 ? Hops : Dops) + (((i64)b * Mc + c) * H + h) * 32768;
-            for (int i = tid; i < 2048; i += kDcThreads)
-                *reinterpret_cast<uint4*>(b0 + i * 16) = reinterpret_cast<const uint4*>(tile)[i];
+            // B: H_[c-1] (dC) or d(dH_c) (dB) of head h, [n][p] hi | lo, K-major (rows n,
+            // K = p): the bulk copy above
         }
         tc::fence_proxy_async_shared();
         tc::tc_fence_before();
         __syncthreads();
-        if (tid == 0) {
+        if (tid == 0 && !tc::mbar_wait(&sm.full[bi], (uint32_t)((u >> 1) & 1), wait_limit_ns, nullptr)) {
+            // no MMA for this unit: the next wait on its mma_done runs out and ends the loop
+            atomicCAS(&g_sbwd_tc_status, 0, 46);
+        } else if (tid == 0) {
             tc::tc_fence_after();
             const uint32_t sa_hi = tc::smem_u32(a_hi), sa_lo = tc::smem_u32(a_lo);
             const uint32_t sb0 = tc::smem_u32(b0), sb1 = tc::smem_u32(b1);
@@ -501,17 +513,22 @@ dcdb_kernel(const __nv_bfloat16* __restrict__ X, const float* __restrict__ dt,
         tc::mma_commit(&sm.drain);
         if (!tc::mbar_wait(&sm.drain, 0, kDrainLimitNs, nullptr)) atomicCAS(&g_sbwd_tc_status, 0, 45);
     }
+    if (tid == 0) {  // never leave a copy in flight behind: the last copy into each buffer
+        for (int k = copied - 1; k >= 0 && k >= copied - 2; --k)
+            if (!tc::mbar_wait(&sm.full[k & 1], (uint32_t)((k >> 1) & 1), kDrainLimitNs, nullptr))
+                atomicCAS(&g_sbwd_tc_status, 0, 47);
+    }
     tc::tc_fence_after();
     if (ok) {
-        // thread (row, half): 64 columns of its token row
-        const int r = tid & (kT - 1), half = tid >> 7;
+        // thread (row, quarter): 32 columns of its token row
+        const int r = tid & (kT - 1), qc = tid >> 7;
         const uint32_t lane_addr = (uint32_t)(32 * (warp & 3)) << 16;
         const i64 tok = tok0 + tt * kT + r;
-        float* dst = (kind == 0 ? dC : dB) + tok * kN + 64 * half;
-        for (int cc = 0; cc < 2; ++cc) {
+        float* dst = (kind == 0 ? dC : dB) + tok * kN + 32 * qc;
+        {
             float v[32];
-            tmem_ld32(tmem + lane_addr + (uint32_t)(64 * half + 32 * cc), v);
-            float4* d4 = reinterpret_cast<float4*>(dst + 32 * cc);
+            tmem_ld32(tmem + lane_addr + (uint32_t)(32 * qc), v);
+            float4* d4 = reinterpret_cast<float4*>(dst);
 #pragma unroll
             for (int q = 0; q < 8; ++q) {
                 float4 o = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);

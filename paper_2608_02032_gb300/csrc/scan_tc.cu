@@ -46,7 +46,11 @@ __device__ int g_scan_tc_status;  // first timeout code since the last read (0 =
 constexpr int kP = 64;
 constexpr int kN = 128;
 constexpr int kT = 128;  // tokens per output tile
+// The tensor-core scan wants H and H / G to be multiples of 8. The output kernel
+// takes a runtime number of heads per CTA (a divisor of H / G, at most
+// kMaxOutHeads) chosen on the host so that its CTAs fill the SMs in few waves.
 constexpr int kHeadsPerCta = 8;
+constexpr int kMaxOutHeads = 16;
 constexpr uint64_t kDrainLimitNs = 2000000000ull;
 constexpr float kLog2e = 1.4426950408889634f;
 
@@ -429,7 +433,7 @@ struct OutSmem {
     float bnorm[256];              // |B_s| of the sources
     float cnorm[kT];               // |C_t| of the tile's rows
     uint32_t bdmax[2];             // max_s |B_s| dt_s of a head (float bits), by head parity
-    float dacc[8][kT][2];          // backward modes: per (head, row) dot product
+    float dacc[kMaxOutHeads][kT][2];  // backward modes: per (head, row) dot product
     uint64_t bar;
     uint64_t hbar[2];              // H_[c-1] tile copy into buffer 0 / 1 landed
     uint32_t tmem_base;
@@ -464,19 +468,19 @@ __global__ void __launch_bounds__(kOutThreads, 1)
 chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restrict__ dt,
                        const float* __restrict__ cum, const __nv_bfloat16* __restrict__ Bm,
                        const __nv_bfloat16* __restrict__ Cm, const uint8_t* __restrict__ Hops,
-                       Tout* __restrict__ Y, int L, int H, int G, int S, int Mc,
+                       Tout* __restrict__ Y, int L, int H, int G, int S, int Mc, int hpc,
                        unsigned long long wait_limit_ns,
                        const __nv_bfloat16* __restrict__ Zd = nullptr, float* __restrict__ dots = nullptr) {
     extern __shared__ uint8_t smem_raw[];
     OutSmem& sm = *reinterpret_cast<OutSmem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                               ~(uintptr_t)1023);
     const int tt = blockIdx.x;  // tile inside the chunk
-    const int c = blockIdx.y / (H / kHeadsPerCta);
-    const int hg = blockIdx.y % (H / kHeadsPerCta);
+    const int c = blockIdx.y / (H / hpc);
+    const int hg = blockIdx.y % (H / hpc);
     const int b = blockIdx.z;
     const int tid = threadIdx.x, warp = tid >> 5;
     const int row = tid & (kT - 1), quarter = tid >> 7;  // token row, quarter of the sources / columns
-    const int h0 = hg * kHeadsPerCta;
+    const int h0 = hg * hpc;
     const int g = h0 / (H / G);
     const int ns = (tt + 1) * kT;  // sources 0 .. ns-1 of the chunk
     const i64 tok0 = (i64)b * L + (i64)c * S;
@@ -487,7 +491,7 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
     auto pos = [&](int k) { return kMode == kOutRev ? S - 1 - k : k; };
     constexpr bool kIntra = kMode != kOutDot;
     if (kMode != kOutY)
-        for (int i = tid; i < kHeadsPerCta * kT * 2; i += kOutThreads) (&sm.dacc[0][0][0])[i] = 0.0f;
+        for (int i = tid; i < hpc * kT * 2; i += kOutThreads) (&sm.dacc[0][0][0])[i] = 0.0f;
 
     if (tid == 0) {
         tc::mbar_init(&sm.bar, 1);
@@ -602,7 +606,7 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
     const i64 tok = tok0 + pos(tl);
     const int tl_warp_max = tt * kT + 32 * (warp & 3) + 31;
     const int s_lo = quarter * (ns / 4), s_hi = s_lo + ns / 4;  // 32 or 64 sources
-    for (int hh = 0; hh < kHeadsPerCta && ok; ++hh) {
+    for (int hh = 0; hh < hpc && ok; ++hh) {
         const int h = h0 + hh;
         // prefetched sources into shared memory (the previous head's MMAs are done)
 #pragma unroll
@@ -632,7 +636,7 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
         // sources ending at r; both factors are at most 1 (cum never rises) when r <= t
         if (tid < ns) sm.bfac[tid] = ex2_approx(sm.c2[tid | 31] - sm.e2[tid]);
         __syncthreads();
-        if (hh + 1 < kHeadsPerCta) {  // lands while this head computes
+        if (hh + 1 < hpc) {  // lands while this head computes
             load_head(h + 1);
             // buffer (hh + 1) & 1 was last read by head hh - 1's MMAs (or the scores), both done
             if (tid == 0 && has_prev) issue_h(hh + 1);
@@ -764,7 +768,7 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
     tc::tc_fence_before();
     __syncthreads();
     if (kMode != kOutY && ok) {  // the per (token, head) dots
-        for (int i = tid; i < kHeadsPerCta * kT; i += kOutThreads) {
+        for (int i = tid; i < hpc * kT; i += kOutThreads) {
             const int hh = i / kT, r = i % kT;
             const i64 tk = tok0 + pos(tt * kT + r);
             dots[tk * H + h0 + hh] = sm.dacc[hh][r][0];
@@ -778,6 +782,29 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
 }
 
 }  // namespace
+
+// Heads per CTA of the output kernel: the divisor d of H / G (d <= kMaxOutHeads)
+// with the least modelled time, waves x (prologue + d heads). The prologue
+// (scores, tile and source staging) costs about two heads' work.
+int out_heads_per_cta(int units, int H, int G) {
+    int dev = 0, nsm = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || nsm <= 0)
+        nsm = 1;
+    const int hg = H / G;
+    int best = kHeadsPerCta;
+    long long best_cost = -1;
+    for (int d = 1; d <= kMaxOutHeads && d <= hg; ++d) {
+        if (hg % d) continue;
+        const long long ctas = (long long)units * (H / d);
+        const long long cost = (ctas + nsm - 1) / nsm * (2 + d);
+        if (best_cost < 0 || cost < best_cost || (cost == best_cost && d > best)) {
+            best = d;
+            best_cost = cost;
+        }
+    }
+    return best;
+}
 
 bool scan_tc_supported(const ScanArgs& a) {
     return a.P == kP && a.N == kN && (a.S == 128 || a.S == 256) &&
@@ -810,10 +837,11 @@ cudaError_t launch_chunk_scan_tc(const ScanArgs& a, unsigned long long wait_limi
         const size_t smem = sizeof(OutSmem) + 1024;
         cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
-        kern<<<dim3(S / kT, M * (H / kHeadsPerCta), B), kOutThreads, smem, stream>>>(
+        const int hpc = out_heads_per_cta(S / kT * M * B, H, G);
+        kern<<<dim3(S / kT, M * (H / hpc), B), kOutThreads, smem, stream>>>(
             (const __nv_bfloat16*)a.X, a.dt, a.cum, (const __nv_bfloat16*)a.Bm,
-            (const __nv_bfloat16*)a.Cm, a.Hops, (Tout*)a.Y, L, H, G, S, M, wait_limit_ns, nullptr,
-            nullptr);
+            (const __nv_bfloat16*)a.Cm, a.Hops, (Tout*)a.Y, L, H, G, S, M, hpc, wait_limit_ns,
+            nullptr, nullptr);
     }
     note_launches(3);
     return cudaGetLastError();
@@ -869,14 +897,15 @@ cudaError_t launch_scan_bwd_output_tc(const ScanArgs& a, const float* cum, const
     const int B = (int)a.B, L = (int)a.L, H = (int)a.H, G = (int)a.G, S = (int)a.S, M = L / S;
     typedef __nv_bfloat16 bf;
     const size_t smem = sizeof(OutSmem) + 1024;
-    const dim3 grid(S / kT, M * (H / kHeadsPerCta), B);
+    const int hpc = out_heads_per_cta(S / kT * M * B, H, G);
+    const dim3 grid(S / kT, M * (H / hpc), B);
     {
         auto kern = chunk_output_tc_kernel<float, kOutDot>;
         cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
         kern<<<grid, kOutThreads, smem, stream>>>((const bf*)a.X, a.dt, cum, (const bf*)a.Bm,
                                                   (const bf*)a.Cm, Hops, nullptr, L, H, G, S, M,
-                                                  wait_limit_ns, (const bf*)dY, rowI);
+                                                  hpc, wait_limit_ns, (const bf*)dY, rowI);
     }
     {
         auto kern = chunk_output_tc_kernel<float, kOutRev>;
@@ -885,7 +914,7 @@ cudaError_t launch_scan_bwd_output_tc(const ScanArgs& a, const float* cum, const
         // sources X <- dY, B <- C, C <- B; the dots take X
         kern<<<grid, kOutThreads, smem, stream>>>((const bf*)dY, a.dt, cum, (const bf*)a.Cm,
                                                   (const bf*)a.Bm, Dops, dX, L, H, G, S, M,
-                                                  wait_limit_ns, (const bf*)a.X, xi);
+                                                  hpc, wait_limit_ns, (const bf*)a.X, xi);
     }
     note_launches(2);
     return cudaGetLastError();

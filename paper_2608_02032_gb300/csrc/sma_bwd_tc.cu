@@ -620,8 +620,8 @@ sma_bwd_rows_kernel(const uint8_t* __restrict__ ops, const __nv_bfloat16* __rest
 }
 
 // ---------------------------------------------------------- memory kernel
-// One CTA per (j, head pair, b), 64-token tiles of the later chunks, double
-// buffered: T += C^T (c_hi + c_lo), G += Q^T (a_hi + a_lo) with C and Q exact
+// One CTA per (two memories j, head pair, b), 32-token tiles of the later chunks,
+// double buffered: T += C^T (c_hi + c_lo), G += Q^T (a_hi + a_lo) with C and Q exact
 // (bf16 inputs, MN-major A) and the scaled B rows split hi + lo:
 // c = g SiLU(z) dY, a = iq dl Ebar / sqrt(N) (Qbar's scale moved onto B).
 constexpr int kMemThreads = 512;
@@ -661,7 +661,9 @@ sma_bwd_mem_kernel(const Tmem* __restrict__ Mem, const float* __restrict__ rM,
     extern __shared__ uint8_t smem_raw[];
     MemSmem& sm = *reinterpret_cast<MemSmem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                               ~(uintptr_t)1023);
-    const int j0 = blockIdx.x * kMemPerCta, hp = blockIdx.y, b = blockIdx.z;
+    // memory pairs in z, the slowest launch index: the heaviest (earliest) memories,
+    // whose later chunks hold the most tokens, start first
+    const int j0 = blockIdx.z * kMemPerCta, hp = blockIdx.x, b = blockIdx.y;
     const int tid = threadIdx.x, warp = tid >> 5;
     const int nm = min(kMemPerCta, Mc - j0);  // memories of this CTA
     const int first = (j0 + 1) * S;           // tokens of the chunks after memory j0
@@ -896,7 +898,7 @@ cudaError_t launch_sma_backward_tc(const SmaBwdArgs& a, void* ws, unsigned long 
         auto k = sma_bwd_mem_kernel<Tmem>;
         if ((e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) != cudaSuccess)
             return e;
-        k<<<dim3((Mc + kMemPerCta - 1) / kMemPerCta, H / 2, Bsz), kMemThreads, smem, stream>>>(
+        k<<<dim3(H / 2, Bsz, (Mc + kMemPerCta - 1) / kMemPerCta), kMemThreads, smem, stream>>>(
             (const Tmem*)a.M, rM, (const __nv_bfloat16*)a.Q, (const __nv_bfloat16*)a.Cm,
             (const __nv_bfloat16*)a.E, (const __nv_bfloat16*)a.z, (const __nv_bfloat16*)a.dY, gbuf, sdl,
             rs, a.dM, L, H, S, Mc, wait_limit_ns);
