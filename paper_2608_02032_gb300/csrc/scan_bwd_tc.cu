@@ -26,6 +26,7 @@
 #include "common.cuh"
 #include "kernels.h"
 #include "tc_ptx.cuh"
+#include "tma.cuh"
 
 namespace dart {
 namespace {
@@ -126,16 +127,18 @@ __host__ __device__ inline int64_t psi_chunk_bytes(int S) { return 2LL * S * S *
 constexpr int kPsiThreads = 512;
 
 struct PsiSmem {
-    uint8_t yt[kT * 128];         // dY rows of the tile: A (rows t, K = p), K-major
-    uint8_t xs[256 * 128];        // X rows of the sources: B (rows s, K = p), K-major
+    uint8_t yt[2][kT * 128];      // dY rows of the tile, heads h and h + 1: A (rows t, K = p), K-major
+    uint8_t xs[2][256 * 128];     // X rows of the sources: B (rows s, K = p), K-major
     uint8_t ct[2][kT * 128];      // kPhi: C rows of the tile, K-major A (two K blocks)
     uint8_t bs[2][256 * 128];     // kPhi: B rows of the sources, K-major B (two K blocks)
-    float c2[256];                // cum log2(e) of tokens 0 .. ns - 1
-    float e2[256];                // c2 - log2(dt): exp2(c2_t - e2_s) = L[t,s] dt_s
-    float bfac[256];              // exp2(c2_r - e2_s), r = last token of s's group of 32
+    float c2[2][256];             // cum log2(e) of tokens 0 .. ns - 1 (by head parity)
+    float e2[2][256];             // c2 - log2(dt): exp2(c2_t - e2_s) = L[t,s] dt_s
+    float bfac[2][256];           // exp2(c2_r - e2_s), r = last token of s's group of 32
     float rowacc[kT];             // kPhi: row sums of the head
     float colacc[256];            // kPhi: column sums of the head
-    uint64_t bar;
+    uint64_t full[2];             // a head's dY and X tiles landed in buffer 0 / 1
+    uint64_t mma[2];              // a head's score chain done (heads of parity 0 / 1)
+    uint64_t drain;
     uint32_t tmem_base;
 };
 
@@ -154,10 +157,14 @@ __device__ __forceinline__ float warp_colsum32(float (&v)[32], int lane) {
     return v[0];
 }
 
+// The heads' dY and X tiles arrive by TMA two heads ahead (double-buffered); in
+// the Psi mode the scores are double-buffered in TMEM too, so head h + 1's MMA
+// chain runs under head h's epilogue. cum and dt of head h + 1 are prefetched
+// into registers during head h.
 template <bool kPhi>
 __global__ void __launch_bounds__(kPsiThreads, 1)
-psi_kernel(const __nv_bfloat16* __restrict__ X, const float* __restrict__ dt,
-           const float* __restrict__ cum, const __nv_bfloat16* __restrict__ dY,
+psi_kernel(const __grid_constant__ CUtensorMap tm_X, const __grid_constant__ CUtensorMap tm_dY,
+           const float* __restrict__ dt, const float* __restrict__ cum,
            const __nv_bfloat16* __restrict__ Bm, const __nv_bfloat16* __restrict__ Cm,
            uint8_t* __restrict__ psi, float* __restrict__ phi_row, float* __restrict__ phi_col,
            int L, int H, int S, int Mc, unsigned long long wait_limit_ns) {
@@ -174,13 +181,20 @@ psi_kernel(const __nv_bfloat16* __restrict__ X, const float* __restrict__ dt,
     const int tl_warp_max = tt * kT + 32 * (warp & 3) + 31;
     const int sq = ns / 4, s_lo = quarter * sq;  // 32 or 64 sources of this thread
     constexpr uint32_t kColCB = 256;
+    const uint32_t head_bytes = (uint32_t)(kT + ns) * 128u;
 
     if (tid == 0) {
-        tc::mbar_init(&sm.bar, 1);
+        for (int u = 0; u < 2; ++u) {
+            tc::mbar_init(&sm.full[u], 1);
+            tc::mbar_init(&sm.mma[u], 1);
+        }
+        tc::mbar_init(&sm.drain, 1);
         tc::fence_barrier_init();
+        tc::tma_prefetch_map(&tm_X);
+        tc::tma_prefetch_map(&tm_dY);
     }
     if (warp == 0) {
-        tc::tmem_alloc(&sm.tmem_base, kPhi ? 512 : 256);
+        tc::tmem_alloc(&sm.tmem_base, 512);
         tc::tmem_relinquish();
     }
     if (kPhi) {
@@ -198,74 +212,115 @@ psi_kernel(const __nv_bfloat16* __restrict__ X, const float* __restrict__ dt,
         for (int i = tid; i < 256; i += kPsiThreads) sm.colacc[i] = 0.0f;
         tc::fence_proxy_async_shared();
     }
+    // cum and dt of head hh for source tid (tid < ns)
+    auto head_c2e2 = [&](int hh, float& c2v, float& e2v) {
+        c2v = cum[(((i64)b * H + hh) * Mc + c) * S + tid] * kLog2e;
+        e2v = c2v - log2f(dt[(tok0 + tid) * H + hh]);  // dt = 0 gives +inf: a zero weight
+    };
+    if (tid < ns) head_c2e2(0, sm.c2[0][tid], sm.e2[0][tid]);
     tc::tc_fence_before();
     __syncthreads();
     tc::tc_fence_after();
     const uint32_t tmem = sm.tmem_base;
-    if (kPhi && tid == 0) {  // C B^T of the tile, committed with the first head's scores
+
+    // thread 0: the dY rows of the tile and the X rows of the sources of head hh into
+    // buffer hh & 1 (boxes of 128 rows x 64 columns at column hh P)
+    auto issue_head = [&](int hh) {
+        const int hb = hh & 1;
+        tc::mbar_arrive_expect_tx(&sm.full[hb], head_bytes);
+        tc::tma_load_2d(sm.yt[hb], &tm_dY, hh * kP, (int)(tok0 + tt * kT), &sm.full[hb]);
+        for (int r0 = 0; r0 < ns; r0 += kT)
+            tc::tma_load_2d(sm.xs[hb] + r0 * 128, &tm_X, hh * kP, (int)(tok0 + r0), &sm.full[hb]);
+    };
+    // thread 0: scores dY X^T of head hh (its tiles landed) into TMEM, committed on mma[hh & 1]
+    auto issue_scores = [&](int hh) {
+        const int hb = hh & 1;
         const uint32_t id = idesc_bf16(false, false, kT, (uint32_t)ns);
-        for (int ks = 0; ks < kN / 16; ++ks) {
-            const uint64_t ad = tc::smem_desc_sw128(tc::smem_u32(sm.ct[ks / 4]) + 32u * (ks % 4), 16u, 1024u);
-            const uint64_t bd = tc::smem_desc_sw128(tc::smem_u32(sm.bs[ks / 4]) + 32u * (ks % 4), 16u, 1024u);
-            mma_ss(tmem + kColCB, ad, bd, id, ks > 0 ? 1u : 0u);
+        const uint32_t dcol = kPhi ? 0u : 256u * (uint32_t)hb;
+        for (int ks = 0; ks < kP / 16; ++ks) {
+            const uint64_t ad = tc::smem_desc_sw128(tc::smem_u32(sm.yt[hb]) + 32u * ks, 16u, 1024u);
+            const uint64_t bd = tc::smem_desc_sw128(tc::smem_u32(sm.xs[hb]) + 32u * ks, 16u, 1024u);
+            mma_ss(tmem + dcol, ad, bd, id, ks > 0 ? 1u : 0u);
+        }
+        tc::mma_commit(&sm.mma[hb]);
+    };
+    int copies = 0, mmas = 0;  // heads whose tiles / score chains thread 0 issued
+    if (tid == 0) {
+        for (int hh = 0; hh < H && hh < 2; ++hh) issue_head(hh);
+        copies = H < 2 ? H : 2;
+        if (kPhi) {  // C B^T of the tile, committed with the first head's scores
+            const uint32_t id = idesc_bf16(false, false, kT, (uint32_t)ns);
+            for (int ks = 0; ks < kN / 16; ++ks) {
+                const uint64_t ad = tc::smem_desc_sw128(tc::smem_u32(sm.ct[ks / 4]) + 32u * (ks % 4), 16u, 1024u);
+                const uint64_t bd = tc::smem_desc_sw128(tc::smem_u32(sm.bs[ks / 4]) + 32u * (ks % 4), 16u, 1024u);
+                mma_ss(tmem + kColCB, ad, bd, id, ks > 0 ? 1u : 0u);
+            }
+        }
+        if (H > 0) {
+            if (tc::mbar_wait(&sm.full[0], 0, wait_limit_ns, nullptr)) {
+                tc::tc_fence_after();
+                issue_scores(0);
+                mmas = 1;
+            } else {
+                atomicCAS(&g_sbwd_tc_status, 0, 48);  // the wait on mma[0] then runs out
+            }
         }
     }
     float acc[kPhi ? 1 : 64];
 #pragma unroll
     for (int i = 0; i < (kPhi ? 1 : 64); ++i) acc[i] = 0.0f;
-    uint32_t phase = 0;
     bool ok = true;
     for (int h = 0; h < H && ok; ++h) {
-        // the head's dY rows of the tile and X rows of the sources (the previous head's
-        // MMA and TMEM reads are done)
-        for (int i = tid; i < kT * 8; i += kPsiThreads) {
-            const int r = i / 8, q = i % 8;
-            *reinterpret_cast<uint4*>(sm.yt + sw128((uint32_t)r, (uint32_t)q * 16u)) =
-                reinterpret_cast<const uint4*>(dY + ((tok0 + tt * kT + r) * H + h) * kP)[q];
-        }
-        for (int i = tid; i < ns * 8; i += kPsiThreads) {
-            const int s = i / 8, q = i % 8;
-            *reinterpret_cast<uint4*>(sm.xs + sw128((uint32_t)s, (uint32_t)q * 16u)) =
-                reinterpret_cast<const uint4*>(X + ((tok0 + s) * H + h) * kP)[q];
-        }
-        if (tid < ns) {
-            const float c2 = cum[(((i64)b * H + h) * Mc + c) * S + tid] * kLog2e;
-            sm.c2[tid] = c2;
-            sm.e2[tid] = c2 - log2f(dt[(tok0 + tid) * H + h]);  // dt = 0 gives +inf: a zero weight
-        }
-        tc::fence_proxy_async_shared();
-        tc::tc_fence_before();
-        __syncthreads();
-        if (tid == 0) {
-            tc::tc_fence_after();
-            const uint32_t id = idesc_bf16(false, false, kT, (uint32_t)ns);
-            for (int ks = 0; ks < kP / 16; ++ks) {
-                const uint64_t ad = tc::smem_desc_sw128(tc::smem_u32(sm.yt) + 32u * ks, 16u, 1024u);
-                const uint64_t bd = tc::smem_desc_sw128(tc::smem_u32(sm.xs) + 32u * ks, 16u, 1024u);
-                mma_ss(tmem, ad, bd, id, ks > 0 ? 1u : 0u);
-            }
-            tc::mma_commit(&sm.bar);
-        }
-        if (tid < ns) sm.bfac[tid] = ex2_approx(sm.c2[tid | 31] - sm.e2[tid]);
-        ok = cta_wait(&sm.bar, phase, wait_limit_ns, 41);
-        phase ^= 1u;
+        const int hb = h & 1;
+        if (tid < ns) sm.bfac[hb][tid] = ex2_approx(sm.c2[hb][tid | 31] - sm.e2[hb][tid]);
+        float nc2 = 0.0f, ne2 = 0.0f;
+        if (h + 1 < H && tid < ns) head_c2e2(h + 1, nc2, ne2);
+        ok = cta_wait(&sm.mma[hb], (uint32_t)((h >> 1) & 1), wait_limit_ns, 41);
         if (!ok) break;
-        const float c2t = sm.c2[tl];
+        // head h + 1's cum and dt into the other slot (its head h - 1 values were last read
+        // before the previous closing barrier)
+        if (h + 1 < H && tid < ns) {
+            sm.c2[hb ^ 1][tid] = nc2;
+            sm.e2[hb ^ 1][tid] = ne2;
+        }
+        if (tid == 0) {
+            // buffer hb's tiles were read by head h's MMAs: head h + 2's go there
+            if (h + 2 < H) {
+                issue_head(h + 2);
+                ++copies;
+            }
+            // Psi mode: head h + 1's scores into the other TMEM buffer (last read by head
+            // h - 1's epilogue, finished at its closing barrier)
+            if (!kPhi && h + 1 < H) {
+                if (tc::mbar_wait(&sm.full[hb ^ 1], (uint32_t)(((h + 1) >> 1) & 1), wait_limit_ns, nullptr)) {
+                    tc::tc_fence_after();
+                    issue_scores(h + 1);
+                    ++mmas;
+                } else {
+                    atomicCAS(&g_sbwd_tc_status, 0, 48);
+                }
+            }
+        }
+        const uint32_t dcol = kPhi ? 0u : 256u * (uint32_t)hb;
+        const float* c2h = sm.c2[hb];
+        const float* e2h = sm.e2[hb];
+        const float* bfh = sm.bfac[hb];
+        const float c2t = c2h[tl];
         float rsum = 0.0f;
 #pragma unroll
         for (int g0 = 0; g0 < 64; g0 += 32) {
             const int s0 = s_lo + g0;
             if (g0 >= sq || s0 > tl_warp_max) continue;  // warp-uniform
             float v[32];
-            tmem_ld32(tmem + lane_addr + (uint32_t)s0, v);
+            tmem_ld32(tmem + lane_addr + dcol + (uint32_t)s0, v);
             // v <- L[t,s] dt_s scores[t,s] (zero for s > t)
             if (s0 + 31 <= tl) {  // the whole group at or before t: factored decay
-                const float a = ex2_approx(c2t - sm.c2[s0 + 31]);
+                const float a = ex2_approx(c2t - c2h[s0 + 31]);
 #pragma unroll
-                for (int i = 0; i < 32; ++i) v[i] *= sm.bfac[s0 + i] * a;
+                for (int i = 0; i < 32; ++i) v[i] *= bfh[s0 + i] * a;
             } else {
 #pragma unroll
-                for (int i = 0; i < 32; ++i) v[i] = s0 + i <= tl ? v[i] * ex2_approx(c2t - sm.e2[s0 + i]) : 0.0f;
+                for (int i = 0; i < 32; ++i) v[i] = s0 + i <= tl ? v[i] * ex2_approx(c2t - e2h[s0 + i]) : 0.0f;
             }
             if constexpr (kPhi) {
                 float w[32];
@@ -295,10 +350,26 @@ psi_kernel(const __nv_bfloat16* __restrict__ X, const float* __restrict__ dt,
             }
         }
         tc::tc_fence_before();
-        __syncthreads();  // shared tiles, sums and TMEM are reused by the next head
+        __syncthreads();  // TMEM reads, slots and sums of head h are done
+        if (kPhi && tid == 0 && h + 1 < H) {  // one TMEM score buffer: head h + 1 starts now
+            tc::tc_fence_after();
+            if (tc::mbar_wait(&sm.full[hb ^ 1], (uint32_t)(((h + 1) >> 1) & 1), wait_limit_ns, nullptr)) {
+                issue_scores(h + 1);
+                ++mmas;
+            } else {
+                atomicCAS(&g_sbwd_tc_status, 0, 48);
+            }
+        }
     }
-    if (!ok) {  // the MMA chain in flight finishes before TMEM is freed
-        if (!tc::mbar_wait(&sm.bar, phase ^ 1u, kDrainLimitNs, nullptr)) atomicCAS(&g_sbwd_tc_status, 0, 42);
+    if (tid == 0) {
+        // never free TMEM under an MMA nor leave a tile copy in flight behind
+        if (!ok && mmas > 0) {
+            tc::mma_commit(&sm.drain);
+            if (!tc::mbar_wait(&sm.drain, 0, kDrainLimitNs, nullptr)) atomicCAS(&g_sbwd_tc_status, 0, 42);
+        }
+        for (int k = copies - 1; k >= 0 && k >= copies - 2; --k)
+            if (!tc::mbar_wait(&sm.full[k & 1], (uint32_t)((k >> 1) & 1), kDrainLimitNs, nullptr))
+                atomicCAS(&g_sbwd_tc_status, 0, 49);
     }
     if (!kPhi && ok) {
         uint8_t* base = psi + (i64)(b * Mc + c) * psi_chunk_bytes(S);
@@ -327,7 +398,7 @@ psi_kernel(const __nv_bfloat16* __restrict__ X, const float* __restrict__ dt,
     if (warp == 0) {
         __syncwarp();
         tc::tc_fence_after();
-        tc::tmem_dealloc(tmem, kPhi ? 512 : 256);
+        tc::tmem_dealloc(tmem, 512);
     }
 }
 
@@ -777,14 +848,19 @@ cudaError_t launch_chunk_scan_backward_tc(const ScanBwdArgs& a, void* ws,
                                        stream)) != cudaSuccess)
         return e;
     if ((e = cudaMemsetAsync(phi_col, 0, (size_t)(f.B * f.L * f.H) * 4, stream)) != cudaSuccess) return e;
+    // X and dY as (B L) x (H P) bf16 matrices, copied in 128 x 64 boxes (one head's rows)
+    CUtensorMap tm_X, tm_dY;
+    if (!encode_bf16_rows_map(&tm_X, f.X, (uint64_t)(f.B * f.L), (uint64_t)(H * kP), (uint64_t)H * kP * 2, kT, kP) ||
+        !encode_bf16_rows_map(&tm_dY, a.dY, (uint64_t)(f.B * f.L), (uint64_t)(H * kP), (uint64_t)H * kP * 2, kT, kP))
+        return cudaErrorNotSupported;
     for (int phi = 0; phi < 2; ++phi) {
         const size_t smem = sizeof(PsiSmem) + 1024;
         auto k = phi ? psi_kernel<true> : psi_kernel<false>;
         if ((e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) != cudaSuccess)
             return e;
         k<<<dim3(S / kT, Mc, B), kPsiThreads, smem, stream>>>(
-            (const __nv_bfloat16*)f.X, f.dt, cum, (const __nv_bfloat16*)a.dY, (const __nv_bfloat16*)f.Bm,
-            (const __nv_bfloat16*)f.Cm, psi, phi_row, phi_col, L, H, S, Mc, wait_limit_ns);
+            tm_X, tm_dY, f.dt, cum, (const __nv_bfloat16*)f.Bm, (const __nv_bfloat16*)f.Cm, psi, phi_row,
+            phi_col, L, H, S, Mc, wait_limit_ns);
     }
     {
         const size_t smem = sizeof(DcSmem) + 1024;

@@ -98,6 +98,20 @@ __device__ __forceinline__ void bulk_g2s(void* smem_dst, const void* gmem_src, u
         : "memory");
 }
 
+// 2D tensor copy global -> shared of one box of the tensor map at (x, y) (x the
+// inner coordinate, in elements; x * element size a multiple of 16 bytes),
+// completion counted on bar. `map` is the address of a __grid_constant__ map.
+__device__ __forceinline__ void tma_load_2d(void* smem_dst, const void* map, int x, int y, uint64_t* bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes "
+        "[%0], [%1, {%2, %3}], [%4];"
+        ::"r"(smem_u32(smem_dst)), "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_u32(bar))
+        : "memory");
+}
+__device__ __forceinline__ void tma_prefetch_map(const void* map) {
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
+}
+
 // 1D bulk copy shared -> global in this thread's bulk group (same size and
 // alignment rules). Shared-memory writes made by ordinary stores must be
 // made visible to the async proxy first (fence_proxy_async_shared).
