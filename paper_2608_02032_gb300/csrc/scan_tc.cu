@@ -63,6 +63,20 @@ __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
     const __nv_bfloat162 v = __floats2bfloat162_rn(a, b);
     return *reinterpret_cast<const uint32_t*>(&v);
 }
+// Packed fp32 pairs (low half first) for the two-wide FMUL.
+__device__ __forceinline__ uint64_t f2_pack(float x, float y) {
+    uint64_t r;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(x), "f"(y));
+    return r;
+}
+__device__ __forceinline__ void f2_unpack(uint64_t v, float& x, float& y) {
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(x), "=f"(y) : "l"(v));
+}
+__device__ __forceinline__ uint64_t f2_mul(uint64_t a, uint64_t b) {
+    uint64_t d;
+    asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+    return d;
+}
 __device__ __forceinline__ uint32_t pack_f16(float a, float b) {
     const __half2 v = __floats2half2_rn(a, b);
     return *reinterpret_cast<const uint32_t*>(&v);
@@ -655,10 +669,13 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
                 for (int i = 0; i < 16; ++i) pk[i] = 0u;
             } else if (s0 + 31 <= tl) {  // the whole group is at or before t: factored decay
                 const float a = ex2_approx(c2t - sm.c2[s0 + 31]) * rscale;
+                const uint64_t a2 = f2_pack(a, a);
 #pragma unroll
-                for (int i = 0; i < 16; ++i) {
-                    const float2 bf = *reinterpret_cast<const float2*>(&sm.bfac[s0 + 2 * i]);
-                    pk[i] = pack_f16(v[2 * i] * bf.x * a, v[2 * i + 1] * bf.y * a);
+                for (int i = 0; i < 16; ++i) {  // packed pairs: (v bfac) a
+                    const uint64_t bf = *reinterpret_cast<const uint64_t*>(&sm.bfac[s0 + 2 * i]);
+                    float w0, w1;
+                    f2_unpack(f2_mul(f2_mul(f2_pack(v[2 * i], v[2 * i + 1]), bf), a2), w0, w1);
+                    pk[i] = pack_f16(w0, w1);
                 }
             } else {  // the group holding t: masked, one exp per element
 #pragma unroll
