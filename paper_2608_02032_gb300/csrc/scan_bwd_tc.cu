@@ -171,7 +171,8 @@ psi_kernel(const __grid_constant__ CUtensorMap tm_X, const __grid_constant__ CUt
     extern __shared__ uint8_t smem_raw[];
     PsiSmem& sm = *reinterpret_cast<PsiSmem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                               ~(uintptr_t)1023);
-    const int tt = blockIdx.x, c = blockIdx.y, b = blockIdx.z;
+    // the tile in z, the slowest launch index: tiles with the most sources start first
+    const int tt = (int)(gridDim.z - 1 - blockIdx.z), c = blockIdx.x, b = blockIdx.y;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int row = tid & (kT - 1), quarter = tid >> 7;
     const int ns = (tt + 1) * kT;
@@ -858,7 +859,7 @@ cudaError_t launch_chunk_scan_backward_tc(const ScanBwdArgs& a, void* ws,
         auto k = phi ? psi_kernel<true> : psi_kernel<false>;
         if ((e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) != cudaSuccess)
             return e;
-        k<<<dim3(S / kT, Mc, B), kPsiThreads, smem, stream>>>(
+        k<<<dim3(Mc, B, S / kT), kPsiThreads, smem, stream>>>(
             tm_X, tm_dY, f.dt, cum, (const __nv_bfloat16*)f.Bm, (const __nv_bfloat16*)f.Cm, psi, phi_row,
             phi_col, L, H, S, Mc, wait_limit_ns);
     }
