@@ -93,7 +93,8 @@ typedef enum {
     DART_OP_SMA_FORWARD = 1,
     DART_OP_DECODE_STEP = 2,
     DART_OP_SMA_BACKWARD = 3,
-    DART_OP_SCAN_BACKWARD = 4
+    DART_OP_SCAN_BACKWARD = 4,
+    DART_OP_PREFILL_HOST = 5
 } dart_op;
 
 /* Human-readable name of a status code (static storage, never NULL). */
@@ -149,6 +150,34 @@ dart_status dart_sma_forward(const dart_dims* dims, const void* M, const float* 
                              const void* Q, const void* Cm, const void* E, const void* z,
                              const void* Y_ssd, void* Y, void* R, float* lse, void* workspace,
                              size_t workspace_bytes, void* stream);
+
+/*
+ * The prefill of one block (dart_chunk_scan then dart_sma_forward) from
+ * host buffers to a host buffer, with the copies overlapped with the kernels.
+ * The heads are taken in groups of 8 when G = 1 and H is a larger multiple of
+ * 8 (one group otherwise): per group the X rows go to the device (a pitched
+ * copy), the scan and SMA kernels run on them, and the group's Y rows come
+ * back, on four streams of the library's own (copy in, two for the kernels
+ * taking the groups in turn, copy out), so that the copies run under the
+ * kernels and neighbouring groups' kernels share the SMs. The shared inputs
+ * (B, C, Q, E, dt, A, z) go first; the gather of a group's dt and gate logits
+ * runs on the device. Per head the result is that of the device entry points.
+ * Inputs:  X (Bsz, L, H, P), Bm, Cm, Q (Bsz, L, G, N), E (Bsz, L, G, P),
+ *          z (Bsz, L, H) in_dtype; dt (Bsz, L, H), A (H) fp32: HOST memory,
+ *          page-locked for the copies to overlap.
+ * Output:  Y (Bsz, L, H, P) out_dtype, HOST memory (page-locked), complete
+ *          once `stream` reaches the point where the call left it.
+ * Workspace: dart_workspace_size(dims, DART_OP_PREFILL_HOST) bytes of device
+ *          memory, 256-byte aligned: device copies of the inputs, each group's
+ *          Y_ssd, Y, memories and their r, and the scan and SMA workspaces.
+ * The call orders itself after the work already on `stream` and leaves
+ * `stream` waiting for its last copy. The four streams are created on the
+ * first call for the current device and kept for the process.
+ */
+dart_status dart_prefill_host(const dart_dims* dims, const void* X, const float* dt, const float* A,
+                              const void* Bm, const void* Cm, const void* Q, const void* E,
+                              const void* z, void* Y, void* workspace, size_t workspace_bytes,
+                              void* stream);
 
 /*
  * One decode step over the chunk-memory cache (the persistent inference

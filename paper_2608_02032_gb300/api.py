@@ -83,6 +83,28 @@ def prefill_forward(X, dt, A, Bm, Cm, Q, E, z, chunk: int, eps: float = 1e-6, wa
     return s, o
 
 
+def prefill_from_host(X, dt, A, Bm, Cm, Q, E, z, chunk: int, eps: float = 1e-6,
+                      out_dtype=torch.float32, Y=None, workspace=None, stream=None):
+    """The prefill (scan, SMA, merge) from host tensors to a host tensor
+    (``dart_prefill_host``): copies overlapped with the kernels, head group by head
+    group. Inputs should be page-locked (``pin_memory()``); ``Y`` (allocated
+    page-locked when not given) is complete once ``stream`` (default: the current
+    stream) is synchronised. ``workspace`` is device memory reused across calls.
+    Returns (Y, workspace)."""
+    Bsz, L, H, P = X.shape
+    G, N = Bm.shape[2], Bm.shape[3]
+    dims = B.make_dims(Bsz, L, H, G, P, N, chunk, _dtype_code(X), B.DART_F32, out_dtype, eps=eps)
+    if Y is None:
+        Y = torch.empty(Bsz, L, H, P, dtype=out_dtype).pin_memory()
+    if workspace is None:
+        workspace = torch.empty(B.dart_workspace_size(dims, B.DART_OP_PREFILL_HOST), dtype=torch.uint8,
+                                device="cuda")
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    B.dart_prefill_host(dims, X, dt, A, Bm, Cm, Q, E, z, Y, workspace, stream)
+    return Y, workspace
+
+
 def decode_step(cache, state, partial, x, dt, A, b, c, q, e, z, pos: int, chunk: int,
                 eps: float = 1e-6, out_dtype=torch.float32):
     """One decode step (``dart_decode_step``); cache, state and partial are updated in place.

@@ -20,7 +20,7 @@ LIB_PATH = os.path.join(_PKG, "libdart.so")
 DART_OK = 0
 DART_F32, DART_BF16 = 0, 1
 DART_OP_CHUNK_SCAN, DART_OP_SMA_FORWARD, DART_OP_DECODE_STEP = 0, 1, 2
-DART_OP_SMA_BACKWARD, DART_OP_SCAN_BACKWARD = 3, 4
+DART_OP_SMA_BACKWARD, DART_OP_SCAN_BACKWARD, DART_OP_PREFILL_HOST = 3, 4, 5
 STATUS_NAMES = {0: "DART_OK", 1: "DART_ERR_INVALID_ARG", 2: "DART_ERR_UNSUPPORTED",
                 3: "DART_ERR_WORKSPACE", 4: "DART_ERR_CUDA", 5: "DART_ERR_TIMEOUT",
                 6: "DART_ERR_TOO_LARGE"}
@@ -31,7 +31,8 @@ DART_DTYPE = {torch.float32: DART_F32, torch.bfloat16: DART_BF16}
 EXPORTED = ("dart_status_string", "dart_last_cuda_error", "dart_workspace_size",
             "dart_chunk_scan", "dart_sma_forward", "dart_decode_step", "dart_sma_forward_noalloc",
             "dart_launch_count", "dart_set_wait_limit_ns", "dart_get_device_status",
-            "dart_sma_backward", "dart_chunk_scan_backward", "dart_test_withhold_copies")
+            "dart_sma_backward", "dart_chunk_scan_backward", "dart_test_withhold_copies",
+            "dart_prefill_host")
 
 
 class DartError(RuntimeError):
@@ -84,6 +85,8 @@ def lib() -> ctypes.CDLL:
         L.dart_chunk_scan.argtypes = [dp] + [_vp] * 10 + [ctypes.c_size_t, _vp]
         L.dart_sma_forward.restype = ctypes.c_int
         L.dart_sma_forward.argtypes = [dp] + [_vp] * 11 + [ctypes.c_size_t, _vp]
+        L.dart_prefill_host.restype = ctypes.c_int
+        L.dart_prefill_host.argtypes = [dp] + [_vp] * 10 + [ctypes.c_size_t, _vp]
         L.dart_decode_step.restype = ctypes.c_int
         L.dart_decode_step.argtypes = ([dp, ctypes.c_int64, ctypes.c_int64] + [_vp] * 14
                                        + [ctypes.c_size_t, _vp])
@@ -113,6 +116,16 @@ def _ptr(t: torch.Tensor | None, name: str):
         raise TypeError(f"{name} must be a torch.Tensor")
     if not t.is_cuda:
         raise ValueError(f"{name} must be a CUDA tensor (the DART library has no CPU path)")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    return _vp(t.data_ptr())
+
+
+def _host_ptr(t: torch.Tensor, name: str):
+    if not isinstance(t, torch.Tensor):
+        raise TypeError(f"{name} must be a torch.Tensor")
+    if t.is_cuda:
+        raise ValueError(f"{name} must be a host tensor (page-locked for the copies to overlap)")
     if not t.is_contiguous():
         raise ValueError(f"{name} must be contiguous")
     return _vp(t.data_ptr())
@@ -179,6 +192,15 @@ def dart_decode_step(dims, pos, m_cap, cache, state, partial, x, dt, A, b, c, q,
         _ptr(partial, "partial"), _ptr(x, "x"), _ptr(dt, "dt"), _ptr(A, "A"), _ptr(b, "b"),
         _ptr(c, "c"), _ptr(q, "q"), _ptr(e, "e"), _ptr(z, "z"), _ptr(y, "y"), _ptr(lse, "lse"),
         w, nb, _stream(stream)))
+
+
+def dart_prefill_host(dims, X, dt, A, Bm, Cm, Q, E, z, Y, workspace=None, stream=None) -> None:
+    """Host tensors in (X, dt, A, Bm, Cm, Q, E, z) and out (Y); a device workspace."""
+    w, nb = _ws(workspace)
+    _check("dart_prefill_host", lib().dart_prefill_host(
+        ctypes.byref(dims), _host_ptr(X, "X"), _host_ptr(dt, "dt"), _host_ptr(A, "A"),
+        _host_ptr(Bm, "Bm"), _host_ptr(Cm, "Cm"), _host_ptr(Q, "Q"), _host_ptr(E, "E"),
+        _host_ptr(z, "z"), _host_ptr(Y, "Y"), w, nb, _stream(stream)))
 
 
 def dart_sma_backward(dims, M, rM, Q, Cm, E, z, lse, dY, dM, dQ, dC, dE, dz, workspace=None,

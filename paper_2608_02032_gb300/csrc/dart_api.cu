@@ -1,6 +1,7 @@
 // C ABI of the DART hot path: host-side validation, workspace layout and
 // kernel dispatch. Declarations and the contract are in include/dart.h.
 #include <atomic>
+#include <mutex>
 
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
@@ -148,6 +149,97 @@ std::atomic<int> g_test_withhold{0};
 
 std::atomic<uint64_t> g_launches{0};
 
+// ------------------------------------------------ host-buffer prefill layout
+constexpr int64_t kHostGroupHeads = 8;  // heads per copy/compute group
+
+size_t dtype_bytes(int t) { return t == DART_F32 ? 4 : 2; }
+
+// Device workspace of dart_prefill_host: the shared inputs, then per group of
+// hg heads its X, dt, z, Y_ssd, Y, memories and r (every group the same size),
+// then one scan and one SMA workspace per compute stream (groups alternate
+// between the two compute streams).
+struct HostLayout {
+    int64_t hg, groups;
+    size_t bm, cm, q, e, dt, z, a;          // shared inputs
+    size_t g0, stride;                      // first group, bytes per group
+    size_t x, dtg, zg, yssd, y, m, rm;      // offsets inside a group
+    size_t scan_ws[2], scan_bytes, sma_ws[2], sma_bytes;
+    size_t total;
+};
+
+HostLayout host_layout(const dart_dims* d) {
+    HostLayout h{};
+    const int64_t B = d->batch, L = d->seqlen, H = d->nheads, G = d->ngroups, P = d->headdim;
+    const int64_t N = d->dstate, M = L / d->chunk;
+    h.hg = (G == 1 && H > kHostGroupHeads && H % kHostGroupHeads == 0) ? kHostGroupHeads : H;
+    h.groups = H / h.hg;
+    const size_t ei = dtype_bytes(d->in_dtype), em = dtype_bytes(d->mem_dtype);
+    const size_t eo = dtype_bytes(d->out_dtype);
+    const size_t rows = (size_t)(B * L);
+    size_t o = 0;
+    auto take = [&o](size_t bytes) {
+        const size_t at = o;
+        o += align256(bytes);
+        return at;
+    };
+    h.bm = take(rows * G * N * ei);
+    h.cm = take(rows * G * N * ei);
+    h.q = take(rows * G * N * ei);
+    h.e = take(rows * G * P * ei);
+    h.dt = take(rows * H * 4);
+    h.z = take(rows * H * ei);
+    h.a = take((size_t)H * 4);
+    h.g0 = o;
+    const size_t hg = (size_t)h.hg;
+    h.x = take(rows * hg * P * ei) - h.g0;
+    h.dtg = take(rows * hg * 4) - h.g0;
+    h.zg = take(rows * hg * ei) - h.g0;
+    h.yssd = take(rows * hg * P * eo) - h.g0;
+    h.y = take(rows * hg * P * eo) - h.g0;
+    h.m = take((size_t)(B * M) * hg * N * P * em) - h.g0;
+    h.rm = take((size_t)(B * M) * hg * N * 4) - h.g0;
+    h.stride = o - h.g0;
+    o = h.g0 + (size_t)h.groups * h.stride;
+    dart_dims dg = *d;
+    dg.nheads = h.hg;
+    h.scan_bytes = scan_ws(&dg).total;
+    h.sma_bytes = sma_ws(&dg);
+    for (int k = 0; k < 2; ++k) {
+        h.scan_ws[k] = take(h.scan_bytes);
+        h.sma_ws[k] = take(h.sma_bytes);
+    }
+    h.total = o;
+    return h;
+}
+
+// The streams of dart_prefill_host (copy in, two for the kernels, copy out) for
+// the current device, created on first use and kept.
+struct HostStreams {
+    cudaStream_t in = nullptr, comp[2] = {nullptr, nullptr}, out = nullptr;
+};
+std::mutex g_host_mu;
+HostStreams g_host_streams[64];
+
+cudaError_t host_streams(HostStreams** hs) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lock(g_host_mu);
+    HostStreams& s = g_host_streams[dev];
+    if (s.in == nullptr) {
+        cudaStream_t t[4];
+        for (int i = 0; i < 4; ++i)
+            if ((e = cudaStreamCreateWithFlags(&t[i], cudaStreamNonBlocking)) != cudaSuccess) return e;
+        s.in = t[0];
+        s.comp[0] = t[1];
+        s.comp[1] = t[2];
+        s.out = t[3];
+    }
+    *hs = &s;
+    return cudaSuccess;
+}
+
 }  // namespace
 
 namespace dart {
@@ -187,6 +279,9 @@ size_t dart_workspace_size(const dart_dims* d, int op) {
             return sma_ws(d);
         case DART_OP_DECODE_STEP:
             return 0;
+        case DART_OP_PREFILL_HOST:
+            if (check_dims(d, true) != DART_OK) return 0;
+            return host_layout(d).total;
         case DART_OP_SMA_BACKWARD:
             if (check_dims(d, true) != DART_OK) return 0;
             if (sma_bwd_uses_tc(d))
@@ -298,6 +393,121 @@ dart_status dart_sma_forward(const dart_dims* d, const void* M, const float* rM,
     a.lse = lse;
     cudaError_t e = dispatch<SmaL>(d, a, s);
     return e == cudaSuccess ? DART_OK : cuda_fail(e);
+}
+
+dart_status dart_prefill_host(const dart_dims* d, const void* X, const float* dt, const float* A,
+                              const void* Bm, const void* Cm, const void* Q, const void* E,
+                              const void* z, void* Y, void* ws, size_t ws_bytes, void* stream) {
+    dart_status st = check_dims(d, true);
+    if (st != DART_OK) return st;
+    const void* req[] = {X, dt, A, Bm, Cm, Q, E, z, Y};
+    for (const void* p : req)
+        if (p == nullptr) return DART_ERR_INVALID_ARG;
+    const HostLayout h = host_layout(d);
+    if (ws == nullptr || ((uintptr_t)ws & 255u) != 0 || ws_bytes < h.total) return DART_ERR_WORKSPACE;
+    HostStreams* hs = nullptr;
+    cudaError_t e = host_streams(&hs);
+    if (e != cudaSuccess) return cuda_fail(e);
+
+    const int64_t B = d->batch, L = d->seqlen, H = d->nheads, G = d->ngroups, P = d->headdim;
+    const int64_t N = d->dstate;
+    const size_t ei = dtype_bytes(d->in_dtype), eo = dtype_bytes(d->out_dtype);
+    const size_t rows = (size_t)(B * L);
+    uint8_t* w = (uint8_t*)ws;
+    cudaStream_t s = (cudaStream_t)stream;
+    const int ng = (int)h.groups;
+    // events: the start on the caller's stream, per group copy-in and kernels done, the end
+    cudaEvent_t start = nullptr, done = nullptr, in_ev[64] = {}, comp_ev[64] = {};
+    if (ng > 64) return DART_ERR_UNSUPPORTED;
+    // events are released once recorded (the driver frees each when its work is done)
+    auto release = [&]() {
+        if (start != nullptr) cudaEventDestroy(start);
+        if (done != nullptr) cudaEventDestroy(done);
+        for (int g = 0; g < ng; ++g) {
+            if (in_ev[g] != nullptr) cudaEventDestroy(in_ev[g]);
+            if (comp_ev[g] != nullptr) cudaEventDestroy(comp_ev[g]);
+        }
+    };
+    auto fail = [&](cudaError_t err) {
+        release();
+        return cuda_fail(err);
+    };
+    const unsigned fl = cudaEventDisableTiming;
+    if ((e = cudaEventCreateWithFlags(&start, fl)) != cudaSuccess) return fail(e);
+    if ((e = cudaEventCreateWithFlags(&done, fl)) != cudaSuccess) return fail(e);
+    for (int g = 0; g < ng; ++g)
+        if ((e = cudaEventCreateWithFlags(&in_ev[g], fl)) != cudaSuccess ||
+            (e = cudaEventCreateWithFlags(&comp_ev[g], fl)) != cudaSuccess)
+            return fail(e);
+    // after the caller's earlier work on `stream`
+    if ((e = cudaEventRecord(start, s)) != cudaSuccess) return fail(e);
+    if ((e = cudaStreamWaitEvent(hs->in, start, 0)) != cudaSuccess) return fail(e);
+    if ((e = cudaStreamWaitEvent(hs->comp[0], start, 0)) != cudaSuccess ||
+        (e = cudaStreamWaitEvent(hs->comp[1], start, 0)) != cudaSuccess)
+        return fail(e);
+    if ((e = cudaStreamWaitEvent(hs->out, start, 0)) != cudaSuccess) return fail(e);
+    // shared inputs, one copy each
+    const struct {
+        size_t off;
+        const void* src;
+        size_t bytes;
+    } shared[] = {{h.bm, Bm, rows * G * N * ei}, {h.cm, Cm, rows * G * N * ei},
+                  {h.q, Q, rows * G * N * ei},   {h.e, E, rows * G * P * ei},
+                  {h.dt, dt, rows * H * 4},      {h.z, z, rows * H * ei},
+                  {h.a, A, (size_t)H * 4}};
+    for (const auto& c : shared)
+        if ((e = cudaMemcpyAsync(w + c.off, c.src, c.bytes, cudaMemcpyHostToDevice, hs->in)) != cudaSuccess)
+            return fail(e);
+    dart_dims dg = *d;
+    dg.nheads = h.hg;
+    const size_t xrow = (size_t)h.hg * P * ei, yrow = (size_t)h.hg * P * eo;
+    for (int g = 0; g < ng; ++g) {
+        const int64_t h0 = (int64_t)g * h.hg;
+        uint8_t* gb = w + h.g0 + (size_t)g * h.stride;
+        // copy in: the group's X rows (pitched)
+        e = cudaMemcpy2DAsync(gb + h.x, xrow, (const uint8_t*)X + (size_t)h0 * P * ei, (size_t)H * P * ei,
+                              xrow, rows, cudaMemcpyHostToDevice, hs->in);
+        if (e != cudaSuccess) return fail(e);
+        if ((e = cudaEventRecord(in_ev[g], hs->in)) != cudaSuccess) return fail(e);
+        // kernels, groups alternating between the two compute streams (so that the
+        // kernels of neighbouring groups share the SMs): the group's dt and z
+        // columns, the scan, the SMA and merge
+        const int k = g & 1;
+        cudaStream_t cs = hs->comp[k];
+        if ((e = cudaStreamWaitEvent(cs, in_ev[g], 0)) != cudaSuccess) return fail(e);
+        const float* dtg = (const float*)(w + h.dt);
+        const void* zg = w + h.z;
+        if (ng > 1) {
+            if ((e = dart::launch_gather_heads(w + h.dt, gb + h.dtg, (int64_t)rows, H, h0, h.hg, 4, cs)) !=
+                    cudaSuccess ||
+                (e = dart::launch_gather_heads(w + h.z, gb + h.zg, (int64_t)rows, H, h0, h.hg, (int)ei, cs)) !=
+                    cudaSuccess)
+                return fail(e);
+            dtg = (const float*)(gb + h.dtg);
+            zg = gb + h.zg;
+        }
+        st = dart_chunk_scan(&dg, gb + h.x, dtg, (const float*)(w + h.a) + h0, w + h.bm, w + h.cm,
+                             gb + h.yssd, gb + h.m, (float*)(gb + h.rm), nullptr, w + h.scan_ws[k],
+                             h.scan_bytes, cs);
+        if (st == DART_OK)
+            st = dart_sma_forward(&dg, gb + h.m, (const float*)(gb + h.rm), w + h.q, w + h.cm, w + h.e, zg,
+                                  gb + h.yssd, gb + h.y, nullptr, nullptr, w + h.sma_ws[k], h.sma_bytes, cs);
+        if (st != DART_OK) {
+            release();
+            return st;
+        }
+        if ((e = cudaEventRecord(comp_ev[g], cs)) != cudaSuccess) return fail(e);
+        // copy out: the group's Y rows (pitched)
+        if ((e = cudaStreamWaitEvent(hs->out, comp_ev[g], 0)) != cudaSuccess) return fail(e);
+        e = cudaMemcpy2DAsync((uint8_t*)Y + (size_t)h0 * P * eo, (size_t)H * P * eo, gb + h.y, yrow, yrow, rows,
+                              cudaMemcpyDeviceToHost, hs->out);
+        if (e != cudaSuccess) return fail(e);
+    }
+    // the caller's stream continues after the last copy out (which follows every kernel)
+    if ((e = cudaEventRecord(done, hs->out)) != cudaSuccess) return fail(e);
+    if ((e = cudaStreamWaitEvent(s, done, 0)) != cudaSuccess) return fail(e);
+    release();
+    return DART_OK;
 }
 
 dart_status dart_decode_step(const dart_dims* d, int64_t pos, int64_t m_cap, void* cache,

@@ -158,6 +158,11 @@ cudaError_t launch_sma_forward_simt(const SmaArgs& a, cudaStream_t stream);
 template <typename Tin, typename Tmem, typename Tout>
 cudaError_t launch_decode_step(const DecodeArgs& a, cudaStream_t stream);
 
+// dst[r, k] = src[r, h0 + k] for r < rows, k < hg (elements of elem_bytes = 2 or 4;
+// src rows of H elements, dst rows of hg).
+cudaError_t launch_gather_heads(const void* src, void* dst, int64_t rows, int64_t H, int64_t h0,
+                                int64_t hg, int elem_bytes, cudaStream_t stream);
+
 // Tensor-core SMA (sma_tc.cu): bf16 token inputs, P = 64, N = 128, S % 128 == 0.
 bool sma_tc_supported(const SmaArgs& a);
 size_t sma_tc_workspace(int64_t B, int64_t Mc, int64_t H);

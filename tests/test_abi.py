@@ -115,6 +115,29 @@ def test_decode_validation(L):
     assert B.STATUS_NAMES[1] == "DART_ERR_INVALID_ARG"
 
 
+def test_prefill_host_validation_and_workspace(L):
+    """The host-buffer prefill: its workspace holds the device copies and one head
+    group's scan and SMA workspaces; missing buffers or a short workspace are refused
+    before any copy or launch."""
+    from paper_2608_02032_gb300 import binding as B
+
+    v = ctypes.c_void_p
+    d = _dims(nheads=32)  # G = 1, H = 32: four groups of 8 heads
+    need = B.dart_workspace_size(d, B.DART_OP_PREFILL_HOST)
+    one = _dims(nheads=8)  # the device sizes of one group of 8 heads
+    per_group_inputs = 512 * 8 * 64 * 2
+    assert need > 4 * per_group_inputs
+    assert need > B.dart_workspace_size(one, B.DART_OP_CHUNK_SCAN)
+    assert B.dart_workspace_size(_dims(headdim=48), B.DART_OP_PREFILL_HOST) == 0
+    host = [v(FAKE)] * 9  # X .. Y (never dereferenced: validation fails first)
+    assert L.dart_prefill_host(ctypes.byref(d), *host, v(FAKE * 256), need - 256, None) == 3
+    assert L.dart_prefill_host(ctypes.byref(d), *host, v(FAKE * 256 + 16), need, None) == 3
+    bad = list(host)
+    bad[4] = None
+    assert L.dart_prefill_host(ctypes.byref(d), *bad, v(FAKE * 256), need, None) == 1
+    assert L.dart_prefill_host(ctypes.byref(_dims(chunk=96)), *host, v(FAKE * 256), need, None) == 2
+
+
 def test_noalloc_rejects_problems_beyond_its_scratch(L):
     """2^20 memory rows is the fixed limit; one more row is refused before any launch."""
     v = ctypes.c_void_p

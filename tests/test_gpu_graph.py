@@ -123,9 +123,12 @@ def test_training_step_replays_from_a_cuda_graph():
     step = _Step(w, train=True)
     ref = {s: _eager(step, s) for s in (43, 44)}
     g = _capture(step)
+    # dA is one sum per head over every token, added by atomics in an order that
+    # varies from run to run (eager or replayed); its spread reaches ~2e-5 of its RMS
+    tol = {"dA": 2e-4}
     for s in (44, 43):
         got = _replay(step, g, s)
         for k in got:
             assert not torch.isnan(got[k]).any(), f"{k}: not written by the replay (seed {s})"
             err = rel_err(host(got[k]), host(ref[s][k]))
-            assert err <= 1e-5, f"{k}: {err:.2e} after replay (seed {s})"
+            assert err <= tol.get(k, 1e-5), f"{k}: {err:.2e} after replay (seed {s})"
