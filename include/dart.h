@@ -171,7 +171,8 @@ dart_status dart_sma_forward(const dart_dims* dims, const void* M, const float* 
  *          memory, 256-byte aligned: device copies of the inputs, each group's
  *          Y_ssd, Y, memories and their r, and the scan and SMA workspaces.
  * The call orders itself after the work already on `stream` and leaves
- * `stream` waiting for its last copy. The four streams are created on the
+ * `stream` waiting for its last copy (also when it fails part way, for what
+ * it had enqueued). The four streams are created on the
  * first call for the current device and kept for the process.
  */
 dart_status dart_prefill_host(const dart_dims* dims, const void* X, const float* dt, const float* A,

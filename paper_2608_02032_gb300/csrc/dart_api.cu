@@ -428,7 +428,24 @@ dart_status dart_prefill_host(const dart_dims* d, const void* X, const float* dt
             if (comp_ev[g] != nullptr) cudaEventDestroy(comp_ev[g]);
         }
     };
+    // on an error after the start: the caller's stream still waits for whatever was
+    // enqueued on the library's streams, so that no copy outlives the caller's buffers
+    bool started = false;
+    auto join = [&]() {
+        if (!started) return;
+        cudaStream_t own[4] = {hs->in, hs->comp[0], hs->comp[1], hs->out};
+        for (cudaStream_t x : own) {
+            cudaEvent_t ev = nullptr;
+            if (cudaEventCreateWithFlags(&ev, cudaEventDisableTiming) == cudaSuccess) {
+                if (cudaEventRecord(ev, x) == cudaSuccess) cudaStreamWaitEvent(s, ev, 0);
+                cudaEventDestroy(ev);
+            } else {
+                cudaStreamSynchronize(x);  // no event to be had: wait here instead
+            }
+        }
+    };
     auto fail = [&](cudaError_t err) {
+        join();
         release();
         return cuda_fail(err);
     };
@@ -441,6 +458,7 @@ dart_status dart_prefill_host(const dart_dims* d, const void* X, const float* dt
             return fail(e);
     // after the caller's earlier work on `stream`
     if ((e = cudaEventRecord(start, s)) != cudaSuccess) return fail(e);
+    started = true;
     if ((e = cudaStreamWaitEvent(hs->in, start, 0)) != cudaSuccess) return fail(e);
     if ((e = cudaStreamWaitEvent(hs->comp[0], start, 0)) != cudaSuccess ||
         (e = cudaStreamWaitEvent(hs->comp[1], start, 0)) != cudaSuccess)
@@ -493,6 +511,7 @@ dart_status dart_prefill_host(const dart_dims* d, const void* X, const float* dt
             st = dart_sma_forward(&dg, gb + h.m, (const float*)(gb + h.rm), w + h.q, w + h.cm, w + h.e, zg,
                                   gb + h.yssd, gb + h.y, nullptr, nullptr, w + h.sma_ws[k], h.sma_bytes, cs);
         if (st != DART_OK) {
+            join();
             release();
             return st;
         }
