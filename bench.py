@@ -438,8 +438,9 @@ def bench_decode(args, dev, world, peaks, Bd, w, cache_slab, state_slab, token_i
 
 
 def bench_train(args, dev, world, peaks, Bd, w, prefill_inputs):
-    """One training step of the layer: forward (scan, SMA + merge) and backward
-    (SMA, scan) on the training workload, inputs resident in HBM."""
+    """One training step of the layer: forward (scan, SMA + merge, keeping the SMA
+    logits) and backward (SMA from those logits, scan) on the training workload,
+    inputs resident in HBM."""
     import torch
 
     inp = prefill_inputs(w, with_grad=True)
@@ -458,6 +459,7 @@ def bench_train(args, dev, world, peaks, Bd, w, prefill_inputs):
     dE, dz = torch.empty(Bsz, L, G, P, **f32), torch.empty(Bsz, L, H, **f32)
     dX, ddt = torch.empty(Bsz, L, H, P, **f32), torch.empty(Bsz, L, H, **f32)
     dA, dB = torch.empty(H, **f32), torch.empty(Bsz, L, G, N, **f32)
+    logits = torch.empty(Bsz, H, M, L, **f32)  # the SMA logits, kept by the forward for the backward
     wsz = lambda op: torch.empty(max(Bd.dart_workspace_size(dims, op), 256), dtype=torch.uint8, device=dev)
     ws_scan, ws_sma = wsz(Bd.DART_OP_CHUNK_SCAN), wsz(Bd.DART_OP_SMA_FORWARD)
     ws_sbwd, ws_cbwd = wsz(Bd.DART_OP_SMA_BACKWARD), wsz(Bd.DART_OP_SCAN_BACKWARD)
@@ -473,11 +475,11 @@ def bench_train(args, dev, world, peaks, Bd, w, prefill_inputs):
         Bd.dart_chunk_scan(dims, d["X"], d["dt"], d["A"], d["Bm"], d["Cm"], Yssd, Mem, rM, None, ws_scan,
                            stream)
         mark()
-        Bd.dart_sma_forward(dims, Mem, rM, d["Q"], d["Cm"], d["E"], d["z"], Yssd, Y, None, lse, ws_sma,
-                            stream)
+        Bd.dart_sma_forward_with_logits(dims, Mem, rM, d["Q"], d["Cm"], d["E"], d["z"], Yssd, Y, None, lse,
+                                        logits, ws_sma, stream)
         mark()
-        Bd.dart_sma_backward(dims, Mem, rM, d["Q"], d["Cm"], d["E"], d["z"], lse, d["dY"], dM, dQ, dC,
-                             dE, dz, ws_sbwd, stream)
+        Bd.dart_sma_backward_with_logits(dims, Mem, rM, d["Q"], d["Cm"], d["E"], d["z"], lse, logits, d["dY"],
+                                         dM, dQ, dC, dE, dz, ws_sbwd, stream)
         mark()
         Bd.dart_chunk_scan_backward(dims, d["X"], d["dt"], d["A"], d["Bm"], d["Cm"], d["dY"], dM, dX,
                                     ddt, dA, dB, dC, ws_cbwd, stream)

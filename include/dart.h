@@ -231,6 +231,26 @@ dart_status dart_sma_backward(const dart_dims* dims, const void* M, const float*
                               void* stream);
 
 /*
+ * Training pair that saves the logits. dart_sma_forward_with_logits is
+ * dart_sma_forward that also writes logits (Bsz, H, M, L) fp32, the entry
+ * (b, h, j, t) holding l_{t,j} for j < t / S (other entries unwritten); lse
+ * is required. It needs the tensor-core path (bf16 inputs, P = 64, N = 128,
+ * S % 128 == 0, H/G even) and gives DART_ERR_UNSUPPORTED elsewhere.
+ * dart_sma_backward_with_logits is dart_sma_backward with those logits: on
+ * the tensor-core path the weights g come from them (the same values as the
+ * recomputation, which it skips); the CUDA-core path recomputes them.
+ */
+dart_status dart_sma_forward_with_logits(const dart_dims* dims, const void* M, const float* rM,
+                                         const void* Q, const void* Cm, const void* E, const void* z,
+                                         const void* Y_ssd, void* Y, void* R, float* lse, float* logits,
+                                         void* workspace, size_t workspace_bytes, void* stream);
+dart_status dart_sma_backward_with_logits(const dart_dims* dims, const void* M, const float* rM,
+                                          const void* Q, const void* Cm, const void* E, const void* z,
+                                          const float* lse, const float* logits, const void* dY, float* dM,
+                                          float* dQ, float* dC, float* dE, float* dz, void* workspace,
+                                          size_t workspace_bytes, void* stream);
+
+/*
  * Backward of dart_chunk_scan (training): gradients of a loss that depends on
  * Y_ssd (through dY) and on the chunk memories (through dM, e.g. the output of
  * dart_sma_backward). Chain rule on the chunked forms of App. A: the states

@@ -57,11 +57,14 @@ class SmaOut:
     Y: torch.Tensor             # (Bsz, L, H, P) gated merge
     R: torch.Tensor | None      # (Bsz, L, H, P) SMA readout
     lse: torch.Tensor           # (Bsz, L, H) fp32 logsumexp over earlier chunks
+    logits: torch.Tensor | None = None  # (Bsz, H, M, L) fp32, saved for the backward
 
 
 def sma_forward(Mem, rM, Q, Cm, E, z, Y_ssd, chunk: int, eps: float = 1e-6, want_R: bool = True,
-                workspace: torch.Tensor | None = None) -> SmaOut:
-    """State-memory attention and gated merge (``dart_sma_forward``)."""
+                workspace: torch.Tensor | None = None, save_logits: bool = False) -> SmaOut:
+    """State-memory attention and gated merge (``dart_sma_forward``). ``save_logits``
+    (tensor-core shapes) also keeps the logits for ``sma_backward``
+    (``dart_sma_forward_with_logits``)."""
     Bsz, L, H, P = Y_ssd.shape
     G, N = Q.shape[2], Q.shape[3]
     dims = B.make_dims(Bsz, L, H, G, P, N, chunk, _dtype_code(Q), _dtype_code(Mem),
@@ -71,15 +74,20 @@ def sma_forward(Mem, rM, Q, Cm, E, z, Y_ssd, chunk: int, eps: float = 1e-6, want
     R = torch.empty_like(Y_ssd) if want_R else None
     lse = torch.empty(Bsz, L, H, dtype=torch.float32, device=dev)
     ws = workspace if workspace is not None else _workspace(dims, B.DART_OP_SMA_FORWARD, dev)
+    if save_logits:
+        logits = torch.empty(Bsz, H, L // chunk, L, dtype=torch.float32, device=dev)
+        B.dart_sma_forward_with_logits(dims, Mem, rM, Q, Cm, E, z, Y_ssd, Y, R, lse, logits, ws)
+        return SmaOut(Y, R, lse, logits)
     B.dart_sma_forward(dims, Mem, rM, Q, Cm, E, z, Y_ssd, Y, R, lse, ws)
     return SmaOut(Y, R, lse)
 
 
 def prefill_forward(X, dt, A, Bm, Cm, Q, E, z, chunk: int, eps: float = 1e-6, want_R=False,
-                    mem_dtype=torch.float32, out_dtype=torch.float32):
-    """Whole DART hot path of one block for a prefill: scan, SMA and merge."""
+                    mem_dtype=torch.float32, out_dtype=torch.float32, save_logits: bool = False):
+    """Whole DART hot path of one block for a prefill: scan, SMA and merge
+    (``save_logits``: keep the SMA logits for ``layer_backward``)."""
     s = chunk_scan(X, dt, A, Bm, Cm, chunk, eps, mem_dtype=mem_dtype, out_dtype=out_dtype)
-    o = sma_forward(s.M, s.rM, Q, Cm, E, z, s.Y_ssd, chunk, eps, want_R=want_R)
+    o = sma_forward(s.M, s.rM, Q, Cm, E, z, s.Y_ssd, chunk, eps, want_R=want_R, save_logits=save_logits)
     return s, o
 
 
@@ -135,8 +143,10 @@ class LayerGrads:
 
 
 def sma_backward(Mem, rM, Q, Cm, E, z, lse, dY, chunk: int, eps: float = 1e-6,
-                 workspace: torch.Tensor | None = None):
-    """Backward of ``sma_forward`` (``dart_sma_backward``): (dM, dQ, dC, dE, dz), all fp32."""
+                 workspace: torch.Tensor | None = None, logits: torch.Tensor | None = None):
+    """Backward of ``sma_forward`` (``dart_sma_backward``, or
+    ``dart_sma_backward_with_logits`` given the forward's saved logits):
+    (dM, dQ, dC, dE, dz), all fp32."""
     Bsz, L, H, P = dY.shape
     G, N = Q.shape[2], Q.shape[3]
     dims = B.make_dims(Bsz, L, H, G, P, N, chunk, _dtype_code(Q), _dtype_code(Mem),
@@ -147,7 +157,10 @@ def sma_backward(Mem, rM, Q, Cm, E, z, lse, dY, chunk: int, eps: float = 1e-6,
     dQ, dC, dE = torch.empty(Q.shape, **f32), torch.empty(Cm.shape, **f32), torch.empty(E.shape, **f32)
     dz = torch.empty(Bsz, L, H, **f32)
     ws = workspace if workspace is not None else _workspace(dims, B.DART_OP_SMA_BACKWARD, dev)
-    B.dart_sma_backward(dims, Mem, rM, Q, Cm, E, z, lse, dY, dM, dQ, dC, dE, dz, ws)
+    if logits is not None:
+        B.dart_sma_backward_with_logits(dims, Mem, rM, Q, Cm, E, z, lse, logits, dY, dM, dQ, dC, dE, dz, ws)
+    else:
+        B.dart_sma_backward(dims, Mem, rM, Q, Cm, E, z, lse, dY, dM, dQ, dC, dE, dz, ws)
     return dM, dQ, dC, dE, dz
 
 
@@ -174,6 +187,7 @@ def layer_backward(X, dt, A, Bm, Cm, Q, E, z, dY, scan: ScanOut, sma: SmaOut, ch
                    eps: float = 1e-6) -> LayerGrads:
     """Backward of ``prefill_forward`` for a loss gradient dY on Y: SMA backward, whose
     memory gradient and dC feed the scan backward."""
-    dM, dQ, dC, dE, dz = sma_backward(scan.M, scan.rM, Q, Cm, E, z, sma.lse, dY, chunk, eps)
+    dM, dQ, dC, dE, dz = sma_backward(scan.M, scan.rM, Q, Cm, E, z, sma.lse, dY, chunk, eps,
+                                      logits=sma.logits)
     dX, ddt, dA, dB, dC = chunk_scan_backward(X, dt, A, Bm, Cm, dY, dM, chunk, dC=dC, eps=eps)
     return LayerGrads(dX, ddt, dA, dB, dC, dQ, dE, dz, dM)

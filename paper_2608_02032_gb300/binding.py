@@ -32,7 +32,7 @@ EXPORTED = ("dart_status_string", "dart_last_cuda_error", "dart_workspace_size",
             "dart_chunk_scan", "dart_sma_forward", "dart_decode_step", "dart_sma_forward_noalloc",
             "dart_launch_count", "dart_set_wait_limit_ns", "dart_get_device_status",
             "dart_sma_backward", "dart_chunk_scan_backward", "dart_test_withhold_copies",
-            "dart_prefill_host")
+            "dart_prefill_host", "dart_sma_forward_with_logits", "dart_sma_backward_with_logits")
 
 
 class DartError(RuntimeError):
@@ -103,6 +103,10 @@ def lib() -> ctypes.CDLL:
         L.dart_test_withhold_copies.restype = None
         L.dart_sma_backward.argtypes = [dp] + [_vp] * 14 + [ctypes.c_size_t, _vp]
         L.dart_sma_backward.restype = ctypes.c_int
+        L.dart_sma_forward_with_logits.restype = ctypes.c_int
+        L.dart_sma_forward_with_logits.argtypes = [dp] + [_vp] * 12 + [ctypes.c_size_t, _vp]
+        L.dart_sma_backward_with_logits.restype = ctypes.c_int
+        L.dart_sma_backward_with_logits.argtypes = [dp] + [_vp] * 15 + [ctypes.c_size_t, _vp]
         L.dart_chunk_scan_backward.argtypes = [dp] + [_vp] * 13 + [ctypes.c_size_t, _vp]
         L.dart_chunk_scan_backward.restype = ctypes.c_int
         _lib = L
@@ -201,6 +205,24 @@ def dart_prefill_host(dims, X, dt, A, Bm, Cm, Q, E, z, Y, workspace=None, stream
         ctypes.byref(dims), _host_ptr(X, "X"), _host_ptr(dt, "dt"), _host_ptr(A, "A"),
         _host_ptr(Bm, "Bm"), _host_ptr(Cm, "Cm"), _host_ptr(Q, "Q"), _host_ptr(E, "E"),
         _host_ptr(z, "z"), _host_ptr(Y, "Y"), w, nb, _stream(stream)))
+
+
+def dart_sma_forward_with_logits(dims, M, rM, Q, Cm, E, z, Y_ssd, Y, R, lse, logits, workspace=None,
+                                 stream=None) -> None:
+    w, nb = _ws(workspace)
+    _check("dart_sma_forward_with_logits", lib().dart_sma_forward_with_logits(
+        ctypes.byref(dims), _ptr(M, "M"), _ptr(rM, "rM"), _ptr(Q, "Q"), _ptr(Cm, "Cm"), _ptr(E, "E"),
+        _ptr(z, "z"), _ptr(Y_ssd, "Y_ssd"), _ptr(Y, "Y"), _ptr(R, "R"), _ptr(lse, "lse"),
+        _ptr(logits, "logits"), w, nb, _stream(stream)))
+
+
+def dart_sma_backward_with_logits(dims, M, rM, Q, Cm, E, z, lse, logits, dY, dM, dQ, dC, dE, dz,
+                                  workspace=None, stream=None) -> None:
+    w, nb = _ws(workspace)
+    _check("dart_sma_backward_with_logits", lib().dart_sma_backward_with_logits(
+        ctypes.byref(dims), _ptr(M, "M"), _ptr(rM, "rM"), _ptr(Q, "Q"), _ptr(Cm, "Cm"), _ptr(E, "E"),
+        _ptr(z, "z"), _ptr(lse, "lse"), _ptr(logits, "logits"), _ptr(dY, "dY"), _ptr(dM, "dM"),
+        _ptr(dQ, "dQ"), _ptr(dC, "dC"), _ptr(dE, "dE"), _ptr(dz, "dz"), w, nb, _stream(stream)))
 
 
 def dart_sma_backward(dims, M, rM, Q, Cm, E, z, lse, dY, dM, dQ, dC, dE, dz, workspace=None,

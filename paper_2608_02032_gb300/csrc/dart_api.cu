@@ -342,18 +342,20 @@ dart_status dart_chunk_scan(const dart_dims* d, const void* X, const float* dt, 
     return e == cudaSuccess ? DART_OK : cuda_fail(e);
 }
 
-dart_status dart_sma_forward(const dart_dims* d, const void* M, const float* rM, const void* Q,
-                             const void* Cm, const void* E, const void* z, const void* Y_ssd,
-                             void* Y, void* R, float* lse, void* ws, size_t ws_bytes,
-                             void* stream) {
+static dart_status sma_forward_impl(const dart_dims* d, const void* M, const float* rM, const void* Q,
+                                    const void* Cm, const void* E, const void* z, const void* Y_ssd,
+                                    void* Y, void* R, float* lse, float* logits, void* ws,
+                                    size_t ws_bytes, void* stream) {
     dart_status st = check_dims(d, true);
     if (st != DART_OK) return st;
     const void* req[] = {M, Q, Cm, E, z, Y_ssd, Y};
     for (const void* p : req)
         if (p == nullptr || !aligned16(p)) return DART_ERR_INVALID_ARG;
-    if ((rM && !aligned16(rM)) || (R && !aligned16(R)) || (lse && !aligned16(lse)))
+    if ((rM && !aligned16(rM)) || (R && !aligned16(R)) || (lse && !aligned16(lse)) ||
+        (logits && !aligned16(logits)))
         return DART_ERR_INVALID_ARG;
     const bool tc = sma_uses_tc(d);
+    if (logits != nullptr && !tc) return DART_ERR_UNSUPPORTED;  // saved by the tensor-core kernel only
     const size_t need = (tc || rM == nullptr) ? sma_ws(d) : 0;
     if (need > 0 && (ws == nullptr || ((uintptr_t)ws & 255u) != 0 || ws_bytes < need))
         return DART_ERR_WORKSPACE;
@@ -362,7 +364,7 @@ dart_status dart_sma_forward(const dart_dims* d, const void* M, const float* rM,
     if (tc) {
         dart::SmaArgs a = sma_args(d);
         a.M = M; a.rM = rM; a.Q = Q; a.Cm = Cm; a.E = E; a.z = z; a.Yssd = Y_ssd; a.Y = Y;
-        a.R = R; a.lse = lse;
+        a.R = R; a.lse = lse; a.logits = logits;
         a.test_withhold = g_test_withhold.load();
         const unsigned long long lim = g_wait_limit_ns.load();
         typedef __nv_bfloat16 bf;
@@ -393,6 +395,21 @@ dart_status dart_sma_forward(const dart_dims* d, const void* M, const float* rM,
     a.lse = lse;
     cudaError_t e = dispatch<SmaL>(d, a, s);
     return e == cudaSuccess ? DART_OK : cuda_fail(e);
+}
+
+dart_status dart_sma_forward(const dart_dims* d, const void* M, const float* rM, const void* Q,
+                             const void* Cm, const void* E, const void* z, const void* Y_ssd,
+                             void* Y, void* R, float* lse, void* ws, size_t ws_bytes,
+                             void* stream) {
+    return sma_forward_impl(d, M, rM, Q, Cm, E, z, Y_ssd, Y, R, lse, nullptr, ws, ws_bytes, stream);
+}
+
+dart_status dart_sma_forward_with_logits(const dart_dims* d, const void* M, const float* rM,
+                                         const void* Q, const void* Cm, const void* E, const void* z,
+                                         const void* Y_ssd, void* Y, void* R, float* lse, float* logits,
+                                         void* ws, size_t ws_bytes, void* stream) {
+    if (logits == nullptr || lse == nullptr) return DART_ERR_INVALID_ARG;
+    return sma_forward_impl(d, M, rM, Q, Cm, E, z, Y_ssd, Y, R, lse, logits, ws, ws_bytes, stream);
 }
 
 dart_status dart_prefill_host(const dart_dims* d, const void* X, const float* dt, const float* A,
@@ -555,21 +572,23 @@ dart_status dart_decode_step(const dart_dims* d, int64_t pos, int64_t m_cap, voi
     return err == cudaSuccess ? DART_OK : cuda_fail(err);
 }
 
-dart_status dart_sma_backward(const dart_dims* d, const void* M, const float* rM, const void* Q,
-                              const void* Cm, const void* E, const void* z, const float* lse,
-                              const void* dY, float* dM, float* dQ, float* dC, float* dE,
-                              float* dz, void* ws, size_t ws_bytes, void* stream) {
+static dart_status sma_backward_impl(const dart_dims* d, const void* M, const float* rM, const void* Q,
+                                     const void* Cm, const void* E, const void* z, const float* lse,
+                                     const float* logits, const void* dY, float* dM, float* dQ, float* dC,
+                                     float* dE, float* dz, void* ws, size_t ws_bytes, void* stream) {
     dart_status st = check_dims(d, true);
     if (st != DART_OK) return st;
     const void* req[] = {M, Q, Cm, E, z, lse, dY, dM, dQ, dC, dE, dz};
     for (const void* p : req)
         if (p == nullptr || !aligned16(p)) return DART_ERR_INVALID_ARG;
-    if (rM != nullptr && !aligned16(rM)) return DART_ERR_INVALID_ARG;
+    if ((rM != nullptr && !aligned16(rM)) || (logits != nullptr && !aligned16(logits)))
+        return DART_ERR_INVALID_ARG;
     const size_t need = dart_workspace_size(d, DART_OP_SMA_BACKWARD);
     if (ws == nullptr || ((uintptr_t)ws & 255u) != 0 || ws_bytes < need) return DART_ERR_WORKSPACE;
     dart::SmaBwdArgs a = sma_bwd_args(d);
     a.M = M; a.rM = rM; a.Q = Q; a.Cm = Cm; a.E = E; a.z = z; a.lse = lse; a.dY = dY;
     a.dM = dM; a.dQ = dQ; a.dC = dC; a.dE = dE; a.dz = dz;
+    a.logits = logits;  // the CUDA-core path recomputes the logits and ignores them
     cudaStream_t s = (cudaStream_t)stream;
     typedef __nv_bfloat16 bf;
     cudaError_t e;
@@ -588,6 +607,24 @@ dart_status dart_sma_backward(const dart_dims* d, const void* M, const float* rM
     else
         return DART_ERR_UNSUPPORTED;
     return e == cudaSuccess ? DART_OK : cuda_fail(e);
+}
+
+dart_status dart_sma_backward(const dart_dims* d, const void* M, const float* rM, const void* Q,
+                              const void* Cm, const void* E, const void* z, const float* lse,
+                              const void* dY, float* dM, float* dQ, float* dC, float* dE,
+                              float* dz, void* ws, size_t ws_bytes, void* stream) {
+    return sma_backward_impl(d, M, rM, Q, Cm, E, z, lse, nullptr, dY, dM, dQ, dC, dE, dz, ws, ws_bytes,
+                             stream);
+}
+
+dart_status dart_sma_backward_with_logits(const dart_dims* d, const void* M, const float* rM,
+                                          const void* Q, const void* Cm, const void* E, const void* z,
+                                          const float* lse, const float* logits, const void* dY, float* dM,
+                                          float* dQ, float* dC, float* dE, float* dz, void* ws,
+                                          size_t ws_bytes, void* stream) {
+    if (logits == nullptr) return DART_ERR_INVALID_ARG;
+    return sma_backward_impl(d, M, rM, Q, Cm, E, z, lse, logits, dY, dM, dQ, dC, dE, dz, ws, ws_bytes,
+                             stream);
 }
 
 dart_status dart_chunk_scan_backward(const dart_dims* d, const void* X, const float* dt,

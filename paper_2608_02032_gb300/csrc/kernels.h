@@ -49,6 +49,7 @@ struct SmaArgs {
     void* R;
     float* lse;
     int test_withhold;  // tensor-core path: issue no operand copies (failure-path test hook)
+    float* logits = nullptr;  // tensor-core path: B x H x Mc x L logits for the backward, or null
 };
 
 struct DecodeArgs {
@@ -86,6 +87,7 @@ struct SmaBwdArgs {
     float* dC;  // B x L x G x N (overwritten)
     float* dE;  // B x L x G x P (overwritten)
     float* dz;  // B x L x H (overwritten)
+    const float* logits = nullptr;  // the forward's logits (B x H x Mc x L) or null: recomputed
 };
 
 // Backward of the chunked scan (scan_bwd.cu). Gradients are fp32.
@@ -177,6 +179,11 @@ template <typename Tmem>
 cudaError_t launch_sma_bwd_stats_tc(const SmaBwdArgs& a, const float* rM, uint8_t* ops,
                                     int pair_bytes, float* scale, float* g, float2* gd,
                                     unsigned long long wait_limit_ns, cudaStream_t stream);
+// The same outputs from a.logits (saved by the forward) instead of the logit chains.
+template <typename Tmem>
+cudaError_t launch_sma_bwd_stats_from_logits(const SmaBwdArgs& a, const float* rM, uint8_t* ops,
+                                             int pair_bytes, float* scale, float* g, float2* gd,
+                                             cudaStream_t stream);
 bool sma_bwd_tc_supported(const SmaBwdArgs& a);
 size_t sma_bwd_tc_workspace(int64_t B, int64_t L, int64_t H, int64_t Mc, int64_t N);
 template <typename Tmem>

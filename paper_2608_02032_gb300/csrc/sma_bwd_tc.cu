@@ -874,7 +874,9 @@ cudaError_t launch_sma_backward_tc(const SmaBwdArgs& a, void* ws, unsigned long 
         e = launch_memory_rms<Tmem>(a.M, rM, a.B * Mc * a.H * a.N, a.P, a.eps, stream);
         if (e != cudaSuccess) return e;
     }
-    e = launch_sma_bwd_stats_tc<Tmem>(a, rM, ops, kPairB, scale, gbuf, gd, wait_limit_ns, stream);
+    e = a.logits != nullptr
+            ? launch_sma_bwd_stats_from_logits<Tmem>(a, rM, ops, kPairB, scale, gbuf, gd, stream)
+            : launch_sma_bwd_stats_tc<Tmem>(a, rM, ops, kPairB, scale, gbuf, gd, wait_limit_ns, stream);
     if (e != cudaSuccess) return e;
     // the row kernels add their head-pair halves into these
     const size_t rows = (size_t)(a.B * a.L);

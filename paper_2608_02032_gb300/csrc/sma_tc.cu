@@ -305,13 +305,14 @@ __device__ __forceinline__ void issue_part(uint32_t d_tmem, uint32_t a_tmem, uin
 // What the backward-statistics variant (kStats) writes instead of the merge:
 // the softmax weights g_{t,j} = exp(l_{t,j} - lse_t) (lse from the forward)
 // and their sum G1_t. It runs the U half of each job only (parts W_hi, W_lo;
-// no value chain).
+// no value chain). The forward variant, when g is given, writes the logits
+// l_{t,j} there instead, for a backward that then needs no statistics pass.
 struct SmaStats {
     float* g;    // B x H x Mc x L
     float2* gd;  // B x L x H: (G1, -) -- the second field is written later
 };
 
-template <typename Tout, bool kStats>
+template <typename Tout, bool kStats, bool kLogits = false>
 __global__ void __launch_bounds__(kThreads, 1)
 sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
               const __nv_bfloat16* __restrict__ Q, const __nv_bfloat16* __restrict__ Cm,
@@ -563,7 +564,7 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
                     for (int i = 0; i < 16; ++i) acc = f2_fma(v[i], eb[16 + i], acc);
                     float lx, ly;
                     f2_unpack(acc, lx, ly);
-                    l = (lx + ly) * lfac;
+                    l = __fmul_rn(lx + ly, lfac);  // rounded: the stored and the recomputed logits agree
                 }
                 const float gw = expf(l - lse_t);
                 G1 += gw;
@@ -580,6 +581,8 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
             float s_next = nj > 0 ? __ldg(scl) : 0.0f;
             const uint32_t ua = tmem + lane_addr + kColU + (uint32_t)(kP * wg);
             const uint32_t va = tmem + lane_addr + kColV + (uint32_t)(kP * wg);  // + 128 per V buffer
+            // training variant: the logits l_{t,j} for the backward (st.g: B x H x Mc x L)
+            float* lgp = kLogits ? st.g + ((i64)b * H + h) * Mc * L + t : nullptr;
             // the merge's Y_ssd row and gate come from L2 if fetched a few jobs ahead
             const i64 rowo_pf = tok * H + h;
             const int pf_job = nj > 4 ? nj - 4 : 0;
@@ -607,8 +610,9 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
                     for (int i = 0; i < 16; ++i) acc = f2_fma(v[i], eb[16 + i], acc);
                     float lx, ly;
                     f2_unpack(acc, lx, ly);
-                    l = (lx + ly) * lfac;
+                    l = __fmul_rn(lx + ly, lfac);  // rounded: the stored and the recomputed logits agree
                 }
+                if constexpr (kLogits) lgp[(i64)j * L] = l;
                 // online softmax; the running sums are rescaled only when the maximum moves
                 if (l > m) {
                     const float sc = expf(m - l);
@@ -715,7 +719,7 @@ cudaError_t launch_sma_forward_tc(const SmaArgs& a, void* ws, unsigned long long
         note_launches(1);
     }
     const size_t smem = sizeof(TcSmem) + 1024;
-    auto kern = sma_tc_kernel<Tout, false>;
+    auto kern = a.logits != nullptr ? sma_tc_kernel<Tout, false, true> : sma_tc_kernel<Tout, false>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     const int items = (L / kRows) * Bsz * (H / kHeadsPerCta);
@@ -724,7 +728,7 @@ cudaError_t launch_sma_forward_tc(const SmaArgs& a, void* ws, unsigned long long
                                             (const __nv_bfloat16*)a.z, (const Tout*)a.Yssd,
                                             (Tout*)a.Y, (Tout*)a.R, a.lse, Bsz, L, H, (int)a.G,
                                             (int)a.S, Mc, a.eps, wait_limit_ns, a.test_withhold,
-                                            kPair, SmaStats{});
+                                            kPair, SmaStats{a.logits, nullptr});
     note_launches(1);
     return cudaGetLastError();
 }
@@ -759,6 +763,48 @@ template cudaError_t launch_sma_bwd_stats_tc<float>(const SmaBwdArgs&, const flo
 template cudaError_t launch_sma_bwd_stats_tc<__nv_bfloat16>(const SmaBwdArgs&, const float*, uint8_t*,
                                                             int, float*, float*, float2*,
                                                             unsigned long long, cudaStream_t);
+
+// g_{t,j} = exp(l_{t,j} - lse_t) for j < t / S and G1_t = sum_j g from the
+// logits the forward saved: the statistics pass's arithmetic in its order,
+// without recomputing the logit chains. One thread per (b, h, t).
+__global__ void sma_g_from_logits_kernel(const float* __restrict__ logits, const float* __restrict__ lse,
+                                         float* __restrict__ g, float2* __restrict__ gd, int L, int H,
+                                         int S, int Mc) {
+    const int t = blockIdx.x * blockDim.x + threadIdx.x, h = blockIdx.y, b = blockIdx.z;
+    if (t >= L) return;
+    const int nj = t / S;
+    const i64 rowo = ((i64)b * L + t) * H + h;
+    const float lse_t = lse[rowo];
+    const i64 base = ((i64)b * H + h) * Mc * L + t;
+    float G1 = 0.0f;
+    for (int j = 0; j < nj; ++j) {
+        const float gw = expf(logits[base + (i64)j * L] - lse_t);
+        G1 += gw;
+        g[base + (i64)j * L] = gw;
+    }
+    gd[rowo] = make_float2(G1, 0.0f);
+}
+
+template <typename Tmem>
+cudaError_t launch_sma_bwd_stats_from_logits(const SmaBwdArgs& a, const float* rM, uint8_t* ops,
+                                             int pair_bytes, float* scale, float* g, float2* gd,
+                                             cudaStream_t stream) {
+    const int Bsz = (int)a.B, L = (int)a.L, H = (int)a.H, Mc = (int)(a.L / a.S);
+    if (Mc > 1) {  // the backward's operand tiles, as in the statistics pass
+        sma_operands_kernel<Tmem><<<dim3(Mc - 1, H, Bsz), 256, 0, stream>>>(
+            (const Tmem*)a.M, rM, ops, scale, Mc, H, a.eps, pair_bytes);
+        note_launches(1);
+    }
+    sma_g_from_logits_kernel<<<dim3((L + 255) / 256, H, Bsz), 256, 0, stream>>>(a.logits, a.lse, g, gd, L, H,
+                                                                                 (int)a.S, Mc);
+    note_launches(1);
+    return cudaGetLastError();
+}
+template cudaError_t launch_sma_bwd_stats_from_logits<float>(const SmaBwdArgs&, const float*, uint8_t*, int,
+                                                             float*, float*, float2*, cudaStream_t);
+template cudaError_t launch_sma_bwd_stats_from_logits<__nv_bfloat16>(const SmaBwdArgs&, const float*,
+                                                                     uint8_t*, int, float*, float*, float2*,
+                                                                     cudaStream_t);
 
 typedef __nv_bfloat16 bf16;
 template cudaError_t launch_sma_forward_tc<float, float>(const SmaArgs&, void*, unsigned long long,

@@ -98,6 +98,35 @@ def test_layer_backward_matches_oracle(w):
         assert err <= _tol(w), f"{name}: {err:.3e}"
 
 
+@pytest.mark.parametrize("w", [CASES[3], CASES[6], CASES[7]], ids=lambda w: w.name)
+def test_layer_backward_with_saved_logits(w):
+    """The training pair that keeps the forward's logits: the backward takes its
+    softmax weights from them instead of recomputing the logit chains. Against the
+    oracle, and against the recomputing backward (the same weights; the gradients
+    differ only by the order of their fp32 atomic additions)."""
+    inp = prefill_inputs(w, with_grad=True)
+    ref = oracle.backward(inp["X"], inp["dt"], inp["A"], inp["Bm"], inp["Cm"], inp["Q"], inp["E"],
+                          inp["z"], inp["dY"], w.chunk, w.eps)
+    X, Bm, Cm, Q, E, z, dY = (dev(inp[k], w.dtype) for k in ("X", "Bm", "Cm", "Q", "E", "z", "dY"))
+    dt, A = dev(inp["dt"], torch.float32), dev(inp["A"], torch.float32)
+    s, o = api.prefill_forward(X, dt, A, Bm, Cm, Q, E, z, w.chunk, w.eps, save_logits=True)
+    assert o.logits is not None
+    gr = api.layer_backward(X, dt, A, Bm, Cm, Q, E, z, dY, s, o, w.chunk, w.eps)
+    s2, o2 = api.prefill_forward(X, dt, A, Bm, Cm, Q, E, z, w.chunk, w.eps)
+    gr2 = api.layer_backward(X, dt, A, Bm, Cm, Q, E, z, dY, s2, o2, w.chunk, w.eps)
+    torch.cuda.synchronize()
+    assert torch.equal(o.Y, o2.Y) and torch.equal(o.lse, o2.lse)  # the forward itself is unchanged
+    names = ["dX", "ddt", "dA", "dB", "dC", "dQ", "dE", "dz"]
+    got = [gr.dX, gr.ddt, gr.dA, gr.dB, gr.dC, gr.dQ, gr.dE, gr.dz]
+    rec = [gr2.dX, gr2.ddt, gr2.dA, gr2.dB, gr2.dC, gr2.dQ, gr2.dE, gr2.dz]
+    # dA: one sum per head over every token, atomics in run-dependent order
+    tol_same = {"dA": 2e-4}
+    for n, g, r, g2 in zip(names, got, ref, rec):
+        assert rel_err(host(g), r) <= _tol(w), n
+        assert rel_err(host(g), host(g2)) <= tol_same.get(n, 1e-5), n
+    assert rel_err(host(gr.dM), host(gr2.dM)) <= 1e-5
+
+
 def test_backward_single_chunk_has_no_sma_gradient():
     """S = L: no token has history, so the SMA gradients are exactly zero."""
     w = Workload("bwd_one_chunk", 1, 2, 128, 32, 16, 128, dtype="f32", seed=2105)
@@ -113,15 +142,16 @@ def test_backward_single_chunk_has_no_sma_gradient():
 
 @pytest.mark.parametrize("name", ["train_b8_l4k_s256", "train_b8_l4k_s128"])
 def test_training_step_full_size_on_one_batch(name):
-    """The training workload at full size (B8 H24 L4096), forward and layer backward
-    through the library exactly as the bench's training step runs them; the oracle
+    """The training workload at full size (B8 H24 L4096), forward (keeping the SMA
+    logits) and layer backward through the library exactly as the bench's training
+    step runs them; the oracle
     computes batch 0 (batches are independent) and every per-batch gradient is
     compared there. dA sums over the batch, so it is checked on the small cases."""
     w = WORKLOADS[name]
     inp = prefill_inputs(w, with_grad=True)
     X, Bm, Cm, Q, E, z, dY = (dev(inp[k], w.dtype) for k in ("X", "Bm", "Cm", "Q", "E", "z", "dY"))
     dt, A = dev(inp["dt"], torch.float32), dev(inp["A"], torch.float32)
-    s, o = api.prefill_forward(X, dt, A, Bm, Cm, Q, E, z, w.chunk, w.eps)
+    s, o = api.prefill_forward(X, dt, A, Bm, Cm, Q, E, z, w.chunk, w.eps, save_logits=True)
     gr = api.layer_backward(X, dt, A, Bm, Cm, Q, E, z, dY, s, o, w.chunk, w.eps)
     torch.cuda.synchronize()
     one = {k: inp[k][:1] for k in ("X", "dt", "Bm", "Cm", "Q", "E", "z", "dY")}
