@@ -18,17 +18,25 @@
  *                     gradients of the two prefill calls for training (the
  *                     paper trains the layer end to end but prints no
  *                     backward; these are the chain rule on the forms above).
+ *   dart_sma_forward_with_logits, dart_sma_backward_with_logits
+ *                     the SMA pair for training that keeps the forward's
+ *                     logits so the backward need not recompute them.
+ *   dart_prefill_host the two prefill calls from host buffers to a host
+ *                     buffer, copies overlapped with the kernels.
  *
  * Conventions shared by every entry point
  *   - Every tensor pointer is a DEVICE pointer owned by the caller, 16-byte
  *     aligned, contiguous and row-major in the shapes given below (the
- *     paper's table of compact tensor shapes, App. B.2). The library keeps
- *     no reference to any pointer after the call returns.
+ *     paper's table of compact tensor shapes, App. B.2), except the host
+ *     buffers of dart_prefill_host. The library keeps no reference to any
+ *     pointer after the call returns.
  *   - The library never allocates device memory. Scratch comes from the
  *     caller's `workspace` (device memory of at least
  *     dart_workspace_size(dims, op) bytes, 256-byte aligned).
  *   - Every call is asynchronous on `stream` (a cudaStream_t; NULL is the
  *     legacy default stream) and does not synchronise the host.
+ *     dart_prefill_host also works on streams of its own (created once per
+ *     device); calls from several host threads share them and run in turn.
  *   - Arguments are validated on the host before anything is launched; a
  *     call that returns an error has written nothing.
  *   - Token and chunk indices are 0-based: token t lies in chunk t / S, the
