@@ -171,7 +171,10 @@ HostLayout host_layout(const dart_dims* d) {
     HostLayout h{};
     const int64_t B = d->batch, L = d->seqlen, H = d->nheads, G = d->ngroups, P = d->headdim;
     const int64_t N = d->dstate, M = L / d->chunk;
-    h.hg = (G == 1 && H > kHostGroupHeads && H % kHostGroupHeads == 0) ? kHostGroupHeads : H;
+    // groups of kHostGroupHeads heads (at most 64 groups), else the whole problem as one
+    h.hg = (G == 1 && H > kHostGroupHeads && H % kHostGroupHeads == 0 && H / kHostGroupHeads <= 64)
+               ? kHostGroupHeads
+               : H;
     h.groups = H / h.hg;
     const size_t ei = dtype_bytes(d->in_dtype), em = dtype_bytes(d->mem_dtype);
     const size_t eo = dtype_bytes(d->out_dtype);
@@ -435,7 +438,6 @@ dart_status dart_prefill_host(const dart_dims* d, const void* X, const float* dt
     const int ng = (int)h.groups;
     // events: the start on the caller's stream, per group copy-in and kernels done, the end
     cudaEvent_t start = nullptr, done = nullptr, in_ev[64] = {}, comp_ev[64] = {};
-    if (ng > 64) return DART_ERR_UNSUPPORTED;
     // events are released once recorded (the driver frees each when its work is done)
     auto release = [&]() {
         if (start != nullptr) cudaEventDestroy(start);

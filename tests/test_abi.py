@@ -129,6 +129,8 @@ def test_prefill_host_validation_and_workspace(L):
     assert need > 4 * per_group_inputs
     assert need > B.dart_workspace_size(one, B.DART_OP_CHUNK_SCAN)
     assert B.dart_workspace_size(_dims(headdim=48), B.DART_OP_PREFILL_HOST) == 0
+    # beyond 64 groups of 8 heads the problem runs as one group (still a valid size)
+    assert B.dart_workspace_size(_dims(nheads=1024), B.DART_OP_PREFILL_HOST) > 0
     host = [v(FAKE)] * 9  # X .. Y (never dereferenced: validation fails first)
     assert L.dart_prefill_host(ctypes.byref(d), *host, v(FAKE * 256), need - 256, None) == 3
     assert L.dart_prefill_host(ctypes.byref(d), *host, v(FAKE * 256 + 16), need, None) == 3
