@@ -437,11 +437,12 @@ dart_status dart_prefill_host(const dart_dims* d, const void* X, const float* dt
     cudaStream_t s = (cudaStream_t)stream;
     const int ng = (int)h.groups;
     // events: the start on the caller's stream, per group copy-in and kernels done, the end
-    cudaEvent_t start = nullptr, done = nullptr, in_ev[64] = {}, comp_ev[64] = {};
+    cudaEvent_t start = nullptr, done = nullptr, sma_ev = nullptr, in_ev[64] = {}, comp_ev[64] = {};
     // events are released once recorded (the driver frees each when its work is done)
     auto release = [&]() {
         if (start != nullptr) cudaEventDestroy(start);
         if (done != nullptr) cudaEventDestroy(done);
+        if (sma_ev != nullptr) cudaEventDestroy(sma_ev);
         for (int g = 0; g < ng; ++g) {
             if (in_ev[g] != nullptr) cudaEventDestroy(in_ev[g]);
             if (comp_ev[g] != nullptr) cudaEventDestroy(comp_ev[g]);
@@ -471,6 +472,7 @@ dart_status dart_prefill_host(const dart_dims* d, const void* X, const float* dt
     const unsigned fl = cudaEventDisableTiming;
     if ((e = cudaEventCreateWithFlags(&start, fl)) != cudaSuccess) return fail(e);
     if ((e = cudaEventCreateWithFlags(&done, fl)) != cudaSuccess) return fail(e);
+    if ((e = cudaEventCreateWithFlags(&sma_ev, fl)) != cudaSuccess) return fail(e);
     for (int g = 0; g < ng; ++g)
         if ((e = cudaEventCreateWithFlags(&in_ev[g], fl)) != cudaSuccess ||
             (e = cudaEventCreateWithFlags(&comp_ev[g], fl)) != cudaSuccess)
@@ -483,16 +485,17 @@ dart_status dart_prefill_host(const dart_dims* d, const void* X, const float* dt
         (e = cudaStreamWaitEvent(hs->comp[1], start, 0)) != cudaSuccess)
         return fail(e);
     if ((e = cudaStreamWaitEvent(hs->out, start, 0)) != cudaSuccess) return fail(e);
-    // shared inputs, one copy each
-    const struct {
+    // shared inputs, one copy each: the scan's first (B, C, dt, A), then, after the
+    // first group's X, the SMA's (Q, E, z), which land under the first group's scan
+    struct Copy {
         size_t off;
         const void* src;
         size_t bytes;
-    } shared[] = {{h.bm, Bm, rows * G * N * ei}, {h.cm, Cm, rows * G * N * ei},
-                  {h.q, Q, rows * G * N * ei},   {h.e, E, rows * G * P * ei},
-                  {h.dt, dt, rows * H * 4},      {h.z, z, rows * H * ei},
-                  {h.a, A, (size_t)H * 4}};
-    for (const auto& c : shared)
+    };
+    const Copy scan_in[] = {{h.bm, Bm, rows * G * N * ei}, {h.cm, Cm, rows * G * N * ei},
+                            {h.dt, dt, rows * H * 4}, {h.a, A, (size_t)H * 4}};
+    const Copy sma_in[] = {{h.q, Q, rows * G * N * ei}, {h.e, E, rows * G * P * ei}, {h.z, z, rows * H * ei}};
+    for (const auto& c : scan_in)
         if ((e = cudaMemcpyAsync(w + c.off, c.src, c.bytes, cudaMemcpyHostToDevice, hs->in)) != cudaSuccess)
             return fail(e);
     dart_dims dg = *d;
@@ -506,6 +509,13 @@ dart_status dart_prefill_host(const dart_dims* d, const void* X, const float* dt
                               xrow, rows, cudaMemcpyHostToDevice, hs->in);
         if (e != cudaSuccess) return fail(e);
         if ((e = cudaEventRecord(in_ev[g], hs->in)) != cudaSuccess) return fail(e);
+        if (g == 0) {  // the SMA's shared inputs follow the first group's X
+            for (const auto& c : sma_in)
+                if ((e = cudaMemcpyAsync(w + c.off, c.src, c.bytes, cudaMemcpyHostToDevice, hs->in)) !=
+                    cudaSuccess)
+                    return fail(e);
+            if ((e = cudaEventRecord(sma_ev, hs->in)) != cudaSuccess) return fail(e);
+        }
         // kernels, groups alternating between the two compute streams (so that the
         // kernels of neighbouring groups share the SMs): the group's dt and z
         // columns, the scan, the SMA and merge
@@ -516,16 +526,21 @@ dart_status dart_prefill_host(const dart_dims* d, const void* X, const float* dt
         const void* zg = w + h.z;
         if (ng > 1) {
             if ((e = dart::launch_gather_heads(w + h.dt, gb + h.dtg, (int64_t)rows, H, h0, h.hg, 4, cs)) !=
-                    cudaSuccess ||
-                (e = dart::launch_gather_heads(w + h.z, gb + h.zg, (int64_t)rows, H, h0, h.hg, (int)ei, cs)) !=
-                    cudaSuccess)
+                cudaSuccess)
                 return fail(e);
             dtg = (const float*)(gb + h.dtg);
-            zg = gb + h.zg;
         }
         st = dart_chunk_scan(&dg, gb + h.x, dtg, (const float*)(w + h.a) + h0, w + h.bm, w + h.cm,
                              gb + h.yssd, gb + h.m, (float*)(gb + h.rm), nullptr, w + h.scan_ws[k],
                              h.scan_bytes, cs);
+        // the SMA's shared inputs (Q, E, z) are there from here on
+        if (st == DART_OK && (e = cudaStreamWaitEvent(cs, sma_ev, 0)) != cudaSuccess) return fail(e);
+        if (st == DART_OK && ng > 1) {
+            if ((e = dart::launch_gather_heads(w + h.z, gb + h.zg, (int64_t)rows, H, h0, h.hg, (int)ei, cs)) !=
+                cudaSuccess)
+                return fail(e);
+            zg = gb + h.zg;
+        }
         if (st == DART_OK)
             st = dart_sma_forward(&dg, gb + h.m, (const float*)(gb + h.rm), w + h.q, w + h.cm, w + h.e, zg,
                                   gb + h.yssd, gb + h.y, nullptr, nullptr, w + h.sma_ws[k], h.sma_bytes, cs);
