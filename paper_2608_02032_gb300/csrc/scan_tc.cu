@@ -349,9 +349,9 @@ struct SpSmem {
 };
 
 __global__ void __launch_bounds__(kSpThreads)
-state_passing_tc_kernel(const float* __restrict__ dH, const float* __restrict__ cum,
+state_passing_tc_kernel(const float* dH, const float* __restrict__ cum,
                         float* __restrict__ final_state, uint8_t* __restrict__ Hops,
-                        float* __restrict__ Hout, int H, int M, int S,
+                        float* Hout, int H, int M, int S,  // Hout may be dH (in place)
                         unsigned long long wait_limit_ns) {
     __shared__ __align__(128) SpSmem sm;
     constexpr int NP = kN * kP;
