@@ -22,7 +22,6 @@ import argparse
 import hashlib
 import json
 import re
-import math
 import os
 import statistics
 import subprocess

@@ -2,7 +2,6 @@
 dart_sma_backward) against the fp64 oracle's hand-derived backward, which the
 CPU tests pin by finite differences. Inputs come from the seeded generators;
 expected values from the oracle on the same (bf16-rounded) inputs."""
-import numpy as np
 import pytest
 import torch
 
