@@ -96,6 +96,25 @@ def test_chunked_scan_of_appendix_a_reproduces_recurrence(oracle_mod, L, S):
             assert _rel(Hlast[b, h], Hprev) < 1e-10
 
 
+def test_scan_outputs_are_linear_in_x(oracle_mod):
+    """For fixed dt, A, B, C the recurrence and the chunk memories are linear in X
+    (App. A): Y_ssd and M_j of a X1 + b X2 are a Y(X1) + b Y(X2) and the same for
+    the memories."""
+    d1 = _rng_inputs(15, 2, 24, 2, 1, 3, 5)
+    X2 = np.random.default_rng(115).standard_normal(d1["X"].shape)
+    a, b = 0.75, -1.5
+    args = (d1["dt"], d1["A"], d1["Bm"], d1["Cm"])
+    Y1, _ = oracle_mod.ssd_recurrence(d1["X"], *args)
+    Y2, _ = oracle_mod.ssd_recurrence(X2, *args)
+    Y3, _ = oracle_mod.ssd_recurrence(a * d1["X"] + b * X2, *args)
+    assert _rel(Y3, a * Y1 + b * Y2) < 1e-12
+    margs = (d1["dt"], d1["A"], d1["Bm"], 8)
+    M1 = oracle_mod.chunk_memories(d1["X"], *margs)
+    M2 = oracle_mod.chunk_memories(X2, *margs)
+    M3 = oracle_mod.chunk_memories(a * d1["X"] + b * X2, *margs)
+    assert _rel(M3, a * M1 + b * M2) < 1e-12
+
+
 def test_decayed_sum_of_memories_is_final_state(oracle_mod):
     """Unrolling App. A eq. (mamba2_chunk_state): H_{L-1} = sum_c A_{e(c)+1:L-1} dH_[c]."""
     L, S, H = 40, 8, 3
@@ -219,6 +238,19 @@ def test_sma_logits_are_scale_invariant_in_q_and_e(oracle_mod):
     R1, l1, g1 = oracle_mod.sma(dH, d["Q"], d["Cm"], d["E"], S, 1e-12, want_g=True)
     R2, l2, g2 = oracle_mod.sma(dH, 7.0 * d["Q"], d["Cm"], 0.25 * d["E"], S, 1e-12, want_g=True)
     assert np.max(np.abs(g1 - g2)) < 1e-9 and _rel(R2, R1) < 1e-9
+
+
+def test_sma_memory_scale_moves_values_not_routing(oracle_mod):
+    """The key path reads r (.) M_j, whose row scale r cancels a uniform scale of M_j
+    (App. B.1), while the value path reads M_j itself: scaling every memory by alpha
+    leaves the weights and lse unchanged (up to eps) and scales R by alpha."""
+    d, dH, S = _small_sma_case(seed=14)
+    alpha = 3.5
+    R1, l1, g1 = oracle_mod.sma(dH, d["Q"], d["Cm"], d["E"], S, 1e-30, want_g=True)
+    R2, l2, g2 = oracle_mod.sma(alpha * dH, d["Q"], d["Cm"], d["E"], S, 1e-30, want_g=True)
+    fin = np.isfinite(l1)
+    assert np.max(np.abs(g1 - g2)) < 1e-12 and np.max(np.abs(l1[fin] - l2[fin])) < 1e-12
+    assert _rel(R2, alpha * R1) < 1e-12
 
 
 def test_sma_is_causal_over_chunks(oracle_mod):
