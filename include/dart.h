@@ -94,7 +94,11 @@ typedef struct {
  * (in, mem, out): (F32, F32, F32), (BF16, F32, F32), (BF16, BF16, F32) and
  * (BF16, BF16, BF16). Accumulation is fp32 in every case. Outputs and
  * memories heavy-tailed enough that rounding them to bf16 costs several
- * percent of their RMS, so fp32 outputs are the default for bf16 inputs. */
+ * percent of their RMS, so fp32 outputs are the default for bf16 inputs.
+ * Size limits: (L / S) H <= 65535 * 64 and Bsz, H <= 65535 (refused with
+ * DART_ERR_UNSUPPORTED); on the tensor-core scan the output kernel's grid also
+ * needs (L / S) H / d <= 65535, d its heads per CTA (8 to 16), so past about
+ * a million (chunk, head) pairs dart_chunk_scan returns DART_ERR_CUDA. */
 
 typedef enum {
     DART_OP_CHUNK_SCAN = 0,
