@@ -192,11 +192,14 @@ def run_reference(args) -> None:
     world, rank, _ = _dist()
     if rank != 0:
         return
+    import oracle
     from paper_2608_02032_gb300.workloads import WORKLOADS, prefill_inputs
 
     w = WORKLOADS[PREFILL]
     inp = prefill_inputs(w)
-    heads = args.ref_heads
+    # one head per oracle thread: its recurrence and memories run over independent
+    # (batch, head) units, so fewer heads than threads would leave cores idle
+    heads = args.ref_heads or max(1, min(w.heads, oracle.num_threads()))
     for _ in range(args.warmup):
         oracle_sample(w, inp, heads)
     times = []
@@ -205,13 +208,15 @@ def run_reference(args) -> None:
         t, threads = oracle_sample(w, inp, heads)
         times.append(t)
     per_step = sum(times) / len(times)
-    # tokens/s of the full workload, extrapolated from the heads sampled
+    # tokens/s of the full workload: the sample covers heads / H of its (token, head) work
     value = w.tokens / (per_step * w.heads / heads)
-    sample = f"{heads} of {w.heads} heads, all {w.seqlen} tokens, full prefill path per step"
+    sample = (f"{heads} of {w.heads} heads, all {w.seqlen} tokens, full prefill path "
+              f"(recurrence, memories, SMA, merge) per step")
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s",
         "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
-        "ms_per_step": per_step * w.heads / heads * 1e3, "higher_is_better": True,
+        "ms_per_step": per_step * 1e3, "higher_is_better": True,
+        "ms_per_full_workload_extrapolated": per_step * w.heads / heads * 1e3,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "config": _config(w),
         "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": threads, "kind": "oracle",
@@ -355,15 +360,20 @@ def run_dart(args) -> None:
     # ---- training step (forward + backward)
     train = None
     if not args.no_train:
-        train = bench_train(args, dev, world, peaks, Bd, WORKLOADS[args.train_workload], prefill_inputs)
+        # the training workload is a sweep over the chunk size: one leg per S
+        train = [bench_train(args, dev, world, peaks, Bd, WORKLOADS[name], prefill_inputs)
+                 for name in args.train_workload.split(",")]
 
     # ---- CPU oracle on a bounded sample (rank 0, N = 1 only)
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        secs, threads = oracle_sample(w, inp, args.cpu_heads)
-        cpu = {"value": w.tokens / (secs * w.heads / args.cpu_heads), "unit": "tokens/s",
+        import oracle
+
+        ch = args.cpu_heads or max(1, min(w.heads, oracle.num_threads()))
+        secs, threads = oracle_sample(w, inp, ch)
+        cpu = {"value": w.tokens / (secs * w.heads / ch), "unit": "tokens/s",
                "cores": threads, "kind": "oracle",
-               "sample": f"{args.cpu_heads} of {w.heads} heads, all {w.seqlen} tokens, full "
+               "sample": f"{ch} of {w.heads} heads, all {w.seqlen} tokens, full "
                          f"prefill path (recurrence, memories, SMA, merge), {secs:.1f} s"}
 
     if rank == 0:
@@ -442,7 +452,9 @@ def bench_decode(args, dev, world, peaks, Bd, w, cache_slab, state_slab, token_i
             "roofline": {"kernel": "decode_step", "bound": "hbm", "achieved": gbs,
                          "peak": peaks["hbm"], "unit": "GB/s", "frac": gbs / peaks["hbm"],
                          "frac_of_nominal": gbs / NOMINAL_HBM_GBS,
-                         "peak_source": f"{peaks['source']} copy bandwidth", "traffic": None}}
+                         "peak_source": f"{peaks['source']} copy bandwidth",
+                         "traffic": _traffic_from_profiles("decode_step_decode_b64.md", "decode.cu")
+                         if w.name == DECODE else None}}
 
 
 def bench_train(args, dev, world, peaks, Bd, w, prefill_inputs):
@@ -519,11 +531,11 @@ def bench_train(args, dev, world, peaks, Bd, w, prefill_inputs):
                          "traffic": None}}
 
 
-def _traffic_from_profiles():
-    """DRAM bytes per SMA launch from the committed ncu summary, while the
+def _traffic_from_profiles(profile: str = "sma_forward_prefill_l16k.md", source: str = "sma_tc.cu"):
+    """DRAM bytes per launch of a kernel from its committed ncu summary, while the
     source hash recorded there matches the current kernel source (else null)."""
-    path = os.path.join(ROOT, "profiles", "sma_forward_prefill_l16k.md")
-    src = os.path.join(ROOT, "paper_2608_02032_gb300", "csrc", "sma_tc.cu")
+    path = os.path.join(ROOT, "profiles", profile)
+    src = os.path.join(ROOT, "paper_2608_02032_gb300", "csrc", source)
     try:
         with open(path) as f:
             text = f.read()
@@ -547,10 +559,13 @@ def main():
     ap.add_argument("--no-decode", action="store_true")
     ap.add_argument("--no-train", action="store_true")
     ap.add_argument("--decode-workload", default=DECODE, help="decode workload (a smaller one for profiling)")
-    ap.add_argument("--train-workload", default="train_b8_l4k_s256")
+    ap.add_argument("--train-workload", default="train_b8_l4k_s256,train_b8_l4k_s128",
+                    help="comma-separated training workloads (one leg each)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--cpu-heads", type=int, default=4, help="heads in the oracle CPU sample")
-    ap.add_argument("--ref-heads", type=int, default=1, help="heads per reference-arm step")
+    ap.add_argument("--cpu-heads", type=int, default=0,
+                    help="heads in the oracle CPU sample (default: one per oracle thread)")
+    ap.add_argument("--ref-heads", type=int, default=0,
+                    help="heads per reference-arm step (default: one per oracle thread)")
     ap.add_argument("--workload", default=PREFILL, help="prefill workload (smaller ones for profiling)")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "dart":

@@ -295,11 +295,17 @@ dart_status dart_chunk_scan_backward(const dart_dims* dims, const void* X, const
  * owns all other device memory; a latency-critical service that forbids
  * allocation after start-up (cudaMalloc and cudaFree can synchronise the
  * device); a process under a fixed device-memory budget.
- * It computes exactly what dart_sma_forward computes when rM is NULL. Its only
- * scratch, the inverse RMS of every memory row, lives in a fixed device array
- * of 2^20 fp32 values (4 MiB) inside the library, which every GPU that loads
- * the library holds until the process exits. It calls no cudaMalloc, no
- * cudaFree and no allocating library routine.
+ * It computes what dart_sma_forward computes when rM is NULL, with the same
+ * definitions, but always on the CUDA-core (FFMA) SMA kernel: there is no
+ * tensor-core path here. Its results therefore equal dart_sma_forward's bit for
+ * bit only on shapes that take the CUDA-core kernel there too; on the
+ * tensor-core shapes (bf16 inputs, P = 64, N = 128, S % 128 == 0, H/G even)
+ * they agree within the bf16-input tolerance (max|err| / RMS <= 2e-2), and the
+ * call is several times slower at long L. Its only scratch, the inverse RMS of
+ * every memory row, lives in a fixed device array of 2^20 fp32 values (4 MiB)
+ * inside the library, which every GPU that loads the library holds until the
+ * process exits. It calls no cudaMalloc, no cudaFree and no allocating library
+ * routine.
  * Arguments: as dart_sma_forward, without rM and the workspace. The caller
  * still passes (and owns) every input and output.
  * Limit: Bsz * (L / S) * H * N <= 2^20 memory rows (e.g. B1 H32 L16384 N128
@@ -307,7 +313,9 @@ dart_status dart_chunk_scan_backward(const dart_dims* dims, const void* X, const
  * is launched.
  * Set-up: the first call on a device looks up the array's device address on
  * that device (with that device current) and caches it; make that first call
- * before any stream capture. All calls share the array and it keeps the last
+ * before any stream capture. The cached address assumes the device context
+ * lives as long as the process: the library does not support cudaDeviceReset
+ * (or a primary-context release) between its calls. All calls share the array and it keeps the last
  * call's contents (every entry read is first written by the same call, so
  * nothing needs clearing). Calls that overlap on the GPU, on any streams,
  * race on the array: serialise them.

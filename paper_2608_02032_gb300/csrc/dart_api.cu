@@ -678,10 +678,11 @@ dart_status dart_chunk_scan_backward(const dart_dims* d, const void* X, const fl
 dart_status dart_get_device_status(void* stream) {
     cudaError_t e = cudaStreamSynchronize((cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(e);
-    const int code = dart::take_tc_status();
-    const int code2 = dart::take_scan_tc_status();
-    const int code3 = dart::take_bwd_tc_status();
-    const int code4 = dart::take_scan_bwd_tc_status();
+    cudaStream_t s = (cudaStream_t)stream;
+    const int code = dart::take_tc_status(s);
+    const int code2 = dart::take_scan_tc_status(s);
+    const int code3 = dart::take_bwd_tc_status(s);
+    const int code4 = dart::take_scan_bwd_tc_status(s);
     if (code < 0 || code2 < 0 || code3 < 0 || code4 < 0) return cuda_fail(cudaGetLastError());
     return (code != 0 || code2 != 0 || code3 != 0 || code4 != 0) ? DART_ERR_TIMEOUT : DART_OK;
 }

@@ -132,7 +132,7 @@ bool scan_tc_supported(const ScanArgs& a);
 template <typename Tmem, typename Tout>
 cudaError_t launch_chunk_scan_tc(const ScanArgs& a, unsigned long long wait_limit_ns,
                                  cudaStream_t stream);
-int take_scan_tc_status();
+int take_scan_tc_status(cudaStream_t stream);
 cudaError_t launch_scan_states_tc(const ScanArgs& a, float* cum, float* Hprev, uint8_t* Hops,
                                   unsigned long long wait_limit_ns, cudaStream_t stream);
 cudaError_t launch_scan_bwd_inter_tc(const ScanArgs& a, const float* cum, const void* dY, float* Z,
@@ -144,7 +144,7 @@ cudaError_t launch_scan_bwd_output_tc(const ScanArgs& a, const float* cum, const
 size_t scan_bwd_tc_workspace(int64_t B, int64_t L, int64_t H, int64_t S);
 cudaError_t launch_chunk_scan_backward_tc(const ScanBwdArgs& a, void* ws,
                                           unsigned long long wait_limit_ns, cudaStream_t stream);
-int take_scan_bwd_tc_status();
+int take_scan_bwd_tc_status(cudaStream_t stream);
 cudaError_t launch_scan_bwd_passing(float* ZD, const float* dM, const float* Hprev, const float* cum,
                                     float* dcum_end, uint8_t* Dops, int B, int H, int S, int Mc,
                                     int NP, cudaStream_t stream);
@@ -172,7 +172,7 @@ template <typename Tmem, typename Tout>
 cudaError_t launch_sma_forward_tc(const SmaArgs& a, void* ws, unsigned long long wait_limit_ns,
                                   cudaStream_t stream);
 // Reads and clears the tensor-core kernels' timeout code (0 = none, -1 = read failed).
-int take_tc_status();
+int take_tc_status(cudaStream_t stream);
 
 // Tensor-core SMA backward (sma_bwd_tc.cu; statistics pass in sma_tc.cu).
 template <typename Tmem>
@@ -189,6 +189,6 @@ size_t sma_bwd_tc_workspace(int64_t B, int64_t L, int64_t H, int64_t Mc, int64_t
 template <typename Tmem>
 cudaError_t launch_sma_backward_tc(const SmaBwdArgs& a, void* ws, unsigned long long wait_limit_ns,
                                    cudaStream_t stream);
-int take_bwd_tc_status();
+int take_bwd_tc_status(cudaStream_t stream);
 
 }  // namespace dart

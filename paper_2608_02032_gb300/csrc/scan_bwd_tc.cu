@@ -878,13 +878,20 @@ cudaError_t launch_chunk_scan_backward_tc(const ScanBwdArgs& a, void* ws,
     return cudaGetLastError();
 }
 
-int take_scan_bwd_tc_status() {
+// Read and clear of the status word in one device-side exchange: a code that a
+// kernel still running on another stream records is either returned now or kept
+// for the next read, never lost between a read and a separate clear.
+__device__ int g_sbwd_tc_status_taken;
+__global__ void take_scan_bwd_tc_status_kernel() { g_sbwd_tc_status_taken = atomicExch(&g_sbwd_tc_status, 0); }
+
+int take_scan_bwd_tc_status(cudaStream_t stream) {
+    take_scan_bwd_tc_status_kernel<<<1, 1, 0, stream>>>();
     int v = 0;
-    if (cudaMemcpyFromSymbol(&v, g_sbwd_tc_status, sizeof(int)) != cudaSuccess) return -1;
-    if (v != 0) {
-        const int zero = 0;
-        cudaMemcpyToSymbol(g_sbwd_tc_status, &zero, sizeof(int));
-    }
+    if (cudaGetLastError() != cudaSuccess ||
+        cudaMemcpyFromSymbolAsync(&v, g_sbwd_tc_status_taken, sizeof(int), 0, cudaMemcpyDeviceToHost, stream) !=
+            cudaSuccess ||
+        cudaStreamSynchronize(stream) != cudaSuccess)
+        return -1;
     return v;
 }
 

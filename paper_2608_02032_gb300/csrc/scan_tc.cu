@@ -942,13 +942,20 @@ template cudaError_t launch_chunk_scan_tc<float, float>(const ScanArgs&, unsigne
 template cudaError_t launch_chunk_scan_tc<bf16, float>(const ScanArgs&, unsigned long long, cudaStream_t);
 template cudaError_t launch_chunk_scan_tc<bf16, bf16>(const ScanArgs&, unsigned long long, cudaStream_t);
 
-int take_scan_tc_status() {
+// Read and clear of the status word in one device-side exchange: a code that a
+// kernel still running on another stream records is either returned now or kept
+// for the next read, never lost between a read and a separate clear.
+__device__ int g_scan_tc_status_taken;
+__global__ void take_scan_tc_status_kernel() { g_scan_tc_status_taken = atomicExch(&g_scan_tc_status, 0); }
+
+int take_scan_tc_status(cudaStream_t stream) {
+    take_scan_tc_status_kernel<<<1, 1, 0, stream>>>();
     int v = 0;
-    if (cudaMemcpyFromSymbol(&v, g_scan_tc_status, sizeof(int)) != cudaSuccess) return -1;
-    if (v != 0) {
-        const int zero = 0;
-        cudaMemcpyToSymbol(g_scan_tc_status, &zero, sizeof(int));
-    }
+    if (cudaGetLastError() != cudaSuccess ||
+        cudaMemcpyFromSymbolAsync(&v, g_scan_tc_status_taken, sizeof(int), 0, cudaMemcpyDeviceToHost, stream) !=
+            cudaSuccess ||
+        cudaStreamSynchronize(stream) != cudaSuccess)
+        return -1;
     return v;
 }
 

@@ -913,13 +913,20 @@ template cudaError_t launch_sma_backward_tc<float>(const SmaBwdArgs&, void*, uns
 template cudaError_t launch_sma_backward_tc<__nv_bfloat16>(const SmaBwdArgs&, void*, unsigned long long,
                                                            cudaStream_t);
 
-int take_bwd_tc_status() {
+// Read and clear of the status word in one device-side exchange: a code that a
+// kernel still running on another stream records is either returned now or kept
+// for the next read, never lost between a read and a separate clear.
+__device__ int g_bwd_tc_status_taken;
+__global__ void take_bwd_tc_status_kernel() { g_bwd_tc_status_taken = atomicExch(&g_bwd_tc_status, 0); }
+
+int take_bwd_tc_status(cudaStream_t stream) {
+    take_bwd_tc_status_kernel<<<1, 1, 0, stream>>>();
     int v = 0;
-    if (cudaMemcpyFromSymbol(&v, g_bwd_tc_status, sizeof(int)) != cudaSuccess) return -1;
-    if (v != 0) {
-        const int zero = 0;
-        cudaMemcpyToSymbol(g_bwd_tc_status, &zero, sizeof(int));
-    }
+    if (cudaGetLastError() != cudaSuccess ||
+        cudaMemcpyFromSymbolAsync(&v, g_bwd_tc_status_taken, sizeof(int), 0, cudaMemcpyDeviceToHost, stream) !=
+            cudaSuccess ||
+        cudaStreamSynchronize(stream) != cudaSuccess)
+        return -1;
     return v;
 }
 
