@@ -14,25 +14,32 @@
 // memory j for two heads of the same group: both heads' tiles side by side
 // make an N = 128 B operand.
 //
-// Precision. Rounding the memory operand to bf16 moves the logits enough to
-// break the 2e-2 parity bar, so W = r (.) M is split into bf16 hi + lo parts
-// (two MMA chains into one accumulator, ~2^-16 relative) and the value path
-// runs in fp16 on M / max|M_j| (scale re-applied in the epilogue). Q is exact
-// (bf16); C is widened to fp16 after a per-row power-of-two scale that puts
-// its largest entry in [2^14, 2^15), which is exact and keeps any bf16 row
-// inside the fp16 range (the scale is undone on R). Qbar's RMS scale and
-// Ebar stay fp32 in the epilogue.
+// Precision. Rounding the memory operand to one 16-bit type moves the logits
+// enough to break the 2e-2 parity bar (fp16: max|err|/RMS(Y) 1.6e-2 at L = 16K
+// in a CPU emulation against the oracle, bf16 far more), so W = r (.) M is
+// split into an fp16 part W16 and its residual 2^12 (W - W16) in e4m3: one
+// chain of eight fp16 MMAs (K = 16) and one of four e4m3 MMAs (K = 32, the
+// kind::f8f6f4 form) into the same accumulator, together ~2^-15 relative.
+// Their A operands are Q itself: fp16 after an exact per-row power-of-two
+// scale that puts its largest entry in [2^14, 2^15) (in TMEM), and e4m3 of
+// the same row scaled 2^-12 further (in shared memory), so both chains
+// accumulate Q W at one scale. The value path runs in fp16 on M / max|M_j|
+// (scale re-applied in the epilogue); C is widened to fp16 after the same kind
+// of row scale (undone on R). Qbar's RMS scale, the row scale and Ebar stay
+// fp32 in the epilogue. Emulated against the oracle at L = 16K, R and Y
+// carry the same error as a bf16 hi + lo split of W (~3e-3, set by the value
+// path); lse's error grows from 5e-6 to 1.6e-5.
 //
-// Cost model (measured on GB300, A in TMEM): a tcgen05.mma with M = 128,
-// K = 16 takes ~64 cycles at N = 128 and ~128 at N = 256, i.e. the full
-// 8192 flop/cycle/SM from N = 128 up. One job is three N = 128 chains of
-// eight MMAs (hi, lo into U; value into V): ~1536 cycles, fed by three
-// 32 KiB operand parts.
+// Cost model (measured on GB300): a tcgen05.mma with M = 128 takes ~64 cycles
+// at N = 128 (K = 16 for 16-bit operands, K = 32 for e4m3), i.e. the full
+// 8192 flop/cycle/SM. One job is twenty such MMAs (W16 and residual into U,
+// value into V), ~1280 cycles, fed by 80 KiB of operands.
 //
-// Kernel 1 (sma_operands_kernel) writes per (memory, pair of heads) the three
-// 32 KiB parts [W_hi h0 | W_hi h1], [W_lo h0 | W_lo h1], [M16 h0 | M16 h1],
-// already in the 128-byte-swizzled shared-memory layout, so each part is one
-// bulk copy.
+// Kernel 1 (sma_operands_kernel) writes per (memory, pair of heads) the
+// 32 KiB part [W16 h0 | W16 h1] (MN-major), the 16 KiB residual part (rows
+// h * 64 + p, K-major) and the 32 KiB part [M16 h0 | M16 h1], already in the
+// 128-byte-swizzled shared-memory layouts, contiguous, so a job's operands
+// are one bulk copy.
 // Kernel 2 (sma_tc_kernel), one CTA per (batch, 128-token tile, 2 heads),
 // grouped by (batch, head pair), heaviest tiles first inside a group:
 //   warp 0      producer: bulk copies of the parts into a 6-stage ring
@@ -44,23 +51,25 @@
 // of U and of V from TMEM, runs the online softmax (the running sum is only
 // rescaled when the maximum moves), and finally writes R = O / d, lse and
 // Y = Y_ssd + SiLU(z) R.
-// TMEM: [0,64) Q (bf16 pairs), [64,128) C (fp16 pairs), [128,256) U,
-// [256,384) and [384,512) V (two buffers, jobs alternate).
+// TMEM: [0,64) Q (fp16 pairs), [64,128) C (fp16 pairs), [128,256) U,
+// [256,384) and [384,512) V (two buffers, jobs alternate). Shared memory:
+// two 80 KiB job buffers and the 16 KiB e4m3 Q tile.
 //
 // Synchronisation, job j, b = j & 1. The MMA thread pays for barrier
 // operations with idle tensor cycles, and most for a wait right after a
 // commit (measured: ~100 cycles each time), so it does all of a job's waits
 // first and commits only between MMA chains: wait u_free (the epilogue has
 // read U of job j - 1), v_free[b] (it has read V of job j - 2) and the
-// job's parts (full[b], one copy), then hi, lo, commit uready[b], V into buffer b, commit
-// vready[b]. The producer refills stages 3b .. 3b+2 once job j - 2 is done
-// with them (uready[b], vready[b]); the epilogue reads U on uready[b] and V on
+// job's parts (full[b], one copy), then W16, residual, commit uready[b], V into buffer
+// b, commit vready[b]. The producer refills job buffer b once job j - 2 is done
+// with it (uready[b], vready[b]); the epilogue reads U on uready[b] and V on
 // vready[b]. Every barrier's waiter is at most one phase behind it, which the
 // parity waits need.
 #include <math.h>
 
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
+#include <cuda_fp8.h>
 
 #include "common.cuh"
 #include "kernels.h"
@@ -77,10 +86,17 @@ constexpr int kN = 128;
 constexpr int kHeadsPerCta = 2;
 constexpr int kTile = kN * kP * 2;            // bytes of one 16-bit N x P operand tile
 constexpr int kPart = kHeadsPerCta * kTile;   // one N = 128 B operand: both heads' tiles
-constexpr int kPartsPerJob = 3;               // W_hi, W_lo, M16
-constexpr int kPair = kPartsPerJob * kPart;   // operand bytes per (memory, head pair)
-constexpr int kStages = 6;                    // ring of kPart-sized stages: two jobs
-static_assert(kStages == 2 * kPartsPerJob, "stage of part p of job j is 3 (j & 1) + p");
+constexpr int kPartsPerJob = 3;               // backward layout parts: W_hi, W_lo, M16 (+ M_hi, M_lo)
+constexpr int kPair = kPartsPerJob * kPart;   // workspace bytes per (memory, head pair)
+constexpr int kStages = 6;                    // ring of kPart-sized stages (192 KiB)
+// forward layout, per (memory, head pair): [W16 h0 | W16 h1], the e4m3 residual
+// (128 rows h * 64 + p of 128 bytes n), [M16 h0 | M16 h1]
+constexpr int kLoPart = kHeadsPerCta * kP * kN;
+constexpr int kOffLo = kPart, kOffV = kPart + kLoPart;
+constexpr int kFwdJob = 2 * kPart + kLoPart;  // 80 KiB
+constexpr int kQ8Off = 2 * kFwdJob;           // the e4m3 Q tile (A of the residual chain) after two jobs
+static_assert(kQ8Off + kRows * kN <= kStages * kPart, "two job buffers and the Q tile fit the ring");
+static_assert(kFwdJob <= kPair, "the forward layout fits the workspace sized for the backward one");
 constexpr int kThreads = 384;
 // Register split: launched at 168 per thread (384 x 168 = 64512 of the 65536
 // of an SM); warpgroup 0 (producer, MMA, two idle warps) drops to 64 and the
@@ -93,13 +109,14 @@ constexpr uint32_t kTmemCols = 512;
 // coalesced) and row slots padded by 16 bytes (a lane's 16-byte accesses to
 // its own row then hit all 32 banks across the warp).
 constexpr int kSlots = 32 * (256 + 16);  // one warp's slots for rows of up to 256 bytes
-static_assert(8 * kSlots <= kPartsPerJob * kPart, "prologue slots fit stages 3..5");
+static_assert(kFwdJob + 8 * kSlots <= kQ8Off, "prologue slots fit job buffer 1");
 static_assert(16 * kSlots <= kStages * kPart, "merge slots fit the ring");
 constexpr uint32_t kColQ = 0, kColC = 64, kColU = 128, kColV = 256;  // V buffer b at kColV + 128 b
 // Bound on the final waits for this CTA's own copies and MMAs (never cut short).
 constexpr uint64_t kDrainLimitNs = 2000000000ull;
 
-constexpr uint32_t kIdescU = tc::idesc_f16(1, true, kRows, kHeadsPerCta * kP);  // bf16, N = 128
+constexpr uint32_t kIdescU = tc::idesc_f16(0, true, kRows, kHeadsPerCta * kP);  // fp16 W16, N = 128
+constexpr uint32_t kIdescLo = tc::idesc_e4m3(kRows, kHeadsPerCta * kP);         // e4m3 residual, N = 128
 constexpr uint32_t kIdescV = tc::idesc_f16(0, true, kRows, kHeadsPerCta * kP);  // fp16, N = 128
 
 // Byte offset of element (n, p) of a 128-row x 128-byte tile in the
@@ -111,9 +128,14 @@ __device__ __forceinline__ uint32_t sw128(int n, int p) {
 
 // ------------------------------------------------------------ kernel 1
 // One block of 256 threads per (j, h, b) memory. Warp w owns rows n = w + 8k;
-// lane owns columns p = lane, lane + 32. Head h = 2 hp + x writes its tile x
-// of each part of ops + ((b Mc + j) (H/2) + hp) pair_bytes: W_hi, W_lo, M16
-// and, when pair_bytes holds five parts (the backward), M split bf16 hi + lo.
+// lane owns columns p = lane, lane + 32. Head h = 2 hp + x writes its share of
+// the operands of memory j for the head pair hp:
+//   pair_bytes == 0 (forward and statistics pass): at ops + ((b Mc + j) (H/2) + hp) kFwdJob
+//     W16 tile x of [W16 h0 | W16 h1], rows x 64 .. x 64 + 63 of the e4m3 residual
+//     part (transposed through shared memory: K-major, the reduction index n along
+//     a row), and tile x of [M16 h0 | M16 h1];
+//   otherwise (the backward's layout, pair_bytes bytes per pair): tile x of each
+//     part W_hi, W_lo, M16 and, when pair_bytes holds five parts, M split bf16 hi + lo.
 template <typename Tmem>
 __global__ void __launch_bounds__(256)
 sma_operands_kernel(const Tmem* __restrict__ M, const float* __restrict__ rM,
@@ -125,11 +147,14 @@ sma_operands_kernel(const Tmem* __restrict__ M, const float* __restrict__ rM,
     const Tmem* src = M + mem * (kN * kP);
     const i64 pair = ((i64)b * Mc + j) * (H / kHeadsPerCta) + h / kHeadsPerCta;
     const int x = h % kHeadsPerCta;
-    uint8_t* dst_hi = ops + pair * pair_bytes + x * kTile;
-    uint8_t* dst_lo = dst_hi + kPart;
-    uint8_t* dst_v = dst_hi + 2 * kPart;
+    const bool fwd = pair_bytes == 0;
+    uint8_t* base = ops + pair * (fwd ? (i64)kFwdJob : (i64)pair_bytes);
+    uint8_t* dst_hi = base + x * kTile;                        // W16 or W_hi
+    uint8_t* dst_lo = fwd ? nullptr : dst_hi + kPart;          // W_lo (backward layout)
+    uint8_t* dst_v = fwd ? base + kOffV + x * kTile : dst_hi + 2 * kPart;
     uint8_t* dst_mb = pair_bytes > kPair ? dst_hi + 3 * kPart : nullptr;  // then + kPart: lo
     __shared__ float s_max[8];
+    __shared__ __align__(16) uint8_t s_res[kP][kN + 16];  // forward: e4m3 residual rows p, bytes n
 
     float v0[16], v1[16], rr[16];
     float amax = 0.0f;
@@ -161,25 +186,45 @@ sma_operands_kernel(const Tmem* __restrict__ M, const float* __restrict__ rM,
             const int p = lane + 32 * half;
             const float v = half ? v1[k] : v0[k];
             const float wv = rr[k] * v;
-            const __nv_bfloat16 hi = __float2bfloat16_rn(wv);
-            const __nv_bfloat16 lo = __float2bfloat16_rn(wv - __bfloat162float(hi));
-            const __half m16 = __float2half_rn(v * inv_s);
             const uint32_t o = sw128(n, p);
-            *reinterpret_cast<__nv_bfloat16*>(dst_hi + o) = hi;
-            *reinterpret_cast<__nv_bfloat16*>(dst_lo + o) = lo;
-            *reinterpret_cast<__half*>(dst_v + o) = m16;
-            if (dst_mb != nullptr) {
-                const __nv_bfloat16 mh = __float2bfloat16_rn(v);
-                *reinterpret_cast<__nv_bfloat16*>(dst_mb + o) = mh;
-                *reinterpret_cast<__nv_bfloat16*>(dst_mb + kPart + o) = __float2bfloat16_rn(v - __bfloat162float(mh));
+            *reinterpret_cast<__half*>(dst_v + o) = __float2half_rn(v * inv_s);
+            if (fwd) {
+                // |W| <= sqrt(P) (r normalises the row), so W16 needs no scale; the
+                // residual is at most 2^-11 |W| <= 2^-8, and 2^12 times it stays
+                // inside e4m3's range
+                const __half w16 = __float2half_rn(wv);
+                *reinterpret_cast<__half*>(dst_hi + o) = w16;
+                const __nv_fp8_e4m3 r8(4096.0f * (wv - __half2float(w16)));
+                s_res[p][n] = r8.__x;
+            } else {
+                const __nv_bfloat16 hi = __float2bfloat16_rn(wv);
+                *reinterpret_cast<__nv_bfloat16*>(dst_hi + o) = hi;
+                *reinterpret_cast<__nv_bfloat16*>(dst_lo + o) = __float2bfloat16_rn(wv - __bfloat162float(hi));
+                if (dst_mb != nullptr) {
+                    const __nv_bfloat16 mh = __float2bfloat16_rn(v);
+                    *reinterpret_cast<__nv_bfloat16*>(dst_mb + o) = mh;
+                    *reinterpret_cast<__nv_bfloat16*>(dst_mb + kPart + o) = __float2bfloat16_rn(v - __bfloat162float(mh));
+                }
             }
+        }
+    }
+    if (fwd) {
+        // the residual rows x 64 + p, 128 bytes each, in the 128-byte swizzle: 512 chunks of 16 bytes
+        __syncthreads();
+        uint8_t* dres = base + kOffLo;
+#pragma unroll
+        for (int i = 0; i < 2; ++i) {
+            const int c = threadIdx.x + 256 * i, p = c >> 3, q = c & 7;
+            const uint32_t row = (uint32_t)(x * kP + p);
+            *reinterpret_cast<uint4*>(dres + row * 128u + (((uint32_t)q ^ (row & 7u)) << 4)) =
+                *reinterpret_cast<const uint4*>(&s_res[p][q * 16]);
         }
     }
 }
 
 // ------------------------------------------------------------ kernel 2
 struct TcSmem {
-    uint8_t stage[kStages][kPart];  // 1024-aligned by placement
+    uint8_t ring[kStages * kPart];  // job buffers, the e4m3 Q tile, row staging; 1024-aligned by placement
     float lq[kRows];                // per-row logit factor 1 / (rms(Q_t) sqrt(N))
     float cdown[kRows];             // per-row power of two undoing C's scale
     uint64_t full[2];        // job j's three parts landed in stages 3b .. 3b+2 (producer -> MMA)
@@ -319,7 +364,7 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
               const __nv_bfloat16* __restrict__ E, const __nv_bfloat16* __restrict__ z,
               const Tout* __restrict__ Yssd, Tout* __restrict__ Y, Tout* __restrict__ R,
               float* __restrict__ lse, int Bsz, int L, int H, int G, int S, int Mc, float eps,
-              unsigned long long wait_limit_ns, int withhold, int pair_bytes, SmaStats st) {
+              unsigned long long wait_limit_ns, int withhold, SmaStats st) {
     extern __shared__ uint8_t smem_raw[];
     TcSmem& sm = *reinterpret_cast<TcSmem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                             ~(uintptr_t)1023);
@@ -371,17 +416,18 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
       asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegsLow));
       if (warp == 0) {
         // ------------------------------------------------------- producer
-        // one 96 KiB copy per job: part p of job j lands in stage 3 (j & 1) + p
+        // one copy per job (80 KiB; the statistics pass takes only W16 and the
+        // residual): job j lands in job buffer j & 1
         if (lane == 0) {
-            const uint8_t* src = ops + ((i64)b * Mc * hpairs + hp) * (i64)pair_bytes;
-            const i64 job_stride = (i64)hpairs * pair_bytes;
+            const uint8_t* src = ops + ((i64)b * Mc * hpairs + hp) * (i64)kFwdJob;
+            const i64 job_stride = (i64)hpairs * kFwdJob;
             bool ok = true;
             int njobs = 0;  // jobs whose copy was issued
             // (withhold: the failure-path test hook; every wait on the operands then runs out)
             for (int j = 0; j < (withhold ? 0 : nj); ++j) {
                 const int ub = j & 1;
-                // stages 3..5 hold the epilogue's row staging until the operands are in TMEM;
-                // stages 3b .. 3b+2 were last used by job j - 2: wait for its U and V
+                // job buffer 1 holds the epilogue's row staging until the operands are in TMEM;
+                // buffer j & 1 was last used by job j - 2: wait for its U and V
                 const uint32_t par = (uint32_t)((j >> 1) & 1) ^ 1u;
                 ok = (j != 1 || tc::mbar_wait(&sm.a_ready, 0, wait_limit_ns, abort)) &&
                      tc::mbar_wait(&sm.uready[ub], par, wait_limit_ns, abort) &&
@@ -390,10 +436,10 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
                     fail(abort, 1);
                     break;
                 }
-                // the job's hi, lo and value parts are contiguous in global and in the ring
-                constexpr uint32_t bytes = kStats ? 2 * kPart : kPair;
+                // the job's parts are contiguous in global and in the ring
+                constexpr uint32_t bytes = kStats ? kOffV : kFwdJob;
                 tc::mbar_arrive_expect_tx(&sm.full[ub], bytes);
-                tc::bulk_g2s(sm.stage[kPartsPerJob * ub], src + j * job_stride, bytes, &sm.full[ub]);
+                tc::bulk_g2s(sm.ring + ub * kFwdJob, src + j * job_stride, bytes, &sm.full[ub]);
                 ++njobs;
             }
             // never leave a copy in flight behind: wait for the last copy into each half
@@ -408,24 +454,29 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
             if (!ok) fail(abort, 2);
             tc::tc_fence_after();
             bool issued = false;
-            // descriptor of stage 0; stage st is kPart * st bytes further (>> 4 in the address field)
-            const uint64_t desc0 = tc::smem_desc_sw128(tc::smem_u32(sm.stage[0]), (uint32_t)kTile, 1024u);
+            // descriptors of job buffer 0 (MN-major W16 / M16, K-major residual) and of the
+            // e4m3 Q tile; buffer 1 is kFwdJob bytes further (>> 4 in the address field)
+            const uint64_t desc0 = tc::smem_desc_sw128(tc::smem_u32(sm.ring), (uint32_t)kTile, 1024u);
+            const uint64_t rdesc0 = tc::smem_desc_sw128(tc::smem_u32(sm.ring + kOffLo), 16u, 1024u);
+            const uint64_t qdesc = tc::smem_desc_sw128(tc::smem_u32(sm.ring + kQ8Off), 16u, 1024u);
             for (int j = 0; ok && j < nj; ++j) {
                 const int ub = j & 1;
-                const int s0 = kPartsPerJob * ub;  // stages of this job's parts: s0, s0 + 1, s0 + 2
                 const uint32_t par = (uint32_t)((j >> 1) & 1);
-                const uint64_t bd = desc0 + (uint64_t)((s0 * kPart) >> 4);
+                const uint64_t boff = (uint64_t)((ub * kFwdJob) >> 4);
+                const uint64_t bd = desc0 + boff;
                 ok = tc::mbar_wait(&sm.u_free, (uint32_t)ub ^ 1u, wait_limit_ns, abort) &&
                      (kStats || tc::mbar_wait(&sm.v_free[ub], par ^ 1u, wait_limit_ns, abort));
                 tc::tc_fence_after();
                 ok = ok && tc::mbar_wait(&sm.full[ub], par, wait_limit_ns, abort);
                 if (!ok) break;
                 issue_part<kIdescU, 0u>(tmem + kColU, tmem + kColQ, bd);
-                issue_part<kIdescU, 1u>(tmem + kColU, tmem + kColQ, bd + (uint64_t)(kPart >> 4));
+#pragma unroll
+                for (uint32_t ks = 0; ks < kN / 32; ++ks)  // residual chain: +32 bytes per K = 32 step
+                    tc::mma_e4m3_ss(tmem + kColU, qdesc + 2u * ks, rdesc0 + boff + 2u * ks, kIdescLo, 1u);
                 tc::mma_commit(&sm.uready[ub]);
                 if (!kStats) {
                     issue_part<kIdescV, 0u>(tmem + kColV + 128u * (uint32_t)ub, tmem + kColC,
-                                            bd + (uint64_t)((2 * kPart) >> 4));
+                                            bd + (uint64_t)(kOffV >> 4));
                     tc::mma_commit(&sm.vready[ub]);
                 }
                 issued = true;
@@ -450,9 +501,9 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
         const i64 tok = (i64)b * L + t;
         const int g = h0 / (H / G);
 
-        // Rows in through shared memory (stages 3..5 are not needed before job 1):
+        // Rows in through shared memory (job buffer 1 is not needed before job 1):
         // Q (warpgroup 0) or C (warpgroup 1), then E, 32 rows per warp.
-        uint8_t* slots = sm.stage[kPartsPerJob] + (warp - 4) * kSlots;
+        uint8_t* slots = sm.ring + kFwdJob + (warp - 4) * kSlots;
         const i64 tok0 = tok - lane;  // first token of this warp's rows
         uint4 av[16];
         uint32_t e2[kP / 2];  // the E row as bf16 pairs; Ebar = E * ie
@@ -469,6 +520,66 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
             const uint4 w = reinterpret_cast<const uint4*>(slots + lane * (2 * kP + 16))[u];
             e2[4 * u] = w.x; e2[4 * u + 1] = w.y; e2[4 * u + 2] = w.z; e2[4 * u + 3] = w.w;
         }
+        // The A operands: the row (Q for warpgroup 0, C for warpgroup 1) as fp16 after an
+        // exact power-of-two scale 2^k that puts its largest entry in [2^14, 2^15)
+        // (cmax = 1.f * 2^(ebits - 127), so k = 141 - ebits), into TMEM
+        float cmax = 0.0f, ssq = 0.0f;
+#pragma unroll
+        for (int u = 0; u < 16; ++u) {
+            const uint32_t cw[4] = {av[u].x, av[u].y, av[u].z, av[u].w};
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const float a = bf_lo(cw[e]), d = bf_hi(cw[e]);
+                cmax = fmaxf(cmax, fmaxf(fabsf(a), fabsf(d)));
+                ssq = fmaf(a, a, fmaf(d, d, ssq));
+            }
+        }
+        const int ebits = (__float_as_int(cmax) >> 23) & 0xff;
+        const int k = cmax > 0.0f ? min(max(141 - ebits, -60), 60) : 0;
+        const float up = __int_as_float((127 + k) << 23);
+        const float down = __int_as_float((127 - k) << 23);
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            uint32_t ca[16];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const uint32_t cw[4] = {av[c * 4 + u].x, av[c * 4 + u].y, av[c * 4 + u].z, av[c * 4 + u].w};
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const __half2 ch = __floats2half2_rn(bf_lo(cw[e]) * up, bf_hi(cw[e]) * up);
+                    ca[u * 4 + e] = *reinterpret_cast<const uint32_t*>(&ch);
+                }
+            }
+            tc::tmem_st16(tmem + lane_addr + (wg == 0 ? kColQ : kColC) + 16u * c, ca);
+        }
+        if (wg == 0) {
+            // Q also as e4m3 at scale 2^(k - 12) (largest entry in [4, 8)): row `row` of the
+            // residual chain's K-major A tile, 128 bytes in the 128-byte swizzle
+            const float up8 = __int_as_float((127 + k - 12) << 23);
+            uint8_t* qrow = sm.ring + kQ8Off + row * 128;
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {  // 16 entries n = 16 q .. 16 q + 15 per chunk
+                uint32_t w4[4];  // bytes in n order (the low half of a bf16 or e4m3 pair first)
+                const uint32_t wds[8] = {av[2 * q].x, av[2 * q].y, av[2 * q].z, av[2 * q].w,
+                                         av[2 * q + 1].x, av[2 * q + 1].y, av[2 * q + 1].z, av[2 * q + 1].w};
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const uint32_t p0 = (uint32_t)__nv_cvt_float2_to_fp8x2(
+                        make_float2(bf_lo(wds[2 * e]) * up8, bf_hi(wds[2 * e]) * up8), __NV_SATFINITE, __NV_E4M3);
+                    const uint32_t p1 = (uint32_t)__nv_cvt_float2_to_fp8x2(
+                        make_float2(bf_lo(wds[2 * e + 1]) * up8, bf_hi(wds[2 * e + 1]) * up8), __NV_SATFINITE,
+                        __NV_E4M3);
+                    w4[e] = (p0 & 0xffffu) | (p1 << 16);
+                }
+                *reinterpret_cast<uint4*>(qrow + (((uint32_t)q ^ ((uint32_t)row & 7u)) << 4)) =
+                    make_uint4(w4[0], w4[1], w4[2], w4[3]);
+            }
+            tc::fence_proxy_async_shared();  // the MMAs read the tile through the async proxy
+            // logit factor: 1 / (rms(Q_t) sqrt(N)), and the row scale undone
+            sm.lq[row] = rsqrtf(ssq / (float)kN + eps) * rsqrtf((float)kN) * down;
+        } else {
+            sm.cdown[row] = down;
+        }
         float sse = 0.0f;
 #pragma unroll
         for (int i = 0; i < kP / 2; ++i) {
@@ -479,54 +590,6 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
         uint64_t eb[kP / 2];  // Ebar row as fp32 pairs
 #pragma unroll
         for (int i = 0; i < kP / 2; ++i) eb[i] = f2_pack(bf_lo(e2[i]) * ie, bf_hi(e2[i]) * ie);
-        if (wg == 0) {
-            // A operand Q (bf16 pairs, exact) into TMEM; 1 / (rms(Q_t) sqrt(N)) to shared memory
-            float ssq = 0.0f;
-#pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                uint32_t qa[16];
-#pragma unroll
-                for (int u = 0; u < 4; ++u) {
-                    const uint32_t qw[4] = {av[c * 4 + u].x, av[c * 4 + u].y, av[c * 4 + u].z, av[c * 4 + u].w};
-#pragma unroll
-                    for (int e = 0; e < 4; ++e) {
-                        qa[u * 4 + e] = qw[e];
-                        const float a = bf_lo(qw[e]), d = bf_hi(qw[e]);
-                        ssq = fmaf(a, a, fmaf(d, d, ssq));
-                    }
-                }
-                tc::tmem_st16(tmem + lane_addr + kColQ + 16u * c, qa);
-            }
-            sm.lq[row] = rsqrtf(ssq / (float)kN + eps) * rsqrtf((float)kN);
-        } else {
-            // A operand C into TMEM as fp16 after an exact power-of-two row scale
-            float cmax = 0.0f;
-#pragma unroll
-            for (int u = 0; u < 16; ++u) {
-                const uint32_t cw[4] = {av[u].x, av[u].y, av[u].z, av[u].w};
-#pragma unroll
-                for (int e = 0; e < 4; ++e) cmax = fmaxf(cmax, fmaxf(fabsf(bf_lo(cw[e])), fabsf(bf_hi(cw[e]))));
-            }
-            // cmax = 1.f * 2^(ebits - 127): scale by 2^k with k = 141 - ebits puts it in [2^14, 2^15)
-            const int ebits = (__float_as_int(cmax) >> 23) & 0xff;
-            const int k = cmax > 0.0f ? min(max(141 - ebits, -60), 60) : 0;
-            const float up = __int_as_float((127 + k) << 23);
-            sm.cdown[row] = __int_as_float((127 - k) << 23);
-#pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                uint32_t ca[16];
-#pragma unroll
-                for (int u = 0; u < 4; ++u) {
-                    const uint32_t cw[4] = {av[c * 4 + u].x, av[c * 4 + u].y, av[c * 4 + u].z, av[c * 4 + u].w};
-#pragma unroll
-                    for (int e = 0; e < 4; ++e) {
-                        const __half2 ch = __floats2half2_rn(bf_lo(cw[e]) * up, bf_hi(cw[e]) * up);
-                        ca[u * 4 + e] = *reinterpret_cast<const uint32_t*>(&ch);
-                    }
-                }
-                tc::tmem_st16(tmem + lane_addr + kColC + 16u * c, ca);
-            }
-        }
         asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
         tc::tc_fence_before();
         tc::mbar_arrive(&sm.a_ready);
@@ -650,7 +713,7 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
                 constexpr int kRowB = kP * (int)sizeof(Tout);
                 const i64 rowo = tok * H + h;
                 const i64 row0 = tok0 * H + h;  // this warp's first output row
-                uint8_t* yslots = sm.stage[0] + (warp - 4) * 2 * kSlots;
+                uint8_t* yslots = sm.ring + (warp - 4) * 2 * kSlots;
                 uint8_t* rslots = yslots + kSlots;
                 const i64 rstride = (i64)H * kRowB;
                 const bool has = nj > 0;
@@ -715,7 +778,7 @@ cudaError_t launch_sma_forward_tc(const SmaArgs& a, void* ws, unsigned long long
     float* scale = (float*)(ops + (size_t)(a.B * Mc * (H / kHeadsPerCta)) * kPair);
     if (Mc > 1) {
         sma_operands_kernel<Tmem><<<dim3(Mc - 1, H, Bsz), 256, 0, stream>>>(
-            (const Tmem*)a.M, a.rM, ops, scale, Mc, H, a.eps, kPair);
+            (const Tmem*)a.M, a.rM, ops, scale, Mc, H, a.eps, 0);  // the forward layout
         note_launches(1);
     }
     const size_t smem = sizeof(TcSmem) + 1024;
@@ -728,7 +791,7 @@ cudaError_t launch_sma_forward_tc(const SmaArgs& a, void* ws, unsigned long long
                                             (const __nv_bfloat16*)a.z, (const Tout*)a.Yssd,
                                             (Tout*)a.Y, (Tout*)a.R, a.lse, Bsz, L, H, (int)a.G,
                                             (int)a.S, Mc, a.eps, wait_limit_ns, a.test_withhold,
-                                            kPair, SmaStats{a.logits, nullptr});
+                                            SmaStats{a.logits, nullptr});
     note_launches(1);
     return cudaGetLastError();
 }
@@ -738,9 +801,12 @@ cudaError_t launch_sma_bwd_stats_tc(const SmaBwdArgs& a, const float* rM, uint8_
                                     int pair_bytes, float* scale, float* g, float2* gd,
                                     unsigned long long wait_limit_ns, cudaStream_t stream) {
     const int Bsz = (int)a.B, L = (int)a.L, H = (int)a.H, Mc = (int)(a.L / a.S);
+    // the statistics pass recomputes the logits exactly as the forward did, from the
+    // forward's operand layout; the backward's own layout (pair_bytes per pair) then
+    // overwrites it for the kernels that follow
     if (Mc > 1) {
         sma_operands_kernel<Tmem><<<dim3(Mc - 1, H, Bsz), 256, 0, stream>>>(
-            (const Tmem*)a.M, rM, ops, scale, Mc, H, a.eps, pair_bytes);
+            (const Tmem*)a.M, rM, ops, scale, Mc, H, a.eps, 0);
         note_launches(1);
     }
     const size_t smem = sizeof(TcSmem) + 1024;
@@ -753,8 +819,13 @@ cudaError_t launch_sma_bwd_stats_tc(const SmaBwdArgs& a, const float* rM, uint8_
                                             (const __nv_bfloat16*)a.Cm, (const __nv_bfloat16*)a.E,
                                             (const __nv_bfloat16*)a.z, nullptr, nullptr, nullptr,
                                             const_cast<float*>(a.lse), Bsz, L, H, (int)a.G,
-                                            (int)a.S, Mc, a.eps, wait_limit_ns, 0, pair_bytes, st);
+                                            (int)a.S, Mc, a.eps, wait_limit_ns, 0, st);
     note_launches(1);
+    if (Mc > 1) {
+        sma_operands_kernel<Tmem><<<dim3(Mc - 1, H, Bsz), 256, 0, stream>>>(
+            (const Tmem*)a.M, rM, ops, scale, Mc, H, a.eps, pair_bytes);
+        note_launches(1);
+    }
     return cudaGetLastError();
 }
 template cudaError_t launch_sma_bwd_stats_tc<float>(const SmaBwdArgs&, const float*, uint8_t*, int,
