@@ -65,7 +65,7 @@ extern "C" {
 typedef enum {
     DART_OK = 0,
     DART_ERR_INVALID_ARG = 1,  /* NULL or misaligned pointer, bad dims, H % G != 0, eps <= 0 */
-    DART_ERR_UNSUPPORTED = 2,  /* valid but not built: L % S != 0, P/N/S outside the set below */
+    DART_ERR_UNSUPPORTED = 2,  /* valid but not built: P/N/S outside the set below, L % S != 0 where required */
     DART_ERR_WORKSPACE = 3,    /* workspace NULL/misaligned or smaller than dart_workspace_size */
     DART_ERR_CUDA = 4,         /* a CUDA call failed; see dart_last_cuda_error() */
     DART_ERR_TIMEOUT = 5,      /* a device-side wait gave up (see dart_get_device_status) */
@@ -82,7 +82,7 @@ typedef struct {
     int64_t ngroups;   /* G, must divide H */
     int64_t headdim;   /* P, value axis of a memory */
     int64_t dstate;    /* N, key axis of a memory (SSD state size) */
-    int64_t chunk;     /* S, chunk size; M = L / S memories per (b, h) */
+    int64_t chunk;     /* S, chunk size; M = ceil(L / S) memories per (b, h) */
     int32_t in_dtype;  /* dart_dtype of the token inputs X, B, C, Q, E, z and x, b, c, q, e, z */
     int32_t mem_dtype; /* dart_dtype of the chunk memories M and the decode cache */
     int32_t out_dtype; /* dart_dtype of the outputs Y_ssd, Y, R and the decode output y */
@@ -90,7 +90,12 @@ typedef struct {
 } dart_dims;
 
 /* Supported sizes: P in {16, 32, 64}, N in {16, 32, 64, 128},
- * S in {16, 32, 64, 128, 256} with L % S == 0. Supported dtype triples
+ * S in {16, 32, 64, 128, 256}. L need not be a multiple of S for
+ * dart_chunk_scan, dart_sma_forward and dart_prefill_host (M = ceil(L / S)
+ * memories; the last holds the partial chunk, e(c) = L - 1, which is the
+ * running partial memory a decode continues from); the backward calls,
+ * dart_sma_forward_with_logits and dart_sma_forward_noalloc need L % S == 0
+ * (DART_ERR_UNSUPPORTED otherwise). Supported dtype triples
  * (in, mem, out): (F32, F32, F32), (BF16, F32, F32), (BF16, BF16, F32) and
  * (BF16, BF16, BF16). Accumulation is fp32 in every case. Outputs and
  * memories heavy-tailed enough that rounding them to bf16 costs several
@@ -131,6 +136,10 @@ size_t dart_workspace_size(const dart_dims* dims, int op);
  *          rM (Bsz, M, H, N) fp32 or NULL: r[n] = (mean_p M[n, p]^2 + eps)^-1/2
  *          of the stored memory (App. B.1);
  *          final_state (Bsz, H, N, P) fp32 or NULL: H_{L-1}.
+ * Ragged L (L % S != 0): the kernels run on copies of the inputs zero-padded to
+ * ceil(L / S) S tokens inside the workspace (a padded token has dt = 0: decay 1,
+ * no write, so states and memories are exactly the L-token ones) and the first L
+ * rows of Y_ssd are copied out; dart_workspace_size includes the copies.
  */
 dart_status dart_chunk_scan(const dart_dims* dims, const void* X, const float* dt,
                             const float* A, const void* Bm, const void* Cm, void* Y_ssd,
@@ -154,7 +163,9 @@ dart_status dart_chunk_scan(const dart_dims* dims, const void* X, const float* d
  *          lse (Bsz, L, H) fp32 or NULL.
  * Workspace: dart_workspace_size(dims, DART_OP_SMA_FORWARD) bytes. Always
  *          needed on the tensor-core path (bf16 inputs, P = 64, N = 128,
- *          S % 128 == 0, H / G even), where it holds each memory's MMA
+ *          L a multiple of 128 after padding to whole chunks, H / G even; any S:
+ *          a 128-token tile spanning several chunks runs the memories of its
+ *          last token and each token keeps its own), where it holds each memory's MMA
  *          operands (48 KiB per memory and head); elsewhere only when rM is
  *          NULL (for r).
  */
@@ -247,7 +258,7 @@ dart_status dart_sma_backward(const dart_dims* dims, const void* M, const float*
  * dart_sma_forward that also writes logits (Bsz, H, M, L) fp32, the entry
  * (b, h, j, t) holding l_{t,j} for j < t / S (other entries unwritten); lse
  * is required. It needs the tensor-core path (bf16 inputs, P = 64, N = 128,
- * S % 128 == 0, H/G even) and gives DART_ERR_UNSUPPORTED elsewhere.
+ * L % 128 == 0, H/G even) and gives DART_ERR_UNSUPPORTED elsewhere.
  * dart_sma_backward_with_logits is dart_sma_backward with those logits: on
  * the tensor-core path the weights g come from them (the same values as the
  * recomputation, which it skips); the CUDA-core path recomputes them.
@@ -299,7 +310,7 @@ dart_status dart_chunk_scan_backward(const dart_dims* dims, const void* X, const
  * definitions, but always on the CUDA-core (FFMA) SMA kernel: there is no
  * tensor-core path here. Its results therefore equal dart_sma_forward's bit for
  * bit only on shapes that take the CUDA-core kernel there too; on the
- * tensor-core shapes (bf16 inputs, P = 64, N = 128, S % 128 == 0, H/G even)
+ * tensor-core shapes (bf16 inputs, P = 64, N = 128, L % 128 == 0, H/G even)
  * they agree within the bf16-input tolerance (max|err| / RMS <= 2e-2), and the
  * call is several times slower at long L. Its only scratch, the inverse RMS of
  * every memory row, lives in a fixed device array of 2^20 fp32 values (4 MiB)

@@ -41,7 +41,7 @@ def chunk_scan(X, dt, A, Bm, Cm, chunk: int, eps: float = 1e-6, final_state: boo
     G, N = Bm.shape[2], Bm.shape[3]
     code = _dtype_code(X)
     dims = B.make_dims(Bsz, L, H, G, P, N, chunk, code, mem_dtype, out_dtype, eps=eps)
-    M = L // chunk
+    M = -(-L // chunk)  # ceil: a ragged last chunk keeps its (partial) memory
     dev = X.device
     Y = torch.empty(X.shape, dtype=out_dtype, device=dev)
     Mem = torch.empty(Bsz, M, H, N, P, dtype=mem_dtype, device=dev)

@@ -67,7 +67,7 @@ template <typename I, typename M, typename O> struct DecodeL {
 };
 
 // Shared validation of the sizes in dims (without the op-specific parts).
-dart_status check_dims(const dart_dims* d, bool need_seqlen) {
+dart_status check_dims(const dart_dims* d, bool need_seqlen, bool ragged_ok = false) {
     if (d == nullptr) return DART_ERR_INVALID_ARG;
     if (d->batch <= 0 || d->nheads <= 0 || d->ngroups <= 0 || d->headdim <= 0 || d->dstate <= 0 ||
         d->chunk <= 0)
@@ -83,9 +83,9 @@ dart_status check_dims(const dart_dims* d, bool need_seqlen) {
     if (!(P == 16 || P == 32 || P == 64)) return DART_ERR_UNSUPPORTED;
     if (!(N == 16 || N == 32 || N == 64 || N == 128)) return DART_ERR_UNSUPPORTED;
     if (!(is_pow2(S) && S >= 16 && S <= 256)) return DART_ERR_UNSUPPORTED;
-    if (need_seqlen && d->seqlen % S != 0) return DART_ERR_UNSUPPORTED;
+    if (need_seqlen && d->seqlen % S != 0 && !ragged_ok) return DART_ERR_UNSUPPORTED;
     // every offset below is computed in 64-bit, but grid dimensions are 32-bit
-    if (need_seqlen && (d->seqlen / S) * d->nheads > 65535 * 64) return DART_ERR_UNSUPPORTED;
+    if (need_seqlen && (d->seqlen + S - 1) / S * d->nheads > 65535 * 64) return DART_ERR_UNSUPPORTED;
     if (d->batch > 65535 || d->nheads > 65535) return DART_ERR_UNSUPPORTED;
     return DART_OK;
 }
@@ -101,6 +101,7 @@ bool scan_uses_tc(const dart_dims* d) {
     return d->in_dtype == DART_BF16 && dart::scan_tc_supported(a);
 }
 
+// Workspace of the scan for L % S == 0.
 ScanWs scan_ws(const dart_dims* d) {
     const i64 M = d->seqlen / d->chunk;
     const size_t states = align256((size_t)(d->batch * M * d->nheads * d->dstate * d->headdim) *
@@ -138,10 +139,90 @@ bool sma_bwd_uses_tc(const dart_dims* d) {
     return d->in_dtype == DART_BF16 && dart::sma_bwd_tc_supported(sma_bwd_args(d));
 }
 
-size_t sma_ws(const dart_dims* d) {
+// Workspace of the SMA forward for L % S == 0.
+size_t sma_ws_aligned(const dart_dims* d) {
     const i64 M = d->seqlen / d->chunk;
     if (sma_uses_tc(d)) return align256(dart::sma_tc_workspace(d->batch, M, d->nheads));
     return align256((size_t)(d->batch * M * d->nheads * d->dstate) * sizeof(float));
+}
+
+// Ragged sequences (L % S != 0). The scan and SMA run unchanged on copies of their
+// token inputs zero-padded to Lp = ceil(L / S) S tokens. A padded token has dt = 0, so
+// its decay is exp(0 A) = 1 and its write term dt B^T X is zero: every state, the
+// final state and every memory are those of the L-token sequence (the last memory
+// holds the partial chunk, whose last token is L - 1), and the first L rows of each
+// output are the outputs. A padded token reads the memories of the chunks before it
+// like any other, but its outputs are dropped.
+bool is_ragged(const dart_dims* d) { return d->seqlen % d->chunk != 0; }
+dart_dims padded_dims(const dart_dims* d) {
+    dart_dims p = *d;
+    p.seqlen = (d->seqlen + d->chunk - 1) / d->chunk * d->chunk;
+    return p;
+}
+size_t dtype_size(int t) { return t == DART_F32 ? 4 : 2; }
+
+// Padded copies of the scan's inputs and output, then the aligned scan workspace.
+struct RaggedScanWs {
+    size_t x, dt, b, c, y, inner, inner_bytes, total;
+};
+RaggedScanWs ragged_scan_ws(const dart_dims* d) {
+    const dart_dims p = padded_dims(d);
+    const size_t rows = (size_t)(p.batch * p.seqlen), ei = dtype_size(d->in_dtype), eo = dtype_size(d->out_dtype);
+    RaggedScanWs w{};
+    size_t o = 0;
+    auto take = [&o](size_t bytes) { const size_t at = o; o += align256(bytes); return at; };
+    w.x = take(rows * d->nheads * d->headdim * ei);
+    w.dt = take(rows * d->nheads * 4);
+    w.b = take(rows * d->ngroups * d->dstate * ei);
+    w.c = take(rows * d->ngroups * d->dstate * ei);
+    w.y = take(rows * d->nheads * d->headdim * eo);
+    w.inner_bytes = scan_ws(&p).total;
+    w.inner = take(w.inner_bytes);
+    w.total = o;
+    return w;
+}
+size_t scan_ws_bytes(const dart_dims* d) { return is_ragged(d) ? ragged_scan_ws(d).total : scan_ws(d).total; }
+
+// Padded copies of the SMA forward's token inputs and outputs, then its aligned workspace.
+struct RaggedSmaWs {
+    size_t q, c, e, z, yssd, y, r, lse, inner, inner_bytes, total;
+};
+RaggedSmaWs ragged_sma_ws(const dart_dims* d) {
+    const dart_dims p = padded_dims(d);
+    const size_t rows = (size_t)(p.batch * p.seqlen), ei = dtype_size(d->in_dtype), eo = dtype_size(d->out_dtype);
+    RaggedSmaWs w{};
+    size_t o = 0;
+    auto take = [&o](size_t bytes) { const size_t at = o; o += align256(bytes); return at; };
+    w.q = take(rows * d->ngroups * d->dstate * ei);
+    w.c = take(rows * d->ngroups * d->dstate * ei);
+    w.e = take(rows * d->ngroups * d->headdim * ei);
+    w.z = take(rows * d->nheads * ei);
+    w.yssd = take(rows * d->nheads * d->headdim * eo);
+    w.y = take(rows * d->nheads * d->headdim * eo);
+    w.r = take(rows * d->nheads * d->headdim * eo);
+    w.lse = take(rows * d->nheads * 4);
+    w.inner_bytes = sma_ws_aligned(&p);
+    w.inner = take(w.inner_bytes);
+    w.total = o;
+    return w;
+}
+size_t sma_ws(const dart_dims* d) { return is_ragged(d) ? ragged_sma_ws(d).total : sma_ws_aligned(d); }
+
+// dst: Bsz blocks of rows_dst rows; src: Bsz blocks of rows_src <= rows_dst rows of row_bytes
+// each. Copies the rows and zeroes the rest of each block (pad) or copies the first
+// rows_dst rows of each source block (unpad, rows_dst <= rows_src).
+cudaError_t pad_rows(void* dst, const void* src, int64_t bsz, int64_t rows_src, int64_t rows_dst,
+                     size_t row_bytes, cudaStream_t s) {
+    cudaError_t e = cudaMemcpy2DAsync(dst, rows_dst * row_bytes, src, rows_src * row_bytes, rows_src * row_bytes,
+                                      (size_t)bsz, cudaMemcpyDeviceToDevice, s);
+    if (e != cudaSuccess || rows_dst == rows_src) return e;
+    return cudaMemset2DAsync((uint8_t*)dst + rows_src * row_bytes, rows_dst * row_bytes, 0,
+                             (rows_dst - rows_src) * row_bytes, (size_t)bsz, s);
+}
+cudaError_t unpad_rows(void* dst, const void* src, int64_t bsz, int64_t rows_src, int64_t rows_dst,
+                       size_t row_bytes, cudaStream_t s) {
+    return cudaMemcpy2DAsync(dst, rows_dst * row_bytes, src, rows_src * row_bytes, rows_dst * row_bytes,
+                             (size_t)bsz, cudaMemcpyDeviceToDevice, s);
 }
 
 std::atomic<unsigned long long> g_wait_limit_ns{2000000000ull};
@@ -170,7 +251,7 @@ struct HostLayout {
 HostLayout host_layout(const dart_dims* d) {
     HostLayout h{};
     const int64_t B = d->batch, L = d->seqlen, H = d->nheads, G = d->ngroups, P = d->headdim;
-    const int64_t N = d->dstate, M = L / d->chunk;
+    const int64_t N = d->dstate, M = (L + d->chunk - 1) / d->chunk;
     // groups of kHostGroupHeads heads (at most 64 groups), else the whole problem as one
     h.hg = (G == 1 && H > kHostGroupHeads && H % kHostGroupHeads == 0 && H / kHostGroupHeads <= 64)
                ? kHostGroupHeads
@@ -205,7 +286,7 @@ HostLayout host_layout(const dart_dims* d) {
     o = h.g0 + (size_t)h.groups * h.stride;
     dart_dims dg = *d;
     dg.nheads = h.hg;
-    h.scan_bytes = scan_ws(&dg).total;
+    h.scan_bytes = scan_ws_bytes(&dg);
     h.sma_bytes = sma_ws(&dg);
     for (int k = 0; k < 2; ++k) {
         h.scan_ws[k] = take(h.scan_bytes);
@@ -275,15 +356,15 @@ int dart_last_cuda_error(void) { return t_last_cuda_error; }
 size_t dart_workspace_size(const dart_dims* d, int op) {
     switch (op) {
         case DART_OP_CHUNK_SCAN:
-            if (check_dims(d, true) != DART_OK) return 0;
-            return scan_ws(d).total;
+            if (check_dims(d, true, true) != DART_OK) return 0;
+            return scan_ws_bytes(d);
         case DART_OP_SMA_FORWARD:
-            if (check_dims(d, true) != DART_OK) return 0;
+            if (check_dims(d, true, true) != DART_OK) return 0;
             return sma_ws(d);
         case DART_OP_DECODE_STEP:
             return 0;
         case DART_OP_PREFILL_HOST:
-            if (check_dims(d, true) != DART_OK) return 0;
+            if (check_dims(d, true, true) != DART_OK) return 0;
             return host_layout(d).total;
         case DART_OP_SMA_BACKWARD:
             if (check_dims(d, true) != DART_OK) return 0;
@@ -309,13 +390,33 @@ size_t dart_workspace_size(const dart_dims* d, int op) {
 dart_status dart_chunk_scan(const dart_dims* d, const void* X, const float* dt, const float* A,
                             const void* Bm, const void* Cm, void* Y_ssd, void* M, float* rM,
                             float* final_state, void* ws, size_t ws_bytes, void* stream) {
-    dart_status st = check_dims(d, true);
+    dart_status st = check_dims(d, true, true);
     if (st != DART_OK) return st;
     const void* req[] = {X, dt, A, Bm, Cm, Y_ssd, M};
     for (const void* p : req)
         if (p == nullptr || !aligned16(p)) return DART_ERR_INVALID_ARG;
     if ((rM && !aligned16(rM)) || (final_state && !aligned16(final_state)))
         return DART_ERR_INVALID_ARG;
+    if (is_ragged(d)) {  // zero-padded copies, the aligned scan, the first L rows of Y_ssd
+        const RaggedScanWs w = ragged_scan_ws(d);
+        if (ws == nullptr || ((uintptr_t)ws & 255u) != 0 || ws_bytes < w.total) return DART_ERR_WORKSPACE;
+        const dart_dims p = padded_dims(d);
+        uint8_t* b = (uint8_t*)ws;
+        cudaStream_t s = (cudaStream_t)stream;
+        const size_t ei = dtype_size(d->in_dtype), eo = dtype_size(d->out_dtype);
+        const int64_t L = d->seqlen, Lp = p.seqlen, H = d->nheads, P = d->headdim, GN = d->ngroups * d->dstate;
+        cudaError_t e;
+        if ((e = pad_rows(b + w.x, X, d->batch, L, Lp, H * P * ei, s)) != cudaSuccess ||
+            (e = pad_rows(b + w.dt, dt, d->batch, L, Lp, H * 4, s)) != cudaSuccess ||
+            (e = pad_rows(b + w.b, Bm, d->batch, L, Lp, GN * ei, s)) != cudaSuccess ||
+            (e = pad_rows(b + w.c, Cm, d->batch, L, Lp, GN * ei, s)) != cudaSuccess)
+            return cuda_fail(e);
+        st = dart_chunk_scan(&p, b + w.x, (const float*)(b + w.dt), A, b + w.b, b + w.c, b + w.y, M, rM,
+                             final_state, b + w.inner, w.inner_bytes, stream);
+        if (st != DART_OK) return st;
+        e = unpad_rows(Y_ssd, b + w.y, d->batch, Lp, L, H * P * eo, s);
+        return e == cudaSuccess ? DART_OK : cuda_fail(e);
+    }
     const ScanWs w = scan_ws(d);
     if (ws == nullptr || ((uintptr_t)ws & 255u) != 0 || ws_bytes < w.total)
         return DART_ERR_WORKSPACE;
@@ -325,6 +426,7 @@ dart_status dart_chunk_scan(const dart_dims* d, const void* X, const float* dt, 
     a.P = d->headdim; a.N = d->dstate; a.S = d->chunk; a.eps = d->eps;
     a.X = X; a.dt = dt; a.A = A; a.Bm = Bm; a.Cm = Cm; a.Y = Y_ssd; a.M = M; a.rM = rM;
     a.final_state = final_state;
+    a.test_withhold = g_test_withhold.load();
     a.cum = (float*)((char*)ws + w.cum_off);
     a.dH32 = (float*)((char*)ws + w.dh_off);
     cudaStream_t s = (cudaStream_t)stream;
@@ -349,7 +451,7 @@ static dart_status sma_forward_impl(const dart_dims* d, const void* M, const flo
                                     const void* Cm, const void* E, const void* z, const void* Y_ssd,
                                     void* Y, void* R, float* lse, float* logits, void* ws,
                                     size_t ws_bytes, void* stream) {
-    dart_status st = check_dims(d, true);
+    dart_status st = check_dims(d, true, logits == nullptr);
     if (st != DART_OK) return st;
     const void* req[] = {M, Q, Cm, E, z, Y_ssd, Y};
     for (const void* p : req)
@@ -357,9 +459,35 @@ static dart_status sma_forward_impl(const dart_dims* d, const void* M, const flo
     if ((rM && !aligned16(rM)) || (R && !aligned16(R)) || (lse && !aligned16(lse)) ||
         (logits && !aligned16(logits)))
         return DART_ERR_INVALID_ARG;
+    if (is_ragged(d)) {  // zero-padded copies, the aligned call, the first L rows of each output
+        const RaggedSmaWs w = ragged_sma_ws(d);
+        if (ws == nullptr || ((uintptr_t)ws & 255u) != 0 || ws_bytes < w.total) return DART_ERR_WORKSPACE;
+        const dart_dims p = padded_dims(d);
+        uint8_t* b = (uint8_t*)ws;
+        cudaStream_t s = (cudaStream_t)stream;
+        const size_t ei = dtype_size(d->in_dtype), eo = dtype_size(d->out_dtype);
+        const int64_t L = d->seqlen, Lp = p.seqlen, H = d->nheads, P = d->headdim, G = d->ngroups;
+        const size_t nrow = (size_t)(G * d->dstate) * ei, erow = (size_t)(G * P) * ei, yrow = (size_t)(H * P) * eo;
+        cudaError_t e;
+        if ((e = pad_rows(b + w.q, Q, d->batch, L, Lp, nrow, s)) != cudaSuccess ||
+            (e = pad_rows(b + w.c, Cm, d->batch, L, Lp, nrow, s)) != cudaSuccess ||
+            (e = pad_rows(b + w.e, E, d->batch, L, Lp, erow, s)) != cudaSuccess ||
+            (e = pad_rows(b + w.z, z, d->batch, L, Lp, (size_t)H * ei, s)) != cudaSuccess ||
+            (e = pad_rows(b + w.yssd, Y_ssd, d->batch, L, Lp, yrow, s)) != cudaSuccess)
+            return cuda_fail(e);
+        st = sma_forward_impl(&p, M, rM, b + w.q, b + w.c, b + w.e, b + w.z, b + w.yssd, b + w.y,
+                              R ? b + w.r : nullptr, lse ? (float*)(b + w.lse) : nullptr, nullptr, b + w.inner,
+                              w.inner_bytes, stream);
+        if (st != DART_OK) return st;
+        if ((e = unpad_rows(Y, b + w.y, d->batch, Lp, L, yrow, s)) != cudaSuccess ||
+            (R && (e = unpad_rows(R, b + w.r, d->batch, Lp, L, yrow, s)) != cudaSuccess) ||
+            (lse && (e = unpad_rows(lse, b + w.lse, d->batch, Lp, L, (size_t)H * 4, s)) != cudaSuccess))
+            return cuda_fail(e);
+        return DART_OK;
+    }
     const bool tc = sma_uses_tc(d);
     if (logits != nullptr && !tc) return DART_ERR_UNSUPPORTED;  // saved by the tensor-core kernel only
-    const size_t need = (tc || rM == nullptr) ? sma_ws(d) : 0;
+    const size_t need = (tc || rM == nullptr) ? sma_ws_aligned(d) : 0;
     if (need > 0 && (ws == nullptr || ((uintptr_t)ws & 255u) != 0 || ws_bytes < need))
         return DART_ERR_WORKSPACE;
 
@@ -418,7 +546,7 @@ dart_status dart_sma_forward_with_logits(const dart_dims* d, const void* M, cons
 dart_status dart_prefill_host(const dart_dims* d, const void* X, const float* dt, const float* A,
                               const void* Bm, const void* Cm, const void* Q, const void* E,
                               const void* z, void* Y, void* ws, size_t ws_bytes, void* stream) {
-    dart_status st = check_dims(d, true);
+    dart_status st = check_dims(d, true, true);
     if (st != DART_OK) return st;
     const void* req[] = {X, dt, A, Bm, Cm, Q, E, z, Y};
     for (const void* p : req)
@@ -606,6 +734,7 @@ static dart_status sma_backward_impl(const dart_dims* d, const void* M, const fl
     a.M = M; a.rM = rM; a.Q = Q; a.Cm = Cm; a.E = E; a.z = z; a.lse = lse; a.dY = dY;
     a.dM = dM; a.dQ = dQ; a.dC = dC; a.dE = dE; a.dz = dz;
     a.logits = logits;  // the CUDA-core path recomputes the logits and ignores them
+    a.test_withhold = g_test_withhold.load();
     cudaStream_t s = (cudaStream_t)stream;
     typedef __nv_bfloat16 bf;
     cudaError_t e;
@@ -664,6 +793,7 @@ dart_status dart_chunk_scan_backward(const dart_dims* d, const void* X, const fl
     f.X = X; f.dt = dt; f.A = A; f.Bm = Bm; f.Cm = Cm;
     a.dY = dY; a.dM = dM; a.dX = dX; a.ddt = ddt; a.dA = dA; a.dB = dB; a.dC = dC;
     a.accumulate_dC = true;
+    f.test_withhold = g_test_withhold.load();
     cudaStream_t s = (cudaStream_t)stream;
     cudaError_t e;
     if (d->in_dtype == DART_F32)

@@ -33,6 +33,7 @@ struct ScanArgs {
     // optional (tensor-core path): the states entering each chunk as bf16 hi | lo
     // tiles in the 128-byte-swizzled shared-memory layout, 32 KiB per (b, c, h)
     uint8_t* Hops;
+    int test_withhold = 0;  // tensor-core path: the state passing issues no copies (failure-path test hook)
 };
 
 struct SmaArgs {
@@ -88,6 +89,7 @@ struct SmaBwdArgs {
     float* dE;  // B x L x G x P (overwritten)
     float* dz;  // B x L x H (overwritten)
     const float* logits = nullptr;  // the forward's logits (B x H x Mc x L) or null: recomputed
+    int test_withhold = 0;  // tensor-core path: the row kernels issue no operand copies (test hook)
 };
 
 // Backward of the chunked scan (scan_bwd.cu). Gradients are fp32.

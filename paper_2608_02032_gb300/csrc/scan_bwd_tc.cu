@@ -646,7 +646,7 @@ __global__ void __launch_bounds__(kBpThreads)
 bwd_passing_tc_kernel(const float* __restrict__ Z, const float* __restrict__ dM,
                       const float* __restrict__ Hprev, const float* __restrict__ cum,
                       float* __restrict__ dcum_end, uint8_t* __restrict__ Dops, int H, int S, int Mc,
-                      unsigned long long wait_limit_ns) {
+                      unsigned long long wait_limit_ns, int withhold) {
     extern __shared__ uint8_t smem_raw[];
     BpSmem& sm = *reinterpret_cast<BpSmem*>((reinterpret_cast<uintptr_t>(smem_raw) + 127) & ~(uintptr_t)127);
     constexpr int NP = kN * kP;
@@ -676,7 +676,8 @@ bwd_passing_tc_kernel(const float* __restrict__ Z, const float* __restrict__ dM,
         if (dM != nullptr) tc::bulk_g2s(sm.m[stg], dM + off, (uint32_t)(kBpSlab * 4), &sm.full[stg]);
         ++issued;
     };
-    if (tid == 0)
+    // (withhold: the failure-path test hook; every wait on the slabs then runs out)
+    if (tid == 0 && !withhold)
         for (int k = 0; k < min(kBpStages, Mc); ++k) issue(k);
     float adj[kBpElems] = {0.0f, 0.0f, 0.0f, 0.0f};
     bool ok = true;
@@ -728,7 +729,7 @@ bwd_passing_tc_kernel(const float* __restrict__ Z, const float* __restrict__ dM,
             float sum = 0.0f;
             for (int w = 0; w < kBpThreads / 32; ++w) sum += sm.red[w];
             atomicAdd(dcum_end + ((i64)b * H + h) * Mc + c, sum);
-            if (k + kBpStages < Mc) issue(k + kBpStages);
+            if (!withhold && k + kBpStages < Mc) issue(k + kBpStages);
         }
         __syncthreads();  // red is reused by the next step
     }
@@ -842,7 +843,7 @@ cudaError_t launch_chunk_scan_backward_tc(const ScanBwdArgs& a, void* ws,
                                       (int)smem)) != cudaSuccess)
             return e;
         bwd_passing_tc_kernel<<<dim3(NP / kBpSlab, H, B), kBpThreads, smem, stream>>>(
-            ZD, a.dM, Hprev, cum, dcum_end, Dops, H, S, Mc, wait_limit_ns);
+            ZD, a.dM, Hprev, cum, dcum_end, Dops, H, S, Mc, wait_limit_ns, a.fwd.test_withhold);
         note_launches(1);
     }
     if ((e = launch_scan_bwd_output_tc(f, cum, Hops, Dops, a.dY, rowI, a.dX, xi, wait_limit_ns,

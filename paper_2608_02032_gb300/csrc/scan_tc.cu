@@ -352,7 +352,7 @@ __global__ void __launch_bounds__(kSpThreads)
 state_passing_tc_kernel(const float* dH, const float* __restrict__ cum,
                         float* __restrict__ final_state, uint8_t* __restrict__ Hops,
                         float* Hout, int H, int M, int S,  // Hout may be dH (in place)
-                        unsigned long long wait_limit_ns) {
+                        unsigned long long wait_limit_ns, int withhold) {
     __shared__ __align__(128) SpSmem sm;
     constexpr int NP = kN * kP;
     const int slab = blockIdx.x, h = blockIdx.y, b = blockIdx.z, tid = threadIdx.x;
@@ -376,7 +376,8 @@ state_passing_tc_kernel(const float* dH, const float* __restrict__ cum,
         tc::bulk_g2s(sm.slab[stg], src + (i64)c * cstride, (uint32_t)(kSpSlab * 4), &sm.full[stg]);
         ++issued;
     };
-    if (tid == 0)
+    // (withhold: the failure-path test hook; every wait on the slabs then runs out)
+    if (tid == 0 && !withhold)
         for (int c = 0; c < min(kSpStages, M); ++c) issue(c);
     float st[kSpElems] = {0.0f, 0.0f, 0.0f, 0.0f};
     bool ok = true;
@@ -420,7 +421,7 @@ state_passing_tc_kernel(const float* dH, const float* __restrict__ cum,
         // every thread has read the stage (and the decays) before it is refilled
         ok = __syncthreads_and(got ? 1 : 0) != 0;
         if (!ok) break;
-        if (tid == 0 && c + kSpStages < M) issue(c + kSpStages);
+        if (tid == 0 && !withhold && c + kSpStages < M) issue(c + kSpStages);
     }
     if (!ok && tid == 0) {  // let the copies in flight land before the CTA exits
         for (int k = c; k < issued; ++k)
@@ -848,7 +849,7 @@ cudaError_t launch_chunk_scan_tc(const ScanArgs& a, unsigned long long wait_limi
     // fp32 memories are the chunk states themselves: the state passing reads them
     state_passing_tc_kernel<<<dim3(kN * kP / kSpSlab, H, B), kSpThreads, 0, stream>>>(
         mem_is_f32 ? (const float*)a.M : a.dH32, a.cum, a.final_state, a.Hops, nullptr, H, M, S,
-        wait_limit_ns);
+        wait_limit_ns, a.test_withhold);
     {
         auto kern = chunk_output_tc_kernel<Tout>;
         const size_t smem = sizeof(OutSmem) + 1024;
@@ -883,7 +884,7 @@ cudaError_t launch_scan_states_tc(const ScanArgs& a0, float* cum, float* Hprev, 
         (const __nv_bfloat16*)a.X, a.dt, a.cum, (const __nv_bfloat16*)a.Bm, nullptr, Hprev, nullptr,
         L, H, G, S, M, a.eps, wait_limit_ns);
     state_passing_tc_kernel<<<dim3(kN * kP / kSpSlab, H, B), kSpThreads, 0, stream>>>(
-        Hprev, a.cum, nullptr, Hops, Hprev, H, M, S, wait_limit_ns);
+        Hprev, a.cum, nullptr, Hops, Hprev, H, M, S, wait_limit_ns, 0);
     note_launches(2);
     return cudaGetLastError();
 }

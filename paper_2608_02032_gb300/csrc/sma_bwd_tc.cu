@@ -210,7 +210,7 @@ sma_bwd_rows_kernel(const uint8_t* __restrict__ ops, const __nv_bfloat16* __rest
                     float* __restrict__ sdl, float2* __restrict__ gd, float2* __restrict__ rs,
                     float* __restrict__ dQC, float* __restrict__ dE, float* __restrict__ dz,
                     const __nv_bfloat16* __restrict__ Cm, int Bsz, int L, int H, int S, int Mc,
-                    float eps, unsigned long long wait_limit_ns) {
+                    float eps, unsigned long long wait_limit_ns, int withhold) {
     extern __shared__ uint8_t smem_raw[];
     RowsSmem& sm = *reinterpret_cast<RowsSmem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                 ~(uintptr_t)1023);
@@ -256,7 +256,8 @@ sma_bwd_rows_kernel(const uint8_t* __restrict__ ops, const __nv_bfloat16* __rest
             bool ok = true;
             int issued = 0;
             const int part0 = kDQ ? 0 : 3;  // W_hi, W_lo or M_hi, M_lo (contiguous)
-            for (int k = 0; k < njobs; ++k) {
+            // (withhold: the failure-path test hook; every wait on the operands then runs out)
+            for (int k = 0; k < (withhold ? 0 : njobs); ++k) {
                 const int sb = k & 1, hp = hp_lo + k / nj, j = k % nj;
                 const uint32_t par = (uint32_t)((k >> 1) & 1) ^ 1u;
                 // stage 1 and the A buffers hold the prologue's row staging until a_ready
@@ -891,7 +892,7 @@ cudaError_t launch_sma_backward_tc(const SmaBwdArgs& a, void* ws, unsigned long 
         k<<<Bsz * (L / kRows) * kRowSplit, kRowsThreads, smem_rows, stream>>>(
             ops, (const __nv_bfloat16*)a.Q, (const __nv_bfloat16*)a.E, (const __nv_bfloat16*)a.z,
             (const __nv_bfloat16*)a.dY, gbuf, sdl, gd, rs, pass == 0 ? a.dC : a.dQ, a.dE, a.dz,
-            (const __nv_bfloat16*)a.Cm, Bsz, L, H, S, Mc, a.eps, wait_limit_ns);
+            (const __nv_bfloat16*)a.Cm, Bsz, L, H, S, Mc, a.eps, wait_limit_ns, a.test_withhold);
         note_launches(1);
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
     }

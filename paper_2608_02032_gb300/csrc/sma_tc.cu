@@ -67,6 +67,8 @@
 // parity waits need.
 #include <math.h>
 
+#include <type_traits>
+
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 #include <cuda_fp8.h>
@@ -382,9 +384,10 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
     const int hp = grp % hpairs;
     const int h0 = hp * kHeadsPerCta;
     const int t0 = tt * kRows;
-    // S is a multiple of the tile height, so every token of the tile lies in
-    // chunk t0 / S and sees exactly the memories j < t0 / S.
-    const int nj = t0 / S;
+    // The tile runs the jobs of its last token, j < (t0 + 127) / S; each token keeps
+    // those of its own history, j < t / S (all of them when S is a multiple of the
+    // tile height: the tile then lies in one chunk).
+    const int nj = (t0 + kRows - 1) / S;
     volatile int* abort = &sm.abort;
 
     if (threadIdx.x == 0) {
@@ -607,6 +610,7 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
             bool ok = true;
             const uint32_t ua = tmem + lane_addr + kColU + (uint32_t)(kP * wg);
             float* gp = st.g + ((i64)b * H + h) * Mc * L + t;  // + j L
+            const int njr = t / S;  // this row's memories
             for (int j = 0; j < nj; ++j) {
                 const int ub = j & 1;
                 if (!warp_wait(&sm.uready[ub], (uint32_t)((j >> 1) & 1), wait_limit_ns, abort)) {
@@ -629,9 +633,11 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
                     f2_unpack(acc, lx, ly);
                     l = __fmul_rn(lx + ly, lfac);  // rounded: the stored and the recomputed logits agree
                 }
-                const float gw = expf(l - lse_t);
-                G1 += gw;
-                gp[(i64)j * L] = gw;
+                if (j < njr) {
+                    const float gw = expf(l - lse_t);
+                    G1 += gw;
+                    gp[(i64)j * L] = gw;
+                }
             }
             if (ok) st.gd[rowo] = make_float2(G1, 0.0f);
         } else {
@@ -640,6 +646,7 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
             for (int i = 0; i < kP / 2; ++i) O[i] = 0ull;
             float m = -INFINITY, dsum = 0.0f;
             bool ok = true;
+            const int njr = t / S;  // this row's memories (the tile's jobs beyond them are skipped)
             const float* scl = scale + (i64)b * Mc * H + h;  // scale of memory j at scl[j H]
             float s_next = nj > 0 ? __ldg(scl) : 0.0f;
             const uint32_t ua = tmem + lane_addr + kColU + (uint32_t)(kP * wg);
@@ -650,62 +657,72 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
             const i64 rowo_pf = tok * H + h;
             const int pf_job = nj > 4 ? nj - 4 : 0;
             if (nj == 0) prefetch_row<kP * (int)sizeof(Tout)>(Yssd + rowo_pf * kP, z + rowo_pf);
-            for (int j = 0; j < nj; ++j) {
+            // one job: U -> logit -> online softmax, V -> weighted sum. kMasked: some lanes
+            // of the warp may be past their history (j >= njr) and skip the softmax update
+            auto job = [&](int j, auto masked) -> bool {
+                constexpr bool kMasked = decltype(masked)::value;
                 const int ub = j & 1;
                 const float s_j = s_next;
                 if (j == pf_job) prefetch_row<kP * (int)sizeof(Tout)>(Yssd + rowo_pf * kP, z + rowo_pf);
                 if (j + 1 < nj) s_next = __ldg(scl + (i64)(j + 1) * H);  // one job ahead
                 if (!warp_wait(&sm.uready[ub], (uint32_t)((j >> 1) & 1), wait_limit_ns, abort)) {
                     fail(abort, 4);
-                    ok = false;
-                    break;
+                    return false;
                 }
                 tc::tc_fence_after();
                 float l;
                 {
                     uint64_t acc = 0ull, v[16];
                     tmem_ld32p(ua, v);
-    #pragma unroll
+#pragma unroll
                     for (int i = 0; i < 16; ++i) acc = f2_fma(v[i], eb[i], acc);
                     tmem_ld32p(ua + 32u, v);
                     warp_release(&sm.u_free);
-    #pragma unroll
+#pragma unroll
                     for (int i = 0; i < 16; ++i) acc = f2_fma(v[i], eb[16 + i], acc);
                     float lx, ly;
                     f2_unpack(acc, lx, ly);
                     l = __fmul_rn(lx + ly, lfac);  // rounded: the stored and the recomputed logits agree
                 }
-                if constexpr (kLogits) lgp[(i64)j * L] = l;
-                // online softmax; the running sums are rescaled only when the maximum moves
-                if (l > m) {
-                    const float sc = expf(m - l);
-                    const uint64_t sc2 = f2_pack(sc, sc);
-    #pragma unroll
-                    for (int i = 0; i < kP / 2; ++i) O[i] = f2_mul(O[i], sc2);
-                    dsum *= sc;
-                    m = l;
+                float w = 0.0f;
+                if (!kMasked || j < njr) {
+                    if constexpr (kLogits) lgp[(i64)j * L] = l;
+                    // online softmax; the running sums are rescaled only when the maximum moves
+                    if (l > m) {
+                        const float sc = expf(m - l);
+                        const uint64_t sc2 = f2_pack(sc, sc);
+#pragma unroll
+                        for (int i = 0; i < kP / 2; ++i) O[i] = f2_mul(O[i], sc2);
+                        dsum *= sc;
+                        m = l;
+                    }
+                    const float pe = expf(l - m);
+                    dsum += pe;
+                    w = pe * s_j;
                 }
-                const float pe = expf(l - m);
-                dsum += pe;
-                const float w = pe * s_j;
                 const uint64_t w2 = f2_pack(w, w);
                 if (!warp_wait(&sm.vready[ub], (uint32_t)((j >> 1) & 1), wait_limit_ns, abort)) {
                     fail(abort, 4);
-                    ok = false;
-                    break;
+                    return false;
                 }
                 tc::tc_fence_after();
                 {
                     uint64_t v[16];
                     tmem_ld32p(va + 128u * ub, v);
-    #pragma unroll
+#pragma unroll
                     for (int i = 0; i < 16; ++i) O[i] = f2_fma(w2, v[i], O[i]);
                     tmem_ld32p(va + 128u * ub + 32u, v);
                     warp_release(&sm.v_free[ub]);
-    #pragma unroll
+#pragma unroll
                     for (int i = 0; i < 16; ++i) O[16 + i] = f2_fma(w2, v[i], O[16 + i]);
                 }
-            }
+                return true;
+            };
+            // jobs every row of the warp keeps (all of them when S >= 128), then the tail
+            const int njw = min(nj, (t0 + 32 * (warp & 3)) / S);
+            int j = 0;
+            for (; ok && j < njw; ++j) ok = job(j, std::false_type{});
+            for (; ok && j < nj; ++j) ok = job(j, std::true_type{});
             if (ok) {
                 // R = O / d (C's row scale undone), lse, gated merge. Every MMA is done
                 // (the last job's V was read, or there were no jobs), so the ring is free
@@ -716,7 +733,7 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
                 uint8_t* yslots = sm.ring + (warp - 4) * 2 * kSlots;
                 uint8_t* rslots = yslots + kSlots;
                 const i64 rstride = (i64)H * kRowB;
-                const bool has = nj > 0;
+                const bool has = njr > 0;
                 const float inv_d = has ? cdown / dsum : 0.0f;
                 const float gate = silu_f32(__bfloat162float(z[rowo]));
                 rows_to_slots<kRowB>(yslots, reinterpret_cast<const uint8_t*>(Yssd + row0 * kP), rstride, lane);
@@ -766,7 +783,7 @@ size_t sma_tc_workspace(int64_t B, int64_t Mc, int64_t H) {
 }
 
 bool sma_tc_supported(const SmaArgs& a) {
-    return a.P == kP && a.N == kN && a.S % kRows == 0 && a.L % kRows == 0 &&
+    return a.P == kP && a.N == kN && a.L % kRows == 0 &&
            a.H % kHeadsPerCta == 0 && (a.H / a.G) % kHeadsPerCta == 0;
 }
 

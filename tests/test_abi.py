@@ -84,10 +84,28 @@ def _scan(L, d, ptrs=None, ws=FAKE, ws_bytes=1 << 40):
 @pytest.mark.parametrize("kw,code", [
     (dict(batch=0), 1), (dict(seqlen=-4), 1), (dict(nheads=3, ngroups=2), 1), (dict(eps=0.0), 1),
     (dict(dtype=7), 1), (dict(headdim=48), 2), (dict(dstate=256), 2), (dict(chunk=96), 2),
-    (dict(seqlen=500), 2), (dict(chunk=512, seqlen=1024), 2),
+    (dict(chunk=512, seqlen=1024), 2),
 ])
 def test_bad_dims_rejected(L, kw, code):
     assert _scan(L, _dims(**kw)) == code
+
+
+def test_ragged_length(L):
+    """L % S != 0: the forward calls take it with a workspace that holds zero-padded
+    copies of the token tensors (L = 500, S = 128 runs as 512 tokens); the backward
+    calls refuse it."""
+    from paper_2608_02032_gb300 import binding as B
+
+    d, d512 = _dims(seqlen=500), _dims(seqlen=512)
+    al = lambda v: (v + 255) // 256 * 256
+    rows = 512  # Bsz 1 x 512 padded tokens; H 2, P 64, G 1, N 128, bf16 inputs, fp32 outputs
+    copies = al(rows * 2 * 64 * 2) + al(rows * 2 * 4) + 2 * al(rows * 128 * 2) + al(rows * 2 * 64 * 4)
+    assert B.dart_workspace_size(d, B.DART_OP_CHUNK_SCAN) == copies + B.dart_workspace_size(d512, B.DART_OP_CHUNK_SCAN)
+    assert B.dart_workspace_size(d, B.DART_OP_SMA_FORWARD) > B.dart_workspace_size(d512, B.DART_OP_SMA_FORWARD)
+    assert _scan(L, d, ws_bytes=100) == 3  # valid sizes, workspace too small
+    v = ctypes.c_void_p
+    assert L.dart_chunk_scan_backward(ctypes.byref(d), *[v(FAKE)] * 12, v(FAKE), 1 << 40, None) == 2
+    assert B.dart_workspace_size(d, B.DART_OP_SCAN_BACKWARD) == 0
 
 
 def test_null_and_misaligned_pointers_rejected(L):

@@ -162,3 +162,39 @@ def test_training_step_full_size_on_one_batch(name):
     print(name, {k: f"{v:.2e}" for k, v in errs.items()})
     for n, err in errs.items():
         assert err <= _tol(w), f"{n}: {err:.3e}"
+
+
+@pytest.mark.parametrize("w", [CASES[0], CASES[6]], ids=lambda w: w.name)
+def test_independent_sma_read_vector(w):
+    """The variant with an independent SMA read vector (the ablation of Sec. 5 that
+    replaces the shared C_t of V_{t,c} = C_t Delta H_[c] by its own projection): the
+    scan reads C, state-memory attention reads C_sma. Forward outputs, and the two
+    read-vector gradients kept apart (dC from the scan backward with no SMA part
+    passed in, dC_sma from the SMA backward), against the oracle run on the same split."""
+    inp = prefill_inputs(w, with_grad=True)
+    g = torch.Generator().manual_seed(w.seed + 77)
+    C_sma = (torch.randn(inp["Cm"].shape, generator=g, dtype=torch.float64) / w.dstate ** 0.5)
+    if w.dtype == "bf16":
+        C_sma = C_sma.to(torch.bfloat16).double()
+    # oracle: the scan with C, SMA and its backward with C_sma
+    Yssd, _ = oracle.ssd_recurrence(inp["X"], inp["dt"], inp["A"], inp["Bm"], inp["Cm"])
+    dH = oracle.chunk_memories(inp["X"], inp["dt"], inp["A"], inp["Bm"], w.chunk)
+    R, lse = oracle.sma(dH, inp["Q"], C_sma, inp["E"], w.chunk, w.eps)
+    Y = oracle.merge(Yssd, inp["z"], R)
+    dMem, dQ, dCs, dE, dz = oracle.sma_backward(dH, inp["Q"], C_sma, inp["E"], inp["z"], inp["dY"], w.chunk, w.eps)
+    dX, ddt, dA, dB, dC = oracle.ssd_backward(inp["X"], inp["dt"], inp["A"], inp["Bm"], inp["Cm"], inp["dY"],
+                                              dMem, w.chunk)
+    # GPU
+    X, Bm, Cm, Q, E, z, dY = (dev(inp[k], w.dtype) for k in ("X", "Bm", "Cm", "Q", "E", "z", "dY"))
+    Cs = dev(C_sma, w.dtype)
+    dt, A = dev(inp["dt"], torch.float32), dev(inp["A"], torch.float32)
+    s = api.chunk_scan(X, dt, A, Bm, Cm, w.chunk, w.eps)
+    o = api.sma_forward(s.M, s.rM, Q, Cs, E, z, s.Y_ssd, w.chunk, w.eps)
+    gM, gQ, gCs, gE, gz = api.sma_backward(s.M, s.rM, Q, Cs, E, z, o.lse, dY, w.chunk, w.eps)
+    gX, gdt, gA, gB, gC = api.chunk_scan_backward(X, dt, A, Bm, Cm, dY, gM, w.chunk, eps=w.eps)
+    torch.cuda.synchronize()
+    tol = _tol(w)
+    for n, got, ref in (("Y", o.Y, Y), ("lse", o.lse, lse), ("dX", gX, dX), ("ddt", gdt, ddt), ("dA", gA, dA),
+                        ("dB", gB, dB), ("dC", gC, dC), ("dC_sma", gCs, dCs), ("dQ", gQ, dQ), ("dE", gE, dE),
+                        ("dz", gz, dz)):
+        assert rel_err(host(got), ref) <= tol, n

@@ -86,6 +86,43 @@ def test_prefill_then_decode_equals_longer_prefill(oracle_mod, dtype):
     assert rel_err(host(cache[:, : (L0 + k) // S]), dH[:, : (L0 + k) // S]) <= tol
 
 
+def test_ragged_prefill_hands_off_mid_chunk_to_decode(oracle_mod):
+    """A prefill of L0 = 300 tokens (S = 128: two full chunks and 44 tokens of a
+    third) on the tensor-core shapes, then decode from pos = 300 across the end of
+    that chunk (pos 383 appends it) into the next: the prefill's last memory is the
+    running partial memory and its final state the running state. Against the
+    oracle prefill of L0 + k tokens: y at every decode position, the completed
+    memories in the cache."""
+    S, L0, k = 128, 300, 100
+    w = Workload("dec_ragged", 2, 2, L0 + k, 64, 128, S, seed=23)
+    inp = prefill_inputs(w)
+    Yssd, dH, R, lse, Y = oracle_mod.forward(inp["X"], inp["dt"], inp["A"], inp["Bm"], inp["Cm"],
+                                             inp["Q"], inp["E"], inp["z"], S, w.eps)
+    pre = {key: dev(inp[key][:, :L0], "bf16") for key in ("X", "Bm", "Cm", "Q", "E", "z")}
+    dt_pre = dev(inp["dt"][:, :L0], torch.float32)
+    A = dev(inp["A"], torch.float32)
+    s, o = api.prefill_forward(pre["X"], dt_pre, A, pre["Bm"], pre["Cm"], pre["Q"], pre["E"], pre["z"], S,
+                               w.eps)
+    s_fs = api.chunk_scan(pre["X"], dt_pre, A, pre["Bm"], pre["Cm"], S, w.eps, final_state=True)
+    torch.cuda.synchronize()
+    assert s.M.shape[1] == 3  # ceil(300 / 128): the third memory is the partial chunk
+    assert rel_err(host(o.Y), Y[:, :L0]) <= TOL["bf16"]
+    m_cap = -(-(L0 + k) // S)
+    cache = torch.zeros(w.batch, m_cap, w.heads, w.dstate, w.headdim, dtype=torch.float32, device="cuda")
+    cache[:, : L0 // S] = s.M[:, : L0 // S]
+    partial = s.M[:, L0 // S].contiguous()  # the running partial memory of chunk 2
+    state = s_fs.final_state.clone()
+    for pos in range(L0, L0 + k):
+        t = {key: dev(inp[src][:, pos], "bf16") for key, src in
+             (("x", "X"), ("b", "Bm"), ("c", "Cm"), ("q", "Q"), ("e", "E"), ("z", "z"))}
+        y, l = api.decode_step(cache, state, partial, t["x"], dev(inp["dt"][:, pos], torch.float32), A,
+                               t["b"], t["c"], t["q"], t["e"], t["z"], pos, S, w.eps)
+        assert rel_err(host(y), Y[:, pos]) <= TOL["bf16"], pos
+        assert rel_err(host(l), lse[:, pos]) <= TOL["bf16"], pos
+    torch.cuda.synchronize()
+    assert rel_err(host(cache[:, :3]), dH[:, :3]) <= TOL["bf16"]
+
+
 def test_decode_mid_chunk_updates_state_and_partial(oracle_mod):
     """pos inside a chunk: the partial memory decays and accumulates (no reset)."""
     w = Workload("dec_mid", 3, 4, 1, 64, 128, 64, seed=31, mem=5, pos=5 * 64 + 17)

@@ -65,6 +65,15 @@ SWEEP = [
     # tensor-core scan shapes (bf16, P 64, N 128, S in {128, 256}, 8 heads per CTA)
     (512, 128, 64, 128, 8, 1, "bf16"),
     (1024, 256, 64, 128, 16, 2, "bf16"),   # G = 2, eight heads per group
+    # ragged L (L % S != 0): the last memory holds the partial chunk
+    (1000, 256, 64, 128, 8, 1, "bf16"),    # tensor-core scan and SMA on 1024 padded tokens
+    (1000, 256, 64, 128, 2, 1, "bf16"),    # CUDA-core scan, tensor-core SMA
+    (300, 64, 32, 32, 2, 1, "f32"),        # CUDA-core path, 5 memories, 44-token last chunk
+    (97, 32, 16, 16, 3, 1, "f32"),         # a last chunk of one token (97 = 3 x 32 + 1)
+    # tensor-core SMA with S < 128: a tile spans chunks, each token keeps its own history
+    (1024, 64, 64, 128, 4, 1, "bf16"),     # S = 64: 16 memories
+    (512, 32, 64, 128, 2, 1, "bf16"),      # S = 32: four chunks per tile
+    (1000, 64, 64, 128, 2, 1, "bf16"),     # S = 64 and ragged (1024 padded tokens)
 ]
 
 
