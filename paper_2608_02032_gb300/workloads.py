@@ -166,3 +166,76 @@ def decode_state(w: Workload, m_cap: int | None = None) -> dict:
         state=torch.stack([decode_state_slab(w, b) for b in range(w.batch)]),
         partial=torch.stack([decode_partial_slab(w, b) for b in range(w.batch)]),
     )
+
+
+# ---------------------------------------------------------------- whole block
+@dataclass(frozen=True)
+class BlockWorkload:
+    """Sizes of one DART block (the hot path inside a Mamba-2 style block): d_inner =
+    H P, in-projection of width 2 d_inner + 3 G N + H + G P + 1."""
+
+    name: str
+    batch: int
+    seqlen: int
+    d_model: int
+    heads: int
+    headdim: int = 64  # P
+    dstate: int = 128  # N
+    chunk: int = 256  # S
+    groups: int = 1
+    conv: int = 4  # convolution width
+    seed: int = 0
+    eps: float = 1e-6  # RMSNorm of Q, E and the memory rows
+    norm_eps: float = 1e-5  # the gated output RMSNorm
+    notes: str = field(default="", compare=False)
+
+    @property
+    def d_inner(self) -> int:
+        return self.heads * self.headdim
+
+    @property
+    def d_in_proj(self) -> int:
+        G, N, P = self.groups, self.dstate, self.headdim
+        return 2 * self.d_inner + 3 * G * N + self.heads + G * P + 1
+
+    @property
+    def tokens(self) -> int:
+        return self.batch * self.seqlen
+
+
+BLOCK_WORKLOADS = {
+    # the DART 380M block shape (d_model 1024, expand 2: 32 heads of 64) at L = 16K
+    "block_l16k": BlockWorkload("block_l16k", 1, 16384, 1024, 32, seed=1010,
+                                notes="B1 L16384 d_model 1024 H32 P64 N128 S256, bf16"),
+    "block_small": BlockWorkload("block_small", 2, 512, 256, 8, chunk=128, seed=1011,
+                                 notes="B2 L512 d_model 256 H8 P64 N128 S128, bf16"),
+}
+
+
+def block_inputs(w: BlockWorkload) -> dict:
+    """Seeded block input and weights as CPU fp32 tensors (U, W_in and W_out bf16-exact).
+
+    U ~ N(0, 1); the in-projection rows ~ N(0, 1/d_model), except the dt rows ~
+    N(0, 0.25/d_model) (with dt_bias ~ N(-2, 0.1^2) the step size is softplus of
+    about N(-2, 0.5^2), as in the hot-path workloads); conv_w, conv_b ~
+    U(-1/sqrt(width), 1/sqrt(width)); A_log ~ U(0, ln 16); D ~ N(1, 0.1^2);
+    norm_w ~ N(1, 0.1^2); W_out ~ N(0, 1/d_inner). Draw order: U, W_in, conv_w,
+    conv_b, dt_bias, A_log, D, norm_w, W_out.
+    """
+    g = torch.Generator().manual_seed(w.seed)
+    d, di, H = w.d_model, w.d_inner, w.heads
+    conv_ch = di + 2 * w.groups * w.dstate
+    U = torch.randn(w.batch, w.seqlen, d, generator=g)
+    W_in = torch.randn(w.d_in_proj, d, generator=g) / math.sqrt(d)
+    dt0 = 2 * di + 2 * w.groups * w.dstate  # first dt row
+    W_in[dt0:dt0 + H] *= 0.5
+    bound = 1.0 / math.sqrt(w.conv)
+    conv_w = (torch.rand(conv_ch, w.conv, generator=g) * 2 - 1) * bound
+    conv_b = (torch.rand(conv_ch, generator=g) * 2 - 1) * bound
+    dt_bias = -2.0 + 0.1 * torch.randn(H, generator=g)
+    A_log = torch.rand(H, generator=g) * math.log(16.0)
+    D = 1.0 + 0.1 * torch.randn(H, generator=g)
+    norm_w = 1.0 + 0.1 * torch.randn(di, generator=g)
+    W_out = torch.randn(d, di, generator=g) / math.sqrt(di)
+    return dict(U=_round(U, "bf16"), W_in=_round(W_in, "bf16"), conv_w=conv_w, conv_b=conv_b,
+                dt_bias=dt_bias, A_log=A_log, D=D, norm_w=norm_w, W_out=_round(W_out, "bf16"))
