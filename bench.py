@@ -364,6 +364,11 @@ def run_dart(args) -> None:
         train = [bench_train(args, dev, world, peaks, Bd, WORKLOADS[name], prefill_inputs)
                  for name in args.train_workload.split(",")]
 
+    # ---- the whole block (projections, convolution, hot path, norm) at the L = 16K shape
+    block = None
+    if not args.no_block:
+        block = bench_block(args, dev, world, peaks, Bd)
+
     # ---- CPU oracle on a bounded sample (rank 0, N = 1 only)
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -399,6 +404,7 @@ def run_dart(args) -> None:
             "gpu_launches": launches, "clocks": clocks, "wall_s_timed": t_wall,
             "decode": dec,
             "train": train,
+            "block": block,
         }
         print(json.dumps(line), flush=True)
     if world > 1:
@@ -455,6 +461,64 @@ def bench_decode(args, dev, world, peaks, Bd, w, cache_slab, state_slab, token_i
                          "peak_source": f"{peaks['source']} copy bandwidth",
                          "traffic": _traffic_from_profiles("decode_step_decode_b64.md", "decode.cu")
                          if w.name == DECODE else None}}
+
+
+def bench_block(args, dev, world, peaks, Bd):
+    """One whole DART block forward (dart_block_forward) on the DART 380M block
+    shape at L = 16K: in-projection, convolution, scan, SMA + merge, D skip, gated
+    RMSNorm, out-projection; inputs and weights resident in HBM."""
+    import torch
+
+    from paper_2608_02032_gb300.workloads import BLOCK_WORKLOADS, block_inputs
+
+    w = BLOCK_WORKLOADS["block_l16k"]
+    inp = block_inputs(w)
+    d = {k: v.to(dev) for k, v in inp.items()}
+    for k in ("U", "W_in", "W_out"):
+        d[k] = d[k].to(torch.bfloat16)
+    dims = Bd.make_block_dims(w.batch, w.seqlen, w.d_model, w.heads, w.groups, w.headdim, w.dstate, w.chunk,
+                              w.conv, Bd.DART_BF16, w.eps, w.norm_eps)
+    out = torch.empty(w.batch, w.seqlen, w.d_model, dtype=torch.bfloat16, device=dev)
+    ws = torch.empty(Bd.dart_block_workspace_size(dims), dtype=torch.uint8, device=dev)
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def step():
+        Bd.dart_block_forward(dims, d["U"], d["W_in"], d["conv_w"], d["conv_b"], d["dt_bias"], d["A_log"],
+                              d["D"], d["norm_w"], d["W_out"], out, ws, stream)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    barrier(world)
+    times = []
+    for _ in range(args.steps):
+        flush.random_(0, 255)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        step()
+        e1.record(stream)
+        times.append((e0, e1))
+    torch.cuda.synchronize()
+    ms = max_over_ranks(sum(a.elapsed_time(b) for a, b in times) / len(times), world, dev)
+    T = w.tokens
+    proj = 2.0 * T * w.d_model * (w.d_in_proj + w.d_inner)
+    pw = block_path_workload(w)
+    flops = proj + sma_flops(pw) + scan_flops(pw)
+    del ws, flush
+    torch.cuda.empty_cache()
+    return {"workload": f"{w.name}: {w.notes}", "tokens_per_s": world * T / (ms / 1e3), "ms_per_step": ms,
+            "flops_per_step": flops, "tflops": flops / (ms / 1e3) / 1e12,
+            "frac_of_peak": flops / (ms / 1e3) / 1e12 / peaks["bf16"],
+            "peak_source": f"{peaks['source']} bf16 dense (burst)",
+            "flops_model": "projections 2 T d_model (D_in + d_inner) + SMA + scan algorithmic flops"}
+
+
+def block_path_workload(bw):
+    """The hot-path workload inside a block workload (for the flop counts)."""
+    from paper_2608_02032_gb300.workloads import Workload
+
+    return Workload(bw.name, bw.batch, bw.heads, bw.seqlen, bw.headdim, bw.dstate, bw.chunk, groups=bw.groups)
 
 
 def bench_train(args, dev, world, peaks, Bd, w, prefill_inputs):
@@ -558,6 +622,7 @@ def main():
     ap.add_argument("--impl", choices=("dart", "reference"), default="dart")
     ap.add_argument("--no-decode", action="store_true")
     ap.add_argument("--no-train", action="store_true")
+    ap.add_argument("--no-block", action="store_true")
     ap.add_argument("--decode-workload", default=DECODE, help="decode workload (a smaller one for profiling)")
     ap.add_argument("--train-workload", default="train_b8_l4k_s256,train_b8_l4k_s128",
                     help="comma-separated training workloads (one leg each)")

@@ -299,6 +299,47 @@ dart_status dart_chunk_scan_backward(const dart_dims* dims, const void* X, const
                                      size_t workspace_bytes, void* stream);
 
 /*
+ * The whole DART block around the hot path, for a prefill (Sec. 3: Q, E and the
+ * gate are projections of the block input U_t, C is shared with the SSM branch
+ * and Y_t = C_t H_t + G_t R_t; for the rest the Mamba-2 block the paper builds
+ * on, with the sizes of App. D.2: head dimension 64, one B, C group,
+ * convolution width 4, RMSNorm):
+ *   zx = U W_in^T, cut into z (d_inner), x (d_inner), B (G N), C (G N), dt (H),
+ *        Q (G N), E (G P), gate (1) in this column order, d_inner = H P;
+ *   x, B, C <- SiLU(causal depthwise convolution, per channel c:
+ *        b[c] + sum_k conv_w[c, k] v[t - width + 1 + k, c], zero before t = 0);
+ *   dt <- softplus(dt + dt_bias), A = -exp(A_log), the gate logit of token t for
+ *        every head (one scalar per token, App. D.2);
+ *   Y = the hot path (dart_chunk_scan, dart_sma_forward) on X, dt, A, B, C, Q, E, gate;
+ *   y = Y + D_h x;  yn = RMSNorm(y * SiLU(z)) * norm_w over d_inner (norm_eps);
+ *   out = yn W_out^T.
+ * Precision: U and the weights W_in, W_out are bf16; the in-projection output, the
+ * memories and Y are fp32; the hot path's token inputs (x, B, C, Q, E, the gate
+ * logit) and yn are rounded to bf16; every accumulation is fp32.
+ * Inputs:  U (Bsz, L, d_model) bf16; W_in (D_in, d_model) bf16 with D_in = 2 d_inner
+ *          + 3 G N + H + G P + 1; conv_w (d_inner + 2 G N, conv_width), conv_b
+ *          (d_inner + 2 G N), dt_bias, A_log, D (H), norm_w (d_inner) fp32;
+ *          W_out (d_model, d_inner) bf16 (nn.Linear layouts).
+ * Output:  out (Bsz, L, d_model) in core.out_dtype (DART_F32 or DART_BF16).
+ * Requires core.in_dtype == DART_BF16, d_model % 8 == 0, H % 8 == 0, H P <= 8192;
+ * L need not be a multiple of S. Workspace: dart_block_workspace_size(dims).
+ */
+typedef struct {
+    dart_dims core;      /* Bsz, L, H, G, P, N, S, eps of the hot path; in_dtype (DART_BF16) and
+                            out_dtype (of the block output); mem_dtype is ignored (fp32 memories) */
+    int64_t d_model;     /* width of U and of the output */
+    int64_t conv_width;  /* 1 .. 8 (4 in the paper) */
+    float norm_eps;      /* epsilon of the output RMSNorm, > 0 */
+} dart_block_dims;
+
+size_t dart_block_workspace_size(const dart_block_dims* dims);
+dart_status dart_block_forward(const dart_block_dims* dims, const void* U, const void* W_in,
+                               const float* conv_w, const float* conv_b, const float* dt_bias,
+                               const float* A_log, const float* D, const float* norm_w,
+                               const void* W_out, void* out, void* workspace, size_t workspace_bytes,
+                               void* stream);
+
+/*
  * dart_sma_forward_noalloc: dart_sma_forward with rM = NULL, for callers that
  * cannot allocate device memory and cannot pass a workspace. The paper has no
  * counterpart; this entry point exists for integration. Typical callers: a

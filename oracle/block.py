@@ -17,7 +17,11 @@ group, convolution width 4, RMSNorm). Readings where the paper says no more:
     residual gate per token"): G_t = SiLU(U_t W_G);
   * D skip after the merge: y = C_t H_t + G_t R_t + D_h x_t;
   * gated RMSNorm over d_inner: RMSNorm(y * SiLU(z)) * w, then the
-    out-projection.
+    out-projection;
+  * precision of the hot path's token inputs: with ``path_dtype="bf16"`` the
+    x, B, C (after the convolution), Q, E and gate logits are rounded to bf16
+    (round to nearest even) before the scan and SMA, the storage type of the
+    bf16 configuration's token inputs; everything else stays fp64.
 
 Weights use ``nn.Linear`` layouts: W_in (D_in x d_model), W_out (d_model x
 d_inner), conv_w (conv channels x width), the tap k multiplying x[t - width + 1 + k].
@@ -82,9 +86,18 @@ def rms_norm_gated(y, z, w, eps: float):
     return g / np.sqrt(np.mean(g * g, axis=-1, keepdims=True) + eps) * _f64(w)
 
 
-def block_inputs_to_path(U, W_in, conv_w, conv_b, dt_bias, A_log, H: int, G: int, N: int, P: int):
+def _bf16(a):
+    """Round to bf16 (nearest even), back in fp64."""
+    import torch
+
+    return torch.from_numpy(np.ascontiguousarray(a)).to(torch.bfloat16).double().numpy()
+
+
+def block_inputs_to_path(U, W_in, conv_w, conv_b, dt_bias, A_log, H: int, G: int, N: int, P: int,
+                         path_dtype: str = "f64"):
     """The in-projection, the convolution and the step-size / decay parameters: the
-    inputs of the hot path (X, dt, A, B, C, Q, E, gate logits per head) and z."""
+    inputs of the hot path (X, dt, A, B, C, Q, E, gate logits per head) and z.
+    ``path_dtype="bf16"`` rounds X, B, C, Q, E and the gate logits to bf16."""
     U, W_in = _f64(U), _f64(W_in)
     Bsz, L, _ = U.shape
     d_inner = H * P
@@ -100,17 +113,21 @@ def block_inputs_to_path(U, W_in, conv_w, conv_b, dt_bias, A_log, H: int, G: int
     Q = parts["Q"].reshape(Bsz, L, G, N)
     E = parts["E"].reshape(Bsz, L, G, P)
     gate = np.broadcast_to(parts["gate"], (Bsz, L, H)).copy()  # one logit per token, every head
+    if path_dtype == "bf16":
+        X, Bm, Cm, Q, E, gate = (_bf16(a) for a in (X, Bm, Cm, Q, E, gate))
+    else:
+        assert path_dtype == "f64", path_dtype
     return dict(X=X, dt=dt, A=A, Bm=Bm, Cm=Cm, Q=Q, E=E, z=gate, zn=parts["z"])
 
 
 def block_forward(U, W_in, conv_w, conv_b, dt_bias, A_log, D, norm_w, W_out, H: int, G: int, N: int,
-                  P: int, S: int, eps: float, norm_eps: float, path=None):
+                  P: int, S: int, eps: float, norm_eps: float, path=None, path_dtype: str = "f64"):
     """Whole DART block for a prefill: returns (out ``Bsz x L x d_model``, intermediates).
 
     ``path``: optional replacement of the hot-path result Y (``Bsz x L x H x P``),
     for tests that pin the surrounding steps alone.
     """
-    p = block_inputs_to_path(U, W_in, conv_w, conv_b, dt_bias, A_log, H, G, N, P)
+    p = block_inputs_to_path(U, W_in, conv_w, conv_b, dt_bias, A_log, H, G, N, P, path_dtype)
     if path is None:
         Yssd, _ = oracle.ssd_recurrence(p["X"], p["dt"], p["A"], p["Bm"], p["Cm"])
         dH = oracle.chunk_memories(p["X"], p["dt"], p["A"], p["Bm"], S)

@@ -191,3 +191,21 @@ def layer_backward(X, dt, A, Bm, Cm, Q, E, z, dY, scan: ScanOut, sma: SmaOut, ch
                                       logits=sma.logits)
     dX, ddt, dA, dB, dC = chunk_scan_backward(X, dt, A, Bm, Cm, dY, dM, chunk, dC=dC, eps=eps)
     return LayerGrads(dX, ddt, dA, dB, dC, dQ, dE, dz, dM)
+
+
+def block_forward(U, W_in, conv_w, conv_b, dt_bias, A_log, D, norm_w, W_out, heads: int, chunk: int = 256,
+                  groups: int = 1, headdim: int = 64, dstate: int = 128, eps: float = 1e-6,
+                  norm_eps: float = 1e-5, out_dtype=torch.float32, workspace=None) -> torch.Tensor:
+    """One whole DART block for a prefill (``dart_block_forward``): in-projection,
+    convolution, the hot path, D skip, gated RMSNorm and out-projection. U and the
+    projection weights are bf16, the small parameters fp32; returns out
+    (Bsz, L, d_model) in ``out_dtype``."""
+    Bsz, L, d_model = U.shape
+    dims = B.make_block_dims(Bsz, L, d_model, heads, groups, headdim, dstate, chunk, conv_w.shape[1],
+                             B.DART_DTYPE[out_dtype], eps, norm_eps)
+    out = torch.empty(Bsz, L, d_model, dtype=out_dtype, device=U.device)
+    ws = workspace
+    if ws is None:
+        ws = torch.empty(max(B.dart_block_workspace_size(dims), 256), dtype=torch.uint8, device=U.device)
+    B.dart_block_forward(dims, U, W_in, conv_w, conv_b, dt_bias, A_log, D, norm_w, W_out, out, ws)
+    return out

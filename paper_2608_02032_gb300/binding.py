@@ -32,7 +32,8 @@ EXPORTED = ("dart_status_string", "dart_last_cuda_error", "dart_workspace_size",
             "dart_chunk_scan", "dart_sma_forward", "dart_decode_step", "dart_sma_forward_noalloc",
             "dart_launch_count", "dart_set_wait_limit_ns", "dart_get_device_status",
             "dart_sma_backward", "dart_chunk_scan_backward", "dart_test_withhold_copies",
-            "dart_prefill_host", "dart_sma_forward_with_logits", "dart_sma_backward_with_logits")
+            "dart_prefill_host", "dart_sma_forward_with_logits", "dart_sma_backward_with_logits",
+            "dart_block_workspace_size", "dart_block_forward")
 
 
 class DartError(RuntimeError):
@@ -50,6 +51,18 @@ class dart_dims(ctypes.Structure):
                 ("chunk", ctypes.c_int64), ("in_dtype", ctypes.c_int32),
                 ("mem_dtype", ctypes.c_int32), ("out_dtype", ctypes.c_int32),
                 ("eps", ctypes.c_float)]
+
+
+class dart_block_dims(ctypes.Structure):
+    _fields_ = [("core", dart_dims), ("d_model", ctypes.c_int64), ("conv_width", ctypes.c_int64),
+                ("norm_eps", ctypes.c_float)]
+
+
+def make_block_dims(batch, seqlen, d_model, nheads, ngroups=1, headdim=64, dstate=128, chunk=256,
+                    conv_width=4, out_dtype=DART_F32, eps=1e-6, norm_eps=1e-5) -> dart_block_dims:
+    """Sizes of one whole block (bf16 input and weights; ``out_dtype`` of its output)."""
+    core = make_dims(batch, seqlen, nheads, ngroups, headdim, dstate, chunk, DART_BF16, DART_F32, out_dtype, eps)
+    return dart_block_dims(core, d_model, conv_width, norm_eps)
 
 
 def _code(dt):
@@ -109,6 +122,11 @@ def lib() -> ctypes.CDLL:
         L.dart_sma_backward_with_logits.argtypes = [dp] + [_vp] * 15 + [ctypes.c_size_t, _vp]
         L.dart_chunk_scan_backward.argtypes = [dp] + [_vp] * 13 + [ctypes.c_size_t, _vp]
         L.dart_chunk_scan_backward.restype = ctypes.c_int
+        bp = ctypes.POINTER(dart_block_dims)
+        L.dart_block_workspace_size.argtypes = [bp]
+        L.dart_block_workspace_size.restype = ctypes.c_size_t
+        L.dart_block_forward.argtypes = [bp] + [_vp] * 11 + [ctypes.c_size_t, _vp]
+        L.dart_block_forward.restype = ctypes.c_int
         _lib = L
     return _lib
 
@@ -241,6 +259,19 @@ def dart_chunk_scan_backward(dims, X, dt, A, Bm, Cm, dY, dM, dX, ddt, dA, dB, dC
         ctypes.byref(dims), _ptr(X, "X"), _ptr(dt, "dt"), _ptr(A, "A"), _ptr(Bm, "Bm"),
         _ptr(Cm, "Cm"), _ptr(dY, "dY"), _ptr(dM, "dM"), _ptr(dX, "dX"), _ptr(ddt, "ddt"),
         _ptr(dA, "dA"), _ptr(dB, "dB"), _ptr(dC, "dC"), w, nb, _stream(stream)))
+
+
+def dart_block_workspace_size(dims: dart_block_dims) -> int:
+    return int(lib().dart_block_workspace_size(ctypes.byref(dims)))
+
+
+def dart_block_forward(dims, U, W_in, conv_w, conv_b, dt_bias, A_log, D, norm_w, W_out, out, workspace=None,
+                       stream=None) -> None:
+    w, nb = _ws(workspace)
+    _check("dart_block_forward", lib().dart_block_forward(
+        ctypes.byref(dims), _ptr(U, "U"), _ptr(W_in, "W_in"), _ptr(conv_w, "conv_w"), _ptr(conv_b, "conv_b"),
+        _ptr(dt_bias, "dt_bias"), _ptr(A_log, "A_log"), _ptr(D, "D"), _ptr(norm_w, "norm_w"),
+        _ptr(W_out, "W_out"), _ptr(out, "out"), w, nb, _stream(stream)))
 
 
 def dart_get_device_status(stream=None) -> None:

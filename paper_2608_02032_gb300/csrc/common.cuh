@@ -105,6 +105,28 @@ __device__ __forceinline__ void store_row16(__nv_bfloat16* dst, const float* v) 
     }
 }
 
+// 8 consecutive bf16 values (16-byte aligned) as floats.
+__device__ __forceinline__ void load_row8(const __nv_bfloat16* src, float* v) {
+    const uint4 u = *reinterpret_cast<const uint4*>(src);
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+        const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w[e]));
+        v[2 * e] = f.x; v[2 * e + 1] = f.y;
+    }
+}
+
+// 8 floats as bf16 (16-byte aligned destination).
+__device__ __forceinline__ void store_row8(__nv_bfloat16* dst, const float* v) {
+    uint32_t w[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+        const __nv_bfloat162 p = __floats2bfloat162_rn(v[2 * e], v[2 * e + 1]);
+        w[e] = *reinterpret_cast<const uint32_t*>(&p);
+    }
+    *reinterpret_cast<uint4*>(dst) = make_uint4(w[0], w[1], w[2], w[3]);
+}
+
 // SiLU(z) = z * sigmoid(z), the SMA residual gate (Sec. 3).
 __device__ __forceinline__ float silu_f32(float z) { return z / (1.0f + expf(-z)); }
 // d SiLU / dz = s (1 + z (1 - s)), s = sigmoid(z)

@@ -324,6 +324,62 @@ cudaError_t host_streams(HostStreams** hs) {
     return cudaSuccess;
 }
 
+// Workspace of dart_block_forward: the in-projection output, the hot path's inputs
+// and outputs, the normalised output, then the scan and SMA workspaces.
+struct BlockWs {
+    int64_t ldz, d_in;
+    size_t zx, x, bm, cm, dt, a, q, e, gate, yssd, y, mem, rm, yn, scan, scan_bytes, sma, sma_bytes, total;
+};
+dart_dims block_core(const dart_block_dims* b) {
+    dart_dims c = b->core;
+    c.in_dtype = DART_BF16;
+    c.mem_dtype = DART_F32;
+    c.out_dtype = DART_F32;
+    return c;
+}
+BlockWs block_ws(const dart_block_dims* b) {
+    const dart_dims c = block_core(b);
+    const int64_t T = c.batch * c.seqlen, H = c.nheads, di = H * c.headdim, GN = c.ngroups * c.dstate;
+    const int64_t GP = c.ngroups * c.headdim, Mc = (c.seqlen + c.chunk - 1) / c.chunk;
+    BlockWs w{};
+    w.d_in = 2 * di + 3 * GN + H + GP + 1;
+    w.ldz = (w.d_in + 7) / 8 * 8;
+    size_t o = 0;
+    auto take = [&o](size_t bytes) { const size_t at = o; o += align256(bytes); return at; };
+    w.zx = take((size_t)(T * w.ldz) * 4);
+    w.x = take((size_t)(T * di) * 2);
+    w.bm = take((size_t)(T * GN) * 2);
+    w.cm = take((size_t)(T * GN) * 2);
+    w.dt = take((size_t)(T * H) * 4);
+    w.a = take((size_t)H * 4);
+    w.q = take((size_t)(T * GN) * 2);
+    w.e = take((size_t)(T * GP) * 2);
+    w.gate = take((size_t)(T * H) * 2);
+    w.yssd = take((size_t)(T * di) * 4);
+    w.y = take((size_t)(T * di) * 4);
+    w.mem = take((size_t)(c.batch * Mc * H * c.dstate * c.headdim) * 4);
+    w.rm = take((size_t)(c.batch * Mc * H * c.dstate) * 4);
+    w.yn = take((size_t)(T * di) * 2);
+    w.scan_bytes = scan_ws_bytes(&c);
+    w.scan = take(w.scan_bytes);
+    w.sma_bytes = sma_ws(&c);
+    w.sma = take(w.sma_bytes);
+    w.total = o;
+    return w;
+}
+dart_status check_block(const dart_block_dims* b) {
+    if (b == nullptr) return DART_ERR_INVALID_ARG;
+    if (b->core.in_dtype != DART_BF16) return DART_ERR_UNSUPPORTED;
+    if (b->core.out_dtype != DART_F32 && b->core.out_dtype != DART_BF16) return DART_ERR_INVALID_ARG;
+    const dart_dims c = block_core(b);
+    const dart_status st = check_dims(&c, true, true);
+    if (st != DART_OK) return st;
+    if (b->d_model <= 0 || !(b->norm_eps > 0.0f) || !dart::block_conv_width_ok(b->conv_width))
+        return DART_ERR_INVALID_ARG;
+    if (b->d_model % 8 != 0 || c.nheads % 8 != 0 || c.nheads * c.headdim > 8192) return DART_ERR_UNSUPPORTED;
+    return DART_OK;
+}
+
 }  // namespace
 
 namespace dart {
@@ -805,6 +861,54 @@ dart_status dart_chunk_scan_backward(const dart_dims* d, const void* X, const fl
     return e == cudaSuccess ? DART_OK : cuda_fail(e);
 }
 
+size_t dart_block_workspace_size(const dart_block_dims* b) {
+    if (check_block(b) != DART_OK) return 0;
+    return block_ws(b).total;
+}
+
+dart_status dart_block_forward(const dart_block_dims* b, const void* U, const void* W_in, const float* conv_w,
+                               const float* conv_b, const float* dt_bias, const float* A_log, const float* D,
+                               const float* norm_w, const void* W_out, void* out, void* ws, size_t ws_bytes,
+                               void* stream) {
+    dart_status st = check_block(b);
+    if (st != DART_OK) return st;
+    const void* req[] = {U, W_in, conv_w, conv_b, dt_bias, A_log, D, norm_w, W_out, out};
+    for (const void* p : req)
+        if (p == nullptr || !aligned16(p)) return DART_ERR_INVALID_ARG;
+    const BlockWs w = block_ws(b);
+    if (ws == nullptr || ((uintptr_t)ws & 255u) != 0 || ws_bytes < w.total) return DART_ERR_WORKSPACE;
+    const dart_dims c = block_core(b);
+    uint8_t* p = (uint8_t*)ws;
+    cudaStream_t s = (cudaStream_t)stream;
+    const unsigned long long lim = g_wait_limit_ns.load();
+    const int64_t T = c.batch * c.seqlen, di = c.nheads * c.headdim;
+    dart::BlockArgs a{};
+    a.B = c.batch; a.L = c.seqlen; a.H = c.nheads; a.G = c.ngroups; a.P = c.headdim; a.N = c.dstate;
+    a.d_model = b->d_model; a.conv_width = b->conv_width; a.norm_eps = b->norm_eps;
+    a.conv_w = conv_w; a.conv_b = conv_b; a.dt_bias = dt_bias; a.A_log = A_log; a.D = D; a.norm_w = norm_w;
+    a.zx = p + w.zx; a.ldz = w.ldz; a.X = p + w.x; a.Bm = p + w.bm; a.Cm = p + w.cm;
+    a.dt = (float*)(p + w.dt); a.A = (float*)(p + w.a); a.Q = p + w.q; a.E = p + w.e; a.gate = p + w.gate;
+    a.Y = (float*)(p + w.y); a.yn = p + w.yn;
+    typedef __nv_bfloat16 bf;
+    cudaError_t e = dart::launch_gemm_tc<float>(U, W_in, (float*)a.zx, T, w.d_in, b->d_model, w.ldz, w.ldz, lim, s);
+    if (e == cudaSuccess) e = dart::launch_block_conv_split(a, s);
+    if (e != cudaSuccess) return cuda_fail(e);
+    st = dart_chunk_scan(&c, a.X, a.dt, a.A, a.Bm, a.Cm, p + w.yssd, p + w.mem, (float*)(p + w.rm), nullptr,
+                         p + w.scan, w.scan_bytes, stream);
+    if (st != DART_OK) return st;
+    st = dart_sma_forward(&c, p + w.mem, (const float*)(p + w.rm), a.Q, a.Cm, a.E, a.gate, p + w.yssd, a.Y,
+                          nullptr, nullptr, p + w.sma, w.sma_bytes, stream);
+    if (st != DART_OK) return st;
+    e = dart::launch_block_norm(a, s);
+    if (e == cudaSuccess)
+        e = b->core.out_dtype == DART_F32
+                ? dart::launch_gemm_tc<float>(a.yn, W_out, (float*)out, T, b->d_model, di, b->d_model,
+                                              b->d_model, lim, s)
+                : dart::launch_gemm_tc<bf>(a.yn, W_out, (bf*)out, T, b->d_model, di, b->d_model, b->d_model,
+                                           lim, s);
+    return e == cudaSuccess ? DART_OK : cuda_fail(e);
+}
+
 dart_status dart_get_device_status(void* stream) {
     cudaError_t e = cudaStreamSynchronize((cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(e);
@@ -813,8 +917,9 @@ dart_status dart_get_device_status(void* stream) {
     const int code2 = dart::take_scan_tc_status(s);
     const int code3 = dart::take_bwd_tc_status(s);
     const int code4 = dart::take_scan_bwd_tc_status(s);
-    if (code < 0 || code2 < 0 || code3 < 0 || code4 < 0) return cuda_fail(cudaGetLastError());
-    return (code != 0 || code2 != 0 || code3 != 0 || code4 != 0) ? DART_ERR_TIMEOUT : DART_OK;
+    const int code5 = dart::take_gemm_status(s);
+    if (code < 0 || code2 < 0 || code3 < 0 || code4 < 0 || code5 < 0) return cuda_fail(cudaGetLastError());
+    return (code != 0 || code2 != 0 || code3 != 0 || code4 != 0 || code5 != 0) ? DART_ERR_TIMEOUT : DART_OK;
 }
 
 void dart_test_withhold_copies(int on) { g_test_withhold.store(on != 0 ? 1 : 0); }

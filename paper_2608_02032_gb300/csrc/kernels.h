@@ -120,6 +120,39 @@ template <typename Tin>
 cudaError_t launch_scan_states(const ScanArgs& a, float* cum, float* Hprev, float* scratch,
                                cudaStream_t stream);
 
+// The whole block (block.cu, gemm_tc.cu): sizes, weights and the workspace buffers.
+struct BlockArgs {
+    int64_t B, L, H, G, P, N, d_model, conv_width;
+    float norm_eps;
+    const float* conv_w;  // (d_inner + 2 G N) x conv_width
+    const float* conv_b;
+    const float* dt_bias;  // H
+    const float* A_log;    // H
+    const float* D;        // H
+    const float* norm_w;   // d_inner
+    // workspace
+    void* zx;     // B L x ldz fp32: the in-projection output
+    int64_t ldz;
+    void* X;      // B L x H P bf16 (after the convolution)
+    void* Bm;     // B L x G N bf16
+    void* Cm;     // B L x G N bf16
+    float* dt;    // B L x H
+    float* A;     // H
+    void* Q;      // B L x G N bf16
+    void* E;      // B L x G P bf16
+    void* gate;   // B L x H bf16 (the token's gate logit for every head)
+    float* Y;     // B L x H P: the hot path's merged output
+    void* yn;     // B L x H P bf16: the normalised, gated output
+};
+cudaError_t launch_block_conv_split(const BlockArgs& a, cudaStream_t stream);
+cudaError_t launch_block_norm(const BlockArgs& a, cudaStream_t stream);
+bool block_conv_width_ok(int64_t w);
+// C (M x ldc, n_store columns written) = A (M x K) B (N x K)^T, bf16 inputs, fp32 accumulation.
+template <typename Tc>
+cudaError_t launch_gemm_tc(const void* A, const void* B, Tc* C, int64_t M, int64_t N, int64_t K, int64_t ldc,
+                           int64_t n_store, unsigned long long wait_limit_ns, cudaStream_t stream);
+int take_gemm_status(cudaStream_t stream);
+
 // Kernels launched by the library (read by dart_launch_count()).
 void note_launches(int n);
 
