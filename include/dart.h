@@ -321,7 +321,7 @@ dart_status dart_chunk_scan_backward(const dart_dims* dims, const void* X, const
  *          (d_inner + 2 G N), dt_bias, A_log, D (H), norm_w (d_inner) fp32;
  *          W_out (d_model, d_inner) bf16 (nn.Linear layouts).
  * Output:  out (Bsz, L, d_model) in core.out_dtype (DART_F32 or DART_BF16).
- * Requires core.in_dtype == DART_BF16, d_model % 8 == 0, H % 8 == 0, H P <= 8192;
+ * Requires core.in_dtype == DART_BF16, d_model % 8 == 0, H % 8 == 0, H P <= 4096;
  * L need not be a multiple of S. Workspace: dart_block_workspace_size(dims).
  */
 typedef struct {

@@ -376,7 +376,7 @@ dart_status check_block(const dart_block_dims* b) {
     if (st != DART_OK) return st;
     if (b->d_model <= 0 || !(b->norm_eps > 0.0f) || !dart::block_conv_width_ok(b->conv_width))
         return DART_ERR_INVALID_ARG;
-    if (b->d_model % 8 != 0 || c.nheads % 8 != 0 || c.nheads * c.headdim > 8192) return DART_ERR_UNSUPPORTED;
+    if (b->d_model % 8 != 0 || c.nheads % 8 != 0 || c.nheads * c.headdim > 4096) return DART_ERR_UNSUPPORTED;
     return DART_OK;
 }
 

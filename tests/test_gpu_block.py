@@ -24,6 +24,7 @@ CASES = [
     BlockWorkload("block_ragged", 1, 300, 128, 8, chunk=128, seed=1012),  # L % S != 0
     BlockWorkload("block_simt", 2, 192, 128, 8, headdim=32, dstate=64, chunk=64, seed=1013),  # CUDA-core path
     BlockWorkload("block_conv2_g2", 1, 256, 192, 8, groups=2, conv=2, chunk=64, seed=1014),
+    BlockWorkload("block_wide", 1, 256, 256, 48, chunk=128, seed=1015),  # d_inner 3072: the wider norm
 ]
 
 
