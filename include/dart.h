@@ -246,6 +246,12 @@ dart_status dart_decode_step(const dart_dims* dims, int64_t pos, int64_t m_cap, 
  * Workspace: dart_workspace_size(dims, DART_OP_SMA_BACKWARD): the weights g and
  *          logit gradients dl of every (memory, token) pair, 2 x Bsz x H x M x L
  *          fp32, plus r when rM is NULL.
+ * Groups: the tensor-core backward (bf16 inputs, P = 64, N = 128, S % 128 == 0,
+ *          L % 128 == 0) sums dQ, dC, dE over all heads of a launch. At G > 1
+ *          with H/G even it runs once per group, on the group's heads and its
+ *          Q, C, E column block copied into contiguous buffers in the workspace,
+ *          and copies the group's gradients back; other G > 1 shapes take the
+ *          CUDA-core kernels.
  */
 dart_status dart_sma_backward(const dart_dims* dims, const void* M, const float* rM,
                               const void* Q, const void* Cm, const void* E, const void* z,
@@ -291,6 +297,11 @@ dart_status dart_sma_backward_with_logits(const dart_dims* dims, const void* M, 
  * Workspace: dart_workspace_size(dims, DART_OP_SCAN_BACKWARD): the within-chunk
  *          cumulative decay, the state entering each chunk and the memory
  *          adjoints (2 x Bsz x M x H x N x P fp32).
+ * Groups: the tensor-core backward (bf16 inputs, P = 64, N = 128, S in {128,
+ *          256}) sums its intra-chunk dB, dC over all heads of a launch. At
+ *          G > 1 with H/G a multiple of 8 it runs once per group on copies of
+ *          the group's slices in the workspace (dC's block is copied in, added
+ *          to and copied back); other G > 1 shapes take the CUDA-core kernels.
  */
 dart_status dart_chunk_scan_backward(const dart_dims* dims, const void* X, const float* dt,
                                      const float* A, const void* Bm, const void* Cm,
@@ -394,9 +405,12 @@ void dart_set_wait_limit_ns(uint64_t limit_ns);
 
 /*
  * Test hook for the failure path of the tensor-core kernels (no counterpart in
- * the paper): while on, tensor-core dart_sma_forward launches issue none of
- * their operand copies, so their pipeline waits can only run out (each bounded
- * by dart_set_wait_limit_ns); the call then reports DART_ERR_TIMEOUT through
+ * the paper): while on, one ring-fed kernel of each tensor-core call issues
+ * none of its copies (dart_sma_forward: the SMA kernel's operands;
+ * dart_chunk_scan: the state passing's chunk slabs; dart_sma_backward: the row
+ * kernels' operands; dart_chunk_scan_backward: the reverse passing's slabs),
+ * so its pipeline waits can only run out (each bounded by
+ * dart_set_wait_limit_ns); the call then reports DART_ERR_TIMEOUT through
  * dart_get_device_status and its outputs are undefined. Process-wide; 0 (the
  * default) turns it off. For tests only.
  */

@@ -139,6 +139,191 @@ bool sma_bwd_uses_tc(const dart_dims* d) {
     return d->in_dtype == DART_BF16 && dart::sma_bwd_tc_supported(sma_bwd_args(d));
 }
 
+// ---- G > 1 on the tensor-core backward. The backward kernels sum over all heads
+// of a call (the SMA row kernels' dQ, dC over head pairs; the scan's intra-chunk
+// dB, dC through the head-summed Psi), so they serve G = 1. A group g is itself
+// a G = 1 problem over its H/G heads: a contiguous slice of every token row (X,
+// dt, z, lse, dY and the per-head gradients), one column block of every B, C, Q,
+// E row, and a slice of every (b, chunk) block of the memories. The grouped path
+// copies a group's inputs into contiguous buffers, runs the G = 1 tensor-core
+// backward on them and copies its gradients back, group after group on the
+// caller's stream (the groups share the buffers).
+dart_dims group_dims(const dart_dims* d) {
+    dart_dims g = *d;
+    g.nheads = d->nheads / d->ngroups;
+    g.ngroups = 1;
+    return g;
+}
+bool sma_bwd_grouped(const dart_dims* d) {
+    if (d->ngroups <= 1 || d->in_dtype != DART_BF16) return false;
+    const dart_dims g = group_dims(d);
+    return sma_bwd_uses_tc(&g);
+}
+bool scan_bwd_grouped(const dart_dims* d) {
+    if (d->ngroups <= 1 || d->in_dtype != DART_BF16) return false;
+    dart::ScanArgs a{};
+    a.B = d->batch; a.L = d->seqlen; a.H = d->nheads / d->ngroups; a.G = 1;
+    a.P = d->headdim; a.N = d->dstate; a.S = d->chunk;
+    return dart::scan_bwd_tc_supported(a);
+}
+
+struct SmaBwdGroupWs {  // byte offsets into the workspace
+    size_t tc, M, rM, Q, C, E, z, lse, dY, logits, dM, dQ, dC, dE, dz, total;
+};
+SmaBwdGroupWs sma_bwd_group_ws(const dart_dims* d) {
+    const size_t B = d->batch, L = d->seqlen, Hg = d->nheads / d->ngroups, P = d->headdim, N = d->dstate,
+                 Mc = d->seqlen / d->chunk;
+    const size_t em = d->mem_dtype == DART_F32 ? 4 : 2, ei = 2;
+    SmaBwdGroupWs w{};
+    size_t o = 0;
+    auto take = [&](size_t bytes) { const size_t at = o; o += align256(bytes); return at; };
+    w.tc = take(dart::sma_bwd_tc_workspace(B, L, Hg, Mc, N));
+    w.M = take(B * Mc * Hg * N * P * em);
+    w.rM = take(B * Mc * Hg * N * 4);
+    w.Q = take(B * L * N * ei);
+    w.C = take(B * L * N * ei);
+    w.E = take(B * L * P * ei);
+    w.z = take(B * L * Hg * ei);
+    w.lse = take(B * L * Hg * 4);
+    w.dY = take(B * L * Hg * P * ei);
+    w.logits = take(B * Hg * Mc * L * 4);
+    w.dM = take(B * Mc * Hg * N * P * 4);
+    w.dQ = take(B * L * N * 4);
+    w.dC = take(B * L * N * 4);
+    w.dE = take(B * L * P * 4);
+    w.dz = take(B * L * Hg * 4);
+    w.total = o;
+    return w;
+}
+
+struct ScanBwdGroupWs {
+    size_t tc, X, dt, Bm, Cm, dY, dM, dX, ddt, dB, dC, total;
+};
+ScanBwdGroupWs scan_bwd_group_ws(const dart_dims* d) {
+    const size_t B = d->batch, L = d->seqlen, Hg = d->nheads / d->ngroups, P = d->headdim, N = d->dstate,
+                 Mc = d->seqlen / d->chunk;
+    ScanBwdGroupWs w{};
+    size_t o = 0;
+    auto take = [&](size_t bytes) { const size_t at = o; o += align256(bytes); return at; };
+    w.tc = take(dart::scan_bwd_tc_workspace(B, L, Hg, d->chunk));
+    w.X = take(B * L * Hg * P * 2);
+    w.dt = take(B * L * Hg * 4);
+    w.Bm = take(B * L * N * 2);
+    w.Cm = take(B * L * N * 2);
+    w.dY = take(B * L * Hg * P * 2);
+    w.dM = take(B * Mc * Hg * N * P * 4);
+    w.dX = take(B * L * Hg * P * 4);
+    w.ddt = take(B * L * Hg * 4);
+    w.dB = take(B * L * N * 4);
+    w.dC = take(B * L * N * 4);
+    w.total = o;
+    return w;
+}
+
+// One group's slice of rows: `rows` rows of `row` bytes, `pitch` bytes apart in the
+// full array, starting `off` bytes in; packed (pitch = row) in the group buffer.
+struct Slice {
+    i64 rows, row, pitch, off;
+};
+cudaError_t gather(void* dst, const void* src, Slice s, cudaStream_t st) {
+    return dart::launch_copy_rows(dst, s.row, (const uint8_t*)src + s.off, s.pitch, s.row, s.rows, st);
+}
+cudaError_t scatter(void* dst, const void* src, Slice s, cudaStream_t st) {
+    return dart::launch_copy_rows((uint8_t*)dst + s.off, s.pitch, src, s.row, s.row, s.rows, st);
+}
+
+cudaError_t sma_backward_grouped(const dart_dims* d, const dart::SmaBwdArgs& f, void* ws,
+                                 unsigned long long lim, cudaStream_t st) {
+    const i64 B = d->batch, L = d->seqlen, H = d->nheads, G = d->ngroups, Hg = H / G, P = d->headdim,
+              N = d->dstate, Mc = d->seqlen / d->chunk;
+    const i64 em = d->mem_dtype == DART_F32 ? 4 : 2, ei = 2;
+    const SmaBwdGroupWs w = sma_bwd_group_ws(d);
+    uint8_t* b = (uint8_t*)ws;
+    const dart_dims gd = group_dims(d);
+    dart::SmaBwdArgs a = sma_bwd_args(&gd);
+    a.test_withhold = f.test_withhold;
+    a.M = b + w.M; a.rM = f.rM != nullptr ? (const float*)(b + w.rM) : nullptr;
+    a.Q = b + w.Q; a.Cm = b + w.C; a.E = b + w.E; a.z = b + w.z; a.lse = (const float*)(b + w.lse);
+    a.dY = b + w.dY; a.logits = f.logits != nullptr ? (const float*)(b + w.logits) : nullptr;
+    a.dM = (float*)(b + w.dM); a.dQ = (float*)(b + w.dQ); a.dC = (float*)(b + w.dC);
+    a.dE = (float*)(b + w.dE); a.dz = (float*)(b + w.dz);
+    cudaError_t e = cudaSuccess;
+    for (i64 g = 0; g < G && e == cudaSuccess; ++g) {
+        const i64 h0 = g * Hg;
+        const Slice mem{B * Mc, Hg * N * P * em, H * N * P * em, h0 * N * P * em};
+        const Slice rms{B * Mc, Hg * N * 4, H * N * 4, h0 * N * 4};
+        const Slice key{B * L, N * ei, G * N * ei, g * N * ei};
+        const Slice val{B * L, P * ei, G * P * ei, g * P * ei};
+        const Slice head_in{B * L, Hg * ei, H * ei, h0 * ei};
+        const Slice head_f32{B * L, Hg * 4, H * 4, h0 * 4};
+        const Slice row_in{B * L, Hg * P * ei, H * P * ei, h0 * P * ei};
+        const Slice lgt{B, Hg * Mc * L * 4, H * Mc * L * 4, h0 * Mc * L * 4};
+        const Slice dmem{B * Mc, Hg * N * P * 4, H * N * P * 4, h0 * N * P * 4};
+        const Slice dkey{B * L, N * 4, G * N * 4, g * N * 4};
+        const Slice dval{B * L, P * 4, G * P * 4, g * P * 4};
+        if ((e = gather((void*)a.M, f.M, mem, st)) != cudaSuccess ||
+            (f.rM != nullptr && (e = gather((void*)a.rM, f.rM, rms, st)) != cudaSuccess) ||
+            (e = gather((void*)a.Q, f.Q, key, st)) != cudaSuccess ||
+            (e = gather((void*)a.Cm, f.Cm, key, st)) != cudaSuccess ||
+            (e = gather((void*)a.E, f.E, val, st)) != cudaSuccess ||
+            (e = gather((void*)a.z, f.z, head_in, st)) != cudaSuccess ||
+            (e = gather((void*)a.lse, f.lse, head_f32, st)) != cudaSuccess ||
+            (e = gather((void*)a.dY, f.dY, row_in, st)) != cudaSuccess ||
+            (f.logits != nullptr && (e = gather((void*)a.logits, f.logits, lgt, st)) != cudaSuccess))
+            break;
+        e = d->mem_dtype == DART_F32 ? dart::launch_sma_backward_tc<float>(a, b + w.tc, lim, st)
+                                     : dart::launch_sma_backward_tc<__nv_bfloat16>(a, b + w.tc, lim, st);
+        if (e != cudaSuccess) break;
+        if ((e = scatter(f.dM, a.dM, dmem, st)) != cudaSuccess || (e = scatter(f.dQ, a.dQ, dkey, st)) != cudaSuccess ||
+            (e = scatter(f.dC, a.dC, dkey, st)) != cudaSuccess || (e = scatter(f.dE, a.dE, dval, st)) != cudaSuccess ||
+            (e = scatter(f.dz, a.dz, head_f32, st)) != cudaSuccess)
+            break;
+    }
+    return e;
+}
+
+cudaError_t scan_backward_grouped(const dart_dims* d, const dart::ScanBwdArgs& f, void* ws,
+                                  unsigned long long lim, cudaStream_t st) {
+    const i64 B = d->batch, L = d->seqlen, H = d->nheads, G = d->ngroups, Hg = H / G, P = d->headdim,
+              N = d->dstate, Mc = d->seqlen / d->chunk;
+    const ScanBwdGroupWs w = scan_bwd_group_ws(d);
+    uint8_t* b = (uint8_t*)ws;
+    dart::ScanBwdArgs a{};
+    dart::ScanArgs& g1 = a.fwd;
+    g1 = f.fwd;
+    g1.H = Hg; g1.G = 1;
+    g1.X = b + w.X; g1.dt = (const float*)(b + w.dt); g1.Bm = b + w.Bm; g1.Cm = b + w.Cm;
+    a.dY = b + w.dY; a.dM = f.dM != nullptr ? (const float*)(b + w.dM) : nullptr;
+    a.dX = (float*)(b + w.dX); a.ddt = (float*)(b + w.ddt); a.dB = (float*)(b + w.dB); a.dC = (float*)(b + w.dC);
+    a.accumulate_dC = true;  // onto the caller's dC block, copied in below
+    cudaError_t e = cudaSuccess;
+    for (i64 g = 0; g < G && e == cudaSuccess; ++g) {
+        const i64 h0 = g * Hg;
+        const Slice row_in{B * L, Hg * P * 2, H * P * 2, h0 * P * 2};
+        const Slice row_f32{B * L, Hg * P * 4, H * P * 4, h0 * P * 4};
+        const Slice head_f32{B * L, Hg * 4, H * 4, h0 * 4};
+        const Slice key{B * L, N * 2, G * N * 2, g * N * 2};
+        const Slice dkey{B * L, N * 4, G * N * 4, g * N * 4};
+        const Slice dmem{B * Mc, Hg * N * P * 4, H * N * P * 4, h0 * N * P * 4};
+        g1.A = f.fwd.A + h0;
+        a.dA = f.dA + h0;
+        if ((e = gather((void*)g1.X, f.fwd.X, row_in, st)) != cudaSuccess ||
+            (e = gather((void*)g1.dt, f.fwd.dt, head_f32, st)) != cudaSuccess ||
+            (e = gather((void*)g1.Bm, f.fwd.Bm, key, st)) != cudaSuccess ||
+            (e = gather((void*)g1.Cm, f.fwd.Cm, key, st)) != cudaSuccess ||
+            (e = gather((void*)a.dY, f.dY, row_in, st)) != cudaSuccess ||
+            (f.dM != nullptr && (e = gather((void*)a.dM, f.dM, dmem, st)) != cudaSuccess) ||
+            (e = gather(a.dC, f.dC, dkey, st)) != cudaSuccess)
+            break;
+        if ((e = dart::launch_chunk_scan_backward<__nv_bfloat16>(a, b + w.tc, lim, st)) != cudaSuccess) break;
+        if ((e = scatter(f.dX, a.dX, row_f32, st)) != cudaSuccess ||
+            (e = scatter(f.ddt, a.ddt, head_f32, st)) != cudaSuccess ||
+            (e = scatter(f.dB, a.dB, dkey, st)) != cudaSuccess || (e = scatter(f.dC, a.dC, dkey, st)) != cudaSuccess)
+            break;
+    }
+    return e;
+}
+
 // Workspace of the SMA forward for L % S == 0.
 size_t sma_ws_aligned(const dart_dims* d) {
     const i64 M = d->seqlen / d->chunk;
@@ -427,6 +612,7 @@ size_t dart_workspace_size(const dart_dims* d, int op) {
             if (sma_bwd_uses_tc(d))
                 return align256(dart::sma_bwd_tc_workspace(d->batch, d->seqlen, d->nheads,
                                                            d->seqlen / d->chunk, d->dstate));
+            if (sma_bwd_grouped(d)) return sma_bwd_group_ws(d).total;
             return align256(dart::sma_bwd_workspace(d->batch, d->seqlen, d->nheads,
                                                     d->seqlen / d->chunk, d->dstate));
         case DART_OP_SCAN_BACKWARD: {
@@ -436,6 +622,7 @@ size_t dart_workspace_size(const dart_dims* d, int op) {
             a.P = d->headdim; a.N = d->dstate; a.S = d->chunk;
             if (d->in_dtype == DART_BF16 && dart::scan_bwd_tc_supported(a))
                 return align256(dart::scan_bwd_tc_workspace(d->batch, d->seqlen, d->nheads, d->chunk));
+            if (scan_bwd_grouped(d)) return scan_bwd_group_ws(d).total;
             return align256(dart::scan_bwd_workspace(d->batch, d->seqlen, d->nheads, d->dstate,
                                                      d->headdim, d->chunk));
         }
@@ -800,6 +987,8 @@ static dart_status sma_backward_impl(const dart_dims* d, const void* M, const fl
             e = dart::launch_sma_backward_tc<float>(a, ws, lim, s);
         else
             e = dart::launch_sma_backward_tc<bf>(a, ws, lim, s);
+    } else if (sma_bwd_grouped(d)) {
+        e = sma_backward_grouped(d, a, ws, g_wait_limit_ns.load(), s);
     } else if (d->in_dtype == DART_F32 && d->mem_dtype == DART_F32)
         e = dart::launch_sma_backward<float, float>(a, ws, s);
     else if (d->in_dtype == DART_BF16 && d->mem_dtype == DART_F32)
@@ -852,7 +1041,9 @@ dart_status dart_chunk_scan_backward(const dart_dims* d, const void* X, const fl
     f.test_withhold = g_test_withhold.load();
     cudaStream_t s = (cudaStream_t)stream;
     cudaError_t e;
-    if (d->in_dtype == DART_F32)
+    if (scan_bwd_grouped(d))
+        e = scan_backward_grouped(d, a, ws, g_wait_limit_ns.load(), s);
+    else if (d->in_dtype == DART_F32)
         e = dart::launch_chunk_scan_backward<float>(a, ws, g_wait_limit_ns.load(), s);
     else if (d->in_dtype == DART_BF16)
         e = dart::launch_chunk_scan_backward<__nv_bfloat16>(a, ws, g_wait_limit_ns.load(), s);

@@ -195,6 +195,9 @@ cudaError_t launch_sma_forward_simt(const SmaArgs& a, cudaStream_t stream);
 template <typename Tin, typename Tmem, typename Tout>
 cudaError_t launch_decode_step(const DecodeArgs& a, cudaStream_t stream);
 
+// dst[r * dst_pitch + i] = src[r * src_pitch + i], i < row_bytes, r < rows (bytes).
+cudaError_t launch_copy_rows(void* dst, int64_t dst_pitch, const void* src, int64_t src_pitch, int64_t row_bytes,
+                             int64_t rows, cudaStream_t stream);
 // dst[r, k] = src[r, h0 + k] for r < rows, k < hg (elements of elem_bytes = 2 or 4;
 // src rows of H elements, dst rows of hg).
 cudaError_t launch_gather_heads(const void* src, void* dst, int64_t rows, int64_t H, int64_t h0,

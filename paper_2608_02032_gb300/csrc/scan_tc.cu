@@ -100,7 +100,21 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
     for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
 
-__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
+// The x16 load without the wait, so that several can be in flight; the caller
+// issues tcgen05.wait::ld before reading any of the registers.
+__device__ __forceinline__ void tmem_ld16_nowait(uint32_t taddr, uint32_t (&r)[16]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+          "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr)
+        : "memory");
+}
+__device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+
+[[maybe_unused]] __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
     uint32_t r[16];
     asm volatile(
         "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
@@ -623,6 +637,26 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
     const int s_lo = quarter * (ns / 4), s_hi = s_lo + ns / 4;  // 32 or 64 sources
     for (int hh = 0; hh < hpc && ok; ++hh) {
         const int h = h0 + hh;
+        // the inter-chunk chain C H_[c-1] needs no W: issued first, it runs under the W pass
+        bool hok = true;
+        if (tid == 0 && has_prev) {
+            tc::tc_fence_after();
+            hok = tc::mbar_wait(&sm.hbar[hh & 1], (uint32_t)((hh >> 1) & 1), wait_limit_ns, nullptr);
+            if (hok) {
+                const uint32_t idb = tc::idesc_f16(1, true, kT, kP);
+                for (int part = 0; part < 2; ++part) {
+                    for (int ks = 0; ks < kN / 16; ++ks) {
+                        const uint64_t ad = tc::smem_desc_sw128(
+                            tc::smem_u32(sm.c_tile[ks / 4]) + 32u * (ks % 4), 16u, 1024u);
+                        const uint64_t bd = tc::smem_desc_sw128(
+                            tc::smem_u32(hbuf(hh & 1) + 16384 * part) + 2048u * ks, 1024u, 1024u);
+                        mma_f16_ss(tmem + kColEx, ad, bd, idb, (part > 0 || ks > 0) ? 1u : 0u);
+                    }
+                }
+            } else {
+                atomicCAS(&g_scan_tc_status, 0, 11);
+            }
+        }
         // prefetched sources into shared memory (the previous head's MMAs are done)
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
@@ -653,7 +687,8 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
         __syncthreads();
         if (hh + 1 < hpc) {  // lands while this head computes
             load_head(h + 1);
-            // buffer (hh + 1) & 1 was last read by head hh - 1's MMAs (or the scores), both done
+            // buffer (hh + 1) & 1 was last read by head hh - 1's MMAs (or the scores), both
+            // done: their commit was waited for before head hh began
             if (tid == 0 && has_prev) issue_h(hh + 1);
         }
 
@@ -699,29 +734,15 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
         tc::fence_proxy_async_shared();
         tc::tc_fence_before();
         __syncthreads();
-        bool hok = true;
         if (tid == 0) {
             tc::tc_fence_after();
-            if (has_prev) hok = tc::mbar_wait(&sm.hbar[hh & 1], (uint32_t)((hh >> 1) & 1), wait_limit_ns, nullptr);
             const uint32_t id16 = tc::idesc_f16(0, true, kT, kP);
             for (int ks = 0; kIntra && ks < ns / 16; ++ks) {
                 const uint64_t bd = tc::smem_desc_sw128(tc::smem_u32(sm.x_src) + 2048u * ks, 1024u, 1024u);
                 tc::mma_f16_ts(tmem + kColIn, tmem + kColW + 8u * ks, bd, id16, ks > 0 ? 1u : 0u);
             }
-            if (has_prev && hok) {
-                const uint32_t idb = tc::idesc_f16(1, true, kT, kP);
-                for (int part = 0; part < 2; ++part) {
-                    for (int ks = 0; ks < kN / 16; ++ks) {
-                        const uint64_t ad = tc::smem_desc_sw128(
-                            tc::smem_u32(sm.c_tile[ks / 4]) + 32u * (ks % 4), 16u, 1024u);
-                        const uint64_t bd = tc::smem_desc_sw128(
-                            tc::smem_u32(hbuf(hh & 1) + 16384 * part) + 2048u * ks, 1024u, 1024u);
-                        mma_f16_ss(tmem + kColEx, ad, bd, idb, (part > 0 || ks > 0) ? 1u : 0u);
-                    }
-                }
-            }
-            if (!hok) atomicCAS(&g_scan_tc_status, 0, 11);
         }
+        // the commit tracks both chains
         ok = commit_and_wait(&sm.bar, phase, wait_limit_ns, 3, hok);
         phase ^= 1u;
         if (!ok) break;
@@ -729,17 +750,16 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
         {
             const float dec = exp2f(c2t);
             float vi[16], ve[16];
-            if (kIntra) {
-                tmem_ld16(tmem + lane_addr + kColIn + 16u * quarter, vi);
-            } else {
+            {
+                uint32_t ri[16], re[16];
+                if (kIntra) tmem_ld16_nowait(tmem + lane_addr + kColIn + 16u * quarter, ri);
+                if (has_prev) tmem_ld16_nowait(tmem + lane_addr + kColEx + 16u * quarter, re);
+                if (kIntra || has_prev) tmem_wait_ld();
 #pragma unroll
-                for (int i = 0; i < 16; ++i) vi[i] = 0.0f;
-            }
-            if (has_prev) {
-                tmem_ld16(tmem + lane_addr + kColEx + 16u * quarter, ve);
-            } else {
-#pragma unroll
-                for (int i = 0; i < 16; ++i) ve[i] = 0.0f;
+                for (int i = 0; i < 16; ++i) {
+                    vi[i] = kIntra ? __uint_as_float(ri[i]) : 0.0f;
+                    ve[i] = has_prev ? __uint_as_float(re[i]) : 0.0f;
+                }
             }
             if (kMode == kOutRev) {
                 // dX = dt Y', and X . (inter part of Y')

@@ -7,7 +7,7 @@ import torch
 
 import oracle
 from helpers import TOL, dev, host, rel_err
-from paper_2608_02032_gb300 import api
+from paper_2608_02032_gb300 import api, binding
 from paper_2608_02032_gb300.workloads import WORKLOADS, Workload, memory_grad_input, prefill_inputs
 
 pytestmark = pytest.mark.gpu
@@ -23,6 +23,10 @@ CASES = [
     # eight heads: the tensor-core scan backward (head groups of 8)
     Workload("bwd_bf16_h8_s256", 1, 8, 1024, 64, 128, 256, seed=2107),
     Workload("bwd_bf16_h8_s128", 2, 8, 512, 64, 128, 128, seed=2108),
+    # G = 2: the tensor-core backward once per group of 8 heads (scan and SMA)
+    Workload("bwd_bf16_h16_g2_s128", 1, 16, 512, 64, 128, 128, groups=2, seed=2109),
+    # G = 2 with 4 heads per group: the SMA backward per group on the tensor cores, the scan on FFMA
+    Workload("bwd_bf16_h8_g2_s256", 2, 8, 1024, 64, 128, 256, groups=2, seed=2110),
 ]
 
 
@@ -78,7 +82,7 @@ def test_sma_backward_matches_oracle(w):
         assert err <= _tol(w), f"{name}: {err:.3e}"
 
 
-@pytest.mark.parametrize("w", [CASES[0], CASES[3], CASES[6]], ids=lambda w: w.name)
+@pytest.mark.parametrize("w", [CASES[0], CASES[3], CASES[6], CASES[8]], ids=lambda w: w.name)
 def test_layer_backward_matches_oracle(w):
     """Forward through the library, then the layer backward: SMA backward's dM and
     dC feed the scan backward."""
@@ -97,7 +101,7 @@ def test_layer_backward_matches_oracle(w):
         assert err <= _tol(w), f"{name}: {err:.3e}"
 
 
-@pytest.mark.parametrize("w", [CASES[3], CASES[6], CASES[7]], ids=lambda w: w.name)
+@pytest.mark.parametrize("w", [CASES[3], CASES[6], CASES[7], CASES[8]], ids=lambda w: w.name)
 def test_layer_backward_with_saved_logits(w):
     """The training pair that keeps the forward's logits: the backward takes its
     softmax weights from them instead of recomputing the logit chains. Against the
@@ -124,6 +128,26 @@ def test_layer_backward_with_saved_logits(w):
         assert rel_err(host(g), r) <= _tol(w), n
         assert rel_err(host(g), host(g2)) <= tol_same.get(n, 1e-5), n
     assert rel_err(host(gr.dM), host(gr2.dM)) <= 1e-5
+
+
+def test_grouped_backward_runs_per_group_on_the_tensor_cores():
+    """At G = 2 with 8 heads per group, each backward runs the G = 1 tensor-core
+    kernels once per group on copied slices: per group at least 7 (scan) and 7
+    (SMA) copies in and 4 and 5 copies out besides the backward's own kernels, far
+    more launches than the CUDA-core backward makes. Parity is checked above."""
+    w = CASES[8]
+    inp = prefill_inputs(w, with_grad=True)
+    X, Bm, Cm, Q, E, z, dY = (dev(inp[k], w.dtype) for k in ("X", "Bm", "Cm", "Q", "E", "z", "dY"))
+    dt, A = dev(inp["dt"], torch.float32), dev(inp["A"], torch.float32)
+    s, o = api.prefill_forward(X, dt, A, Bm, Cm, Q, E, z, w.chunk, w.eps)
+    torch.cuda.synchronize()
+    n0 = binding.dart_launch_count()
+    gM, gQ, gC, gE, gz = api.sma_backward(s.M, s.rM, Q, Cm, E, z, o.lse, dY, w.chunk, w.eps)
+    n1 = binding.dart_launch_count()
+    api.chunk_scan_backward(X, dt, A, Bm, Cm, dY, gM, w.chunk, dC=gC, eps=w.eps)
+    n2 = binding.dart_launch_count()
+    torch.cuda.synchronize()
+    assert n1 - n0 >= 2 * (7 + 5) and n2 - n1 >= 2 * (7 + 4), (n1 - n0, n2 - n1)
 
 
 def test_backward_single_chunk_has_no_sma_gradient():
