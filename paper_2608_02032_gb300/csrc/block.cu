@@ -25,82 +25,64 @@ namespace {
 constexpr int kMaxConv = 8;
 
 // The convolution of the in-projection's x, B, C blocks (columns di .. di + conv_ch
-// of zx). A block of 256 threads covers 256 channels x 64 tokens: warp r takes the
-// tokens tok0 + 8 r .. + 7, lane c the channels 8 c .. 8 c + 7 of the block's range
-// (a warp's loads of one row are 1 KiB contiguous). Each thread keeps its channels'
-// taps and a window of the last W input rows in registers, so every row is loaded
-// once per thread: W - 1 rows before its first token, then one per token.
-constexpr int kConvTok = 64, kConvCh = 256;
+// of zx). A block of 256 threads covers 128 channels x 128 tokens: warp r takes the
+// tokens tok0 + 16 r .. + 15, lane c the channels 4 c .. 4 c + 3 of the block's range
+// (a warp's loads of one row are 512 contiguous bytes). Each thread loads the W - 1
+// rows before its first token and its 16 rows up front, all in flight at once, and
+// keeps its channels' taps in registers. A group of 4 channels never straddles x, B
+// and C (di and GN are multiples of 4).
+constexpr int kConvTok = 16, kConvWarps = 8, kConvCh = 128;
 template <int W>
 __global__ void __launch_bounds__(256)
 block_conv_kernel(const float* __restrict__ zx, int ldz, int64_t T, int L, int di, int conv_ch,
                   const float* __restrict__ conv_w, const float* __restrict__ conv_b,
                   __nv_bfloat16* __restrict__ X, __nv_bfloat16* __restrict__ Bm, __nv_bfloat16* __restrict__ Cm,
                   int GN) {
-    const int c0 = kConvCh * blockIdx.y + 8 * (threadIdx.x & 31);  // channel within x | B | C
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int c0 = kConvCh * blockIdx.y + 4 * lane;  // channel within x | B | C
     if (c0 >= conv_ch) return;
-    const i64 tok0 = (i64)kConvTok * blockIdx.x + 8 * (threadIdx.x >> 5);
+    const i64 tok0 = ((i64)blockIdx.x * kConvWarps + warp) * kConvTok;
     if (tok0 >= T) return;
-    float w[8][W], bias[8];
+    float w[4][W], bias[4];
 #pragma unroll
-    for (int e = 0; e < 8; ++e) {
+    for (int e = 0; e < 4; ++e) {
         bias[e] = conv_b[c0 + e];
 #pragma unroll
         for (int k = 0; k < W; ++k) w[e][k] = conv_w[(c0 + e) * W + k];
     }
     __nv_bfloat16* dst = c0 < di ? X + c0 : c0 < di + GN ? Bm + (c0 - di) : Cm + (c0 - di - GN);
     const int ld_dst = c0 < di ? di : GN;
-    auto load = [&](i64 tok, float (&v)[8]) {
-        const float* src = zx + tok * ldz + di + c0;
-        const float4 u0 = *reinterpret_cast<const float4*>(src);
-        const float4 u1 = *reinterpret_cast<const float4*>(src + 4);
-        v[0] = u0.x; v[1] = u0.y; v[2] = u0.z; v[3] = u0.w; v[4] = u1.x; v[5] = u1.y; v[6] = u1.z; v[7] = u1.w;
-    };
-    // win[k] holds the row of token tok - (W - 1) + k (zeros before the sequence start)
-    float win[W][8];
+    // v[r] holds the row of token tok0 - (W - 1) + r (zeros outside 0 .. T - 1)
+    constexpr int kR = W - 1 + kConvTok;
+    float4 v[kR];
+#pragma unroll
+    for (int r = 0; r < kR; ++r) {
+        const i64 tk = tok0 - (W - 1) + r;
+        v[r] = tk >= 0 && tk < T ? *reinterpret_cast<const float4*>(zx + tk * ldz + di + c0)
+                                 : make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+    }
     const int t0 = (int)(tok0 % L);
 #pragma unroll
-    for (int k = 0; k < W - 1; ++k) {
-        const int back = W - 1 - k;
-        if (t0 - back >= 0) {
-            load(tok0 - back, win[k]);
-        } else {
+    for (int i = 0; i < kConvTok; ++i) {
+        if (tok0 + i >= T) break;
+        const int pos = (t0 + i) % L;  // position in its sequence: taps further back read zeros
+        float acc[4] = {bias[0], bias[1], bias[2], bias[3]};
 #pragma unroll
-            for (int e = 0; e < 8; ++e) win[k][e] = 0.0f;
+        for (int k = 0; k < W; ++k) {
+            if (W - 1 - k <= pos) {
+                const float4 x = v[i + k];
+                acc[0] = fmaf(w[0][k], x.x, acc[0]);
+                acc[1] = fmaf(w[1][k], x.y, acc[1]);
+                acc[2] = fmaf(w[2][k], x.z, acc[2]);
+                acc[3] = fmaf(w[3][k], x.w, acc[3]);
+            }
         }
-    }
-    const bool full = tok0 + 8 <= T;
-    float nxt[4][8];  // the rows of four tokens, loaded together ahead of their arithmetic
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-        const i64 tok = tok0 + i;
-        if ((i & 3) == 0) {
-#pragma unroll
-            for (int u = 0; u < 4; ++u)
-                if (full || tok + u < T) load(tok + u, nxt[u]);
-        }
-        if (!full && tok >= T) break;
-        if (i > 0 && (t0 + i) % L == 0) {  // a new sequence starts: nothing before it
-#pragma unroll
-            for (int k = 0; k < W - 1; ++k)
-#pragma unroll
-                for (int e = 0; e < 8; ++e) win[k][e] = 0.0f;
-        }
-#pragma unroll
-        for (int e = 0; e < 8; ++e) win[W - 1][e] = nxt[i & 3][e];
-        float acc[8];
-#pragma unroll
-        for (int e = 0; e < 8; ++e) {
-            acc[e] = bias[e];
-#pragma unroll
-            for (int k = 0; k < W; ++k) acc[e] = fmaf(w[e][k], win[k][e], acc[e]);
-            acc[e] = silu_f32(acc[e]);
-        }
-        store_row8(dst + tok * ld_dst, acc);
-#pragma unroll
-        for (int k = 0; k < W - 1; ++k)
-#pragma unroll
-            for (int e = 0; e < 8; ++e) win[k][e] = win[k + 1][e];
+        const __nv_bfloat162 lo = __floats2bfloat162_rn(silu_f32(acc[0]), silu_f32(acc[1]));
+        const __nv_bfloat162 hi = __floats2bfloat162_rn(silu_f32(acc[2]), silu_f32(acc[3]));
+        uint2 o;
+        o.x = *reinterpret_cast<const uint32_t*>(&lo);
+        o.y = *reinterpret_cast<const uint32_t*>(&hi);
+        *reinterpret_cast<uint2*>(dst + (tok0 + i) * ld_dst) = o;
     }
 }
 
@@ -149,23 +131,32 @@ block_norm_kernel(const float* __restrict__ Y, const __nv_bfloat16* __restrict__
     const int groups = di / 8;
     float g[kNormGroups][8];
     float ss = 0.0f;
+    // every group of the lane: no early exit, so that all its loads are in flight together
 #pragma unroll
     for (int j = 0; j < kNormGroups; ++j) {
         const int q = lane + 32 * j;
-        if (q >= groups) break;
-        const int c0 = 8 * q;
-        const float4 y0 = *reinterpret_cast<const float4*>(Y + tok * di + c0);
-        const float4 y1 = *reinterpret_cast<const float4*>(Y + tok * di + c0 + 4);
-        const float4 z0 = *reinterpret_cast<const float4*>(zx + tok * ldz + c0);  // z: the first column block
-        const float4 z1 = *reinterpret_cast<const float4*>(zx + tok * ldz + c0 + 4);
+        const bool live = q < groups;
+        const int c0 = live ? 8 * q : 0;
+        const float4 zero = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+        const float4 y0 = live ? *reinterpret_cast<const float4*>(Y + tok * di + c0) : zero;
+        const float4 y1 = live ? *reinterpret_cast<const float4*>(Y + tok * di + c0 + 4) : zero;
+        const float4 z0 = live ? *reinterpret_cast<const float4*>(zx + tok * ldz + c0) : zero;  // z: the first block
+        const float4 z1 = live ? *reinterpret_cast<const float4*>(zx + tok * ldz + c0 + 4) : zero;
+        const uint4 xr = live ? *reinterpret_cast<const uint4*>(X + tok * di + c0) : make_uint4(0u, 0u, 0u, 0u);
+        const uint32_t xw[4] = {xr.x, xr.y, xr.z, xr.w};
         float xv[8];
-        load_row8(X + tok * di + c0, xv);
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&xw[e]));
+            xv[2 * e] = f.x;
+            xv[2 * e + 1] = f.y;
+        }
         const float yv[8] = {y0.x, y0.y, y0.z, y0.w, y1.x, y1.y, y1.z, y1.w};
         const float zv[8] = {z0.x, z0.y, z0.z, z0.w, z1.x, z1.y, z1.z, z1.w};
-        const float d = D[c0 / P];  // 8 channels never straddle heads (P % 8 == 0)
+        const float d = live ? D[c0 / P] : 0.0f;  // 8 channels never straddle heads (P % 8 == 0)
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
-            g[j][e] = fmaf(d, xv[e], yv[e]) * silu_f32(zv[e]);
+            g[j][e] = fmaf(d, xv[e], yv[e]) * silu_f32(zv[e]);  // 0 for a dead group
             ss = fmaf(g[j][e], g[j][e], ss);
         }
     }
@@ -190,8 +181,9 @@ cudaError_t launch_block_conv_split(const BlockArgs& a, cudaStream_t stream) {
     const int di = (int)(a.H * a.P), GN = (int)(a.G * a.N), GP = (int)(a.G * a.P);
     const int64_t T = a.B * a.L;
     const int conv_ch = di + 2 * GN;
-    if ((T + kConvTok - 1) / kConvTok > 0x7fffffff) return cudaErrorInvalidValue;
-    const dim3 grid((unsigned)((T + kConvTok - 1) / kConvTok), (unsigned)((conv_ch + kConvCh - 1) / kConvCh));
+    constexpr int kBlockTok = kConvTok * kConvWarps;
+    if ((T + kBlockTok - 1) / kBlockTok > 0x7fffffff) return cudaErrorInvalidValue;
+    const dim3 grid((unsigned)((T + kBlockTok - 1) / kBlockTok), (unsigned)((conv_ch + kConvCh - 1) / kConvCh));
     auto conv = [&](auto kw) {
         block_conv_kernel<decltype(kw)::value><<<grid, 256, 0, stream>>>(
             (const float*)a.zx, (int)a.ldz, T, (int)a.L, di, conv_ch, a.conv_w, a.conv_b, (__nv_bfloat16*)a.X,
