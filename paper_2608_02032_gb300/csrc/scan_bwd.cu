@@ -374,7 +374,8 @@ cudaError_t launch_scan_bwd_passing(float* ZD, const float* dM, const float* Hpr
     return cudaGetLastError();
 }
 
-bool scan_bwd_tc_supported(const ScanArgs& f) { return f.G == 1 && scan_tc_supported(f); }
+// The backward's output-kernel modes run 128-token tiles inside a chunk: S in {128, 256}.
+bool scan_bwd_tc_supported(const ScanArgs& f) { return f.G == 1 && f.S >= 128 && scan_tc_supported(f); }
 
 template <typename Tin>
 cudaError_t launch_chunk_scan_backward(const ScanBwdArgs& a, void* ws, unsigned long long wait_limit_ns,

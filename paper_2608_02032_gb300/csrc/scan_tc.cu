@@ -1,5 +1,5 @@
 // Chunked SSD scan on the 5th-generation tensor cores for bf16 token inputs,
-// P = 64, N = 128, S in {128, 256} (Sec. 2; Sec. 3 "Chunk State Memories";
+// P = 64, N = 128, S in {64, 128, 256} (Sec. 2; Sec. 3 "Chunk State Memories";
 // App. A chunked scan). The chunk-state and chunk-output kernels run on the
 // tensor cores, the state passing streams the chunk states through shared
 // memory with bulk copies; the within-chunk cumsum is shared with the FFMA
@@ -25,6 +25,8 @@
 //   (one 32 KiB bulk copy per head, double-buffered). A CPU emulation against the oracle gives
 //   max|err|/RMS(Y) = 2.1e-3 with the exact row maximum as the scale (5.4e-3
 //   without a row scale, 4.2e-2 with plain bf16).
+//   With S = 64 the tile holds one chunk: rows 64 .. 127 are idle (zero C rows,
+//   nothing stored) and the 64 sources are two groups of 32 per row.
 // TMEM of the output kernel: scores [0, 256), W [256, 384), intra accumulator
 // [384, 448), inter accumulator [448, 512).
 #include <math.h>
@@ -511,7 +513,9 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
     const int row = tid & (kT - 1), quarter = tid >> 7;  // token row, quarter of the sources / columns
     const int h0 = hg * hpc;
     const int g = h0 / (H / G);
-    const int ns = (tt + 1) * kT;  // sources 0 .. ns-1 of the chunk
+    // sources 0 .. ns-1 of the chunk; with S = 64 the 128-row tile holds one chunk and
+    // its rows S .. 127 are idle (zero C rows, nothing stored)
+    const int ns = min((tt + 1) * kT, S);
     const i64 tok0 = (i64)b * L + (i64)c * S;
     const uint32_t lane_addr = (uint32_t)(32 * (warp & 3)) << 16;
     const bool has_prev = kMode == kOutRev || c > 0;
@@ -548,7 +552,9 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
     // C of the tile: row t, K-major, two K blocks of 64 (16-byte chunks, swizzled)
     for (int i = tid; i < kT * 16; i += kOutThreads) {
         const int t = i / 16, q = i % 16;
-        const uint4 v = reinterpret_cast<const uint4*>(Cm + ((tok0 + pos(tt * kT + t)) * G + g) * kN)[q];
+        const uint4 v = tt * kT + t < S
+                            ? reinterpret_cast<const uint4*>(Cm + ((tok0 + pos(tt * kT + t)) * G + g) * kN)[q]
+                            : make_uint4(0u, 0u, 0u, 0u);
         *reinterpret_cast<uint4*>(sm.c_tile[q / 8] + sw128((uint32_t)t, (uint32_t)(q % 8) * 16u)) = v;
     }
     // B of the sources: row s, K-major
@@ -573,7 +579,8 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
         }
         sm.bnorm[tid] = sqrtf(ss);
     }
-    if (tid < kT) {
+    if (tid < kT && tt * kT + tid >= S) sm.cnorm[tid] = 0.0f;
+    if (tid < kT && tt * kT + tid < S) {
         const uint4* crow = reinterpret_cast<const uint4*>(Cm + ((tok0 + pos(tt * kT + tid)) * G + g) * kN);
         float ss = 0.0f;
 #pragma unroll 4
@@ -634,7 +641,10 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
     const int tl = tt * kT + row;  // this thread's token inside the chunk (kernel order)
     const i64 tok = tok0 + pos(tl);
     const int tl_warp_max = tt * kT + 32 * (warp & 3) + 31;
-    const int s_lo = quarter * (ns / 4), s_hi = s_lo + ns / 4;  // 32 or 64 sources
+    // this thread's sources: a quarter of them (32 or 64) for ns >= 128, else 32 per
+    // thread for the first two quarters (ns = 64) and none for the others
+    const int per_q = ns >= 128 ? ns / 4 : 32;
+    const int s_lo = quarter * per_q, s_hi = min(s_lo + per_q, ns);
     for (int hh = 0; hh < hpc && ok; ++hh) {
         const int h = h0 + hh;
         // the inter-chunk chain C H_[c-1] needs no W: issued first, it runs under the W pass
@@ -694,7 +704,7 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
 
         // W row of this thread over its quarter of the sources, scaled by the bound
         // 1 / (|C_t| max_s |B_s| dt_s) and stored fp16 in one pass
-        const float c2t = sm.c2[tl];
+        const float c2t = sm.c2[min(tl, ns - 1)];  // an idle row (tl >= S) reads a live entry
         const float bound = sm.cnorm[row] * __uint_as_float(sm.bdmax[hh & 1]);
         const float wmax = bound > 0.0f ? bound : 1.0f;  // undone on the intra accumulator
         const float rscale = 1.0f / wmax;
@@ -724,7 +734,7 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
             }
             tc::tmem_st16(tmem + lane_addr + kColW + (uint32_t)(s0 / 2), pk);
         };
-        for (int s0 = s_lo; kIntra && s0 < s_hi; s0 += 32) {  // s_hi - s_lo is 32 or 64
+        for (int s0 = s_lo; kIntra && s0 < s_hi; s0 += 32) {  // s_hi - s_lo is 0, 32 or 64
             const bool live = s0 <= tl_warp_max;
             float v[32];
             if (live) tmem_ld32(tmem + lane_addr + kColSc + (uint32_t)s0, v);
@@ -779,7 +789,7 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
 #pragma unroll
                 for (int i = 0; i < 16; ++i) vi[i] = fmaf(wmax, vi[i], dec * ve[i]);
                 if (kMode == kOutY) {
-                    store_row16(Y + (tok * H + h) * kP + 16 * quarter, vi);
+                    if (tl < S) store_row16(Y + (tok * H + h) * kP + 16 * quarter, vi);
                 } else {  // dY . (inter part of Y); vi holds only that part here
                     float zv[16];
                     load_row16(Zd + (tok * H + h) * kP + 16 * quarter, zv);
@@ -845,7 +855,7 @@ int out_heads_per_cta(int units, int H, int G) {
 }
 
 bool scan_tc_supported(const ScanArgs& a) {
-    return a.P == kP && a.N == kN && (a.S == 128 || a.S == 256) &&
+    return a.P == kP && a.N == kN && (a.S == 64 || a.S == 128 || a.S == 256) &&
            a.H % kHeadsPerCta == 0 && (a.H / a.G) % kHeadsPerCta == 0;
 }
 
@@ -875,8 +885,9 @@ cudaError_t launch_chunk_scan_tc(const ScanArgs& a, unsigned long long wait_limi
         const size_t smem = sizeof(OutSmem) + 1024;
         cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
-        const int hpc = out_heads_per_cta(S / kT * M * B, H, G);
-        kern<<<dim3(S / kT, M * (H / hpc), B), kOutThreads, smem, stream>>>(
+        const int tiles = S >= kT ? S / kT : 1;  // S = 64: one tile, half of its rows idle
+        const int hpc = out_heads_per_cta(tiles * M * B, H, G);
+        kern<<<dim3(tiles, M * (H / hpc), B), kOutThreads, smem, stream>>>(
             (const __nv_bfloat16*)a.X, a.dt, a.cum, (const __nv_bfloat16*)a.Bm,
             (const __nv_bfloat16*)a.Cm, a.Hops, (Tout*)a.Y, L, H, G, S, M, hpc, wait_limit_ns,
             nullptr, nullptr);

@@ -53,18 +53,20 @@ SWEEP = [
     (768, 256, 64, 128, 4, 2, "bf16"),   # M = 3, two groups
     (320, 64, 32, 32, 2, 1, "bf16"),     # ragged last token tile inside chunks
     (1024, 128, 64, 128, 2, 1, "bf16"),
-    # tensor-core SMA shapes (bf16, P 64, N 128, S % 128 == 0, two heads per job; CTA pairs
-    # over two 128-token tiles when L % 256 == 0, one CTA per tile otherwise)
+    # tensor-core SMA shapes (bf16, P 64, N 128, two heads per job, one CTA per 128-token tile)
     (512, 128, 64, 128, 4, 1, "bf16"),     # first tile of each chunk ... M = 4
     (256, 128, 64, 128, 4, 1, "bf16"),     # M = 2
     (128, 128, 64, 128, 4, 1, "bf16"),     # M = 1: only chunk-0 tiles
-    (384, 128, 64, 128, 4, 1, "bf16"),     # L not a multiple of 256: single-CTA kernel, M = 3
-    (768, 128, 64, 128, 2, 1, "bf16"),     # CTA pairs across chunks (S = 128), M = 6
+    (384, 128, 64, 128, 4, 1, "bf16"),     # L not a multiple of 256, M = 3
+    (768, 128, 64, 128, 2, 1, "bf16"),     # M = 6
     (1024, 256, 64, 128, 8, 1, "bf16"),    # two head groups
     (768, 256, 64, 128, 8, 2, "bf16"),     # G = 2, four heads per group
-    # tensor-core scan shapes (bf16, P 64, N 128, S in {128, 256}, 8 heads per CTA)
+    # tensor-core scan shapes (bf16, P 64, N 128, S in {64, 128, 256}, 8 heads per CTA)
     (512, 128, 64, 128, 8, 1, "bf16"),
     (1024, 256, 64, 128, 16, 2, "bf16"),   # G = 2, eight heads per group
+    (1024, 64, 64, 128, 8, 1, "bf16"),     # S = 64: one chunk per 128-row tile, rows 64 .. 127 idle
+    (512, 64, 64, 128, 16, 2, "bf16"),     # S = 64, G = 2
+    (1000, 64, 64, 128, 8, 1, "bf16"),     # S = 64 and ragged: 1024 padded tokens
     # ragged L (L % S != 0): the last memory holds the partial chunk
     (1000, 256, 64, 128, 8, 1, "bf16"),    # tensor-core scan and SMA on 1024 padded tokens
     (1000, 256, 64, 128, 2, 1, "bf16"),    # CUDA-core scan, tensor-core SMA
