@@ -113,6 +113,11 @@ constexpr uint32_t kTmemCols = 512;
 constexpr int kSlots = 32 * (256 + 16);  // one warp's slots for rows of up to 256 bytes
 static_assert(kFwdJob + 8 * kSlots <= kQ8Off, "prologue slots fit job buffer 1");
 static_assert(16 * kSlots <= kStages * kPart, "merge slots fit the ring");
+static_assert(8 * kSlots <= kFwdJob, "one job buffer holds every epilogue warp's merge slots");
+// E rows of the prologue: 32 rows of 128 bytes per quadrant, 16-byte chunks XORed with
+// the row, in the ring's tail after the e4m3 Q tile (untouched by copies and the merge)
+constexpr int kEOff = kQ8Off + kRows * kN;
+static_assert(kEOff + 4 * 32 * 2 * kP <= kStages * kPart, "the E rows fit the ring's tail");
 constexpr uint32_t kColQ = 0, kColC = 64, kColU = 128, kColV = 256;  // V buffer b at kColV + 128 b
 // Bound on the final waits for this CTA's own copies and MMAs (never cut short).
 constexpr uint64_t kDrainLimitNs = 2000000000ull;
@@ -331,6 +336,21 @@ __device__ __forceinline__ void slots_to_rows(uint8_t* base, i64 stride, const u
             *reinterpret_cast<const uint4*>(slots + (i * kRpi + lane / kCpr) * (RB + 16) + (lane % kCpr) * 16);
 }
 
+// rows_to_slots without the registers: cp.async copies straight into the slots
+// (completed by cp_async_wait_all).
+template <int RB>
+__device__ __forceinline__ void rows_to_slots_async(uint8_t* slots, const uint8_t* base, i64 stride, int lane) {
+    constexpr int kCpr = RB / 16, kRpi = 32 / kCpr;
+#pragma unroll
+    for (int i = 0; i < kCpr; ++i) {
+        const uint32_t dst = tc::smem_u32(slots + (i * kRpi + lane / kCpr) * (RB + 16) + (lane % kCpr) * 16);
+        const uint8_t* src = base + (i64)(i * kRpi + lane / kCpr) * stride + (lane % kCpr) * 16;
+        asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+    }
+    asm volatile("cp.async.commit_group;" ::: "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
+
 // Prefetches an RB-byte row and one gate value into L2.
 template <int RB, typename T>
 __device__ __forceinline__ void prefetch_row(const T* row, const __nv_bfloat16* zv) {
@@ -504,23 +524,45 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
         const i64 tok = (i64)b * L + t;
         const int g = h0 / (H / G);
 
-        // Rows in through shared memory (job buffer 1 is not needed before job 1):
-        // Q (warpgroup 0) or C (warpgroup 1), then E, 32 rows per warp.
+        // Rows in through shared memory, 32 rows per warp, in one round trip: Q (warpgroup 0)
+        // or C (warpgroup 1) into padded slots in job buffer 1 (not needed before job 1),
+        // and E, which warpgroup 0 loads for both into the ring's tail (kEOff).
         uint8_t* slots = sm.ring + kFwdJob + (warp - 4) * kSlots;
+        uint8_t* eslots = sm.ring + kEOff + (warp & 3) * (32 * 2 * kP);  // rows of the quadrant
         const i64 tok0 = tok - lane;  // first token of this warp's rows
         uint4 av[16];
         uint32_t e2[kP / 2];  // the E row as bf16 pairs; Ebar = E * ie
-        rows_to_slots<2 * kN>(slots, reinterpret_cast<const uint8_t*>((wg == 0 ? Q : Cm) + (tok0 * G + g) * kN),
-                              (i64)G * kN * 2, lane);
+        {
+            const uint8_t* qc = reinterpret_cast<const uint8_t*>((wg == 0 ? Q : Cm) + (tok0 * G + g) * kN);
+            const uint8_t* er = reinterpret_cast<const uint8_t*>(E + (tok0 * G + g) * kP);
+            const i64 qs = (i64)G * kN * 2, es = (i64)G * kP * 2;
+            uint4 v[16], ev[8];  // whole rows per warp access: 2 rows of Q or C, 4 of E
+#pragma unroll
+            for (int i = 0; i < 16; ++i)
+                v[i] = *reinterpret_cast<const uint4*>(qc + (i64)(2 * i + lane / 16) * qs + (lane % 16) * 16);
+            if (wg == 0) {
+#pragma unroll
+                for (int i = 0; i < 8; ++i)
+                    ev[i] = *reinterpret_cast<const uint4*>(er + (i64)(4 * i + lane / 8) * es + (lane % 8) * 16);
+            }
+#pragma unroll
+            for (int i = 0; i < 16; ++i)
+                *reinterpret_cast<uint4*>(slots + (2 * i + lane / 16) * (2 * kN + 16) + (lane % 16) * 16) = v[i];
+            if (wg == 0) {
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    const int r = 4 * i + lane / 8, c = lane % 8;
+                    *reinterpret_cast<uint4*>(eslots + r * 128 + ((c ^ (r & 7)) << 4)) = ev[i];
+                }
+            }
+        }
         __syncwarp();
 #pragma unroll
         for (int u = 0; u < 16; ++u) av[u] = reinterpret_cast<const uint4*>(slots + lane * (2 * kN + 16))[u];
-        __syncwarp();
-        rows_to_slots<2 * kP>(slots, reinterpret_cast<const uint8_t*>(E + (tok0 * G + g) * kP), (i64)G * kP * 2, lane);
-        __syncwarp();
+        asm volatile("bar.sync 2, 256;" ::: "memory");  // warpgroup 0's E rows are staged
 #pragma unroll
         for (int u = 0; u < 8; ++u) {
-            const uint4 w = reinterpret_cast<const uint4*>(slots + lane * (2 * kP + 16))[u];
+            const uint4 w = *reinterpret_cast<const uint4*>(eslots + lane * 128 + ((u ^ (lane & 7)) << 4));
             e2[4 * u] = w.x; e2[4 * u + 1] = w.y; e2[4 * u + 2] = w.z; e2[4 * u + 3] = w.w;
         }
         // The A operands: the row (Q for warpgroup 0, C for warpgroup 1) as fp16 after an
@@ -659,11 +701,21 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
             if (nj == 0) prefetch_row<kP * (int)sizeof(Tout)>(Yssd + rowo_pf * kP, z + rowo_pf);
             // one job: U -> logit -> online softmax, V -> weighted sum. kMasked: some lanes
             // of the warp may be past their history (j >= njr) and skip the softmax update
+            // The merge's Y_ssd rows land in the job buffer of job nj - 2 (done) while the last
+            // job runs: cp.async straight into this warp's slots there.
+            uint8_t* yslots_last = sm.ring + (nj & 1) * kFwdJob + (warp - 4) * kSlots;
+            float zlast = 0.0f;
             auto job = [&](int j, auto masked) -> bool {
                 constexpr bool kMasked = decltype(masked)::value;
                 const int ub = j & 1;
                 const float s_j = s_next;
                 if (j == pf_job) prefetch_row<kP * (int)sizeof(Tout)>(Yssd + rowo_pf * kP, z + rowo_pf);
+                if (j == nj - 1) {
+                    rows_to_slots_async<kP * (int)sizeof(Tout)>(
+                        yslots_last, reinterpret_cast<const uint8_t*>(Yssd + (tok0 * H + h) * kP),
+                        (i64)H * kP * (i64)sizeof(Tout), lane);
+                    zlast = __bfloat162float(z[rowo_pf]);
+                }
                 if (j + 1 < nj) s_next = __ldg(scl + (i64)(j + 1) * H);  // one job ahead
                 if (!warp_wait(&sm.uready[ub], (uint32_t)((j >> 1) & 1), wait_limit_ns, abort)) {
                     fail(abort, 4);
@@ -723,20 +775,24 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
             int j = 0;
             for (; ok && j < njw; ++j) ok = job(j, std::false_type{});
             for (; ok && j < nj; ++j) ok = job(j, std::true_type{});
+            if (nj > 0) cp_async_wait_all();  // also when a wait gave up: no copy outlives the CTA
             if (ok) {
                 // R = O / d (C's row scale undone), lse, gated merge. Every MMA is done
                 // (the last job's V was read, or there were no jobs), so the ring is free
-                // for the row transposes: Y_ssd in, Y and R out.
+                // for the row transposes: Y_ssd in (already there when there were jobs),
+                // Y and R out.
                 constexpr int kRowB = kP * (int)sizeof(Tout);
                 const i64 rowo = tok * H + h;
                 const i64 row0 = tok0 * H + h;  // this warp's first output row
-                uint8_t* yslots = sm.ring + (warp - 4) * 2 * kSlots;
-                uint8_t* rslots = yslots + kSlots;
+                uint8_t* yslots = nj > 0 ? yslots_last : sm.ring + (warp - 4) * 2 * kSlots;
+                uint8_t* rslots = nj > 0 ? sm.ring + ((nj - 1) & 1) * kFwdJob + (warp - 4) * kSlots
+                                         : yslots + kSlots;
                 const i64 rstride = (i64)H * kRowB;
                 const bool has = njr > 0;
                 const float inv_d = has ? cdown / dsum : 0.0f;
-                const float gate = silu_f32(__bfloat162float(z[rowo]));
-                rows_to_slots<kRowB>(yslots, reinterpret_cast<const uint8_t*>(Yssd + row0 * kP), rstride, lane);
+                const float gate = silu_f32(nj > 0 ? zlast : __bfloat162float(z[rowo]));
+                if (nj == 0)
+                    rows_to_slots<kRowB>(yslots, reinterpret_cast<const uint8_t*>(Yssd + row0 * kP), rstride, lane);
                 float r[kP];
     #pragma unroll
                 for (int i = 0; i < kP / 2; ++i) {
