@@ -71,6 +71,16 @@ def scan_flops(w) -> float:
     return w.batch * w.nchunks * (w.heads * per_ch + w.groups * per_grp)
 
 
+def scan_bytes(w) -> float:
+    """Algorithmic HBM bytes of the forward scan with bf16 token inputs and fp32
+    outputs: X, B, C (bf16) and dt read once; Y_ssd, the chunk memories and their
+    inverse RMS (fp32) written once."""
+    T = w.batch * w.seqlen
+    reads = T * (w.heads * w.headdim * 2 + 2 * w.groups * w.dstate * 2 + w.heads * 4)
+    writes = T * w.heads * w.headdim * 4 + w.batch * w.nchunks * w.heads * w.dstate * (w.headdim + 1) * 4
+    return float(reads + writes)
+
+
 def decode_bytes(w, m_cap) -> int:
     """HBM bytes one decode step must move: the whole cache of completed memories,
     the running state (read + write), the partial memory (write; read unless the
@@ -396,6 +406,10 @@ def run_dart(args) -> None:
                          "algorithmic_flops_per_launch": sma_flops(w),
                          "ms_per_launch": sma_avg, "traffic": traffic},
             "layer": {"scan_ms": ms - sma_avg, "sma_ms": sma_avg,
+                      "scan_roofline": {"bound": "hbm", "algorithmic_bytes": scan_bytes(w),
+                                        "achieved": scan_bytes(w) / ((ms - sma_avg) / 1e3) / 1e9,
+                                        "peak": peaks["hbm"], "unit": "GB/s",
+                                        "frac": scan_bytes(w) / ((ms - sma_avg) / 1e3) / 1e9 / peaks["hbm"]},
                       "layer_tflops": (sma_flops(w) + scan_flops(w)) / (ms / 1e3) / 1e12,
                       "layer_frac": (sma_flops(w) + scan_flops(w)) / (ms / 1e3) / 1e12 / peaks["bf16"]},
             "cpu_baseline": cpu,
