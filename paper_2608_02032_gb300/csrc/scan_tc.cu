@@ -258,15 +258,47 @@ chunk_state_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restri
         asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
     }
     __syncthreads();  // b_rows is overwritten by the staging buffers below
-    const uint32_t d_col = (uint32_t)(S / 2);  // accumulator after the A operand
+    // two accumulators after the A operand (64 columns each): head hh's MMAs run into
+    // buffer hh & 1 while the epilogue of head hh - 1 reads the other
+    const uint32_t d_col = (uint32_t)(S / 2);
     constexpr uint32_t idesc = tc::idesc_f16(1, true, kN, kP);
     uint32_t phase = 0;
     bool ok = true;
+    // epilogue of head hh from its accumulator: row n of the memory, columns 32 half ..
+    // 32 half + 31
+    auto epilogue = [&](int hh) {
+        const int h = h0 + hh;
+        const i64 mrow = ((((i64)b * Mc + c) * H + h) * kN + n);
+        float ss = 0.0f;
+        {
+            float v[32];
+            tmem_ld32(tmem + lane_addr + d_col + 64u * (uint32_t)(hh & 1) + 32u * half, v);
+            if (dH32 != nullptr) {
+                float4* d32 = reinterpret_cast<float4*>(dH32 + mrow * kP + 32 * half);
+#pragma unroll
+                for (int q = 0; q < 8; ++q)
+                    d32[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+            }
+            if (!kZ) {
+                store_row32(Mout + mrow * kP + 32 * half, v);
+#pragma unroll
+                for (int i = 0; i < 32; ++i) {
+                    const float sv = stored_value<Tmem>(v[i]);
+                    ss = fmaf(sv, sv, ss);
+                }
+            }
+        }
+        if (half == 1) sm.ssq[n] = ss;
+        tc::tc_fence_before();
+        __syncthreads();  // ssq; the accumulator is free for head hh + 2
+        if (!kZ && half == 0 && rM != nullptr) rM[mrow] = rsqrtf((ss + sm.ssq[n]) / (float)kP + eps);
+    };
     for (int hh = 0; hh < kStateHeads && ok; ++hh) {
         const int h = h0 + hh;
         if (tid < S) sm.w[tid] = kZ ? expf(nx.cumv) : expf(nx.cend - nx.cumv) * nx.dtv;
-        __syncthreads();
-        // stage (w (.) X_h) as bf16 hi / lo, rows s, 128-byte swizzle
+        __syncthreads();  // also: ssq of head hh - 2 read
+        // stage (w (.) X_h) as bf16 hi / lo, rows s, 128-byte swizzle (the MMAs of head
+        // hh - 1, the last to read these buffers, were waited for)
 #pragma unroll
         for (int k = 0; k < 8; ++k) {
             if (k < xiters) {
@@ -294,44 +326,27 @@ chunk_state_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restri
         __syncthreads();
         if (tid == 0) {
             tc::tc_fence_after();
+            const uint32_t dcur = tmem + d_col + 64u * (uint32_t)(hh & 1);
             for (int part = 0; part < 2; ++part) {
                 const uint32_t base = tc::smem_u32(sm.wx[part]);
                 for (int ks = 0; ks < S / 16; ++ks) {
                     const uint64_t bd = tc::smem_desc_sw128(base + 2048u * ks, 1024u, 1024u);
-                    tc::mma_f16_ts(tmem + d_col, tmem + 8u * ks, bd, idesc,
-                                   (part > 0 || ks > 0) ? 1u : 0u);
+                    tc::mma_f16_ts(dcur, tmem + 8u * ks, bd, idesc, (part > 0 || ks > 0) ? 1u : 0u);
                 }
             }
+            tc::mma_commit(&sm.bar);
         }
-        ok = commit_and_wait(&sm.bar, phase, wait_limit_ns, 1);
-        phase ^= 1u;
-        if (!ok) break;
-        // epilogue: row n of the memory, columns 32 half .. 32 half + 31
-        const i64 mrow = ((((i64)b * Mc + c) * H + h) * kN + n);
-        float ss = 0.0f;
+        if (hh > 0) epilogue(hh - 1);  // under this head's MMAs
+        // this head's MMAs done: its accumulator is complete and the staging buffers free
         {
-            float v[32];
-            tmem_ld32(tmem + lane_addr + d_col + 32u * half, v);
-            if (dH32 != nullptr) {
-                float4* d32 = reinterpret_cast<float4*>(dH32 + mrow * kP + 32 * half);
-#pragma unroll
-                for (int q = 0; q < 8; ++q)
-                    d32[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
-            }
-            if (!kZ) {
-                store_row32(Mout + mrow * kP + 32 * half, v);
-#pragma unroll
-                for (int i = 0; i < 32; ++i) {
-                    const float sv = stored_value<Tmem>(v[i]);
-                    ss = fmaf(sv, sv, ss);
-                }
-            }
+            const bool got = tc::mbar_wait(&sm.bar, phase, wait_limit_ns, nullptr);
+            if (!got) atomicCAS(&g_scan_tc_status, 0, 1);
+            ok = __syncthreads_and(got ? 1 : 0) != 0;
+            tc::tc_fence_after();
         }
-        if (half == 1) sm.ssq[n] = ss;
-        tc::tc_fence_before();
-        __syncthreads();  // the accumulator and the staging buffers are reused
-        if (!kZ && half == 0 && rM != nullptr) rM[mrow] = rsqrtf((ss + sm.ssq[n]) / (float)kP + eps);
+        phase ^= 1u;
     }
+    if (ok) epilogue(kStateHeads - 1);
     if (!ok) {  // a wait ran out: let the MMAs in flight finish before freeing TMEM
         if (!tc::mbar_wait(&sm.bar, phase ^ 1u, kDrainLimitNs, nullptr))
             atomicCAS(&g_scan_tc_status, 0, 9);
