@@ -204,7 +204,7 @@ cudaError_t launch_copy_rows(void* dst, int64_t dst_pitch, const void* src, int6
 cudaError_t launch_gather_heads(const void* src, void* dst, int64_t rows, int64_t H, int64_t h0,
                                 int64_t hg, int elem_bytes, cudaStream_t stream);
 
-// Tensor-core SMA (sma_tc.cu): bf16 token inputs, P = 64, N = 128, S % 128 == 0.
+// Tensor-core SMA (sma_tc.cu): bf16 token inputs, P = 64, N = 128, L % 128 == 0, any S.
 bool sma_tc_supported(const SmaArgs& a);
 size_t sma_tc_workspace(int64_t B, int64_t Mc, int64_t H);
 template <typename Tmem, typename Tout>

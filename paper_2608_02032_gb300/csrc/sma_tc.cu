@@ -1,6 +1,7 @@
 // State-memory attention forward + gated merge on the 5th-generation tensor
 // cores (tcgen05, TMEM, bulk async copies), for bf16 token inputs with
-// P = 64, N = 128 and S a multiple of 128 (Sec. 3 value/key readouts, chunk
+// P = 64, N = 128 and L a multiple of 128; for S < 128 a tile spans several
+// chunks and each row keeps its own history (Sec. 3 value/key readouts, chunk
 // logit, softmax over earlier chunks and R_t; App. B.1 normalised score
 // branch; Alg. 1 streaming order; Sec. 3 gated merge).
 //
@@ -42,7 +43,7 @@
 // are one bulk copy.
 // Kernel 2 (sma_tc_kernel), one CTA per (batch, 128-token tile, 2 heads),
 // grouped by (batch, head pair), heaviest tiles first inside a group:
-//   warp 0      producer: bulk copies of the parts into a 6-stage ring
+//   warp 0      producer: one bulk copy per job into two 80 KiB job buffers
 //   warp 1      TMEM allocation; one thread issues the MMAs
 //   warps 2, 3  idle (they complete warpgroup 0 for the register split)
 //   warps 4..7  epilogue warpgroup 0: head 0 of the pair (stages Q)
@@ -52,8 +53,10 @@
 // rescaled when the maximum moves), and finally writes R = O / d, lse and
 // Y = Y_ssd + SiLU(z) R.
 // TMEM: [0,64) Q (fp16 pairs), [64,128) C (fp16 pairs), [128,256) U,
-// [256,384) and [384,512) V (two buffers, jobs alternate). Shared memory:
-// two 80 KiB job buffers and the 16 KiB e4m3 Q tile.
+// [256,384) and [384,512) V (two buffers, jobs alternate). Shared memory
+// (192 KiB): two 80 KiB job buffers, the 16 KiB e4m3 Q tile and a 16 KiB tail
+// where the prologue stages the E rows; the prologue's Q / C rows and the
+// merge's Y_ssd, Y and R rows pass through job buffers no copy is using.
 //
 // Synchronisation, job j, b = j & 1. The MMA thread pays for barrier
 // operations with idle tensor cycles, and most for a wait right after a
@@ -371,8 +374,8 @@ __device__ __forceinline__ void issue_part(uint32_t d_tmem, uint32_t a_tmem, uin
 
 // What the backward-statistics variant (kStats) writes instead of the merge:
 // the softmax weights g_{t,j} = exp(l_{t,j} - lse_t) (lse from the forward)
-// and their sum G1_t. It runs the U half of each job only (parts W_hi, W_lo;
-// no value chain). The forward variant, when g is given, writes the logits
+// and their sum G1_t. It runs the U half of each job only (the W16 part and
+// the e4m3 residual of the forward layout; no value chain). The forward variant, when g is given, writes the logits
 // l_{t,j} there instead, for a backward that then needs no statistics pass.
 struct SmaStats {
     float* g;    // B x H x Mc x L

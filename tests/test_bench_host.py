@@ -31,6 +31,17 @@ def test_decode_bytes_of_the_b64_workload():
     assert cache + state + part < n < cache + state + part + 2 ** 20
 
 
+def test_scan_bytes_of_the_l16k_workload():
+    """The forward scan's algorithmic HBM bytes: bf16 X, B, C and fp32 dt in;
+    fp32 Y_ssd, memories and their inverse RMS out (64 chunks)."""
+    w = WORKLOADS["prefill_l16k"]
+    T = 16384
+    reads = T * 32 * 64 * 2 + 2 * T * 128 * 2 + T * 32 * 4
+    writes = T * 32 * 64 * 4 + 64 * 32 * 128 * 64 * 4 + 64 * 32 * 128 * 4
+    assert bench.scan_bytes(w) == reads + writes
+    assert 279e6 < bench.scan_bytes(w) < 281e6
+
+
 def _free_port():
     with socket.socket() as s:
         s.bind(("127.0.0.1", 0))
