@@ -280,6 +280,36 @@ dart_status dart_sma_backward_with_logits(const dart_dims* dims, const void* M, 
                                           size_t workspace_bytes, void* stream);
 
 /*
+ * Prefill pair that hands the SMA its operands from the scan (no counterpart in
+ * the paper: a fusion of data movement). The tensor-core SMA forward reads each
+ * memory M_j as operand tiles per memory and pair of heads:
+ *   W = r_j (.) M_j as fp16 and the e4m3 residual 2^12 (W - fp16(W));
+ *   M_j / max|M_j| as fp16, with the scale max|M_j|.
+ * dart_sma_forward builds them from M and rM in a pass of its own.
+ * dart_chunk_scan_with_tiles is dart_chunk_scan that also writes those tiles from
+ * the chunk-state kernel, which holds each memory in registers as it computes it,
+ * into `tiles`. dart_sma_forward_with_tiles is dart_sma_forward that reads them
+ * instead of M and rM. The results equal the two regular calls' bit for bit; the
+ * tile-building pass and its re-read of M are saved.
+ * tiles:   caller-owned device buffer of dart_sma_tiles_size(dims) bytes, 256-byte
+ *          aligned, an opaque layout; valid for the dims and the memories of the
+ *          dart_chunk_scan_with_tiles call that wrote it.
+ * Other arguments, outputs and the scan's workspace as for dart_chunk_scan and
+ * dart_sma_forward; dart_sma_forward_with_tiles takes no workspace.
+ * Requires the tensor-core paths of both calls: bf16 inputs, P = 64, N = 128,
+ * S in {64, 128, 256}, H/G a multiple of 8, L a multiple of 128 and of S.
+ * dart_sma_tiles_size returns 0 elsewhere, and the calls DART_ERR_UNSUPPORTED.
+ */
+size_t dart_sma_tiles_size(const dart_dims* dims);
+dart_status dart_chunk_scan_with_tiles(const dart_dims* dims, const void* X, const float* dt,
+                                       const float* A, const void* Bm, const void* Cm, void* Y_ssd,
+                                       void* M, float* rM, float* final_state, void* tiles,
+                                       void* workspace, size_t workspace_bytes, void* stream);
+dart_status dart_sma_forward_with_tiles(const dart_dims* dims, const void* tiles, const void* Q,
+                                        const void* Cm, const void* E, const void* z, const void* Y_ssd,
+                                        void* Y, void* R, float* lse, void* stream);
+
+/*
  * Backward of dart_chunk_scan (training): gradients of a loss that depends on
  * Y_ssd (through dY) and on the chunk memories (through dM, e.g. the output of
  * dart_sma_backward). Chain rule on the chunked forms of App. A: the states

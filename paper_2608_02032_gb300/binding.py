@@ -33,7 +33,8 @@ EXPORTED = ("dart_status_string", "dart_last_cuda_error", "dart_workspace_size",
             "dart_launch_count", "dart_set_wait_limit_ns", "dart_get_device_status",
             "dart_sma_backward", "dart_chunk_scan_backward", "dart_test_withhold_copies",
             "dart_prefill_host", "dart_sma_forward_with_logits", "dart_sma_backward_with_logits",
-            "dart_block_workspace_size", "dart_block_forward")
+            "dart_block_workspace_size", "dart_block_forward", "dart_sma_tiles_size",
+            "dart_chunk_scan_with_tiles", "dart_sma_forward_with_tiles")
 
 
 class DartError(RuntimeError):
@@ -126,6 +127,12 @@ def lib() -> ctypes.CDLL:
         L.dart_block_workspace_size.argtypes = [bp]
         L.dart_block_workspace_size.restype = ctypes.c_size_t
         L.dart_block_forward.argtypes = [bp] + [_vp] * 11 + [ctypes.c_size_t, _vp]
+        L.dart_sma_tiles_size.restype = ctypes.c_size_t
+        L.dart_sma_tiles_size.argtypes = [dp]
+        L.dart_chunk_scan_with_tiles.restype = ctypes.c_int
+        L.dart_chunk_scan_with_tiles.argtypes = [dp] + [_vp] * 11 + [ctypes.c_size_t, _vp]
+        L.dart_sma_forward_with_tiles.restype = ctypes.c_int
+        L.dart_sma_forward_with_tiles.argtypes = [dp] + [_vp] * 10
         L.dart_block_forward.restype = ctypes.c_int
         _lib = L
     return _lib
@@ -186,6 +193,26 @@ def dart_chunk_scan(dims, X, dt, A, Bm, Cm, Y_ssd, M, rM=None, final_state=None,
         ctypes.byref(dims), _ptr(X, "X"), _ptr(dt, "dt"), _ptr(A, "A"), _ptr(Bm, "Bm"),
         _ptr(Cm, "Cm"), _ptr(Y_ssd, "Y_ssd"), _ptr(M, "M"), _ptr(rM, "rM"),
         _ptr(final_state, "final_state"), w, nb, _stream(stream)))
+
+
+def dart_sma_tiles_size(dims) -> int:
+    return int(lib().dart_sma_tiles_size(ctypes.byref(dims)))
+
+
+def dart_chunk_scan_with_tiles(dims, X, dt, A, Bm, Cm, Y_ssd, M, rM, final_state, tiles, workspace=None,
+                               stream=None) -> None:
+    w, nb = _ws(workspace)
+    _check("dart_chunk_scan_with_tiles", lib().dart_chunk_scan_with_tiles(
+        ctypes.byref(dims), _ptr(X, "X"), _ptr(dt, "dt"), _ptr(A, "A"), _ptr(Bm, "Bm"),
+        _ptr(Cm, "Cm"), _ptr(Y_ssd, "Y_ssd"), _ptr(M, "M"), _ptr(rM, "rM"),
+        _ptr(final_state, "final_state"), _ptr(tiles, "tiles"), w, nb, _stream(stream)))
+
+
+def dart_sma_forward_with_tiles(dims, tiles, Q, Cm, E, z, Y_ssd, Y, R=None, lse=None, stream=None) -> None:
+    _check("dart_sma_forward_with_tiles", lib().dart_sma_forward_with_tiles(
+        ctypes.byref(dims), _ptr(tiles, "tiles"), _ptr(Q, "Q"), _ptr(Cm, "Cm"), _ptr(E, "E"),
+        _ptr(z, "z"), _ptr(Y_ssd, "Y_ssd"), _ptr(Y, "Y"), _ptr(R, "R"), _ptr(lse, "lse"),
+        _stream(stream)))
 
 
 def dart_sma_forward(dims, M, rM, Q, Cm, E, z, Y_ssd, Y, R=None, lse=None, workspace=None,

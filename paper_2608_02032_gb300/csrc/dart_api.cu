@@ -630,9 +630,10 @@ size_t dart_workspace_size(const dart_dims* d, int op) {
     return 0;
 }
 
-dart_status dart_chunk_scan(const dart_dims* d, const void* X, const float* dt, const float* A,
-                            const void* Bm, const void* Cm, void* Y_ssd, void* M, float* rM,
-                            float* final_state, void* ws, size_t ws_bytes, void* stream) {
+static dart_status chunk_scan_impl(const dart_dims* d, const void* X, const float* dt, const float* A,
+                                   const void* Bm, const void* Cm, void* Y_ssd, void* M, float* rM,
+                                   float* final_state, uint8_t* tiles, void* ws, size_t ws_bytes,
+                                   void* stream) {
     dart_status st = check_dims(d, true, true);
     if (st != DART_OK) return st;
     const void* req[] = {X, dt, A, Bm, Cm, Y_ssd, M};
@@ -676,6 +677,7 @@ dart_status dart_chunk_scan(const dart_dims* d, const void* X, const float* dt, 
     cudaError_t e;
     if (scan_uses_tc(d)) {
         a.Hops = (uint8_t*)ws + w.hops_off;
+        a.sma_tiles = tiles;
         typedef __nv_bfloat16 bf;
         const unsigned long long lim = g_wait_limit_ns.load();
         if (d->mem_dtype == DART_F32)
@@ -687,6 +689,63 @@ dart_status dart_chunk_scan(const dart_dims* d, const void* X, const float* dt, 
     } else {
         e = dispatch<ScanL>(d, a, s);
     }
+    return e == cudaSuccess ? DART_OK : cuda_fail(e);
+}
+
+dart_status dart_chunk_scan(const dart_dims* d, const void* X, const float* dt, const float* A,
+                            const void* Bm, const void* Cm, void* Y_ssd, void* M, float* rM,
+                            float* final_state, void* ws, size_t ws_bytes, void* stream) {
+    return chunk_scan_impl(d, X, dt, A, Bm, Cm, Y_ssd, M, rM, final_state, nullptr, ws, ws_bytes, stream);
+}
+
+// The SMA operand tiles built by the scan: both calls on their tensor-core paths,
+// whole chunks.
+static bool tiles_supported(const dart_dims* d) {
+    return check_dims(d, true) == DART_OK && scan_uses_tc(d) && sma_uses_tc(d);
+}
+
+size_t dart_sma_tiles_size(const dart_dims* d) {
+    if (!tiles_supported(d)) return 0;
+    return dart::sma_tiles_bytes(d->batch, d->seqlen / d->chunk, d->nheads);
+}
+
+dart_status dart_chunk_scan_with_tiles(const dart_dims* d, const void* X, const float* dt, const float* A,
+                                       const void* Bm, const void* Cm, void* Y_ssd, void* M, float* rM,
+                                       float* final_state, void* tiles, void* ws, size_t ws_bytes,
+                                       void* stream) {
+    dart_status st = check_dims(d, true);
+    if (st != DART_OK) return st;
+    if (!tiles_supported(d)) return DART_ERR_UNSUPPORTED;
+    if (tiles == nullptr || ((uintptr_t)tiles & 255u) != 0) return DART_ERR_INVALID_ARG;
+    return chunk_scan_impl(d, X, dt, A, Bm, Cm, Y_ssd, M, rM, final_state, (uint8_t*)tiles, ws, ws_bytes,
+                           stream);
+}
+
+dart_status dart_sma_forward_with_tiles(const dart_dims* d, const void* tiles, const void* Q, const void* Cm,
+                                        const void* E, const void* z, const void* Y_ssd, void* Y, void* R,
+                                        float* lse, void* stream) {
+    dart_status st = check_dims(d, true);
+    if (st != DART_OK) return st;
+    if (!tiles_supported(d)) return DART_ERR_UNSUPPORTED;
+    if (tiles == nullptr || ((uintptr_t)tiles & 255u) != 0) return DART_ERR_INVALID_ARG;
+    const void* req[] = {Q, Cm, E, z, Y_ssd, Y};
+    for (const void* p : req)
+        if (p == nullptr || !aligned16(p)) return DART_ERR_INVALID_ARG;
+    if ((R && !aligned16(R)) || (lse && !aligned16(lse))) return DART_ERR_INVALID_ARG;
+    dart::SmaArgs a = sma_args(d);
+    a.M = nullptr; a.rM = nullptr; a.Q = Q; a.Cm = Cm; a.E = E; a.z = z; a.Yssd = Y_ssd; a.Y = Y;
+    a.R = R; a.lse = lse; a.tiles = (const uint8_t*)tiles;
+    a.test_withhold = g_test_withhold.load();
+    const unsigned long long lim = g_wait_limit_ns.load();
+    cudaStream_t s = (cudaStream_t)stream;
+    typedef __nv_bfloat16 bf;
+    cudaError_t e;
+    if (d->mem_dtype == DART_F32)
+        e = dart::launch_sma_forward_tc<float, float>(a, nullptr, lim, s);
+    else if (d->out_dtype == DART_F32)
+        e = dart::launch_sma_forward_tc<bf, float>(a, nullptr, lim, s);
+    else
+        e = dart::launch_sma_forward_tc<bf, bf>(a, nullptr, lim, s);
     return e == cudaSuccess ? DART_OK : cuda_fail(e);
 }
 

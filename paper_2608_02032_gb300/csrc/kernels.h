@@ -34,6 +34,9 @@ struct ScanArgs {
     // tiles in the 128-byte-swizzled shared-memory layout, 32 KiB per (b, c, h)
     uint8_t* Hops;
     int test_withhold = 0;  // tensor-core path: the state passing issues no copies (failure-path test hook)
+    // optional (tensor-core path): the SMA forward's operand tiles and scales, written by
+    // the chunk-state epilogue (layout of sma_tiles_bytes), or null
+    uint8_t* sma_tiles = nullptr;
 };
 
 struct SmaArgs {
@@ -51,6 +54,9 @@ struct SmaArgs {
     float* lse;
     int test_withhold;  // tensor-core path: issue no operand copies (failure-path test hook)
     float* logits = nullptr;  // tensor-core path: B x H x Mc x L logits for the backward, or null
+    // tensor-core path: operand tiles already built (by the chunk-state kernel), or null;
+    // M and rM are then not read
+    const uint8_t* tiles = nullptr;
 };
 
 struct DecodeArgs {
@@ -204,6 +210,20 @@ cudaError_t launch_copy_rows(void* dst, int64_t dst_pitch, const void* src, int6
 cudaError_t launch_gather_heads(const void* src, void* dst, int64_t rows, int64_t H, int64_t h0,
                                 int64_t hg, int elem_bytes, cudaStream_t stream);
 
+// The SMA forward's operand tiles (P = 64, N = 128): per (b, memory, head pair) an
+// 80 KiB job (fp16 W = r M, its e4m3 residual, fp16 M / max|M|) at
+// ((b Mc + j) (H / 2) + hp) * 80 KiB, then one fp32 scale max|M| per (b, j, h) at
+// sma_tiles_scale_offset. Written by the tensor-core chunk-state kernel or by the
+// SMA's own operand kernel; read by the SMA kernel.
+size_t sma_tiles_bytes(int64_t B, int64_t Mc, int64_t H);
+// Byte layout of one job: [W16 h0 | W16 h1] (MN-major, 128-byte swizzle, rows n),
+// the e4m3 residual 2^12 (W - W16) (K-major: rows x 64 + p of 128 bytes over n, the
+// same swizzle), [M16 h0 | M16 h1] (as W16).
+constexpr int kSmaTile = 128 * 64 * 2;
+constexpr int kSmaOffLo = 2 * kSmaTile;
+constexpr int kSmaOffV = kSmaOffLo + 2 * 64 * 128;
+constexpr int kSmaJob = kSmaOffV + 2 * kSmaTile;
+size_t sma_tiles_scale_offset(int64_t B, int64_t Mc, int64_t H);
 // Tensor-core SMA (sma_tc.cu): bf16 token inputs, P = 64, N = 128, L % 128 == 0, any S.
 bool sma_tc_supported(const SmaArgs& a);
 size_t sma_tc_workspace(int64_t B, int64_t Mc, int64_t H);

@@ -35,6 +35,7 @@
 
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
+#include <cuda_fp8.h>
 
 #include "common.cuh"
 #include "kernels.h"
@@ -168,7 +169,9 @@ struct StateSmem {
         __nv_bfloat16 b_rows[256 * kN];  // the chunk's B rows (only while building A)
     };
     float w[256];
-    float ssq[kN];  // sum of squares of the second half of each memory row
+    float ssq[2][kN];  // sum of squares of each half of each memory row
+    float smax[8];     // per warp: max |M| of its rows and half (SMA tiles)
+    uint8_t s_res[kP][kN + 16];  // SMA tiles: e4m3 residual rows p, bytes n
     uint64_t bar;
     uint32_t tmem_base;
 };
@@ -187,7 +190,8 @@ chunk_state_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restri
                       const float* __restrict__ cum, const __nv_bfloat16* __restrict__ Bm,
                       float* __restrict__ dH32, Tmem* __restrict__ Mout, float* __restrict__ rM,
                       int L, int H, int G, int S, int Mc, float eps,
-                      unsigned long long wait_limit_ns) {
+                      unsigned long long wait_limit_ns, uint8_t* __restrict__ tiles,
+                      float* __restrict__ tile_scale) {
     extern __shared__ uint8_t smem_raw[];
     StateSmem& sm = *reinterpret_cast<StateSmem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                   ~(uintptr_t)1023);
@@ -266,32 +270,83 @@ chunk_state_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restri
     bool ok = true;
     // epilogue of head hh from its accumulator: row n of the memory, columns 32 half ..
     // 32 half + 31
+    // With `tiles`, the epilogue also writes the SMA forward's operands of the memory
+    // (the layout of sma_operands_kernel, the same arithmetic): W16 = fp16(r M), the
+    // e4m3 residual of 2^12 (W - W16) transposed through shared memory, M16 =
+    // fp16(M / max|M|) and the scale max|M|. The last memory has no later token to read it.
+    const bool tiled = !kZ && tiles != nullptr && c < Mc - 1;
     auto epilogue = [&](int hh) {
         const int h = h0 + hh;
         const i64 mrow = ((((i64)b * Mc + c) * H + h) * kN + n);
-        float ss = 0.0f;
-        {
-            float v[32];
-            tmem_ld32(tmem + lane_addr + d_col + 64u * (uint32_t)(hh & 1) + 32u * half, v);
-            if (dH32 != nullptr) {
-                float4* d32 = reinterpret_cast<float4*>(dH32 + mrow * kP + 32 * half);
+        float ss = 0.0f, am = 0.0f;
+        float v[32];
+        tmem_ld32(tmem + lane_addr + d_col + 64u * (uint32_t)(hh & 1) + 32u * half, v);
+        if (dH32 != nullptr) {
+            float4* d32 = reinterpret_cast<float4*>(dH32 + mrow * kP + 32 * half);
 #pragma unroll
-                for (int q = 0; q < 8; ++q)
-                    d32[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
-            }
-            if (!kZ) {
-                store_row32(Mout + mrow * kP + 32 * half, v);
+            for (int q = 0; q < 8; ++q)
+                d32[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+        }
+        if (!kZ) {
+            store_row32(Mout + mrow * kP + 32 * half, v);
 #pragma unroll
-                for (int i = 0; i < 32; ++i) {
-                    const float sv = stored_value<Tmem>(v[i]);
-                    ss = fmaf(sv, sv, ss);
-                }
+            for (int i = 0; i < 32; ++i) {
+                v[i] = stored_value<Tmem>(v[i]);  // the memory as stored (bf16-rounded for bf16 memories)
+                ss = fmaf(v[i], v[i], ss);
+                am = fmaxf(am, fabsf(v[i]));
             }
         }
-        if (half == 1) sm.ssq[n] = ss;
+        sm.ssq[half][n] = ss;
+        if (tiled) {
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) am = fmaxf(am, __shfl_xor_sync(0xffffffffu, am, o));
+            if ((tid & 31) == 0) sm.smax[warp] = am;
+        }
         tc::tc_fence_before();
-        __syncthreads();  // ssq; the accumulator is free for head hh + 2
-        if (!kZ && half == 0 && rM != nullptr) rM[mrow] = rsqrtf((ss + sm.ssq[n]) / (float)kP + eps);
+        __syncthreads();  // ssq, smax; the accumulator is free for head hh + 2
+        const float r = rsqrtf((sm.ssq[0][n] + sm.ssq[1][n]) / (float)kP + eps);
+        if (!kZ && half == 0 && rM != nullptr) rM[mrow] = r;
+        if (tiled) {
+            float smx = 0.0f;
+#pragma unroll
+            for (int w = 0; w < 8; ++w) smx = fmaxf(smx, sm.smax[w]);
+            const float inv_s = smx > 0.0f ? 1.0f / smx : 1.0f;
+            const int x = h & 1;
+            uint8_t* job = tiles + (((i64)b * Mc + c) * (H / 2) + h / 2) * (i64)kSmaJob;
+            if (tid == 0) tile_scale[((i64)b * Mc + c) * H + h] = smx > 0.0f ? smx : 1.0f;
+            // row n, columns p = 32 half .. 32 half + 31: four 16-byte chunks of 8 fp16
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                uint32_t wq[4], mq[4];
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const int i = 8 * q + 2 * e;
+                    const float w0 = r * v[i], w1 = r * v[i + 1];
+                    const __half h0w = __float2half_rn(w0), h1w = __float2half_rn(w1);
+                    // |W| <= sqrt(P) (r normalises the row): W16 needs no scale, and 2^12 times
+                    // the residual (at most 2^-11 |W|) stays inside e4m3's range
+                    const __nv_fp8_e4m3 r0(4096.0f * (w0 - __half2float(h0w)));
+                    const __nv_fp8_e4m3 r1(4096.0f * (w1 - __half2float(h1w)));
+                    sm.s_res[32 * half + i][n] = r0.__x;
+                    sm.s_res[32 * half + i + 1][n] = r1.__x;
+                    wq[e] = (uint32_t)__half_as_ushort(h0w) | ((uint32_t)__half_as_ushort(h1w) << 16);
+                    const __half m0 = __float2half_rn(v[i] * inv_s), m1 = __float2half_rn(v[i + 1] * inv_s);
+                    mq[e] = (uint32_t)__half_as_ushort(m0) | ((uint32_t)__half_as_ushort(m1) << 16);
+                }
+                const uint32_t o = sw128((uint32_t)n, (uint32_t)(64 * half + 16 * q));
+                *reinterpret_cast<uint4*>(job + x * kSmaTile + o) = make_uint4(wq[0], wq[1], wq[2], wq[3]);
+                *reinterpret_cast<uint4*>(job + kSmaOffV + x * kSmaTile + o) = make_uint4(mq[0], mq[1], mq[2], mq[3]);
+            }
+            __syncthreads();  // the residual rows are complete
+            // rows x 64 + p, 128 bytes each, in the 128-byte swizzle: 512 chunks of 16 bytes
+#pragma unroll
+            for (int k2 = 0; k2 < 2; ++k2) {
+                const int ci = tid + kStateThreads * k2, p = ci >> 3, q = ci & 7;
+                const uint32_t row = (uint32_t)(x * kP + p);
+                *reinterpret_cast<uint4*>(job + kSmaOffLo + row * 128u + (((uint32_t)q ^ (row & 7u)) << 4)) =
+                    *reinterpret_cast<const uint4*>(&sm.s_res[p][q * 16]);
+            }
+        }
     };
     for (int hh = 0; hh < kStateHeads && ok; ++hh) {
         const int h = h0 + hh;
@@ -887,9 +942,12 @@ cudaError_t launch_chunk_scan_tc(const ScanArgs& a, unsigned long long wait_limi
         const size_t smem = sizeof(StateSmem) + 1024;
         cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
+        uint8_t* tiles = a.sma_tiles;
+        float* tile_scale = tiles != nullptr ? (float*)(tiles + sma_tiles_scale_offset(a.B, M, a.H)) : nullptr;
         kern<<<dim3(M, H / kStateHeads, B), kStateThreads, smem, stream>>>(
             (const __nv_bfloat16*)a.X, a.dt, a.cum, (const __nv_bfloat16*)a.Bm,
-            mem_is_f32 ? nullptr : a.dH32, (Tmem*)a.M, a.rM, L, H, G, S, M, a.eps, wait_limit_ns);
+            mem_is_f32 ? nullptr : a.dH32, (Tmem*)a.M, a.rM, L, H, G, S, M, a.eps, wait_limit_ns, tiles,
+            tile_scale);
     }
     // fp32 memories are the chunk states themselves: the state passing reads them
     state_passing_tc_kernel<<<dim3(kN * kP / kSpSlab, H, B), kSpThreads, 0, stream>>>(
@@ -928,7 +986,7 @@ cudaError_t launch_scan_states_tc(const ScanArgs& a0, float* cum, float* Hprev, 
         return e;
     kern<<<dim3(M, H / kStateHeads, B), kStateThreads, smem, stream>>>(
         (const __nv_bfloat16*)a.X, a.dt, a.cum, (const __nv_bfloat16*)a.Bm, nullptr, Hprev, nullptr,
-        L, H, G, S, M, a.eps, wait_limit_ns);
+        L, H, G, S, M, a.eps, wait_limit_ns, nullptr, nullptr);
     state_passing_tc_kernel<<<dim3(kN * kP / kSpSlab, H, B), kSpThreads, 0, stream>>>(
         Hprev, a.cum, nullptr, Hops, Hprev, H, M, S, wait_limit_ns, 0);
     note_launches(2);
@@ -945,7 +1003,7 @@ cudaError_t launch_scan_bwd_inter_tc(const ScanArgs& a, const float* cum, const 
     if (e != cudaSuccess) return e;
     kern<<<dim3(M, H / kStateHeads, B), kStateThreads, smem, stream>>>(
         (const __nv_bfloat16*)dY, a.dt, cum, (const __nv_bfloat16*)a.Cm, Z, nullptr, nullptr, L, H, G,
-        S, M, a.eps, wait_limit_ns);
+        S, M, a.eps, wait_limit_ns, nullptr, nullptr);
     note_launches(1);
     return cudaGetLastError();
 }

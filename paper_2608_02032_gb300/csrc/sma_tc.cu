@@ -99,6 +99,8 @@ constexpr int kStages = 6;                    // ring of kPart-sized stages (192
 constexpr int kLoPart = kHeadsPerCta * kP * kN;
 constexpr int kOffLo = kPart, kOffV = kPart + kLoPart;
 constexpr int kFwdJob = 2 * kPart + kLoPart;  // 80 KiB
+static_assert(kFwdJob == kSmaJob && kOffLo == kSmaOffLo && kOffV == kSmaOffV && kTile == kSmaTile,
+              "the forward layout is the one the chunk-state kernel writes");
 constexpr int kQ8Off = 2 * kFwdJob;           // the e4m3 Q tile (A of the residual chain) after two jobs
 static_assert(kQ8Off + kRows * kN <= kStages * kPart, "two job buffers and the Q tile fit the ring");
 static_assert(kFwdJob <= kPair, "the forward layout fits the workspace sized for the backward one");
@@ -835,6 +837,13 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
 
 }  // namespace
 
+size_t sma_tiles_scale_offset(int64_t B, int64_t Mc, int64_t H) {
+    return ((size_t)(B * Mc * (H / kHeadsPerCta)) * kFwdJob + 255) & ~(size_t)255;
+}
+size_t sma_tiles_bytes(int64_t B, int64_t Mc, int64_t H) {
+    return sma_tiles_scale_offset(B, Mc, H) + (((size_t)(B * Mc * H) * sizeof(float) + 255) & ~(size_t)255);
+}
+
 size_t sma_tc_workspace(int64_t B, int64_t Mc, int64_t H) {
     const size_t ops = (size_t)(B * Mc * (H / kHeadsPerCta)) * kPair;
     const size_t sc = (size_t)(B * Mc * H) * sizeof(float);
@@ -850,12 +859,21 @@ template <typename Tmem, typename Tout>
 cudaError_t launch_sma_forward_tc(const SmaArgs& a, void* ws, unsigned long long wait_limit_ns,
                                   cudaStream_t stream) {
     const int Bsz = (int)a.B, L = (int)a.L, H = (int)a.H, Mc = (int)(a.L / a.S);
-    uint8_t* ops = (uint8_t*)ws;
-    float* scale = (float*)(ops + (size_t)(a.B * Mc * (H / kHeadsPerCta)) * kPair);
-    if (Mc > 1) {
-        sma_operands_kernel<Tmem><<<dim3(Mc - 1, H, Bsz), 256, 0, stream>>>(
-            (const Tmem*)a.M, a.rM, ops, scale, Mc, H, a.eps, 0);  // the forward layout
-        note_launches(1);
+    const uint8_t* ops;
+    const float* scale;
+    if (a.tiles != nullptr) {  // built by the chunk-state kernel
+        ops = a.tiles;
+        scale = (const float*)(a.tiles + sma_tiles_scale_offset(a.B, Mc, a.H));
+    } else {
+        uint8_t* w = (uint8_t*)ws;
+        float* sc = (float*)(w + (size_t)(a.B * Mc * (H / kHeadsPerCta)) * kPair);
+        if (Mc > 1) {
+            sma_operands_kernel<Tmem><<<dim3(Mc - 1, H, Bsz), 256, 0, stream>>>(
+                (const Tmem*)a.M, a.rM, w, sc, Mc, H, a.eps, 0);  // the forward layout
+            note_launches(1);
+        }
+        ops = w;
+        scale = sc;
     }
     const size_t smem = sizeof(TcSmem) + 1024;
     auto kern = a.logits != nullptr ? sma_tc_kernel<Tout, false, true> : sma_tc_kernel<Tout, false>;

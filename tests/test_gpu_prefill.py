@@ -213,3 +213,67 @@ def test_l16k_workload_sampled_heads_and_tokens(oracle_mod):
         assert rel_err(got["R"][0, toks, h], R) <= TOL["bf16"]
         assert rel_err(got["lse"][0, toks, h], lse) <= TOL["bf16"]
         assert rel_err(got["Y"][0, toks, h], Y) <= TOL["bf16"]
+
+
+TILE_CASES = [
+    # (B, H, G, L, S, mem, out): the tensor-core shapes of both calls
+    (1, 8, 1, 1024, 256, "f32", "f32"),
+    (2, 16, 2, 512, 128, "f32", "f32"),   # G = 2
+    (1, 8, 1, 512, 64, "f32", "f32"),     # S = 64: a tile spans two chunks in the SMA
+    (1, 8, 1, 512, 128, "bf16", "bf16"),  # bf16 memories: the tiles hold the stored (rounded) values
+]
+
+
+@pytest.mark.parametrize("Bsz,H,G,L,S,mem,out", TILE_CASES)
+def test_sma_tiles_from_the_scan_match_the_regular_calls_bit_for_bit(oracle_mod, Bsz, H, G, L, S, mem, out):
+    """dart_chunk_scan_with_tiles + dart_sma_forward_with_tiles: the chunk-state kernel
+    writes the SMA's operand tiles; every output equals the regular pair's, bit for
+    bit, and the oracle's within the bf16 tolerance."""
+    w = Workload("tiles", Bsz, H, L, 64, 128, S, groups=G, seed=3300 + L + S + H)
+    inp = prefill_inputs(w)
+    tdt = {"f32": torch.float32, "bf16": torch.bfloat16}
+    X, Bm, Cm, Q, E, z = (dev(inp[k], "bf16") for k in ("X", "Bm", "Cm", "Q", "E", "z"))
+    dtv, A = dev(inp["dt"], torch.float32), dev(inp["A"], torch.float32)
+    dims = binding.make_dims(Bsz, L, H, G, 64, 128, S, binding.DART_BF16, binding.DART_DTYPE[tdt[mem]],
+                             binding.DART_DTYPE[tdt[out]], eps=w.eps)
+    nb = binding.dart_sma_tiles_size(dims)
+    assert nb > 0
+    Mc = L // S
+    outs = []
+    for fused in (False, True):
+        Yssd = torch.empty(Bsz, L, H, 64, dtype=tdt[out], device="cuda")
+        M = torch.empty(Bsz, Mc, H, 128, 64, dtype=tdt[mem], device="cuda")
+        rM = torch.empty(Bsz, Mc, H, 128, dtype=torch.float32, device="cuda")
+        Y, R = torch.empty_like(Yssd), torch.empty_like(Yssd)
+        lse = torch.empty(Bsz, L, H, dtype=torch.float32, device="cuda")
+        ws = torch.empty(binding.dart_workspace_size(dims, binding.DART_OP_CHUNK_SCAN), dtype=torch.uint8,
+                         device="cuda")
+        if fused:
+            tiles = torch.full((nb,), 0xFF, dtype=torch.uint8, device="cuda")  # NaN-poisoned
+            binding.dart_chunk_scan_with_tiles(dims, X, dtv, A, Bm, Cm, Yssd, M, rM, None, tiles, ws)
+            binding.dart_sma_forward_with_tiles(dims, tiles, Q, Cm, E, z, Yssd, Y, R, lse)
+        else:
+            binding.dart_chunk_scan(dims, X, dtv, A, Bm, Cm, Yssd, M, rM, None, ws)
+            wss = torch.empty(binding.dart_workspace_size(dims, binding.DART_OP_SMA_FORWARD), dtype=torch.uint8,
+                              device="cuda")
+            binding.dart_sma_forward(dims, M, rM, Q, Cm, E, z, Yssd, Y, R, lse, wss)
+        torch.cuda.synchronize()
+        outs.append((Yssd, M, rM, Y, R, lse))
+    for name, a, b in zip(("Y_ssd", "M", "rM", "Y", "R", "lse"), outs[0], outs[1]):
+        assert torch.equal(a, b), name
+    if mem == "f32" and out == "f32":
+        ref = oracle_prefill(inp, w)
+        for name, got in (("Y", outs[1][3]), ("R", outs[1][4]), ("lse", outs[1][5])):
+            assert rel_err(host(got), ref[name]) <= TOL["bf16"], name
+
+
+def test_sma_tiles_refuse_other_shapes():
+    dims = lambda **kw: binding.make_dims(kw.get("B", 1), kw.get("L", 512), kw.get("H", 8), kw.get("G", 1),
+                                         kw.get("P", 64), kw.get("N", 128), kw.get("S", 128),
+                                         kw.get("dt", binding.DART_BF16), eps=1e-6)
+    assert binding.dart_sma_tiles_size(dims()) > 0
+    for bad in (dict(L=500), dict(H=4), dict(P=32), dict(dt=binding.DART_F32), dict(S=32)):
+        assert binding.dart_sma_tiles_size(dims(**bad)) == 0, bad
+    with pytest.raises(binding.DartError):
+        t = torch.empty(1 << 20, dtype=torch.uint8, device="cuda")
+        binding.dart_sma_forward_with_tiles(dims(H=4), t, t, t, t, t, t, t)
