@@ -430,6 +430,7 @@ struct HostLayout {
     size_t g0, stride;                      // first group, bytes per group
     size_t x, dtg, zg, yssd, y, m, rm;      // offsets inside a group
     size_t scan_ws[2], scan_bytes, sma_ws[2], sma_bytes;
+    size_t tiles[2], tiles_bytes;  // the SMA's operand tiles from the scan (0: not on this shape)
     size_t total;
 };
 
@@ -472,10 +473,12 @@ HostLayout host_layout(const dart_dims* d) {
     dart_dims dg = *d;
     dg.nheads = h.hg;
     h.scan_bytes = scan_ws_bytes(&dg);
-    h.sma_bytes = sma_ws(&dg);
+    h.tiles_bytes = dart_sma_tiles_size(&dg);
+    h.sma_bytes = h.tiles_bytes > 0 ? 0 : sma_ws(&dg);  // the tiles replace the SMA's workspace
     for (int k = 0; k < 2; ++k) {
         h.scan_ws[k] = take(h.scan_bytes);
         h.sma_ws[k] = take(h.sma_bytes);
+        h.tiles[k] = take(h.tiles_bytes);
     }
     h.total = o;
     return h;
@@ -960,8 +963,10 @@ dart_status dart_prefill_host(const dart_dims* d, const void* X, const float* dt
                 return fail(e);
             dtg = (const float*)(gb + h.dtg);
         }
-        st = dart_chunk_scan(&dg, gb + h.x, dtg, (const float*)(w + h.a) + h0, w + h.bm, w + h.cm,
-                             gb + h.yssd, gb + h.m, (float*)(gb + h.rm), nullptr, w + h.scan_ws[k],
+        // the scan writes the SMA's operand tiles where both run on the tensor cores
+        uint8_t* tiles = h.tiles_bytes > 0 ? w + h.tiles[k] : nullptr;
+        st = chunk_scan_impl(&dg, gb + h.x, dtg, (const float*)(w + h.a) + h0, w + h.bm, w + h.cm,
+                             gb + h.yssd, gb + h.m, (float*)(gb + h.rm), nullptr, tiles, w + h.scan_ws[k],
                              h.scan_bytes, cs);
         // the SMA's shared inputs (Q, E, z) are there from here on
         if (st == DART_OK && (e = cudaStreamWaitEvent(cs, sma_ev, 0)) != cudaSuccess) return fail(e);
@@ -971,7 +976,10 @@ dart_status dart_prefill_host(const dart_dims* d, const void* X, const float* dt
                 return fail(e);
             zg = gb + h.zg;
         }
-        if (st == DART_OK)
+        if (st == DART_OK && tiles != nullptr)
+            st = dart_sma_forward_with_tiles(&dg, tiles, w + h.q, w + h.cm, w + h.e, zg, gb + h.yssd, gb + h.y,
+                                             nullptr, nullptr, cs);
+        else if (st == DART_OK)
             st = dart_sma_forward(&dg, gb + h.m, (const float*)(gb + h.rm), w + h.q, w + h.cm, w + h.e, zg,
                                   gb + h.yssd, gb + h.y, nullptr, nullptr, w + h.sma_ws[k], h.sma_bytes, cs);
         if (st != DART_OK) {
