@@ -516,7 +516,9 @@ cudaError_t host_streams(HostStreams** hs) {
 // and outputs, the normalised output, then the scan and SMA workspaces.
 struct BlockWs {
     int64_t ldz, d_in;
-    size_t zx, x, bm, cm, dt, a, q, e, gate, yssd, y, mem, rm, yn, scan, scan_bytes, sma, sma_bytes, total;
+    size_t zx, x, bm, cm, dt, a, q, e, gate, yssd, y, mem, rm, yn, scan, scan_bytes, sma, sma_bytes;
+    size_t tiles, tiles_bytes;  // the SMA's operand tiles from the scan (0: not on this shape)
+    size_t total;
 };
 dart_dims block_core(const dart_block_dims* b) {
     dart_dims c = b->core;
@@ -550,8 +552,10 @@ BlockWs block_ws(const dart_block_dims* b) {
     w.yn = take((size_t)(T * di) * 2);
     w.scan_bytes = scan_ws_bytes(&c);
     w.scan = take(w.scan_bytes);
-    w.sma_bytes = sma_ws(&c);
+    w.tiles_bytes = dart_sma_tiles_size(&c);
+    w.sma_bytes = w.tiles_bytes > 0 ? 0 : sma_ws(&c);  // the tiles replace the SMA's workspace
     w.sma = take(w.sma_bytes);
+    w.tiles = take(w.tiles_bytes);
     w.total = o;
     return w;
 }
@@ -1151,11 +1155,16 @@ dart_status dart_block_forward(const dart_block_dims* b, const void* U, const vo
     cudaError_t e = dart::launch_gemm_tc<float>(U, W_in, (float*)a.zx, T, w.d_in, b->d_model, w.ldz, w.ldz, lim, s);
     if (e == cudaSuccess) e = dart::launch_block_conv_split(a, s);
     if (e != cudaSuccess) return cuda_fail(e);
-    st = dart_chunk_scan(&c, a.X, a.dt, a.A, a.Bm, a.Cm, p + w.yssd, p + w.mem, (float*)(p + w.rm), nullptr,
-                         p + w.scan, w.scan_bytes, stream);
+    // the scan writes the SMA's operand tiles where both run on the tensor cores
+    uint8_t* tiles = w.tiles_bytes > 0 ? p + w.tiles : nullptr;
+    st = chunk_scan_impl(&c, a.X, a.dt, a.A, a.Bm, a.Cm, p + w.yssd, p + w.mem, (float*)(p + w.rm), nullptr,
+                         tiles, p + w.scan, w.scan_bytes, stream);
     if (st != DART_OK) return st;
-    st = dart_sma_forward(&c, p + w.mem, (const float*)(p + w.rm), a.Q, a.Cm, a.E, a.gate, p + w.yssd, a.Y,
-                          nullptr, nullptr, p + w.sma, w.sma_bytes, stream);
+    st = tiles != nullptr
+             ? dart_sma_forward_with_tiles(&c, tiles, a.Q, a.Cm, a.E, a.gate, p + w.yssd, a.Y, nullptr, nullptr,
+                                           stream)
+             : dart_sma_forward(&c, p + w.mem, (const float*)(p + w.rm), a.Q, a.Cm, a.E, a.gate, p + w.yssd,
+                                a.Y, nullptr, nullptr, p + w.sma, w.sma_bytes, stream);
     if (st != DART_OK) return st;
     e = dart::launch_block_norm(a, s);
     if (e == cudaSuccess)
