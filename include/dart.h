@@ -192,7 +192,9 @@ dart_status dart_sma_forward(const dart_dims* dims, const void* M, const float* 
  *          once `stream` reaches the point where the call left it.
  * Workspace: dart_workspace_size(dims, DART_OP_PREFILL_HOST) bytes of device
  *          memory, 256-byte aligned: device copies of the inputs, each group's
- *          Y_ssd, Y, memories and their r, and the scan and SMA workspaces.
+ *          Y_ssd, Y, memories and their r, and the scan and SMA workspaces. On
+ *          the shapes of dart_chunk_scan_with_tiles each group's scan writes
+ *          the SMA's operand tiles, which take the SMA workspace's place.
  * The call orders itself after the work already on `stream` and leaves
  * `stream` waiting for its last copy (also when it fails part way, for what
  * it had enqueued). The four streams are created on the
@@ -363,7 +365,10 @@ dart_status dart_chunk_scan_backward(const dart_dims* dims, const void* X, const
  *          W_out (d_model, d_inner) bf16 (nn.Linear layouts).
  * Output:  out (Bsz, L, d_model) in core.out_dtype (DART_F32 or DART_BF16).
  * Requires core.in_dtype == DART_BF16, d_model % 8 == 0, H % 8 == 0, H P <= 4096;
- * L need not be a multiple of S. Workspace: dart_block_workspace_size(dims).
+ * L need not be a multiple of S. Workspace: dart_block_workspace_size(dims): zx,
+ * the hot path's inputs and outputs, yn, the scan's workspace and either the SMA's
+ * workspace or, on the shapes of dart_chunk_scan_with_tiles, the SMA's operand tiles
+ * (written by the scan).
  */
 typedef struct {
     dart_dims core;      /* Bsz, L, H, G, P, N, S, eps of the hot path; in_dtype (DART_BF16) and

@@ -67,6 +67,8 @@ SWEEP = [
     (1024, 64, 64, 128, 8, 1, "bf16"),     # S = 64: one chunk per 128-row tile, rows 64 .. 127 idle
     (512, 64, 64, 128, 16, 2, "bf16"),     # S = 64, G = 2
     (1000, 64, 64, 128, 8, 1, "bf16"),     # S = 64 and ragged: 1024 padded tokens
+    (100, 256, 64, 128, 8, 1, "bf16"),     # L < S: one partial chunk, no token has history
+    (129, 128, 64, 128, 8, 1, "bf16"),     # one full chunk and a one-token chunk: only the last token reads a memory
     # ragged L (L % S != 0): the last memory holds the partial chunk
     (1000, 256, 64, 128, 8, 1, "bf16"),    # tensor-core scan and SMA on 1024 padded tokens
     (1000, 256, 64, 128, 2, 1, "bf16"),    # CUDA-core scan, tensor-core SMA
