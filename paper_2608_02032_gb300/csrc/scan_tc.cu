@@ -619,51 +619,59 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
     };
     __syncthreads();  // barriers initialised before any copy
     if (tid == 0 && has_prev) issue_h(0);
-    // C of the tile: row t, K-major, two K blocks of 64 (16-byte chunks, swizzled)
-    for (int i = tid; i < kT * 16; i += kOutThreads) {
-        const int t = i / 16, q = i % 16;
-        const uint4 v = tt * kT + t < S
-                            ? reinterpret_cast<const uint4*>(Cm + ((tok0 + pos(tt * kT + t)) * G + g) * kN)[q]
-                            : make_uint4(0u, 0u, 0u, 0u);
-        *reinterpret_cast<uint4*>(sm.c_tile[q / 8] + sw128((uint32_t)t, (uint32_t)(q % 8) * 16u)) = v;
-    }
-    // B of the sources: row s, K-major
-    for (int i = tid; kIntra && i < ns * 16; i += kOutThreads) {
-        const int s = i / 16, q = i % 16;
-        const uint4 v = reinterpret_cast<const uint4*>(Bm + ((tok0 + pos(s)) * G + g) * kN)[q];
-        *reinterpret_cast<uint4*>(sm.b_src[q / 8] + sw128((uint32_t)s, (uint32_t)(q % 8) * 16u)) = v;
-    }
-    // row norms for the W scale bound: thread tid < ns takes |B_tid|, tid < kT takes |C_tid|
-    if (kIntra && tid < ns) {
-        const uint4* brow = reinterpret_cast<const uint4*>(Bm + ((tok0 + pos(tid)) * G + g) * kN);
+    // C of the tile and B of the sources, K-major (row t or s, two K blocks of 64, 16-byte
+    // chunks, swizzled). Every load of a thread is issued before any store; the 16 lanes
+    // of a half-warp hold one row, and their squares give its norm for the W scale bound
+    // (|C_t|, |B_s|) without a second pass over the rows.
+    constexpr int kCIt = kT * 16 / kOutThreads;    // 4 pieces of C per thread
+    constexpr int kBItMax = 256 * 16 / kOutThreads;  // up to 8 pieces of B
+    const int bit = kIntra ? ns * 16 / kOutThreads : 0;  // 2, 4 or 8 (ns = 64, 128, 256)
+    auto sumsq8 = [](const uint4 v) {
+        const uint32_t w[4] = {v.x, v.y, v.z, v.w};
         float ss = 0.0f;
-#pragma unroll 4
-        for (int q = 0; q < 16; ++q) {
-            const uint4 v = brow[q];
-            const uint32_t w[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
-            for (int e = 0; e < 4; ++e) {
-                const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w[e]));
-                ss = fmaf(f.x, f.x, fmaf(f.y, f.y, ss));
+        for (int e = 0; e < 4; ++e) {
+            const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w[e]));
+            ss = fmaf(f.x, f.x, fmaf(f.y, f.y, ss));
+        }
+        return ss;
+    };
+    auto half_sum = [](float ss) {  // over the 16 lanes of a half-warp
+#pragma unroll
+        for (int o = 8; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+        return ss;
+    };
+    {
+        uint4 cv[kCIt], bv[kBItMax];
+#pragma unroll
+        for (int k = 0; k < kCIt; ++k) {
+            const int i = tid + k * kOutThreads, t = i / 16, q = i % 16;
+            cv[k] = tt * kT + t < S ? reinterpret_cast<const uint4*>(Cm + ((tok0 + pos(tt * kT + t)) * G + g) * kN)[q]
+                                    : make_uint4(0u, 0u, 0u, 0u);
+        }
+#pragma unroll
+        for (int k = 0; k < kBItMax; ++k) {
+            if (k < bit) {
+                const int i = tid + k * kOutThreads, sidx = i / 16, q = i % 16;
+                bv[k] = reinterpret_cast<const uint4*>(Bm + ((tok0 + pos(sidx)) * G + g) * kN)[q];
             }
         }
-        sm.bnorm[tid] = sqrtf(ss);
-    }
-    if (tid < kT && tt * kT + tid >= S) sm.cnorm[tid] = 0.0f;
-    if (tid < kT && tt * kT + tid < S) {
-        const uint4* crow = reinterpret_cast<const uint4*>(Cm + ((tok0 + pos(tt * kT + tid)) * G + g) * kN);
-        float ss = 0.0f;
-#pragma unroll 4
-        for (int q = 0; q < 16; ++q) {
-            const uint4 v = crow[q];
-            const uint32_t w[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
-            for (int e = 0; e < 4; ++e) {
-                const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w[e]));
-                ss = fmaf(f.x, f.x, fmaf(f.y, f.y, ss));
+        for (int k = 0; k < kCIt; ++k) {
+            const int i = tid + k * kOutThreads, t = i / 16, q = i % 16;
+            *reinterpret_cast<uint4*>(sm.c_tile[q / 8] + sw128((uint32_t)t, (uint32_t)(q % 8) * 16u)) = cv[k];
+            const float ss = half_sum(sumsq8(cv[k]));
+            if (q == 0) sm.cnorm[t] = sqrtf(ss);
+        }
+#pragma unroll
+        for (int k = 0; k < kBItMax; ++k) {
+            if (k < bit) {  // uniform over the block
+                const int i = tid + k * kOutThreads, sidx = i / 16, q = i % 16;
+                *reinterpret_cast<uint4*>(sm.b_src[q / 8] + sw128((uint32_t)sidx, (uint32_t)(q % 8) * 16u)) = bv[k];
+                const float ss = half_sum(sumsq8(bv[k]));
+                if (q == 0) sm.bnorm[sidx] = sqrtf(ss);
             }
         }
-        sm.cnorm[tid] = sqrtf(ss);
     }
     if (tid < 2) sm.bdmax[tid] = 0u;
     tc::fence_proxy_async_shared();
