@@ -1,5 +1,6 @@
 // C ABI of the DART hot path: host-side validation, workspace layout and
 // kernel dispatch. Declarations and the contract are in include/dart.h.
+#include <algorithm>
 #include <atomic>
 #include <mutex>
 
@@ -98,7 +99,7 @@ bool scan_uses_tc(const dart_dims* d) {
     dart::ScanArgs a{};
     a.B = d->batch; a.L = d->seqlen; a.H = d->nheads; a.G = d->ngroups;
     a.P = d->headdim; a.N = d->dstate; a.S = d->chunk;
-    return d->in_dtype == DART_BF16 && dart::scan_tc_supported(a);
+    return d->in_dtype == DART_BF16 && dart::scan_fwd_tc_supported(a);
 }
 
 // Workspace of the scan for L % S == 0.
@@ -416,16 +417,35 @@ std::atomic<int> g_test_withhold{0};
 std::atomic<uint64_t> g_launches{0};
 
 // ------------------------------------------------ host-buffer prefill layout
-constexpr int64_t kHostGroupHeads = 8;  // heads per copy/compute group
+constexpr int kMaxHostGroups = 64;
 
 size_t dtype_bytes(int t) { return t == DART_F32 ? 4 : 2; }
 
-// Device workspace of dart_prefill_host: the shared inputs, then per group of
-// hg heads its X, dt, z, Y_ssd, Y, memories and r (every group the same size),
-// then one scan and one SMA workspace per compute stream (groups alternate
-// between the two compute streams).
+// Heads of each copy/compute group of dart_prefill_host. G = 1 with H a multiple
+// of 8 above 8 (at most 64 groups): 4-head groups at both ends, 8-head groups
+// between them, so that the first group's kernels start after the shortest
+// copy-in and the last group's copy-out, which nothing runs under, is the
+// shortest. Any other shape: one group of all heads. Returns the group count.
+int host_groups(const dart_dims* d, int64_t* gh) {
+    const int64_t H = d->nheads;
+    if (d->ngroups != 1 || H <= 8 || H % 8 != 0 || H / 8 + 1 > kMaxHostGroups) {
+        gh[0] = H;
+        return 1;
+    }
+    int n = 0;
+    gh[n++] = 4;
+    for (int64_t h = 4; h < H - 4; h += 8) gh[n++] = 8;
+    gh[n++] = 4;
+    return n;
+}
+
+// Device workspace of dart_prefill_host: the shared inputs, then per group its X,
+// dt, z, Y_ssd, Y, memories and r (every group sized for the largest), then one
+// scan workspace and one set of SMA tiles (or SMA workspace) per compute stream
+// (groups alternate between the two compute streams).
 struct HostLayout {
-    int64_t hg, groups;
+    int64_t groups, hmax;
+    int64_t gh[kMaxHostGroups], gfirst[kMaxHostGroups];  // heads of each group, its first head
     size_t bm, cm, q, e, dt, z, a;          // shared inputs
     size_t g0, stride;                      // first group, bytes per group
     size_t x, dtg, zg, yssd, y, m, rm;      // offsets inside a group
@@ -438,11 +458,11 @@ HostLayout host_layout(const dart_dims* d) {
     HostLayout h{};
     const int64_t B = d->batch, L = d->seqlen, H = d->nheads, G = d->ngroups, P = d->headdim;
     const int64_t N = d->dstate, M = (L + d->chunk - 1) / d->chunk;
-    // groups of kHostGroupHeads heads (at most 64 groups), else the whole problem as one
-    h.hg = (G == 1 && H > kHostGroupHeads && H % kHostGroupHeads == 0 && H / kHostGroupHeads <= 64)
-               ? kHostGroupHeads
-               : H;
-    h.groups = H / h.hg;
+    h.groups = host_groups(d, h.gh);
+    for (int64_t g = 0, h0 = 0; g < h.groups; h0 += h.gh[g], ++g) {
+        h.gfirst[g] = h0;
+        h.hmax = std::max(h.hmax, h.gh[g]);
+    }
     const size_t ei = dtype_bytes(d->in_dtype), em = dtype_bytes(d->mem_dtype);
     const size_t eo = dtype_bytes(d->out_dtype);
     const size_t rows = (size_t)(B * L);
@@ -460,7 +480,7 @@ HostLayout host_layout(const dart_dims* d) {
     h.z = take(rows * H * ei);
     h.a = take((size_t)H * 4);
     h.g0 = o;
-    const size_t hg = (size_t)h.hg;
+    const size_t hg = (size_t)h.hmax;
     h.x = take(rows * hg * P * ei) - h.g0;
     h.dtg = take(rows * hg * 4) - h.g0;
     h.zg = take(rows * hg * ei) - h.g0;
@@ -470,10 +490,17 @@ HostLayout host_layout(const dart_dims* d) {
     h.rm = take((size_t)(B * M) * hg * N * 4) - h.g0;
     h.stride = o - h.g0;
     o = h.g0 + (size_t)h.groups * h.stride;
+    // workspaces for the largest group (their sizes grow with the heads); the tiles
+    // only where every group's shape takes them
     dart_dims dg = *d;
-    dg.nheads = h.hg;
+    dg.nheads = h.hmax;
     h.scan_bytes = scan_ws_bytes(&dg);
     h.tiles_bytes = dart_sma_tiles_size(&dg);
+    for (int64_t g = 0; g < h.groups && h.tiles_bytes > 0; ++g) {
+        dart_dims dk = *d;
+        dk.nheads = h.gh[g];
+        if (dart_sma_tiles_size(&dk) == 0) h.tiles_bytes = 0;
+    }
     h.sma_bytes = h.tiles_bytes > 0 ? 0 : sma_ws(&dg);  // the tiles replace the SMA's workspace
     for (int k = 0; k < 2; ++k) {
         h.scan_ws[k] = take(h.scan_bytes);
@@ -874,7 +901,8 @@ dart_status dart_prefill_host(const dart_dims* d, const void* X, const float* dt
     cudaStream_t s = (cudaStream_t)stream;
     const int ng = (int)h.groups;
     // events: the start on the caller's stream, per group copy-in and kernels done, the end
-    cudaEvent_t start = nullptr, done = nullptr, sma_ev = nullptr, in_ev[64] = {}, comp_ev[64] = {};
+    cudaEvent_t start = nullptr, done = nullptr, sma_ev = nullptr, in_ev[kMaxHostGroups] = {},
+                comp_ev[kMaxHostGroups] = {};
     // events are released once recorded (the driver frees each when its work is done)
     auto release = [&]() {
         if (start != nullptr) cudaEventDestroy(start);
@@ -935,11 +963,11 @@ dart_status dart_prefill_host(const dart_dims* d, const void* X, const float* dt
     for (const auto& c : scan_in)
         if ((e = cudaMemcpyAsync(w + c.off, c.src, c.bytes, cudaMemcpyHostToDevice, hs->in)) != cudaSuccess)
             return fail(e);
-    dart_dims dg = *d;
-    dg.nheads = h.hg;
-    const size_t xrow = (size_t)h.hg * P * ei, yrow = (size_t)h.hg * P * eo;
     for (int g = 0; g < ng; ++g) {
-        const int64_t h0 = (int64_t)g * h.hg;
+        const int64_t h0 = h.gfirst[g], hg = h.gh[g];
+        dart_dims dg = *d;
+        dg.nheads = hg;
+        const size_t xrow = (size_t)hg * P * ei, yrow = (size_t)hg * P * eo;
         uint8_t* gb = w + h.g0 + (size_t)g * h.stride;
         // copy in: the group's X rows (pitched)
         e = cudaMemcpy2DAsync(gb + h.x, xrow, (const uint8_t*)X + (size_t)h0 * P * ei, (size_t)H * P * ei,
@@ -962,7 +990,7 @@ dart_status dart_prefill_host(const dart_dims* d, const void* X, const float* dt
         const float* dtg = (const float*)(w + h.dt);
         const void* zg = w + h.z;
         if (ng > 1) {
-            if ((e = dart::launch_gather_heads(w + h.dt, gb + h.dtg, (int64_t)rows, H, h0, h.hg, 4, cs)) !=
+            if ((e = dart::launch_gather_heads(w + h.dt, gb + h.dtg, (int64_t)rows, H, h0, hg, 4, cs)) !=
                 cudaSuccess)
                 return fail(e);
             dtg = (const float*)(gb + h.dtg);
@@ -975,7 +1003,7 @@ dart_status dart_prefill_host(const dart_dims* d, const void* X, const float* dt
         // the SMA's shared inputs (Q, E, z) are there from here on
         if (st == DART_OK && (e = cudaStreamWaitEvent(cs, sma_ev, 0)) != cudaSuccess) return fail(e);
         if (st == DART_OK && ng > 1) {
-            if ((e = dart::launch_gather_heads(w + h.z, gb + h.zg, (int64_t)rows, H, h0, h.hg, (int)ei, cs)) !=
+            if ((e = dart::launch_gather_heads(w + h.z, gb + h.zg, (int64_t)rows, H, h0, hg, (int)ei, cs)) !=
                 cudaSuccess)
                 return fail(e);
             zg = gb + h.zg;

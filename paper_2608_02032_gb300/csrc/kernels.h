@@ -169,8 +169,10 @@ cudaError_t launch_chunk_cumsum(const ScanArgs& a, cudaStream_t stream);
 cudaError_t launch_state_passing(const ScanArgs& a, cudaStream_t stream);
 
 // Tensor-core scan (scan_tc.cu): bf16 inputs, P = 64, N = 128, S in {64, 128, 256}
-// (the backward helpers: S in {128, 256}).
+// (the backward helpers: S in {128, 256}). The forward (launch_chunk_scan_tc) takes
+// H and H / G multiples of 4; the backward helpers multiples of 8.
 bool scan_tc_supported(const ScanArgs& a);
+bool scan_fwd_tc_supported(const ScanArgs& a);
 template <typename Tmem, typename Tout>
 cudaError_t launch_chunk_scan_tc(const ScanArgs& a, unsigned long long wait_limit_ns,
                                  cudaStream_t stream);

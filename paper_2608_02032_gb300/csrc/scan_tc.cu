@@ -49,9 +49,11 @@ __device__ int g_scan_tc_status;  // first timeout code since the last read (0 =
 constexpr int kP = 64;
 constexpr int kN = 128;
 constexpr int kT = 128;  // tokens per output tile
-// The tensor-core scan wants H and H / G to be multiples of 8. The output kernel
-// takes a runtime number of heads per CTA (a divisor of H / G, at most
-// kMaxOutHeads) chosen on the host so that its CTAs fill the SMs in few waves.
+// The tensor-core scan's backward wants H and H / G to be multiples of 8, its
+// forward multiples of kStateHeads (4, the chunk-state kernel's heads per CTA).
+// The output kernel takes a runtime number of heads per CTA (a divisor of H / G,
+// at most kMaxOutHeads) chosen on the host so that its CTAs fill the SMs in few
+// waves.
 constexpr int kHeadsPerCta = 8;
 constexpr int kMaxOutHeads = 16;
 constexpr uint64_t kDrainLimitNs = 2000000000ull;
@@ -935,6 +937,11 @@ int out_heads_per_cta(int units, int H, int G) {
 bool scan_tc_supported(const ScanArgs& a) {
     return a.P == kP && a.N == kN && (a.S == 64 || a.S == 128 || a.S == 256) &&
            a.H % kHeadsPerCta == 0 && (a.H / a.G) % kHeadsPerCta == 0;
+}
+
+bool scan_fwd_tc_supported(const ScanArgs& a) {
+    return a.P == kP && a.N == kN && (a.S == 64 || a.S == 128 || a.S == 256) &&
+           a.H % kStateHeads == 0 && (a.H / a.G) % kStateHeads == 0;
 }
 
 template <typename Tmem, typename Tout>

@@ -53,7 +53,8 @@ SWEEP = [
     (768, 256, 64, 128, 4, 2, "bf16"),   # M = 3, two groups
     (320, 64, 32, 32, 2, 1, "bf16"),     # ragged last token tile inside chunks
     (1024, 128, 64, 128, 2, 1, "bf16"),
-    # tensor-core SMA shapes (bf16, P 64, N 128, two heads per job, one CTA per 128-token tile)
+    # tensor-core SMA shapes (bf16, P 64, N 128, two heads per job, one CTA per 128-token tile);
+    # at H = 4 the scan runs on the tensor cores too
     (512, 128, 64, 128, 4, 1, "bf16"),     # first tile of each chunk ... M = 4
     (256, 128, 64, 128, 4, 1, "bf16"),     # M = 2
     (128, 128, 64, 128, 4, 1, "bf16"),     # M = 1: only chunk-0 tiles
@@ -61,8 +62,10 @@ SWEEP = [
     (768, 128, 64, 128, 2, 1, "bf16"),     # M = 6
     (1024, 256, 64, 128, 8, 1, "bf16"),    # two head groups
     (768, 256, 64, 128, 8, 2, "bf16"),     # G = 2, four heads per group
-    # tensor-core scan shapes (bf16, P 64, N 128, S in {64, 128, 256}, 8 heads per CTA)
+    # tensor-core scan shapes (bf16, P 64, N 128, S in {64, 128, 256}, H / G a multiple of 4)
     (512, 128, 64, 128, 8, 1, "bf16"),
+    (1024, 256, 64, 128, 4, 1, "bf16"),    # four heads: one chunk-state CTA per chunk
+    (512, 256, 64, 128, 12, 1, "bf16"),    # twelve heads: three chunk-state CTAs, output heads per CTA divide 12
     (1024, 256, 64, 128, 16, 2, "bf16"),   # G = 2, eight heads per group
     (1024, 64, 64, 128, 8, 1, "bf16"),     # S = 64: one chunk per 128-row tile, rows 64 .. 127 idle
     (512, 64, 64, 128, 16, 2, "bf16"),     # S = 64, G = 2
@@ -223,6 +226,8 @@ TILE_CASES = [
     (2, 16, 2, 512, 128, "f32", "f32"),   # G = 2
     (1, 8, 1, 512, 64, "f32", "f32"),     # S = 64: a tile spans two chunks in the SMA
     (1, 8, 1, 512, 128, "bf16", "bf16"),  # bf16 memories: the tiles hold the stored (rounded) values
+    (2, 4, 1, 512, 256, "f32", "f32"),    # four heads: one chunk-state CTA per chunk
+    (1, 12, 1, 768, 128, "f32", "f32"),   # twelve heads
 ]
 
 
@@ -274,8 +279,9 @@ def test_sma_tiles_refuse_other_shapes():
                                          kw.get("P", 64), kw.get("N", 128), kw.get("S", 128),
                                          kw.get("dt", binding.DART_BF16), eps=1e-6)
     assert binding.dart_sma_tiles_size(dims()) > 0
-    for bad in (dict(L=500), dict(H=4), dict(P=32), dict(dt=binding.DART_F32), dict(S=32)):
+    assert binding.dart_sma_tiles_size(dims(H=4)) > 0
+    for bad in (dict(L=500), dict(H=2), dict(H=6), dict(P=32), dict(dt=binding.DART_F32), dict(S=32)):
         assert binding.dart_sma_tiles_size(dims(**bad)) == 0, bad
     with pytest.raises(binding.DartError):
         t = torch.empty(1 << 20, dtype=torch.uint8, device="cuda")
-        binding.dart_sma_forward_with_tiles(dims(H=4), t, t, t, t, t, t, t)
+        binding.dart_sma_forward_with_tiles(dims(H=6), t, t, t, t, t, t, t)
