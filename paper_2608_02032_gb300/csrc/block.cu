@@ -116,16 +116,16 @@ block_split_kernel(const float* __restrict__ zx, int ldz, int64_t T, int di, int
 }
 
 // y = Y + D_h x, g = y SiLU(z), yn = g / sqrt(mean(g^2) + eps) w over d_inner, bf16:
-// one warp per token (8 per block), lane l taking the 8-channel groups l, l + 32, ...
+// one warp per token (4 per block), lane l taking the 8-channel groups l, l + 32, ...
 // (at most kNormGroups per lane, kept in registers between the two passes:
 // d_inner <= kNormGroups x 32 x 8).
 template <int kNormGroups>
-__global__ void __launch_bounds__(256)
+__global__ void __launch_bounds__(128)
 block_norm_kernel(const float* __restrict__ Y, const __nv_bfloat16* __restrict__ X,
                   const float* __restrict__ zx, int ldz, const float* __restrict__ D,
                   const float* __restrict__ norm_w, __nv_bfloat16* __restrict__ yn, int64_t T, int di, int P,
                   float eps) {
-    const i64 tok = (i64)blockIdx.x * 8 + (threadIdx.x >> 5);
+    const i64 tok = (i64)blockIdx.x * 4 + (threadIdx.x >> 5);
     const int lane = threadIdx.x & 31;
     if (tok >= T) return;
     const int groups = di / 8;
@@ -168,9 +168,13 @@ block_norm_kernel(const float* __restrict__ Y, const __nv_bfloat16* __restrict__
         const int q = lane + 32 * j;
         if (q >= groups) break;
         const int c0 = 8 * q;
+        // norm_w is 16-byte aligned (checked by the entry point) and c0 a multiple of 8
+        const float4 w0 = *reinterpret_cast<const float4*>(norm_w + c0);
+        const float4 w1 = *reinterpret_cast<const float4*>(norm_w + c0 + 4);
+        const float wv[8] = {w0.x, w0.y, w0.z, w0.w, w1.x, w1.y, w1.z, w1.w};
         float o[8];
 #pragma unroll
-        for (int e = 0; e < 8; ++e) o[e] = g[j][e] * inv * norm_w[c0 + e];
+        for (int e = 0; e < 8; ++e) o[e] = g[j][e] * inv * wv[e];
         store_row8(yn + tok * di + c0, o);
     }
 }
@@ -212,7 +216,7 @@ cudaError_t launch_block_norm(const BlockArgs& a, cudaStream_t stream) {
     const int64_t T = a.B * a.L;
     if (di > 16 * 32 * 8) return cudaErrorInvalidValue;
     auto kern = di <= 8 * 32 * 8 ? block_norm_kernel<8> : block_norm_kernel<16>;
-    kern<<<(unsigned)((T + 7) / 8), 256, 0, stream>>>(
+    kern<<<(unsigned)((T + 3) / 4), 128, 0, stream>>>(
         a.Y, (const __nv_bfloat16*)a.X, (const float*)a.zx, (int)a.ldz, a.D, a.norm_w, (__nv_bfloat16*)a.yn, T,
         di, (int)a.P, a.norm_eps);
     note_launches(1);

@@ -418,39 +418,39 @@ std::atomic<uint64_t> g_launches{0};
 
 // ------------------------------------------------ host-buffer prefill layout
 constexpr int kMaxHostGroups = 64;
+constexpr int kHostComp = 3;  // compute streams of dart_prefill_host (groups take them in turn)
 
 size_t dtype_bytes(int t) { return t == DART_F32 ? 4 : 2; }
 
-// Heads of each copy/compute group of dart_prefill_host. G = 1 with H a multiple
-// of 8 above 8 (at most 64 groups): 4-head groups at both ends, 8-head groups
-// between them, so that the first group's kernels start after the shortest
-// copy-in and the last group's copy-out, which nothing runs under, is the
-// shortest. Any other shape: one group of all heads. Returns the group count.
+// Heads of each copy/compute group of dart_prefill_host: groups of 4 heads for
+// G = 1 with H a multiple of 4 above 4 (at most 64 groups), else one group of all
+// heads. Small groups start the first kernels after a short copy-in and leave a
+// short copy-out after the last; three compute streams run neighbouring groups'
+// kernels side by side, which makes up for the small grids of 4-head kernels.
+// Returns the group count.
 int host_groups(const dart_dims* d, int64_t* gh) {
     const int64_t H = d->nheads;
-    if (d->ngroups != 1 || H <= 8 || H % 8 != 0 || H / 8 + 1 > kMaxHostGroups) {
+    if (d->ngroups != 1 || H <= 4 || H % 4 != 0 || H / 4 > kMaxHostGroups) {
         gh[0] = H;
         return 1;
     }
-    int n = 0;
-    gh[n++] = 4;
-    for (int64_t h = 4; h < H - 4; h += 8) gh[n++] = 8;
-    gh[n++] = 4;
-    return n;
+    for (int64_t g = 0; g < H / 4; ++g) gh[g] = 4;
+    return (int)(H / 4);
 }
 
 // Device workspace of dart_prefill_host: the shared inputs, then per group its X,
 // dt, z, Y_ssd, Y, memories and r (every group sized for the largest), then one
 // scan workspace and one set of SMA tiles (or SMA workspace) per compute stream
-// (groups alternate between the two compute streams).
+// (groups take the compute streams in turn).
 struct HostLayout {
     int64_t groups, hmax;
+    int nc;  // compute streams in use
     int64_t gh[kMaxHostGroups], gfirst[kMaxHostGroups];  // heads of each group, its first head
     size_t bm, cm, q, e, dt, z, a;          // shared inputs
     size_t g0, stride;                      // first group, bytes per group
     size_t x, dtg, zg, yssd, y, m, rm;      // offsets inside a group
-    size_t scan_ws[2], scan_bytes, sma_ws[2], sma_bytes;
-    size_t tiles[2], tiles_bytes;  // the SMA's operand tiles from the scan (0: not on this shape)
+    size_t scan_ws[kHostComp], scan_bytes, sma_ws[kHostComp], sma_bytes;
+    size_t tiles[kHostComp], tiles_bytes;  // the SMA's operand tiles from the scan (0: not on this shape)
     size_t total;
 };
 
@@ -502,7 +502,8 @@ HostLayout host_layout(const dart_dims* d) {
         if (dart_sma_tiles_size(&dk) == 0) h.tiles_bytes = 0;
     }
     h.sma_bytes = h.tiles_bytes > 0 ? 0 : sma_ws(&dg);  // the tiles replace the SMA's workspace
-    for (int k = 0; k < 2; ++k) {
+    h.nc = (int)std::min<int64_t>(kHostComp, h.groups);
+    for (int k = 0; k < h.nc; ++k) {
         h.scan_ws[k] = take(h.scan_bytes);
         h.sma_ws[k] = take(h.sma_bytes);
         h.tiles[k] = take(h.tiles_bytes);
@@ -511,10 +512,10 @@ HostLayout host_layout(const dart_dims* d) {
     return h;
 }
 
-// The streams of dart_prefill_host (copy in, two for the kernels, copy out) for
-// the current device, created on first use and kept.
+// The streams of dart_prefill_host (copy in, kHostComp for the kernels, copy out)
+// for the current device, created on first use and kept.
 struct HostStreams {
-    cudaStream_t in = nullptr, comp[2] = {nullptr, nullptr}, out = nullptr;
+    cudaStream_t in = nullptr, comp[kHostComp] = {}, out = nullptr;
 };
 std::mutex g_host_mu;
 HostStreams g_host_streams[64];
@@ -527,13 +528,12 @@ cudaError_t host_streams(HostStreams** hs) {
     std::lock_guard<std::mutex> lock(g_host_mu);
     HostStreams& s = g_host_streams[dev];
     if (s.in == nullptr) {
-        cudaStream_t t[4];
-        for (int i = 0; i < 4; ++i)
+        cudaStream_t t[kHostComp + 2];
+        for (int i = 0; i < kHostComp + 2; ++i)
             if ((e = cudaStreamCreateWithFlags(&t[i], cudaStreamNonBlocking)) != cudaSuccess) return e;
         s.in = t[0];
-        s.comp[0] = t[1];
-        s.comp[1] = t[2];
-        s.out = t[3];
+        for (int k = 0; k < kHostComp; ++k) s.comp[k] = t[1 + k];
+        s.out = t[kHostComp + 1];
     }
     *hs = &s;
     return cudaSuccess;
@@ -918,7 +918,8 @@ dart_status dart_prefill_host(const dart_dims* d, const void* X, const float* dt
     bool started = false;
     auto join = [&]() {
         if (!started) return;
-        cudaStream_t own[4] = {hs->in, hs->comp[0], hs->comp[1], hs->out};
+        cudaStream_t own[kHostComp + 2] = {hs->in, hs->out};
+        for (int k = 0; k < kHostComp; ++k) own[2 + k] = hs->comp[k];
         for (cudaStream_t x : own) {
             cudaEvent_t ev = nullptr;
             if (cudaEventCreateWithFlags(&ev, cudaEventDisableTiming) == cudaSuccess) {
@@ -946,9 +947,8 @@ dart_status dart_prefill_host(const dart_dims* d, const void* X, const float* dt
     if ((e = cudaEventRecord(start, s)) != cudaSuccess) return fail(e);
     started = true;
     if ((e = cudaStreamWaitEvent(hs->in, start, 0)) != cudaSuccess) return fail(e);
-    if ((e = cudaStreamWaitEvent(hs->comp[0], start, 0)) != cudaSuccess ||
-        (e = cudaStreamWaitEvent(hs->comp[1], start, 0)) != cudaSuccess)
-        return fail(e);
+    for (int k = 0; k < h.nc; ++k)
+        if ((e = cudaStreamWaitEvent(hs->comp[k], start, 0)) != cudaSuccess) return fail(e);
     if ((e = cudaStreamWaitEvent(hs->out, start, 0)) != cudaSuccess) return fail(e);
     // shared inputs, one copy each: the scan's first (B, C, dt, A), then, after the
     // first group's X, the SMA's (Q, E, z), which land under the first group's scan
@@ -981,10 +981,10 @@ dart_status dart_prefill_host(const dart_dims* d, const void* X, const float* dt
                     return fail(e);
             if ((e = cudaEventRecord(sma_ev, hs->in)) != cudaSuccess) return fail(e);
         }
-        // kernels, groups alternating between the two compute streams (so that the
-        // kernels of neighbouring groups share the SMs): the group's dt and z
+        // kernels, groups taking the compute streams in turn (so that the kernels
+        // of neighbouring groups share the SMs): the group's dt and z
         // columns, the scan, the SMA and merge
-        const int k = g & 1;
+        const int k = g % h.nc;
         cudaStream_t cs = hs->comp[k];
         if ((e = cudaStreamWaitEvent(cs, in_ev[g], 0)) != cudaSuccess) return fail(e);
         const float* dtg = (const float*)(w + h.dt);

@@ -140,11 +140,11 @@ def test_prefill_host_validation_and_workspace(L):
     from paper_2608_02032_gb300 import binding as B
 
     v = ctypes.c_void_p
-    d = _dims(nheads=32)  # G = 1, H = 32: groups of 4, 8, 8, 8 and 4 heads
+    d = _dims(nheads=32)  # G = 1, H = 32: eight groups of 4 heads
     need = B.dart_workspace_size(d, B.DART_OP_PREFILL_HOST)
-    one = _dims(nheads=8)  # the device sizes of one group of 8 heads
-    per_group_inputs = 512 * 8 * 64 * 2
-    assert need > 5 * per_group_inputs  # five groups, each sized for the largest
+    one = _dims(nheads=4)  # the device sizes of one group of 4 heads
+    per_group_inputs = 512 * 4 * 64 * 2
+    assert need > 8 * per_group_inputs
     assert need > B.dart_workspace_size(one, B.DART_OP_CHUNK_SCAN)
     assert B.dart_workspace_size(_dims(headdim=48), B.DART_OP_PREFILL_HOST) == 0
     # beyond 64 groups the problem runs as one group (still a valid size)

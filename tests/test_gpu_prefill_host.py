@@ -21,10 +21,11 @@ def _inputs(w):
 
 
 @pytest.mark.parametrize("w", [
-    Workload("host_h32", 1, 32, 2048, 64, 128, 256, seed=51),              # groups of 4, 8, 8, 8, 4 heads
-    Workload("host_b2_h16", 2, 16, 1024, 64, 128, 128, seed=52),           # 4, 8, 4 heads, S = 128
-    Workload("host_h24", 1, 24, 1024, 64, 128, 64, seed=57),               # 4, 8, 8, 4 heads, S = 64
-    Workload("host_h6", 1, 6, 512, 64, 128, 128, seed=53),                 # one group (H < 8)
+    Workload("host_h32", 1, 32, 2048, 64, 128, 256, seed=51),              # eight groups of 4 heads
+    Workload("host_b2_h16", 2, 16, 1024, 64, 128, 128, seed=52),           # four groups, S = 128
+    Workload("host_h24", 1, 24, 1024, 64, 128, 64, seed=57),               # six groups, S = 64
+    Workload("host_h8", 1, 8, 512, 64, 128, 256, seed=58),                 # two groups: fewer than the streams
+    Workload("host_h6", 1, 6, 512, 64, 128, 128, seed=53),                 # one group (H % 4 != 0)
     Workload("host_g2", 1, 16, 512, 64, 128, 128, groups=2, seed=54),      # one group (G = 2)
     Workload("host_small", 1, 16, 512, 32, 64, 64, seed=55),               # the CUDA-core kernels
 ], ids=lambda w: w.name)
