@@ -129,6 +129,17 @@ __device__ __forceinline__ void store_row8(__nv_bfloat16* dst, const float* v) {
 
 // SiLU(z) = z * sigmoid(z), the SMA residual gate (Sec. 3).
 __device__ __forceinline__ float silu_f32(float z) { return z / (1.0f + expf(-z)); }
+
+// Programmatic dependent launch (PTX griddepcontrol). launch_dependents: a kernel
+// launched next on the stream with programmatic stream serialization may start
+// once every CTA of this grid has executed it or exited. wait: blocks the thread
+// until the grid this one was launched after has completed and its memory
+// operations are visible; it returns at once in a kernel launched without that
+// attribute (the stream order has already done it).
+__device__ __forceinline__ void griddep_launch_dependents() {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 // d SiLU / dz = s (1 + z (1 - s)), s = sigmoid(z)
 __device__ __forceinline__ float silu_grad_f32(float z) {
     const float s = 1.0f / (1.0f + expf(-z));

@@ -995,19 +995,25 @@ dart_status dart_prefill_host(const dart_dims* d, const void* X, const float* dt
                 return fail(e);
             dtg = (const float*)(gb + h.dtg);
         }
+        // the SMA's shared inputs (Q, E, z), then the group's z columns: for the first
+        // group after its scan (they land under it), for the others before it (long
+        // there by then), so that their SMA kernel directly follows the scan's last
+        // kernel and may start under its last wave
+        auto sma_inputs = [&]() -> cudaError_t {
+            cudaError_t err = cudaStreamWaitEvent(cs, sma_ev, 0);
+            if (err == cudaSuccess && ng > 1) {
+                err = dart::launch_gather_heads(w + h.z, gb + h.zg, (int64_t)rows, H, h0, hg, (int)ei, cs);
+                zg = gb + h.zg;
+            }
+            return err;
+        };
+        if (g > 0 && (e = sma_inputs()) != cudaSuccess) return fail(e);
         // the scan writes the SMA's operand tiles where both run on the tensor cores
         uint8_t* tiles = h.tiles_bytes > 0 ? w + h.tiles[k] : nullptr;
         st = chunk_scan_impl(&dg, gb + h.x, dtg, (const float*)(w + h.a) + h0, w + h.bm, w + h.cm,
                              gb + h.yssd, gb + h.m, (float*)(gb + h.rm), nullptr, tiles, w + h.scan_ws[k],
                              h.scan_bytes, cs);
-        // the SMA's shared inputs (Q, E, z) are there from here on
-        if (st == DART_OK && (e = cudaStreamWaitEvent(cs, sma_ev, 0)) != cudaSuccess) return fail(e);
-        if (st == DART_OK && ng > 1) {
-            if ((e = dart::launch_gather_heads(w + h.z, gb + h.zg, (int64_t)rows, H, h0, hg, (int)ei, cs)) !=
-                cudaSuccess)
-                return fail(e);
-            zg = gb + h.zg;
-        }
+        if (st == DART_OK && g == 0 && (e = sma_inputs()) != cudaSuccess) return fail(e);
         if (st == DART_OK && tiles != nullptr)
             st = dart_sma_forward_with_tiles(&dg, tiles, w + h.q, w + h.cm, w + h.e, zg, gb + h.yssd, gb + h.y,
                                              nullptr, nullptr, cs);

@@ -577,6 +577,9 @@ chunk_output_tc_kernel(const __nv_bfloat16* __restrict__ X, const float* __restr
     extern __shared__ uint8_t smem_raw[];
     OutSmem& sm = *reinterpret_cast<OutSmem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                               ~(uintptr_t)1023);
+    // the SMA kernel that follows may take the SMs this grid's last wave leaves idle: it
+    // reads nothing this kernel writes before its own griddep_wait
+    griddep_launch_dependents();
     const int tt = blockIdx.x;  // tile inside the chunk
     const int c = blockIdx.y / (H / hpc);
     const int hg = blockIdx.y % (H / hpc);

@@ -716,6 +716,7 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
                 const float s_j = s_next;
                 if (j == pf_job) prefetch_row<kP * (int)sizeof(Tout)>(Yssd + rowo_pf * kP, z + rowo_pf);
                 if (j == nj - 1) {
+                    griddep_wait();  // Y_ssd: the kernel launched before this one is done
                     rows_to_slots_async<kP * (int)sizeof(Tout)>(
                         yslots_last, reinterpret_cast<const uint8_t*>(Yssd + (tok0 * H + h) * kP),
                         (i64)H * kP * (i64)sizeof(Tout), lane);
@@ -796,8 +797,10 @@ sma_tc_kernel(const uint8_t* __restrict__ ops, const float* __restrict__ scale,
                 const bool has = njr > 0;
                 const float inv_d = has ? cdown / dsum : 0.0f;
                 const float gate = silu_f32(nj > 0 ? zlast : __bfloat162float(z[rowo]));
-                if (nj == 0)
+                if (nj == 0) {
+                    griddep_wait();
                     rows_to_slots<kRowB>(yslots, reinterpret_cast<const uint8_t*>(Yssd + row0 * kP), rstride, lane);
+                }
                 float r[kP];
     #pragma unroll
                 for (int i = 0; i < kP / 2; ++i) {
@@ -880,12 +883,26 @@ cudaError_t launch_sma_forward_tc(const SmaArgs& a, void* ws, unsigned long long
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     const int items = (L / kRows) * Bsz * (H / kHeadsPerCta);
-    kern<<<items, kThreads, smem, stream>>>(ops, scale, (const __nv_bfloat16*)a.Q,
-                                            (const __nv_bfloat16*)a.Cm, (const __nv_bfloat16*)a.E,
-                                            (const __nv_bfloat16*)a.z, (const Tout*)a.Yssd,
-                                            (Tout*)a.Y, (Tout*)a.R, a.lse, Bsz, L, H, (int)a.G,
-                                            (int)a.S, Mc, a.eps, wait_limit_ns, a.test_withhold,
-                                            SmaStats{a.logits, nullptr});
+    // Programmatic stream serialization: after the scan's output kernel (which lets
+    // its dependents start once all its CTAs run), this grid's CTAs take the SMs that
+    // kernel's last wave leaves idle. Only Y_ssd comes from that kernel, and every
+    // thread reads it after griddep_wait. After any other kernel the launch waits for
+    // it to finish, as a plain launch does.
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)items);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    e = cudaLaunchKernelEx(&cfg, kern, ops, scale, (const __nv_bfloat16*)a.Q, (const __nv_bfloat16*)a.Cm,
+                           (const __nv_bfloat16*)a.E, (const __nv_bfloat16*)a.z, (const Tout*)a.Yssd, (Tout*)a.Y,
+                           (Tout*)a.R, a.lse, Bsz, L, H, (int)a.G, (int)a.S, Mc, a.eps, wait_limit_ns,
+                           a.test_withhold, SmaStats{a.logits, nullptr});
+    if (e != cudaSuccess) return e;
     note_launches(1);
     return cudaGetLastError();
 }
