@@ -110,15 +110,6 @@ __device__ __forceinline__ void warp_arrive(uint64_t* bar) {
     if ((threadIdx.x & 31) == 0) tc::mbar_arrive(bar);
 }
 
-// Bounded wait by every thread of the CTA, then a CTA-wide AND of the outcome.
-__device__ __forceinline__ bool cta_and_wait(uint64_t* bar, uint32_t parity, uint64_t limit_ns, int code) {
-    const bool got = tc::mbar_wait(bar, parity, limit_ns, nullptr);
-    if (!got) atomicCAS(&g_bwd_tc_status, 0, code);
-    const bool all = __syncthreads_and(got ? 1 : 0) != 0;
-    tc::tc_fence_after();
-    return all;
-}
-
 // Splits 8 floats into bf16 hi and lo words.
 __device__ __forceinline__ void split_bf16x8(const float* v, uint4& hi, uint4& lo) {
     uint32_t hw[4], lw[4];
@@ -621,34 +612,50 @@ sma_bwd_rows_kernel(const uint8_t* __restrict__ ops, const __nv_bfloat16* __rest
 }
 
 // ---------------------------------------------------------- memory kernel
-// One CTA per (two memories j, head pair, b), 32-token tiles of the later chunks,
-// double buffered: T += C^T (c_hi + c_lo), G += Q^T (a_hi + a_lo) with C and Q exact
-// (bf16 inputs, MN-major A) and the scaled B rows split hi + lo:
+// One CTA per (two memories j, head pair, b), 32-token tiles of the later chunks:
+// T += C^T (c_hi + c_lo), G += Q^T (a_hi + a_lo) with C and Q exact (bf16 inputs,
+// MN-major A) and the scaled B rows split hi + lo:
 // c = g SiLU(z) dY, a = iq dl Ebar / sqrt(N) (Qbar's scale moved onto B).
-constexpr int kMemThreads = 512;
+// A tile's global rows (C, Q in the MMA layout; dY, E, g, dl, z, (iq, ie) as they
+// are) land by cp.async in a three-stage ring, two tiles ahead of the one being
+// formed, so the loads' latency hides under a whole tile of work; the B operands
+// are double-buffered. Warps 0..15 form the B operands; warp 16 issues the MMAs,
+// so no forming warp waits for the issue: full[b] (one arrival per forming warp)
+// hands a tile's operands to the MMA warp, mma_done[b] hands buffer b back.
+constexpr int kMemFormThreads = 512;
+constexpr int kMemThreads = kMemFormThreads + 32;
 constexpr int kMT = 32;          // tokens per staged tile (K of one MMA chain: 2 steps)
 constexpr int kBlk = kMT * 128;  // one 64-column MN block of kMT rows
 constexpr int kMemPerCta = 2;    // memories per CTA, sharing the staged C and Q rows
+constexpr int kMemStages = 3;    // tiles in flight in the input ring
 
 struct MemSmem {
-    // per buffer: C^T, Q^T (two 64-row blocks of n each); per memory c_hi, c_lo, a_hi,
-    // a_lo (one 64-column block per head each)
-    uint8_t bc[2][2 * kBlk];
-    uint8_t bq[2][2 * kBlk];
+    uint8_t bc[kMemStages][2 * kBlk];  // C^T, Q^T of a tile (two 64-row blocks of n each)
+    uint8_t bq[kMemStages][2 * kBlk];
+    // per buffer and memory: c_hi, c_lo, a_hi, a_lo (one 64-column block per head each)
     uint8_t bm[2][kMemPerCta][4][2 * kBlk];
+    uint8_t dy[kMemStages][kMT][2][kP * 2];  // dY rows of the two heads, bf16
+    uint8_t ee[kMemStages][kMT][kP * 2];     // E rows, bf16
+    float gb[kMemStages][kMemPerCta][2][kMT];  // g per (memory, head, token)
+    float dl[kMemStages][kMemPerCta][2][kMT];  // dl per (memory, head, token)
+    uint32_t zz[kMemStages][kMT];              // z of the two heads (a bf16 pair) per token
+    float2 rq[kMemStages][kMT];                // (iq, ie) per token
+    uint64_t full[2];
     uint64_t mma_done[2];
     uint64_t drain;
     uint32_t tmem_base;
+    int abort;
 };
 
-// One tile's global data for one thread, prefetched into registers while the
-// previous tile's MMAs run: row tid >> 4 of C and Q (16-byte piece tid & 15),
-// and for head x = tid >> 8, row (tid >> 3) & 31: dY and E (piece tid & 7)
-// with the factors of c and a for both memories.
-struct MemRegs {
-    uint4 cv, qv, dv, ev;
-    float fg[kMemPerCta], fd[kMemPerCta];
-};
+__device__ __forceinline__ void cp_async16(void* dst, const void* src) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(tc::smem_u32(dst)), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async4(void* dst, const void* src) {
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(tc::smem_u32(dst)), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait1() { asm volatile("cp.async.wait_group 1;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait0() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
 
 template <typename Tmem>
 __global__ void __launch_bounds__(kMemThreads, 1)
@@ -672,89 +679,146 @@ sma_bwd_mem_kernel(const Tmem* __restrict__ Mem, const float* __restrict__ rM,
     const float rsn = rsqrtf((float)kN);
 
     if (tid == 0) {
+        tc::mbar_init(&sm.full[0], kMemFormThreads / 32);
+        tc::mbar_init(&sm.full[1], kMemFormThreads / 32);
         tc::mbar_init(&sm.mma_done[0], 1);
         tc::mbar_init(&sm.mma_done[1], 1);
         tc::mbar_init(&sm.drain, 1);
+        sm.abort = 0;
         tc::fence_barrier_init();
     }
     if (warp == 0) {
         tc::tmem_alloc(&sm.tmem_base, 512);
         tc::tmem_relinquish();
     }
+    const bool former = tid < kMemFormThreads;
     const int cr = tid >> 4, cq = tid & 15;                      // C / Q row, piece
     const int ex = tid >> 8, er = (tid >> 3) & 31, eq = tid & 7;  // head, dY / E row, piece
     const int eh = 2 * hp + ex;
-    MemRegs nx;
-    auto prefetch = [&](int it) {
-        const i64 tok0 = (i64)b * L + first + it * kMT;
-        nx.cv = reinterpret_cast<const uint4*>(Cm + (tok0 + cr) * kN)[cq];
-        nx.qv = reinterpret_cast<const uint4*>(Q + (tok0 + cr) * kN)[cq];
-        const i64 tok = tok0 + er;
-        const float2 q = rs[tok];
-        nx.dv = reinterpret_cast<const uint4*>(dY + (tok * H + eh) * kP)[eq];
-        nx.ev = reinterpret_cast<const uint4*>(E + tok * kP)[eq];
-        const float gate = silu_f32(__bfloat162float(z[tok * H + eh]));
-        const int t = first + it * kMT + er;  // position in the sequence
-#pragma unroll
-        for (int m = 0; m < kMemPerCta; ++m) {
-            const int j = j0 + m;
-            // memory j sees tokens of later chunks only (its factors are zero before)
-            const bool live = m < nm && t >= (j + 1) * S;
-            const i64 sidx = (((i64)b * H + eh) * Mc + j) * L + t;
-            nx.fg[m] = live ? gbuf[sidx] * gate : 0.0f;
-            nx.fd[m] = live ? dlbuf[sidx] * q.x * q.y * rsn : 0.0f;
+    // the copies of tile `it` into ring stage it % kMemStages (one commit group per
+    // tile and thread, empty past the last tile)
+    auto issue = [&](int it) {
+        if (it < ntiles) {
+            const int st = it % kMemStages;
+            const i64 tok0 = (i64)b * L + first + it * kMT;
+            const uint32_t o = (uint32_t)(cq >> 3) * kBlk + sw128((uint32_t)cr, (uint32_t)(cq & 7) * 16u);
+            cp_async16(sm.bc[st] + o, Cm + (tok0 + cr) * kN + 8 * cq);
+            cp_async16(sm.bq[st] + o, Q + (tok0 + cr) * kN + 8 * cq);
+            cp_async16(&sm.dy[st][er][ex][16 * eq], dY + ((tok0 + er) * H + eh) * kP + 8 * eq);
+            if (tid < 256) {
+                cp_async16(&sm.ee[st][tid >> 3][16 * (tid & 7)], E + (tok0 + (tid >> 3)) * kP + 8 * (tid & 7));
+            } else if (tid < 320) {  // g (256 .. 287) and dl (288 .. 319): 4 tokens a thread
+                const int i = tid - 256, which = i >> 5, m = (i >> 4) & 1, x = (i >> 3) & 1, pc = i & 7;
+                if (m < nm) {  // the other memory's rows lie past this CTA's last one
+                    const i64 sidx = (((i64)b * H + 2 * hp + x) * Mc + j0 + m) * L + first + it * kMT + 4 * pc;
+                    cp_async16(which ? &sm.dl[st][m][x][4 * pc] : &sm.gb[st][m][x][4 * pc],
+                               (which ? dlbuf : gbuf) + sidx);
+                }
+            } else if (tid < 352) {  // z of both heads for token tid - 320
+                const int r = tid - 320;
+                cp_async4(&sm.zz[st][r], z + (tok0 + r) * H + 2 * hp);
+            } else if (tid < 368) {  // (iq, ie) of two tokens
+                const int r = 2 * (tid - 352);
+                cp_async16(&sm.rq[st][r], rs + tok0 + r);
+            }
         }
+        cp_async_commit();
     };
-    if (ntiles > 0) prefetch(0);
+    if (former) {
+        issue(0);
+        issue(1);
+    }
     tc::tc_fence_before();
     __syncthreads();
     tc::tc_fence_after();
     const uint32_t tmem = sm.tmem_base;
-    constexpr uint32_t idM = idesc_bf16(true, true, kN, 2 * kP);  // A and B MN-major
+    volatile int* abort = &sm.abort;
 
     bool ok = true;
-    int issued = 0;  // tiles whose MMAs were issued
-    for (int it = 0; it < ntiles; ++it) {
-        const int bi = it & 1;
-        // buffer bi was read by the MMAs of tile it - 2
-        if (it >= 2) {
-            ok = cta_and_wait(&sm.mma_done[bi], (uint32_t)(((it - 2) >> 1) & 1), wait_limit_ns, 31);
-            if (!ok) break;
-        }
-        // C and Q rows: token r, columns n -> block n / 64, row r, bytes 2 (n % 64)
-        {
-            const uint32_t o = (uint32_t)(cq >> 3) * kBlk + sw128((uint32_t)cr, (uint32_t)(cq & 7) * 16u);
-            *reinterpret_cast<uint4*>(sm.bc[bi] + o) = nx.cv;
-            *reinterpret_cast<uint4*>(sm.bq[bi] + o) = nx.qv;
-        }
-        // c and a rows split hi / lo: memory m, token r, head x, columns p -> block x, row r
-        {
-            const uint32_t o = (uint32_t)ex * kBlk + sw128((uint32_t)er, (uint32_t)eq * 16u);
-            const uint32_t dw[4] = {nx.dv.x, nx.dv.y, nx.dv.z, nx.dv.w};
-            const uint32_t ew[4] = {nx.ev.x, nx.ev.y, nx.ev.z, nx.ev.w};
+    if (former) {
+        for (int it = 0; it < ntiles; ++it) {
+            const int bi = it & 1, st = it % kMemStages;
+            cp_async_wait1();  // this thread's copies of tile it (tile it + 1's may be in flight)
+            // everyone's copies, and one decision for all forming threads: stop if any of
+            // them has seen a wait give up (a forming warp's or the MMA thread's)
+            const uint32_t seen = *abort != 0 ? 1u : 0u;
+            uint32_t stop;
+            asm volatile(
+                "{\n\t.reg .pred p, q;\n\t"
+                "setp.ne.u32 q, %1, 0;\n\t"
+                "bar.red.or.pred p, 1, %2, q;\n\t"
+                "selp.u32 %0, 1, 0, p;\n\t}"
+                : "=r"(stop)
+                : "r"(seen), "n"(kMemFormThreads)
+                : "memory");
+            if (stop) break;
+            // c and a rows split hi / lo: memory m, token r, head x, columns p -> block x,
+            // row r. Buffer bi was read by the MMAs of tile it - 2, waited at the end of
+            // tile it - 1.
+            {
+                const int t = first + it * kMT + er;  // position in the sequence
+                const uint32_t zw = sm.zz[st][er];
+                const float gate = silu_f32(ex ? bf_hi(zw) : bf_lo(zw));
+                const float2 q = sm.rq[st][er];
+                const uint4 dv = *reinterpret_cast<const uint4*>(&sm.dy[st][er][ex][16 * eq]);
+                const uint4 ev = *reinterpret_cast<const uint4*>(&sm.ee[st][er][16 * eq]);
+                const uint32_t dw[4] = {dv.x, dv.y, dv.z, dv.w};
+                const uint32_t ew[4] = {ev.x, ev.y, ev.z, ev.w};
+                const uint32_t o = (uint32_t)ex * kBlk + sw128((uint32_t)er, (uint32_t)eq * 16u);
 #pragma unroll
-            for (int m = 0; m < kMemPerCta; ++m) {
-                float gv[8], av[8];
+                for (int m = 0; m < kMemPerCta; ++m) {
+                    // memory j sees tokens of later chunks only (its factors are zero before)
+                    const bool live = m < nm && t >= (j0 + m + 1) * S;
+                    const float fg = live ? sm.gb[st][m][ex][er] * gate : 0.0f;
+                    const float fd = live ? sm.dl[st][m][ex][er] * q.x * q.y * rsn : 0.0f;
+                    float gv[8], av[8];
 #pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    gv[2 * e] = bf_lo(dw[e]) * nx.fg[m];
-                    gv[2 * e + 1] = bf_hi(dw[e]) * nx.fg[m];
-                    av[2 * e] = bf_lo(ew[e]) * nx.fd[m];
-                    av[2 * e + 1] = bf_hi(ew[e]) * nx.fd[m];
+                    for (int e = 0; e < 4; ++e) {
+                        gv[2 * e] = bf_lo(dw[e]) * fg;
+                        gv[2 * e + 1] = bf_hi(dw[e]) * fg;
+                        av[2 * e] = bf_lo(ew[e]) * fd;
+                        av[2 * e + 1] = bf_hi(ew[e]) * fd;
+                    }
+                    uint4 hi, lo;
+                    split_bf16x8(gv, hi, lo);
+                    *reinterpret_cast<uint4*>(sm.bm[bi][m][0] + o) = hi;
+                    *reinterpret_cast<uint4*>(sm.bm[bi][m][1] + o) = lo;
+                    split_bf16x8(av, hi, lo);
+                    *reinterpret_cast<uint4*>(sm.bm[bi][m][2] + o) = hi;
+                    *reinterpret_cast<uint4*>(sm.bm[bi][m][3] + o) = lo;
                 }
-                uint4 hi, lo;
-                split_bf16x8(gv, hi, lo);
-                *reinterpret_cast<uint4*>(sm.bm[bi][m][0] + o) = hi;
-                *reinterpret_cast<uint4*>(sm.bm[bi][m][1] + o) = lo;
-                split_bf16x8(av, hi, lo);
-                *reinterpret_cast<uint4*>(sm.bm[bi][m][2] + o) = hi;
-                *reinterpret_cast<uint4*>(sm.bm[bi][m][3] + o) = lo;
+            }
+            // the copied C and Q rows and the stored B rows, to the MMA warp
+            tc::fence_proxy_async_shared();
+            __syncwarp();
+            if ((tid & 31) == 0) tc::mbar_arrive(&sm.full[bi]);
+            // tile it + 2 goes to the stage of tile it - 1, whose MMAs read its C and Q
+            // rows (and leave buffer bi ^ 1 free for tile it + 1)
+            if (it >= 1 && !warp_wait(&sm.mma_done[bi ^ 1], (uint32_t)(((it - 1) >> 1) & 1), wait_limit_ns, abort)) {
+                fail(abort, 31);
+                ok = false;
+            }
+            if (ok) issue(it + 2);
+            else cp_async_commit();  // keeps this thread's group count; the barrier then breaks
+        }
+        cp_async_wait0();  // also when a wait gave up: no copy outlives the CTA
+        // the last tile's MMAs (and with them every earlier one) are done
+        if (ok && !*abort && ntiles > 0) {
+            const int last = ntiles - 1;
+            if (!warp_wait(&sm.mma_done[last & 1], (uint32_t)((last >> 1) & 1), wait_limit_ns, abort)) {
+                fail(abort, 32);
             }
         }
-        tc::fence_proxy_async_shared();
-        tc::tc_fence_before();
-        __syncthreads();
-        if (tid == 0) {
+    } else if (tid == kMemFormThreads) {
+        // the MMA thread: tile it's operands on full[it & 1], its MMAs into mma_done[it & 1]
+        constexpr uint32_t idM = idesc_bf16(true, true, kN, 2 * kP);  // A and B MN-major
+        int issued = 0;
+        for (int it = 0; it < ntiles; ++it) {
+            const int bi = it & 1, st = it % kMemStages;
+            if (!tc::mbar_wait(&sm.full[bi], (uint32_t)((it >> 1) & 1), wait_limit_ns, abort)) {
+                fail(abort, 34);
+                break;
+            }
             tc::tc_fence_after();
             const int tb = first + it * kMT;
             for (int m = 0; m < nm; ++m) {
@@ -765,30 +829,27 @@ sma_bwd_mem_kernel(const Tmem* __restrict__ Mem, const float* __restrict__ rM,
                 for (int part = 0; part < 2; ++part)
                     for (int ks = 0; ks < kMT / 16; ++ks) {
                         const uint32_t acc = (!fresh || part > 0 || ks > 0) ? 1u : 0u;
-                        const uint64_t ac = tc::smem_desc_sw128(tc::smem_u32(sm.bc[bi]) + 2048u * ks, (uint32_t)kBlk, 1024u);
+                        const uint64_t ac = tc::smem_desc_sw128(tc::smem_u32(sm.bc[st]) + 2048u * ks, (uint32_t)kBlk, 1024u);
                         const uint64_t bgd = tc::smem_desc_sw128(tc::smem_u32(sm.bm[bi][m][part]) + 2048u * ks,
                                                                  (uint32_t)kBlk, 1024u);
                         mma_ss(d, ac, bgd, idM, acc);
-                        const uint64_t aq = tc::smem_desc_sw128(tc::smem_u32(sm.bq[bi]) + 2048u * ks, (uint32_t)kBlk, 1024u);
+                        const uint64_t aq = tc::smem_desc_sw128(tc::smem_u32(sm.bq[st]) + 2048u * ks, (uint32_t)kBlk, 1024u);
                         const uint64_t bdd = tc::smem_desc_sw128(tc::smem_u32(sm.bm[bi][m][2 + part]) + 2048u * ks,
                                                                  (uint32_t)kBlk, 1024u);
                         mma_ss(d + 128u, aq, bdd, idM, acc);
                     }
             }
             tc::mma_commit(&sm.mma_done[bi]);
+            issued = it + 1;
         }
-        issued = it + 1;
-        if (it + 1 < ntiles) prefetch(it + 1);  // lands while these MMAs run
+        if (*abort && issued > 0) {  // let the MMAs in flight finish before TMEM is freed
+            tc::mma_commit(&sm.drain);
+            if (!tc::mbar_wait(&sm.drain, 0, kDrainLimitNs, nullptr)) atomicCAS(&g_bwd_tc_status, 0, 33);
+        }
     }
-    // the last tile's MMAs (and with them every earlier one) are done
-    if (ok && ntiles > 0) {
-        const int last = ntiles - 1;
-        ok = cta_and_wait(&sm.mma_done[last & 1], (uint32_t)((last >> 1) & 1), wait_limit_ns, 32);
-    }
-    if (!ok && issued > 0 && tid == 0) {  // let the MMAs in flight finish before TMEM is freed
-        tc::mma_commit(&sm.drain);
-        if (!tc::mbar_wait(&sm.drain, 0, kDrainLimitNs, nullptr)) atomicCAS(&g_bwd_tc_status, 0, 33);
-    }
+    tc::tc_fence_before();
+    __syncthreads();
+    ok = !*abort;
     tc::tc_fence_after();
     const int m = tid >> 8;
     if (ok && m < nm) {
