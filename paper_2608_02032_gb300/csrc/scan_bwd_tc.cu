@@ -404,15 +404,22 @@ psi_kernel(const __grid_constant__ CUtensorMap tm_X, const __grid_constant__ CUt
 }
 
 // ---------------------------------------------------------------- dC / dB
-constexpr int kDcThreads = 512;
+// Warps 0..15 stage each unit's register-formed operand part; warp 16 issues the
+// unit's bulk copy and its MMAs. formed[b] (one arrival per staging warp) and
+// full[b] (the copy) hand buffer b to the MMA thread, mma_done[b] hands it back,
+// so no staging warp waits for the MMA issue.
+constexpr int kDcFormThreads = 512;
+constexpr int kDcThreads = kDcFormThreads + 32;
 constexpr int kUnit = 16384;  // one operand slot
 
 struct DcSmem {
     uint8_t slot[2][4][kUnit];  // per buffer: A hi, A lo, B (or B hi), B lo
     uint64_t full[2];           // the unit's 32 KiB bulk-copied part landed in buffer 0 / 1
+    uint64_t formed[2];         // the staging warps' part is in buffer 0 / 1
     uint64_t mma_done[2];
     uint64_t drain;
     uint32_t tmem_base;
+    int abort;
 };
 
 // kind 0: dC rows of a 128-token tile (accumulated into dC); kind 1: dB rows.
@@ -441,9 +448,11 @@ dcdb_kernel(const __nv_bfloat16* __restrict__ X, const float* __restrict__ dt,
     if (tid == 0) {
         for (int u = 0; u < 2; ++u) {
             tc::mbar_init(&sm.full[u], 1);
+            tc::mbar_init(&sm.formed[u], kDcFormThreads / 32);
             tc::mbar_init(&sm.mma_done[u], 1);
         }
         tc::mbar_init(&sm.drain, 1);
+        sm.abort = 0;
         tc::fence_barrier_init();
     }
     if (warp == 0) {
@@ -455,25 +464,109 @@ dcdb_kernel(const __nv_bfloat16* __restrict__ X, const float* __restrict__ dt,
     tc::tc_fence_after();
     const uint32_t tmem = sm.tmem_base;
     const float* cumb = cum + (i64)b * H * Mc * S;  // + (h Mc + c) S + t
+    volatile int* abort = &sm.abort;
+    auto fail_code = [&](int code) {
+        *abort = 1;
+        atomicCAS(&g_sbwd_tc_status, 0, code);
+    };
 
-    bool ok = true;
-    int issued = 0;   // units whose MMAs were issued
-    int copied = 0;   // units whose bulk copy was issued (thread 0)
-    for (int u = 0; u < nunits; ++u) {
-        const int bi = u & 1;
-        if (u >= 2) {
-            ok = cta_wait(&sm.mma_done[bi], (uint32_t)(((u - 2) >> 1) & 1), wait_limit_ns, 43);
-            if (!ok) break;
+    if (tid < kDcFormThreads) {
+        for (int u = 0; u < nunits; ++u) {
+            const int bi = u & 1;
+            // buffer bi was read by the MMAs of unit u - 2
+            if (u >= 2) {
+                const bool got = tc::mbar_wait(&sm.mma_done[bi], (uint32_t)(((u - 2) >> 1) & 1), wait_limit_ns, abort);
+                if (!__all_sync(0xffffffffu, got)) {
+                    if ((tid & 31) == 0) fail_code(43);
+                    break;
+                }
+            }
+            uint8_t* a_hi = sm.slot[bi][0];
+            uint8_t* a_lo = sm.slot[bi][1];
+            uint8_t* b0 = sm.slot[bi][2];
+            if (u < nintra) {
+                // B: 64 token rows of B (dC) or C (dB), MN-major N = 128: [n block][64 rows][128 bytes]
+                const int r0 = kind == 0 ? 64 * u : tt * kT + 64 * u;
+                const __nv_bfloat16* src = kind == 0 ? Bm : Cm;
+                uint4 v[2];
+#pragma unroll
+                for (int k = 0; k < 2; ++k) {
+                    const int i = tid + k * kDcFormThreads, r = i / 16, q = i % 16;
+                    v[k] = reinterpret_cast<const uint4*>(src + (tok0 + r0 + r) * kN)[q];
+                }
+#pragma unroll
+                for (int k = 0; k < 2; ++k) {
+                    const int i = tid + k * kDcFormThreads, r = i / 16, q = i % 16;
+                    *reinterpret_cast<uint4*>(b0 + (q / 8) * 8192 + sw128((uint32_t)r, (uint32_t)(q % 8) * 16u)) = v[k];
+                }
+            } else {
+                const int h = u - nintra;
+                // A: exp(cum_t) dY_t (dC) or exp(cum_end - cum_s) dt_s X_s (dB) of head h, K = p, split
+                const float* cumh = cumb + ((i64)h * Mc + c) * S;
+                const float cend = kind == 0 ? 0.0f : cumh[S - 1];
+                uint4 w[2];
+                float f[2];
+#pragma unroll
+                for (int k = 0; k < 2; ++k) {  // every load of the thread in flight at once
+                    const int i = tid + k * kDcFormThreads, r = i / 8, q = i % 8;
+                    const int t = tt * kT + r;
+                    const i64 tok = tok0 + t;
+                    if (kind == 0) {
+                        f[k] = cumh[t];
+                        w[k] = reinterpret_cast<const uint4*>(dY + (tok * H + h) * kP)[q];
+                    } else {
+                        f[k] = dt[tok * H + h];
+                        w[k] = reinterpret_cast<const uint4*>(X + (tok * H + h) * kP)[q];
+                    }
+                }
+#pragma unroll
+                for (int k = 0; k < 2; ++k) {
+                    const int i = tid + k * kDcFormThreads, r = i / 8, q = i % 8;
+                    const int t = tt * kT + r;
+                    const float fk = kind == 0 ? expf(f[k]) : expf(cend - cumh[t]) * f[k];
+                    const uint32_t ww[4] = {w[k].x, w[k].y, w[k].z, w[k].w};
+                    float v[8];
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        v[2 * e] = bf_lo(ww[e]) * fk;
+                        v[2 * e + 1] = bf_hi(ww[e]) * fk;
+                    }
+                    uint4 hi, lo;
+                    split8(v, hi, lo);
+                    const uint32_t o = sw128((uint32_t)r, (uint32_t)q * 16u);
+                    *reinterpret_cast<uint4*>(a_hi + o) = hi;
+                    *reinterpret_cast<uint4*>(a_lo + o) = lo;
+                }
+                // B: H_[c-1] (dC) or d(dH_c) (dB) of head h, [n][p] hi | lo, K-major (rows n,
+                // K = p): the MMA thread's bulk copy
+            }
+            tc::fence_proxy_async_shared();
+            __syncwarp();
+            if ((tid & 31) == 0) tc::mbar_arrive(&sm.formed[bi]);
         }
-        uint8_t* a_hi = sm.slot[bi][0];
-        uint8_t* a_lo = sm.slot[bi][1];
-        uint8_t* b0 = sm.slot[bi][2];
-        uint8_t* b1 = sm.slot[bi][3];
-        const bool intra = u < nintra;
-        // Every unit has one 32 KiB part that is already laid out in global memory: the
-        // Psi blocks (intra) or the H / d(dH) operand tile (per head); bulk copies bring
-        // it in while the threads stage the rest.
-        if (tid == 0) {
+        // the last unit's MMAs (and with them every earlier one) are done
+        if (!*abort && nunits > 0) {
+            const int last = nunits - 1;
+            const bool got = tc::mbar_wait(&sm.mma_done[last & 1], (uint32_t)((last >> 1) & 1), wait_limit_ns, abort);
+            if (!__all_sync(0xffffffffu, got) && (tid & 31) == 0) fail_code(44);
+        }
+    } else if (tid == kDcFormThreads) {
+        int issued = 0;  // units whose MMAs were issued
+        int copied = 0;  // units whose bulk copy was issued
+        for (int u = 0; u < nunits; ++u) {
+            const int bi = u & 1;
+            if (u >= 2 && !tc::mbar_wait(&sm.mma_done[bi], (uint32_t)(((u - 2) >> 1) & 1), wait_limit_ns, abort)) {
+                fail_code(43);
+                break;
+            }
+            uint8_t* a_hi = sm.slot[bi][0];
+            uint8_t* a_lo = sm.slot[bi][1];
+            uint8_t* b0 = sm.slot[bi][2];
+            uint8_t* b1 = sm.slot[bi][3];
+            const bool intra = u < nintra;
+            // Every unit has one 32 KiB part that is already laid out in global memory: the
+            // Psi blocks (intra) or the H / d(dH) operand tile (per head); the bulk copy
+            // brings it in while the staging warps form the rest.
             tc::mbar_arrive_expect_tx(&sm.full[bi], 32768u);
             if (!intra) {
                 const int h = u - nintra;
@@ -496,57 +589,14 @@ dcdb_kernel(const __nv_bfloat16* __restrict__ X, const float* __restrict__ dt,
                                      8192u, &sm.full[bi]);
             }
             copied = u + 1;
-        }
-        if (intra) {
-            // B: 64 token rows of B (dC) or C (dB), MN-major N = 128: [n block][64 rows][128 bytes]
-            const int r0 = kind == 0 ? 64 * u : tt * kT + 64 * u;
-            const __nv_bfloat16* src = kind == 0 ? Bm : Cm;
-            for (int i = tid; i < 64 * 16; i += kDcThreads) {
-                const int r = i / 16, q = i % 16;
-                const uint4 v = reinterpret_cast<const uint4*>(src + (tok0 + r0 + r) * kN)[q];
-                *reinterpret_cast<uint4*>(b0 + (q / 8) * 8192 + sw128((uint32_t)r, (uint32_t)(q % 8) * 16u)) = v;
+            if (!tc::mbar_wait(&sm.formed[bi], (uint32_t)((u >> 1) & 1), wait_limit_ns, abort)) {
+                fail_code(48);
+                break;
             }
-        } else {
-            const int h = u - nintra;
-            // A: exp(cum_t) dY_t (dC) or exp(cum_end - cum_s) dt_s X_s (dB) of head h, K = p, split
-            const float* cumh = cumb + ((i64)h * Mc + c) * S;
-            const float cend = cumh[S - 1];
-            for (int i = tid; i < kT * 8; i += kDcThreads) {
-                const int r = i / 8, q = i % 8;
-                const int t = tt * kT + r;
-                const i64 tok = tok0 + t;
-                float f;
-                uint4 w;
-                if (kind == 0) {
-                    f = expf(cumh[t]);
-                    w = reinterpret_cast<const uint4*>(dY + (tok * H + h) * kP)[q];
-                } else {
-                    f = expf(cend - cumh[t]) * dt[tok * H + h];
-                    w = reinterpret_cast<const uint4*>(X + (tok * H + h) * kP)[q];
-                }
-                const uint32_t ww[4] = {w.x, w.y, w.z, w.w};
-                float v[8];
-#pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    v[2 * e] = bf_lo(ww[e]) * f;
-                    v[2 * e + 1] = bf_hi(ww[e]) * f;
-                }
-                uint4 hi, lo;
-                split8(v, hi, lo);
-                const uint32_t o = sw128((uint32_t)r, (uint32_t)q * 16u);
-                *reinterpret_cast<uint4*>(a_hi + o) = hi;
-                *reinterpret_cast<uint4*>(a_lo + o) = lo;
+            if (!tc::mbar_wait(&sm.full[bi], (uint32_t)((u >> 1) & 1), wait_limit_ns, abort)) {
+                fail_code(46);
+                break;
             }
-            // B: H_[c-1] (dC) or d(dH_c) (dB) of head h, [n][p] hi | lo, K-major (rows n,
-            // K = p): the bulk copy above
-        }
-        tc::fence_proxy_async_shared();
-        tc::tc_fence_before();
-        __syncthreads();
-        if (tid == 0 && !tc::mbar_wait(&sm.full[bi], (uint32_t)((u >> 1) & 1), wait_limit_ns, nullptr)) {
-            // no MMA for this unit: the next wait on its mma_done runs out and ends the loop
-            atomicCAS(&g_sbwd_tc_status, 0, 46);
-        } else if (tid == 0) {
             tc::tc_fence_after();
             const uint32_t sa_hi = tc::smem_u32(a_hi), sa_lo = tc::smem_u32(a_lo);
             const uint32_t sb0 = tc::smem_u32(b0), sb1 = tc::smem_u32(b1);
@@ -574,24 +624,21 @@ dcdb_kernel(const __nv_bfloat16* __restrict__ X, const float* __restrict__ dt,
                 }
             }
             tc::mma_commit(&sm.mma_done[bi]);
+            issued = u + 1;
         }
-        issued = u + 1;
-    }
-    if (ok && nunits > 0) {
-        const int last = nunits - 1;
-        ok = cta_wait(&sm.mma_done[last & 1], (uint32_t)((last >> 1) & 1), wait_limit_ns, 44);
-    }
-    if (!ok && issued > 0 && tid == 0) {
-        tc::mma_commit(&sm.drain);
-        if (!tc::mbar_wait(&sm.drain, 0, kDrainLimitNs, nullptr)) atomicCAS(&g_sbwd_tc_status, 0, 45);
-    }
-    if (tid == 0) {  // never leave a copy in flight behind: the last copy into each buffer
+        if (*abort && issued > 0) {  // let the MMAs in flight finish before TMEM is freed
+            tc::mma_commit(&sm.drain);
+            if (!tc::mbar_wait(&sm.drain, 0, kDrainLimitNs, nullptr)) atomicCAS(&g_sbwd_tc_status, 0, 45);
+        }
+        // never leave a copy in flight behind: the last copy into each buffer
         for (int k = copied - 1; k >= 0 && k >= copied - 2; --k)
             if (!tc::mbar_wait(&sm.full[k & 1], (uint32_t)((k >> 1) & 1), kDrainLimitNs, nullptr))
                 atomicCAS(&g_sbwd_tc_status, 0, 47);
     }
+    tc::tc_fence_before();
+    __syncthreads();
     tc::tc_fence_after();
-    if (ok) {
+    if (!*abort && tid < kDcFormThreads) {
         // thread (row, quarter): 32 columns of its token row
         const int r = tid & (kT - 1), qc = tid >> 7;
         const uint32_t lane_addr = (uint32_t)(32 * (warp & 3)) << 16;
