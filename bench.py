@@ -320,6 +320,7 @@ def run_dart(args) -> None:
 
     for _ in range(args.warmup):
         step()
+        step(split=True)
     torch.cuda.synchronize()
 
     # ---- kernel-level timing, inputs resident in HBM
