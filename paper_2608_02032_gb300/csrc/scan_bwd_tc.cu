@@ -471,8 +471,47 @@ dcdb_kernel(const __nv_bfloat16* __restrict__ X, const float* __restrict__ dt,
     };
 
     if (tid < kDcFormThreads) {
+        // a unit's global inputs for this thread, loaded one unit ahead: intra, w = two
+        // pieces of B (dC) or C (dB) rows; per head, w = two pieces of dY (dC) or X (dB)
+        // rows, f = cum_t (dC) or dt_s (dB), g = cum_s and e = cum_end (dB)
+        struct DcRegs {
+            uint4 w[2];
+            float f[2], g[2], e;
+        };
+        auto load_unit = [&](int u, DcRegs& R) {
+            if (u < nintra) {
+                const int r0 = kind == 0 ? 64 * u : tt * kT + 64 * u;
+                const __nv_bfloat16* src = kind == 0 ? Bm : Cm;
+#pragma unroll
+                for (int k = 0; k < 2; ++k) {
+                    const int i = tid + k * kDcFormThreads, r = i / 16, q = i % 16;
+                    R.w[k] = reinterpret_cast<const uint4*>(src + (tok0 + r0 + r) * kN)[q];
+                }
+            } else {
+                const int h = u - nintra;
+                const float* cumh = cumb + ((i64)h * Mc + c) * S;
+                R.e = kind == 0 ? 0.0f : cumh[S - 1];
+#pragma unroll
+                for (int k = 0; k < 2; ++k) {
+                    const int i = tid + k * kDcFormThreads, r = i / 8, q = i % 8;
+                    const int t = tt * kT + r;
+                    const i64 tok = tok0 + t;
+                    if (kind == 0) {
+                        R.f[k] = cumh[t];
+                        R.w[k] = reinterpret_cast<const uint4*>(dY + (tok * H + h) * kP)[q];
+                    } else {
+                        R.f[k] = dt[tok * H + h];
+                        R.g[k] = cumh[t];
+                        R.w[k] = reinterpret_cast<const uint4*>(X + (tok * H + h) * kP)[q];
+                    }
+                }
+            }
+        };
+        DcRegs cur, nxt;
+        if (nunits > 0) load_unit(0, cur);
         for (int u = 0; u < nunits; ++u) {
             const int bi = u & 1;
+            if (u + 1 < nunits) load_unit(u + 1, nxt);  // in flight under this unit's wait and stores
             // buffer bi was read by the MMAs of unit u - 2
             if (u >= 2) {
                 const bool got = tc::mbar_wait(&sm.mma_done[bi], (uint32_t)(((u - 2) >> 1) & 1), wait_limit_ns, abort);
@@ -486,45 +525,18 @@ dcdb_kernel(const __nv_bfloat16* __restrict__ X, const float* __restrict__ dt,
             uint8_t* b0 = sm.slot[bi][2];
             if (u < nintra) {
                 // B: 64 token rows of B (dC) or C (dB), MN-major N = 128: [n block][64 rows][128 bytes]
-                const int r0 = kind == 0 ? 64 * u : tt * kT + 64 * u;
-                const __nv_bfloat16* src = kind == 0 ? Bm : Cm;
-                uint4 v[2];
 #pragma unroll
                 for (int k = 0; k < 2; ++k) {
                     const int i = tid + k * kDcFormThreads, r = i / 16, q = i % 16;
-                    v[k] = reinterpret_cast<const uint4*>(src + (tok0 + r0 + r) * kN)[q];
-                }
-#pragma unroll
-                for (int k = 0; k < 2; ++k) {
-                    const int i = tid + k * kDcFormThreads, r = i / 16, q = i % 16;
-                    *reinterpret_cast<uint4*>(b0 + (q / 8) * 8192 + sw128((uint32_t)r, (uint32_t)(q % 8) * 16u)) = v[k];
+                    *reinterpret_cast<uint4*>(b0 + (q / 8) * 8192 + sw128((uint32_t)r, (uint32_t)(q % 8) * 16u)) = cur.w[k];
                 }
             } else {
-                const int h = u - nintra;
                 // A: exp(cum_t) dY_t (dC) or exp(cum_end - cum_s) dt_s X_s (dB) of head h, K = p, split
-                const float* cumh = cumb + ((i64)h * Mc + c) * S;
-                const float cend = kind == 0 ? 0.0f : cumh[S - 1];
-                uint4 w[2];
-                float f[2];
-#pragma unroll
-                for (int k = 0; k < 2; ++k) {  // every load of the thread in flight at once
-                    const int i = tid + k * kDcFormThreads, r = i / 8, q = i % 8;
-                    const int t = tt * kT + r;
-                    const i64 tok = tok0 + t;
-                    if (kind == 0) {
-                        f[k] = cumh[t];
-                        w[k] = reinterpret_cast<const uint4*>(dY + (tok * H + h) * kP)[q];
-                    } else {
-                        f[k] = dt[tok * H + h];
-                        w[k] = reinterpret_cast<const uint4*>(X + (tok * H + h) * kP)[q];
-                    }
-                }
 #pragma unroll
                 for (int k = 0; k < 2; ++k) {
                     const int i = tid + k * kDcFormThreads, r = i / 8, q = i % 8;
-                    const int t = tt * kT + r;
-                    const float fk = kind == 0 ? expf(f[k]) : expf(cend - cumh[t]) * f[k];
-                    const uint32_t ww[4] = {w[k].x, w[k].y, w[k].z, w[k].w};
+                    const float fk = kind == 0 ? expf(cur.f[k]) : expf(cur.e - cur.g[k]) * cur.f[k];
+                    const uint32_t ww[4] = {cur.w[k].x, cur.w[k].y, cur.w[k].z, cur.w[k].w};
                     float v[8];
 #pragma unroll
                     for (int e = 0; e < 4; ++e) {
@@ -543,6 +555,7 @@ dcdb_kernel(const __nv_bfloat16* __restrict__ X, const float* __restrict__ dt,
             tc::fence_proxy_async_shared();
             __syncwarp();
             if ((tid & 31) == 0) tc::mbar_arrive(&sm.formed[bi]);
+            cur = nxt;
         }
         // the last unit's MMAs (and with them every earlier one) are done
         if (!*abort && nunits > 0) {
