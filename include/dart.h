@@ -37,6 +37,14 @@
  *     legacy default stream) and does not synchronise the host.
  *     dart_prefill_host also works on streams of its own (created once per
  *     device); calls from several host threads share them and run in turn.
+ *   - Stream order holds as for plain launches, with one overlap inside it:
+ *     the tensor-core SMA kernel (dart_sma_forward, _with_tiles and
+ *     _with_logits on their tensor-core shapes) is launched with programmatic
+ *     stream serialization. When the kernel just before it on the stream is
+ *     the scan's output kernel, which writes only Y_ssd, its CTAs may start
+ *     while that kernel's last CTAs still run, and they read Y_ssd only after
+ *     it has completed. After any other kernel, copy or event it starts once
+ *     that work is done.
  *   - Arguments are validated on the host before anything is launched; a
  *     call that returns an error has written nothing.
  *   - Token and chunk indices are 0-based: token t lies in chunk t / S, the
