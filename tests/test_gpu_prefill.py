@@ -74,6 +74,7 @@ SWEEP = [
     (129, 128, 64, 128, 8, 1, "bf16"),     # one full chunk and a one-token chunk: only the last token reads a memory
     # ragged L (L % S != 0): the last memory holds the partial chunk
     (1000, 256, 64, 128, 8, 1, "bf16"),    # tensor-core scan and SMA on 1024 padded tokens
+    (1000, 256, 64, 128, 4, 1, "bf16"),    # the same with four heads (one chunk-state CTA per chunk)
     (1000, 256, 64, 128, 2, 1, "bf16"),    # CUDA-core scan, tensor-core SMA
     (300, 64, 32, 32, 2, 1, "f32"),        # CUDA-core path, 5 memories, 44-token last chunk
     (97, 32, 16, 16, 3, 1, "f32"),         # a last chunk of one token (97 = 3 x 32 + 1)
