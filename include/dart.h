@@ -148,6 +148,9 @@ size_t dart_workspace_size(const dart_dims* dims, int op);
  * ceil(L / S) S tokens inside the workspace (a padded token has dt = 0: decay 1,
  * no write, so states and memories are exactly the L-token ones) and the first L
  * rows of Y_ssd are copied out; dart_workspace_size includes the copies.
+ * The tensor-core kernels serve bf16 inputs with P = 64, N = 128, S in
+ * {64, 128, 256} and H, H / G multiples of 4; every other shape runs on the
+ * CUDA-core kernels.
  */
 dart_status dart_chunk_scan(const dart_dims* dims, const void* X, const float* dt,
                             const float* A, const void* Bm, const void* Cm, void* Y_ssd,
@@ -185,12 +188,12 @@ dart_status dart_sma_forward(const dart_dims* dims, const void* M, const float* 
 /*
  * The prefill of one block (dart_chunk_scan then dart_sma_forward) from
  * host buffers to a host buffer, with the copies overlapped with the kernels.
- * The heads are taken in groups of 8 when G = 1 and H is a larger multiple of
- * 8 (one group otherwise): per group the X rows go to the device (a pitched
- * copy), the scan and SMA kernels run on them, and the group's Y rows come
- * back, on four streams of the library's own (copy in, two for the kernels
- * taking the groups in turn, copy out), so that the copies run under the
- * kernels and neighbouring groups' kernels share the SMs. The shared inputs
+ * The heads are taken in groups of 4 when G = 1 and H is a larger multiple of
+ * 4 with at most 64 groups (one group otherwise): per group the X rows go to
+ * the device (a pitched copy), the scan and SMA kernels run on them, and the
+ * group's Y rows come back, on five streams of the library's own (copy in,
+ * three for the kernels taking the groups in turn, copy out), so that the
+ * copies run under the kernels and neighbouring groups' kernels share the SMs. The shared inputs
  * (B, C, Q, E, dt, A, z) go first; the gather of a group's dt and gate logits
  * runs on the device. Per head the result is that of the device entry points.
  * Inputs:  X (Bsz, L, H, P), Bm, Cm, Q (Bsz, L, G, N), E (Bsz, L, G, P),
@@ -307,7 +310,7 @@ dart_status dart_sma_backward_with_logits(const dart_dims* dims, const void* M, 
  * Other arguments, outputs and the scan's workspace as for dart_chunk_scan and
  * dart_sma_forward; dart_sma_forward_with_tiles takes no workspace.
  * Requires the tensor-core paths of both calls: bf16 inputs, P = 64, N = 128,
- * S in {64, 128, 256}, H/G a multiple of 8, L a multiple of 128 and of S.
+ * S in {64, 128, 256}, H and H/G multiples of 4, L a multiple of 128 and of S.
  * dart_sma_tiles_size returns 0 elsewhere, and the calls DART_ERR_UNSUPPORTED.
  */
 size_t dart_sma_tiles_size(const dart_dims* dims);
